@@ -1,0 +1,356 @@
+"""Pins of the CPU oracle against what the paper and the mathematics fix (no GPU).
+
+Each pin reaches the oracle's result by another route: PyTorch's scaled_dot_product_attention
+and F.linear (library routines for softmax attention and the output projection), numpy's
+reduceat (block sums), the paper's closed forms (Eq. 4, 9, 14-16), brute-force search over
+every drop set, and invariants (scale, permutation, track-best, schedule totals).
+"""
+import itertools
+import math
+
+import numpy as np
+import pytest
+import torch
+import torch.nn.functional as F
+
+import oracle as O
+import synth
+
+torch.set_default_dtype(torch.float64)
+
+
+# ---------------------------------------------------------------------------------------
+# small layers
+# ---------------------------------------------------------------------------------------
+def small_layer(n_tokens=778, n_special=10, heads=2, d_model=128, seed=1):
+    d = synth.make_random_layer(n_tokens, heads, d_model, seed)
+    X = {k: synth.bf16_to_f32(v).astype(np.float64) for k, v in d.items()}
+    return X, n_special
+
+
+def sdpa(q, k, v, mask=None):
+    """Library softmax attention in float64: q [M, d], k/v [L, d], mask [M, L] bool."""
+    t = lambda a: torch.from_numpy(np.ascontiguousarray(a))[None, None]
+    m = None if mask is None else torch.from_numpy(mask)[None, None]
+    return F.scaled_dot_product_attention(t(q), t(k), t(v), attn_mask=m)[0, 0].numpy()
+
+
+def pooled_output_via_library(pooled, h, i, D=None):
+    """Renormalised pooled attention output of row (h, i) with the blocks of D masked."""
+    q = pooled.Qb[h, i][None]
+    mask = None if D is None else (~np.asarray(D, dtype=bool))[None]
+    return sdpa(q, pooled.Kb[h], pooled.Vb[h], mask)[0]
+
+
+def residual_drift_via_library(pooled, W_o, h, i, D):
+    """||y_masked - y_dense||^2 with y = F.linear(concat_h pooled outputs, W_o): the change
+    the masked attention sublayer leaves in the residual stream (Sec. 3, Eq. 11-12)."""
+    H = pooled.heads
+    dense = np.concatenate([pooled_output_via_library(pooled, g, i) for g in range(H)])
+    masked = dense.copy()
+    d_h = pooled.Qb.shape[2]
+    masked[h * d_h:(h + 1) * d_h] = pooled_output_via_library(pooled, h, i, D)
+    W = torch.from_numpy(W_o)
+    y0 = F.linear(torch.from_numpy(dense), W)
+    y1 = F.linear(torch.from_numpy(masked), W)
+    return float(((y1 - y0) ** 2).sum())
+
+
+@pytest.fixture(scope="module")
+def layer():
+    X, ns = small_layer()
+    pooled = O.pool(X["Q"], X["K"], X["V"], ns)
+    return X, pooled
+
+
+# ---------------------------------------------------------------------------------------
+# pooling and the pooled attention map
+# ---------------------------------------------------------------------------------------
+def test_shapes_of_the_block_grid():
+    wl = synth.WORKLOADS["vggt_v32"]
+    assert O.n_blocks(wl.n_tokens) == 687
+    assert O.n_candidates(wl.n_tokens, wl.n_special) == 684
+    wl1 = synth.WORKLOADS["tiny_v2"]
+    assert (O.n_blocks(wl1.n_tokens), O.n_candidates(wl1.n_tokens, wl1.n_special)) == (43, 42)
+    assert int(wl1.budgets()[0]) == 21 and int(wl.budgets()[0]) == 68
+
+
+def test_pool_blocks_matches_reduceat(layer):
+    X, pooled = layer
+    N = X["Q"].shape[0]
+    starts = np.arange(0, N, 64)
+    counts = np.diff(np.append(starts, N))
+    for name, got in (("Q", pooled.Qb), ("K", pooled.Kb), ("V", pooled.Vb)):
+        ref = np.add.reduceat(X[name], starts, axis=0) / counts[:, None, None]
+        np.testing.assert_allclose(got, np.transpose(ref, (1, 0, 2)), rtol=1e-13, atol=1e-13)
+    assert counts[-1] == N - 64 * (len(starts) - 1) == 10   # ragged tail block
+
+
+def test_dense_pooled_output_is_library_attention(layer):
+    """Eq. 1 with P from the pooled softmax equals softmax attention at block level."""
+    _, pooled = layer
+    for h in range(pooled.heads):
+        for i in (0, 5, pooled.nb - 1):
+            P_i, vbar = O.row_quantities(pooled, h, i)
+            assert abs(P_i.sum() - 1) < 1e-13 and (P_i > 0).all()
+            np.testing.assert_allclose(vbar, pooled_output_via_library(pooled, h, i),
+                                       rtol=1e-12, atol=1e-13)
+
+
+def test_single_block_masking_identity(layer):
+    """Eq. 3-4: masking block j gives v_bar + P/(1-P) (v_bar - V_j) exactly."""
+    _, pooled = layer
+    h, i = 1, 3
+    P_i, vbar = O.row_quantities(pooled, h, i)
+    for j in range(pooled.nb):
+        D = np.zeros(pooled.nb, dtype=bool)
+        D[j] = True
+        direct = pooled_output_via_library(pooled, h, i, D)
+        closed = vbar + P_i[j] / (1 - P_i[j]) * (vbar - pooled.Vb[h, j])
+        np.testing.assert_allclose(direct, closed, rtol=1e-11, atol=1e-12)
+
+
+# ---------------------------------------------------------------------------------------
+# drift score and objective
+# ---------------------------------------------------------------------------------------
+def test_drift_score_equals_gram_expansion(layer):
+    """Eq. 6 == Eq. 9: s_ij = P_ij sqrt(v^T M v - 2 v^T M V_j + V_j^T M V_j), M = W^T W."""
+    X, pooled = layer
+    d_h = 64
+    for h in range(pooled.heads):
+        WOh = O.head_projection(X["W_o"], h, d_h)
+        M = WOh.T @ WOh                                              # Eq. 8
+        P_i, vbar = O.row_quantities(pooled, h, 4)
+        _, _, r = O.residual_contributions(P_i, vbar, pooled.Vb[h], WOh)
+        s = O.drift_scores(r)
+        Vb = pooled.Vb[h]
+        q = vbar @ M @ vbar - 2 * (Vb @ M @ vbar) + np.einsum("jd,de,je->j", Vb, M, Vb)
+        np.testing.assert_allclose(s, P_i * np.sqrt(np.maximum(q, 0)), rtol=1e-9)
+
+
+def test_objective_equals_measured_residual_drift(layer):
+    """Eq. 10-12: G/K^2 from the contribution vectors equals the change the masked
+    attention output leaves after the output projection, for random drop sets."""
+    X, pooled = layer
+    rng = np.random.default_rng(0)
+    for h in range(pooled.heads):
+        for i in (0, 7, 11):
+            for size in (1, 3, 6, 12):
+                D = np.zeros(pooled.nb, dtype=bool)
+                D[rng.choice(pooled.n_cand, size, replace=False)] = True
+                J = O.drift_of(pooled, X["W_o"], h, i, D)
+                ref = residual_drift_via_library(pooled, X["W_o"], h, i, D)
+                assert J == pytest.approx(ref, rel=1e-9, abs=1e-18)
+
+
+def test_single_drop_objective_is_squared_cut_key(layer):
+    """Sec. 4.3: for D = {j}, Eq. 12 reduces to the square of the Eq. 7 key."""
+    X, pooled = layer
+    h, i = 0, 2
+    P_i, vbar = O.row_quantities(pooled, h, i)
+    _, _, r = O.residual_contributions(P_i, vbar, pooled.Vb[h], O.head_projection(X["W_o"], h, 64))
+    key = O.cut_keys(O.drift_scores(r), P_i)
+    for j in range(pooled.n_cand):
+        D = np.zeros(pooled.nb, dtype=bool)
+        D[j] = True
+        assert O.objective(D, P_i, r)[0] == pytest.approx(key[j] ** 2, rel=1e-11)
+
+
+def test_round_gains_match_closed_form(layer):
+    """Eq. 14-16: the directly recomputed gains equal G/K^2 - (G + dG)/(K + u)^2 with
+    dG = -/+ 2 d^T M g + s^2 computed from M_h = W_O^h^T W_O^h."""
+    X, pooled = layer
+    h, i = 1, 6
+    WOh = O.head_projection(X["W_o"], h, 64)
+    M = WOh.T @ WOh
+    P_i, vbar = O.row_quantities(pooled, h, i)
+    _, dvec, r = O.residual_contributions(P_i, vbar, pooled.Vb[h], WOh)
+    s = O.drift_scores(r)
+    D = np.zeros(pooled.nb, dtype=bool)
+    D[[0, 2, 3, 7, 9, 10]] = True
+    J, a, K = O.objective(D, P_i, r)
+    g = dvec[D].sum(0)
+    G = g @ M @ g
+    assert J == pytest.approx(G / K ** 2, rel=1e-11)
+    inD, gr, outD, gd = O.round_gains(D, pooled.n_cand, P_i, r, J, a, K)
+    for k, gain in zip(inD, gr):
+        dG = -2 * dvec[k] @ M @ g + s[k] ** 2                       # Eq. 14
+        assert gain == pytest.approx(G / K ** 2 - (G + dG) / (K + P_i[k]) ** 2, rel=1e-8)
+    for k, gain in zip(outD, gd):
+        dG = 2 * dvec[k] @ M @ g + s[k] ** 2                        # Eq. 15
+        assert gain == pytest.approx(G / K ** 2 - (G + dG) / (K - P_i[k]) ** 2, rel=1e-8)
+
+
+# ---------------------------------------------------------------------------------------
+# selection
+# ---------------------------------------------------------------------------------------
+def test_swap_schedule_totals():
+    """Eq. 17: rho 2^-(r+1) c per round, at most rho (1 - 2^-R) c in total; paper default
+    rho = 0.5, R = 5 gives 0.484 c."""
+    assert O.swap_schedule(68, 3, 0.5) == [17, 8, 4]
+    assert O.swap_schedule(214, 3, 0.5) == [53, 26, 13]
+    assert O.swap_schedule(21, 2, 0.5) == [5, 2]
+    for c in range(2, 400):
+        for R in range(0, 8):
+            assert sum(O.swap_schedule(c, R, 0.5)) <= 0.5 * (1 - 2.0 ** -R) * c + 1e-12
+    assert 0.5 * (1 - 2 ** -5) == pytest.approx(0.484, abs=5e-4)
+
+
+def test_initial_selection_single_drop_is_brute_force_optimum(layer):
+    """|D| = 1: the Eq. 7 selection drops the block whose removal leaves the least drift,
+    found by measuring every single-block removal through the library path."""
+    X, pooled = layer
+    c = pooled.n_cand - 1
+    for h in range(pooled.heads):
+        for i in (0, 4, 9):
+            sel = O.ress_select(pooled, X["W_o"], [c] * pooled.heads, 0, rows=[(h, i)])[(h, i)]
+            drifts = []
+            for j in range(pooled.n_cand):
+                D = np.zeros(pooled.nb, dtype=bool)
+                D[j] = True
+                drifts.append(residual_drift_via_library(pooled, X["W_o"], h, i, D))
+            assert np.nonzero(sel.D0)[0].tolist() == [int(np.argmin(drifts))]
+
+
+@pytest.mark.parametrize("c", [3, 6, 9])
+def test_brute_force_bounds_restoration(layer, c):
+    """Track-best restoration lands between the exhaustive optimum of Eq. 2 and the
+    initial selection: J_opt <= J_ReSS <= J_0, and the returned set has the claimed J."""
+    X, pooled = layer
+    n = pooled.n_cand
+    assert n == 12
+    W = X["W_o"]
+    for h in range(pooled.heads):
+        for i in (1, 8):
+            sel = O.ress_select(pooled, W, [c] * pooled.heads, 5, rows=[(h, i)])[(h, i)]
+            P_i, vbar = O.row_quantities(pooled, h, i)
+            _, _, r = O.residual_contributions(P_i, vbar, pooled.Vb[h], O.head_projection(W, h, 64))
+            best = math.inf
+            for comb in itertools.combinations(range(n), n - c):
+                D = np.zeros(pooled.nb, dtype=bool)
+                D[list(comb)] = True
+                best = min(best, O.objective(D, P_i, r)[0])
+            assert sel.D_best[:n].sum() == n - c and not sel.D_best[n:].any()
+            assert best <= sel.J_best * (1 + 1e-12)
+            assert sel.J_best <= sel.J0
+            measured = residual_drift_via_library(pooled, W, h, i, sel.D_best)
+            assert sel.J_best == pytest.approx(measured, rel=1e-9)
+
+
+def test_track_best_and_monotone_in_rounds(layer):
+    """J_best = min(J_0, J after each round) and, since m_r does not depend on R, one
+    more round never raises J_best."""
+    X, pooled = layer
+    rows = [(h, i) for h in range(pooled.heads) for i in range(pooled.n_cand)]
+    prev = None
+    for R in range(0, 7):
+        sel = O.ress_select(pooled, X["W_o"], [5] * pooled.heads, R, rows=rows)
+        for key, s in sel.items():
+            assert s.J_best == min([s.J0] + s.J_trace)
+            assert len(s.J_trace) == R
+            if prev is not None:
+                assert s.J_best <= prev[key].J_best
+                assert s.J_trace[:R - 1] == prev[key].J_trace
+        prev = sel
+
+
+def test_budget_is_preserved_and_special_blocks_kept(layer):
+    X, pooled = layer
+    sel = O.ress_select(pooled, X["W_o"], [4, 7], 3)
+    for (h, i), s in sel.items():
+        kept = s.kept()
+        if i >= pooled.n_cand:
+            assert s.dense and kept.tolist() == list(range(pooled.nb)) and s.J_best == 0
+        else:
+            assert int((kept < pooled.n_cand).sum()) == [4, 7][h]
+            assert kept[-1] == pooled.nb - 1 and np.all(np.diff(kept) > 0)
+
+
+def test_scale_invariance(layer):
+    """W_o -> alpha W_o leaves every choice unchanged and scales J by alpha^2."""
+    X, pooled = layer
+    a = 3.0
+    s1 = O.ress_select(pooled, X["W_o"], [5, 5], 3)
+    s2 = O.ress_select(pooled, a * X["W_o"], [5, 5], 3)
+    for k in s1:
+        assert (s1[k].D_best == s2[k].D_best).all()
+        assert s2[k].J_best == pytest.approx(a * a * s1[k].J_best, rel=1e-10, abs=1e-30)
+
+
+def test_candidate_permutation_equivariance():
+    """Permuting whole candidate key blocks (tokens of K and V) permutes the drop sets."""
+    X, ns = small_layer(seed=3)
+    pooled = O.pool(X["Q"], X["K"], X["V"], ns)
+    perm = np.random.default_rng(5).permutation(pooled.n_cand)
+    tok = np.arange(X["K"].shape[0])
+    newtok = tok.copy()
+    for dst, src in enumerate(perm):
+        newtok[dst * 64:(dst + 1) * 64] = tok[src * 64:(src + 1) * 64]
+    pooled2 = O.pool(X["Q"], X["K"][newtok], X["V"][newtok], ns)
+    rows = [(h, i) for h in range(2) for i in range(0, 12, 3)]
+    s1 = O.ress_select(pooled, X["W_o"], [5, 5], 3, rows=rows)
+    s2 = O.ress_select(pooled2, X["W_o"], [5, 5], 3, rows=rows)
+    for k in rows:
+        assert (s2[k].D_best[:12] == s1[k].D_best[:12][perm]).all()
+        assert s2[k].J_best == pytest.approx(s1[k].J_best, rel=1e-9)
+
+
+def test_deterministic(layer):
+    X, pooled = layer
+    a = O.ress_select(pooled, X["W_o"], [6, 6], 4)
+    b = O.ress_select(pooled, X["W_o"], [6, 6], 4)
+    for k in a:
+        assert (a[k].D_best == b[k].D_best).all() and a[k].J_best == b[k].J_best
+
+
+# ---------------------------------------------------------------------------------------
+# token-level attention
+# ---------------------------------------------------------------------------------------
+def _token_mask(kept, N, H, nb):
+    mask = np.zeros((H, N, N), dtype=bool)
+    for (h, i), cols in kept.items():
+        for j in cols:
+            mask[h, i * 64:min(N, i * 64 + 64), j * 64:min(N, j * 64 + 64)] = True
+    return mask
+
+
+def test_zero_sparsity_is_dense_attention(layer):
+    """c_h = |P| keeps every block; the output equals library dense attention."""
+    X, pooled = layer
+    sel = O.ress_select(pooled, X["W_o"], [pooled.n_cand] * 2, 3)
+    kept = {k: s.kept() for k, s in sel.items()}
+    assert all(len(v) == pooled.nb for v in kept.values())
+    out = O.block_sparse_attention(X["Q"], X["K"], X["V"], kept, list(kept))
+    N = X["Q"].shape[0]
+    for h in range(2):
+        ref = sdpa(X["Q"][:, h], X["K"][:, h], X["V"][:, h])
+        for i in range(pooled.nb):
+            np.testing.assert_allclose(out[(h, i)], ref[i * 64:min(N, i * 64 + 64)],
+                                       rtol=1e-10, atol=1e-12)
+
+
+def test_block_sparse_attention_is_masked_library_attention(layer):
+    """Sec. 3 step (3): exact attention over the kept blocks, renormalised among them,
+    equals library attention with the dropped blocks masked out."""
+    X, pooled = layer
+    sel = O.ress_select(pooled, X["W_o"], [3, 8], 2)
+    kept = {k: s.kept() for k, s in sel.items()}
+    out = O.block_sparse_attention(X["Q"], X["K"], X["V"], kept, list(kept))
+    N = X["Q"].shape[0]
+    mask = _token_mask(kept, N, 2, pooled.nb)
+    for h in range(2):
+        ref = sdpa(X["Q"][:, h], X["K"][:, h], X["V"][:, h], mask[h])
+        for i in range(pooled.nb):
+            np.testing.assert_allclose(out[(h, i)], ref[i * 64:min(N, i * 64 + 64)],
+                                       rtol=1e-10, atol=1e-12)
+
+
+def test_csr_layout(layer):
+    X, pooled = layer
+    sel = O.ress_select(pooled, X["W_o"], [3, 8], 2)
+    rp, ci = O.csr_from_selection(sel, 2, pooled.nb)
+    assert rp[0] == 0 and rp[-1] == ci.size
+    ns = pooled.nb - pooled.n_cand
+    lens = np.diff(rp).reshape(2, pooled.nb)
+    assert (lens[0, :pooled.n_cand] == 3 + ns).all() and (lens[1, :pooled.n_cand] == 8 + ns).all()
+    assert (lens[:, pooled.n_cand:] == pooled.nb).all()
