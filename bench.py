@@ -1,0 +1,485 @@
+#!/usr/bin/env python
+"""Benchmark of the ReSS hot path: one sparsified global-attention layer of a 3D ViT.
+
+One step = ress_forward over one layer of synthetic inputs resident in HBM: block scoring
+and the initial selection, R restoration rounds, the kept-block lists, and the
+block-sparse attention.  Prints one JSON line (rank 0).
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+                  [--workload vggt_v32] [--sweep]
+
+N > 1 runs as independent replicas (one per GPU, launched by torchrun): the method has no
+exchange step, so there is no collective on the data path.  --impl reference times the
+CPU oracle (float64 numpy) on a bounded sample of the same workload, extrapolated.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+
+METRIC = "ReSS layer ms & kept-FLOP TFLOP/s at 32 views/90% sparsity; select overhead %"
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--warmup", type=int, default=10)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", default="vggt_v32")
+    ap.add_argument("--cpu-budget", type=float, default=15.0, help="seconds of oracle work")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--sweep", action="store_true", help="64-view sparsity x rounds sweep lines")
+    return ap.parse_args()
+
+
+def peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            p = json.load(f)
+        return p["hbm_gbs"], p["bf16_tflops"], p.get("bf16_tflops_sustained"), "measured"
+    except Exception:
+        return 6800.0, 1900.0, 1700.0, "fallback"
+
+
+# ----------------------------------------------------------------------------------------
+# work accounting
+# ----------------------------------------------------------------------------------------
+def kept_flops(row_ptr, col_idx, N, H, nb):
+    """4 * 64 * sum over rows of (valid query tokens) x (valid keys of the kept blocks)."""
+    tok = np.minimum(64, N - 64 * np.arange(nb)).astype(np.int64)
+    lens = np.diff(row_ptr.astype(np.int64))
+    keys = np.add.reduceat(tok[col_idx[:row_ptr[-1]]], row_ptr[:-1].astype(np.int64)) if col_idx.size else 0
+    keys = np.where(lens > 0, keys, 0)
+    q = np.tile(tok, H)
+    return 4.0 * 64.0 * float((q * keys).sum())
+
+
+def selection_bytes(N, H, nb, ld, rounds, csr_entries):
+    """Algorithmic bytes of scoring + restoration: read Q, K, V once; write P and q; per
+    round read P, q, t and read/write the drop masks; write the CSR."""
+    mat = H * nb * nb * 4
+    score = 3 * N * H * 64 * 2 + 2 * mat
+    per_round = 3 * mat + 2 * H * nb * math.ceil(nb / 32) * 4
+    return score + rounds * per_round + 4 * (csr_entries + H * nb + 1)
+
+
+# ----------------------------------------------------------------------------------------
+# clocks during the timed region
+# ----------------------------------------------------------------------------------------
+class ClockSampler:
+    FIELDS = ("uuid,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, uuid):
+        self.uuid = uuid
+        self.rows = []
+        self.proc = None
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", f"--query-gpu={self.FIELDS}",
+                                          "--format=csv,noheader,nounits", "-lms", "100"],
+                                         stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.thread = threading.Thread(target=self._read, daemon=True)
+            self.thread.start()
+        except Exception:
+            self.proc = None
+        return self
+
+    def _read(self):
+        for line in self.proc.stdout:
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) == 9:
+                self.rows.append(parts)
+
+    def __exit__(self, *a):
+        if self.proc:
+            time.sleep(0.15)
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=2)
+            except Exception:
+                self.proc.kill()
+
+    def summary(self):
+        rows = [r for r in self.rows if not self.uuid or self.uuid in r[0]] or self.rows
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"], "samples": 0}
+        def num(x):
+            try:
+                return float(x)
+            except ValueError:
+                return None
+        sm = [num(r[1]) for r in rows if num(r[1]) is not None]
+        reasons = set()
+        for r in rows:
+            for name, v in zip(("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"), r[5:9]):
+                if v.lower() == "active":
+                    reasons.add(name)
+        return {"sm_mhz": float(np.median(sm)) if sm else None,
+                "sm_max_mhz": num(rows[0][2]), "reasons": sorted(reasons),
+                "power_w_max": max((num(r[3]) or 0.0) for r in rows), "samples": len(rows)}
+
+
+# ----------------------------------------------------------------------------------------
+# CPU oracle timing (bounded sample, extrapolated)
+# ----------------------------------------------------------------------------------------
+def _oracle_rows(args):
+    pooled, W_o, c_h, rounds, rho, rows = args
+    import oracle as O
+    t = time.perf_counter()
+    O.ress_select(pooled, W_o, c_h, rounds, rho, rows=rows)
+    return time.perf_counter() - t
+
+
+def _oracle_attn(args):
+    X, kept, rows = args
+    import oracle as O
+    t = time.perf_counter()
+    O.block_sparse_attention(*X, kept, rows)
+    return time.perf_counter() - t
+
+
+def oracle_layer_seconds(wl, bits, kept, pool_exec, workers, budget_s, rng):
+    """Extrapolated seconds of the oracle for the whole layer, measured on a sample."""
+    import oracle as O
+    import synth
+    X = [synth.bf16_to_f32(bits[k]) for k in ("Q", "K", "V")]
+    t0 = time.perf_counter()
+    pooled = O.pool(*X, wl.n_special)
+    t_pool = time.perf_counter() - t0
+    W = synth.bf16_to_f32(bits["W_o"]).astype(np.float64)
+    H, nb, nc = wl.heads, wl.n_blocks, wl.n_candidates
+    c_h = wl.budgets()
+    sparse_rows = [(h, i) for h in range(H) for i in range(nc)]
+    # calibrate one row, then size the sample to about half of the budget per stage
+    t1 = _oracle_rows((pooled, W, c_h, wl.rounds, wl.rho, [sparse_rows[0]]))
+    n_sel = int(min(len(sparse_rows), max(workers, 0.5 * budget_s * workers / max(t1, 1e-4))))
+    pick = rng.choice(len(sparse_rows), n_sel, replace=False)
+    srows = [sparse_rows[k] for k in pick]
+    chunks = [srows[k::workers] for k in range(workers)]
+    t0 = time.perf_counter()
+    list(pool_exec.map(_oracle_rows, [(pooled, W, c_h, wl.rounds, wl.rho, ch) for ch in chunks if ch]))
+    t_sel = (time.perf_counter() - t0) * len(sparse_rows) / n_sel
+    # attention: sample rows (sparse and dense) and scale by kept FLOPs
+    all_rows = [(h, i) for h in range(H) for i in range(nb)]
+    N = wl.n_tokens
+    tok = np.minimum(64, N - 64 * np.arange(nb))
+    def row_flops(r):
+        return 4 * 64 * tok[r[1]] * tok[kept[r]].sum()
+    total = sum(row_flops(r) for r in all_rows)
+    t1 = _oracle_attn((X, {all_rows[0]: kept[all_rows[0]]}, [all_rows[0]]))
+    per_flop = t1 / max(row_flops(all_rows[0]), 1)
+    n_att = int(min(len(all_rows), max(workers, 0.5 * budget_s * workers / max(per_flop * total / len(all_rows), 1e-4))))
+    pick = rng.choice(len(all_rows), n_att, replace=False)
+    arows = [all_rows[k] for k in pick]
+    f_sample = sum(row_flops(r) for r in arows)
+    chunks = [arows[k::workers] for k in range(workers)]
+    t0 = time.perf_counter()
+    list(pool_exec.map(_oracle_attn, [(X, {r: kept[r] for r in ch}, ch) for ch in chunks if ch]))
+    t_att = (time.perf_counter() - t0) * total / max(f_sample, 1)
+    sample = (f"pooling of all {nb} blocks; ReSS selection on {n_sel} of {len(sparse_rows)} candidate "
+              f"rows; token attention on {n_att} of {len(all_rows)} rows; extrapolated linearly by "
+              f"rows (selection) and kept FLOPs (attention); {workers} worker processes, 1 BLAS "
+              f"thread each")
+    return t_pool + t_sel + t_att, dict(pool_s=t_pool, select_s=t_sel, attn_s=t_att), sample
+
+
+def make_pool(workers):
+    os.environ.setdefault("OPENBLAS_NUM_THREADS", "1")
+    os.environ.setdefault("OMP_NUM_THREADS", "1")
+    os.environ.setdefault("MKL_NUM_THREADS", "1")
+    import multiprocessing as mp
+    from concurrent.futures import ProcessPoolExecutor
+    return ProcessPoolExecutor(max_workers=workers, mp_context=mp.get_context("spawn"))
+
+
+# ----------------------------------------------------------------------------------------
+# reference arm: the oracle as the timed implementation
+# ----------------------------------------------------------------------------------------
+def run_reference(a, wl):
+    import synth
+    import oracle as O
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    workers = os.cpu_count() or 1
+    pool_exec = make_pool(workers)
+    bits = synth.make_inputs(wl)
+    X = [synth.bf16_to_f32(bits[k]) for k in ("Q", "K", "V")]
+    # kept lists from the oracle's own selection on a row sample would differ per row; the
+    # attention cost depends only on the list lengths, which the budget fixes
+    nb, nc, H = wl.n_blocks, wl.n_candidates, wl.heads
+    c = int(wl.budgets()[0])
+    rng = np.random.default_rng(0)
+    kept = {}
+    for h in range(H):
+        for i in range(nb):
+            kept[(h, i)] = np.arange(nb) if i >= nc else np.sort(np.concatenate(
+                [rng.choice(nc, c, replace=False), np.arange(nc, nb)]))
+    N = wl.n_tokens
+    tok = np.minimum(64, N - 64 * np.arange(nb))
+    flops = sum(4 * 64 * tok[i] * tok[kept[(h, i)]].sum() for (h, i) in kept)
+    per_step = max(2.0, min(8.0, 150.0 / max(a.steps + a.warmup, 1)))
+    times = []
+    for s in range(a.warmup + a.steps):
+        t, parts, sample = oracle_layer_seconds(wl, bits, kept, pool_exec, workers, per_step,
+                                                np.random.default_rng(s))
+        if s >= a.warmup:
+            times.append(t)
+    del X
+    t = float(np.mean(times))
+    val = flops / t / 1e12
+    line = {"metric": METRIC, "value": val, "unit": "TFLOP/s", "impl": "reference",
+            "n_gpus": a.gpus, "steps": a.steps, "warmup": a.warmup, "ms_per_step": t * 1e3,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic", "config": {"workload": wl.name, "views": wl.views, "heads": wl.heads,
+                                             "tokens": N, "sparsity": wl.sparsity, "rounds": wl.rounds},
+            "layer_ms": t * 1e3, "stage_s": parts,
+            "cpu_baseline": {"value": val, "unit": "TFLOP/s", "cores": workers, "kind": "oracle",
+                             "sample": sample},
+            "e2e": {"value": val, "unit": "TFLOP/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+    pool_exec.shutdown()
+
+
+# ----------------------------------------------------------------------------------------
+# our arm
+# ----------------------------------------------------------------------------------------
+def run_ours(a, wl):
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    pool_exec = None
+    workers = os.cpu_count() or 1
+    if rank == 0 and world == 1 and not a.no_cpu_baseline:
+        pool_exec = make_pool(workers)  # spawned before the first CUDA call
+    import torch
+    import synth
+    torch.cuda.set_device(local)
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    import paper_2609_35593_gb300 as ress
+
+    bits = synth.make_inputs(wl)
+    dev = lambda b: torch.from_numpy(b.view(np.int16)).view(torch.bfloat16).cuda()
+    Q, K, V, W = (dev(bits[k]) for k in ("Q", "K", "V", "W_o"))
+    c_h = wl.budgets()
+    N, H = wl.n_tokens, wl.heads
+    d = ress.dims(N, H, wl.n_special, wl.d_model)
+    buf = ress.Buffers(d, c_h)
+    nb = buf.nb
+    ress.prepare_wo(d, W, buf.F)  # model-load time (Eq. 8), outside the step
+    stream = torch.cuda.current_stream()
+
+    def step():
+        ress.forward(d, Q, K, V, buf.F, c_h, wl.rounds, wl.rho, buf.ws, buf.row_ptr, buf.col_idx,
+                     buf.O, buf.J_best)
+
+    for _ in range(max(a.warmup, 3)):
+        step()
+    ress.status(buf.ws)
+    torch.cuda.synchronize()
+
+    props = torch.cuda.get_device_properties(local)
+    uuid = str(getattr(props, "uuid", "") or "")
+    if dist:
+        dist.barrier()
+    torch.cuda.synchronize()
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with ClockSampler(uuid) as clk:
+        ev0.record(stream)
+        for _ in range(a.steps):
+            step()
+        ev1.record(stream)
+        torch.cuda.synchronize()
+    ms = ev0.elapsed_time(ev1) / a.steps
+    ress.status(buf.ws)
+    if dist:
+        t = torch.tensor([ms], device="cuda")
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+
+    # ---- stage breakdown (same work, events between the three calls) ---------------
+    nst = max(20, min(200, a.steps))
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(4)] for _ in range(nst)]
+    for k in range(nst):
+        e = evs[k]
+        e[0].record(stream)
+        ress.score(d, Q, K, V, buf.F, c_h, buf.ws)
+        e[1].record(stream)
+        ress.restore(d, c_h, wl.rounds, wl.rho, buf.ws, buf.row_ptr, buf.col_idx, buf.J_best)
+        e[2].record(stream)
+        ress.sparse_attn(d, Q, K, V, buf.row_ptr, buf.col_idx, buf.O, buf.ws)
+        e[3].record(stream)
+    torch.cuda.synchronize()
+    st = np.array([[e[i].elapsed_time(e[i + 1]) for i in range(3)] for e in evs])
+    score_ms, restore_ms, attn_ms = (float(x) for x in np.median(st, axis=0))
+
+    rp = buf.row_ptr.cpu().numpy()
+    ci = buf.col_idx.cpu().numpy()
+    flops = kept_flops(rp, ci, N, H, nb)
+    hbm, bf16, bf16_sus, peak_kind = peaks()
+
+    # ---- dense run of the same attention kernel (no block dropped) -------------------
+    dense = None
+    if wl.name == "vggt_v32":
+        rpd = torch.arange(0, H * nb * nb + 1, nb, dtype=torch.int32, device="cuda")
+        cid = torch.arange(nb, dtype=torch.int32, device="cuda").repeat(H * nb)
+        Od = torch.empty_like(buf.O)
+        for _ in range(3):
+            ress.sparse_attn(d, Q, K, V, rpd, cid, Od, buf.ws)
+        torch.cuda.synchronize()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        nd = 10
+        e0.record(stream)
+        for _ in range(nd):
+            ress.sparse_attn(d, Q, K, V, rpd, cid, Od, buf.ws)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        dms = e0.elapsed_time(e1) / nd
+        dfl = kept_flops(rpd.cpu().numpy(), cid.cpu().numpy(), N, H, nb)
+        dense = {"attn_ms": dms, "tflops": dfl / dms / 1e9, "frac_of_bf16_peak": dfl / dms / 1e9 / bf16,
+                 "speedup_of_sparse_layer": dms / ms}
+        ress.status(buf.ws)
+        del Od, rpd, cid
+
+    # ---- end to end through the public API with host buffers -------------------------
+    hQ, hK, hV = (t.cpu().pin_memory() for t in (Q, K, V))
+    hO = torch.empty(buf.O.shape, dtype=torch.bfloat16).pin_memory()
+    dQ, dK, dV = (torch.empty_like(t) for t in (Q, K, V))
+    ne = max(10, min(50, a.steps))
+    for _ in range(2):
+        dQ.copy_(hQ, non_blocking=True); dK.copy_(hK, non_blocking=True); dV.copy_(hV, non_blocking=True)
+        ress.forward(d, dQ, dK, dV, buf.F, c_h, wl.rounds, wl.rho, buf.ws, buf.row_ptr, buf.col_idx, buf.O, buf.J_best)
+        hO.copy_(buf.O, non_blocking=True)
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(ne):
+        dQ.copy_(hQ, non_blocking=True); dK.copy_(hK, non_blocking=True); dV.copy_(hV, non_blocking=True)
+        ress.forward(d, dQ, dK, dV, buf.F, c_h, wl.rounds, wl.rho, buf.ws, buf.row_ptr, buf.col_idx, buf.O, buf.J_best)
+        hO.copy_(buf.O, non_blocking=True)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    ems = e0.elapsed_time(e1) / ne
+    ress.status(buf.ws)
+    h2d = 3 * N * H * 64 * 2
+    d2h = N * H * 64 * 2
+
+    # ---- realised drift and sparsity ---------------------------------------------------
+    Jb = buf.J_best.cpu().numpy().astype(np.float64)
+    J0 = buf.ws_view("J0", torch.float32).cpu().numpy()[:H * nb].astype(np.float64)
+    cand_rows = np.tile(np.arange(nb) < wl.n_candidates, H)
+    kept_pairs = int(np.diff(rp.astype(np.int64)).sum())
+
+    sel_bytes = selection_bytes(N, H, nb, buf.layout.ld, wl.rounds, ci.size)
+    sel_ms = score_ms + restore_ms
+    line = {
+        "metric": METRIC, "value": flops / ms / 1e9 * world, "unit": "TFLOP/s", "n_gpus": world,
+        "steps": a.steps, "warmup": a.warmup, "ms_per_step": ms, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic (seeded VGGT-shaped Q/K/V and W_o; inputs 3x larger than L2, no flush)",
+        "config": {"workload": wl.name, "views": wl.views, "heads": H, "tokens": N, "head_dim": 64,
+                   "block": 64, "sparsity": wl.sparsity, "rounds": wl.rounds, "rho": wl.rho,
+                   "c_h": int(c_h[0]), "parallelism": f"replicas{world}",
+                   "l2": "inputs larger than L2 (270 MB Q/K/V at 32 views)"},
+        "layer_ms": ms, "stage_ms": {"score": score_ms, "restore": restore_ms, "attn": attn_ms},
+        "select_overhead_pct": 100.0 * sel_ms / (sel_ms + attn_ms),
+        "attn_tflops": flops / attn_ms / 1e9,
+        "selection": {"algorithmic_bytes": sel_bytes, "gbs": sel_bytes / sel_ms / 1e6,
+                      "frac_of_hbm": sel_bytes / sel_ms / 1e6 / hbm, "hbm_peak_gbs": hbm},
+        "kept_tflop": flops / 1e12, "realized_pair_sparsity": 1.0 - kept_pairs / (H * nb * nb),
+        "drift": {"sum_J_best": float(Jb[cand_rows].sum()), "sum_J0": float(J0[cand_rows].sum())},
+        "dense": dense,
+        "roofline": {"bound": "tensor", "kernel": "k_attn (ress_sparse_attn)",
+                     "achieved": flops / attn_ms / 1e9, "peak": bf16, "unit": "TFLOP/s",
+                     "frac": flops / attn_ms / 1e9 / bf16, "traffic": None,
+                     "peak_kind": f"{peak_kind} bf16 burst"},
+        "gpu_launches": a.steps * (3 + wl.rounds + 1 + 2),
+        "e2e": {"value": flops / ems / 1e9 * world, "unit": "TFLOP/s", "ms_per_step": ems,
+                "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
+        "clocks": clk.summary(),
+    }
+
+    if pool_exec is not None:
+        kept = {(h, i): ci[rp[h * nb + i]:rp[h * nb + i + 1]] for h in range(H) for i in range(nb)}
+        t, parts, sample = oracle_layer_seconds(wl, bits, kept, pool_exec, workers, a.cpu_budget,
+                                                np.random.default_rng(0))
+        line["cpu_baseline"] = {"value": flops / t / 1e12, "unit": "TFLOP/s", "cores": workers,
+                                "kind": "oracle", "sample": sample, "layer_s": t, "stage_s": parts}
+        pool_exec.shutdown()
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+
+    if a.sweep and rank == 0:
+        sweep(a)
+    if dist:
+        dist.destroy_process_group()
+
+
+def sweep(a):
+    """64 views: sparsity x rounds, realised drift, selection and attention time per point."""
+    import torch
+    import synth
+    import paper_2609_35593_gb300 as ress
+    base = synth.WORKLOADS["vggt_v64"]
+    bits = synth.make_inputs(base)
+    dev = lambda b: torch.from_numpy(b.view(np.int16)).view(torch.bfloat16).cuda()
+    Q, K, V, W = (dev(bits[k]) for k in ("Q", "K", "V", "W_o"))
+    for s, R in synth.SWEEP_V64:
+        wl = base.with_(sparsity=s, rounds=R)
+        c_h = wl.budgets()
+        d = ress.dims(wl.n_tokens, wl.heads, wl.n_special, wl.d_model)
+        buf = ress.Buffers(d, c_h)
+        ress.prepare_wo(d, W, buf.F)
+        evs = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
+        res = []
+        for k in range(6):
+            evs[0].record()
+            ress.score(d, Q, K, V, buf.F, c_h, buf.ws)
+            evs[1].record()
+            ress.restore(d, c_h, R, wl.rho, buf.ws, buf.row_ptr, buf.col_idx, buf.J_best)
+            evs[2].record()
+            ress.sparse_attn(d, Q, K, V, buf.row_ptr, buf.col_idx, buf.O, buf.ws)
+            evs[3].record()
+            torch.cuda.synchronize()
+            if k >= 2:
+                res.append([evs[i].elapsed_time(evs[i + 1]) for i in range(3)])
+        ress.status(buf.ws)
+        m = np.median(np.array(res), axis=0)
+        nb = buf.nb
+        Jb = buf.J_best.cpu().numpy().reshape(wl.heads, nb)[:, :wl.n_candidates]
+        print(json.dumps({"sweep": "vggt_v64", "sparsity": s, "rounds": R, "c_h": int(c_h[0]),
+                          "sum_J_best": float(Jb.astype(np.float64).sum()),
+                          "select_ms": float(m[0] + m[1]), "attn_ms": float(m[2])}), flush=True)
+        del buf
+
+
+def main():
+    a = parse()
+    import synth
+    wl = synth.WORKLOADS[a.workload]
+    if a.impl == "reference":
+        run_reference(a, wl)
+    else:
+        run_ours(a, wl)
+
+
+if __name__ == "__main__":
+    main()

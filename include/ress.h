@@ -1,0 +1,160 @@
+/*
+ * ress.h -- C ABI of the ReSS (Residual-Restoring Sparse Attention) hot path on GB300.
+ *
+ * One sparsified global-attention layer of a 3D vision transformer:
+ *   ress_score       block pooling, pooled attention map, block drift scores and the
+ *                    initial selection (Sec. 4.1-4.2, Eq. 1, 5-9)
+ *   ress_restore     R budget-neutral restoration rounds with track-best and the kept-block
+ *                    lists (Sec. 4.3, Eq. 10-17)
+ *   ress_sparse_attn exact attention over the kept 64x64 blocks (Sec. 3 step (3))
+ *   ress_forward     the three in order on one stream
+ *
+ * Conventions shared by every call
+ *   - Pointers named "device" point to GPU memory owned by the caller; the library never
+ *     allocates, frees or retains memory.  Host pointers are read before the call returns.
+ *   - bf16 tensors are passed as uint16_t bit patterns.  Q, K, V and O are [N, H, 64]
+ *     row-major (token, head, channel): one token is H*128 contiguous bytes.  Their base
+ *     addresses must be 16-byte aligned.
+ *   - Every call is asynchronous on `stream` (a cudaStream_t; NULL = legacy default
+ *     stream) and validates all host-visible arguments before it launches anything.  On a
+ *     validation error nothing is launched.
+ *   - Return value: RESS_OK (0) or a negative ress_status code; ress_last_error() gives a
+ *     message for the calling thread.  No C++ exception crosses the ABI.
+ *   - Device-side failures (a bounded wait that gave up, an out-of-range index in a
+ *     caller-built CSR) are recorded in a status word inside the workspace; read it with
+ *     ress_status() after the stream work completes.  Kernels never trap.
+ *   - Fixed constants: head_dim = 64, block = 64 (64x64 block grid), eps = 1e-4 (Eq. 7).
+ *   - Results are deterministic: the same inputs give the same bits (Appendix B.4).
+ */
+#ifndef RESS_H
+#define RESS_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define RESS_ABI_VERSION 1
+#define RESS_HEAD_DIM 64
+#define RESS_BLOCK 64
+#define RESS_MAX_HEADS 32
+#define RESS_MAX_BLOCKS 4096 /* key blocks per sequence: 262144 tokens */
+
+typedef enum {
+  RESS_OK = 0,
+  RESS_EINVAL = -1,       /* null/misaligned pointer, inconsistent sizes or budgets      */
+  RESS_EWORKSPACE = -2,   /* workspace or output buffer smaller than required            */
+  RESS_EUNSUPPORTED = -3, /* head_dim != 64, block != 64, too many heads or blocks        */
+  RESS_ECUDA = -4,        /* a CUDA runtime call or kernel launch failed                  */
+  RESS_ETIMEOUT = -5,     /* a bounded device-side wait gave up (status word)             */
+  RESS_EDEVICE = -6       /* a device-side argument check failed (status word)            */
+} ress_status_code;
+
+/* Shape of one global-attention layer.  Special tokens (camera/register) are the last
+ * n_special tokens of the sequence (Sec. 3, "excluded from sparsification"): key blocks
+ * that contain any of them are always kept, query blocks that contain any of them attend
+ * densely.  The remaining key blocks form the candidate set P of Sec. 4.1, of size
+ * (n_tokens - n_special) / 64 (rounded down). */
+typedef struct {
+  int32_t n_tokens;  /* N >= 1                                                    */
+  int32_t n_heads;   /* H, 1..RESS_MAX_HEADS                                      */
+  int32_t head_dim;  /* d_h, must be 64                                           */
+  int32_t block;     /* block size, must be 64                                    */
+  int32_t n_special; /* trailing special tokens, 0..N-1                           */
+  int32_t d_model;   /* d: rows of the output projection W_o ([d, H*64])          */
+} ress_dims;
+
+/* Byte offsets of the arrays inside the workspace (for inspection and tests).  All
+ * arrays are float32 unless noted; row strides are in elements. */
+typedef struct {
+  int64_t status;      /* uint32 status word (first device-side error, sticky)          */
+  int64_t counter;     /* uint32 tile-scheduler counters of the attention kernel        */
+  int64_t qbar, kbar, vbar, ztil; /* [H, nb, 64] block means; z~_j = F_h V_j              */
+  int64_t ytil, gtil;  /* [H, nb, 64] y~_i = F_h v_bar_i (Eq. 1); g~ = F_h g (Eq. 10)    */
+  int64_t P, q, t;     /* [H, nb, ld] pooled P_ij, q_ij = ||F_h e_ij||^2 (Eq. 9), gains;
+                          t doubles as the attention kernel's pair-list scratch            */
+  int64_t K, G, J, Jbest, J0; /* [H, nb] remaining mass, G, J of Eq. 12                  */
+  int64_t dmask, bmask; /* uint32 [H, nb, words] current and best drop sets (bit j)      */
+  int64_t plen;        /* int32 [H, ceil(nb/2)] union lengths of query-block pairs          */
+  int64_t ld;          /* row stride of P, q, t                                          */
+  int64_t words;       /* uint32 words per drop-set bitmask = ceil(nb / 32)              */
+  int64_t total;       /* bytes                                                          */
+} ress_ws_layout;
+
+/* Message describing the last error returned on the calling thread ("" if none). */
+const char* ress_last_error(void);
+int32_t ress_abi_version(void);
+
+/* Number of key blocks nb = ceil(N / 64) and candidate blocks |P|; -1 on bad dims. */
+int32_t ress_num_blocks(const ress_dims* dims);
+int32_t ress_num_candidates(const ress_dims* dims);
+
+/* Workspace needed by ress_score / ress_restore / ress_sparse_attn / ress_forward
+ * (0 on invalid dims).  The same workspace serves every call on that layer shape; it
+ * must be 256-byte aligned and must not be shared by calls that may overlap on the GPU. */
+size_t ress_workspace_bytes(const ress_dims* dims);
+int ress_workspace_layout(const ress_dims* dims, ress_ws_layout* out);
+
+/* Entries of col_idx that ress_restore writes for the budgets c_h (host array [H]):
+ * every candidate query row keeps c_h + (nb - |P|) blocks, every special query row keeps
+ * all nb blocks.  -1 on invalid arguments. */
+int64_t ress_csr_capacity(const ress_dims* dims, const int32_t* c_h_host);
+
+/* Eq. 8 at model-load time.  W_o: device bf16 [d_model, H*64] (Linear.weight layout,
+ * out x in; head h owns columns 64h..64h+63, i.e. W_O^h).  F: device float32 [H, 64, 64]
+ * receives an upper-triangular F_h with F_h^T F_h = M_h = W_O^h^T W_O^h (Cholesky factor,
+ * computed in float64; a zero pivot of a rank-deficient M_h yields a zero row).  The
+ * scoring kernels use ||F_h e||^2 = e^T M_h e, the Gram form of Eq. 9. */
+int ress_prepare_wo(const ress_dims* dims, const uint16_t* W_o, float* F, void* stream);
+
+/* Sec. 4.1-4.2: pooled attention map P (softmax over all key blocks of the block-mean
+ * logits q_bar . k_bar / 8), the dense pooled output (Eq. 1), q_ij = ||F_h (v_bar_i - V_j)||^2
+ * (Eq. 9), drift scores s = P sqrt(q) (Eq. 6) and the initial selection: per candidate
+ * query row the c_h candidate blocks with the largest s / max(1 - P, 1e-4) (Eq. 7), ties to
+ * the lower block index.  Writes P, q, the initial drop sets and their objective J_0
+ * (Eq. 10-12) into the workspace.  c_h_host: host int32 [H], 1 <= c_h <= |P|. */
+int ress_score(const ress_dims* dims, const uint16_t* Q, const uint16_t* K, const uint16_t* V,
+               const float* F, const int32_t* c_h_host, void* ws, size_t ws_bytes,
+               void* stream);
+
+/* Sec. 4.3: `rounds` budget-neutral swap rounds on the drop sets left by ress_score.
+ * Round r exchanges m_r = floor(rho c_h / 2^(r+1)) blocks (Eq. 17), capped by the sizes of
+ * the two sides: the m_r restores and the m_r drops with the largest exact decrease of
+ * J (Eq. 13-16), both taken from the round-start state.  The set with the smallest J seen
+ * (track-best, strict <) is returned as kept-block lists in CSR form over the H*nb query
+ * rows (h-major): row_ptr device int32 [H*nb + 1], col_idx device int32 [col_capacity] with
+ * ascending block indices; col_capacity >= ress_csr_capacity().  Optional device outputs
+ * (NULL to skip): J_best float [H*nb] (0 for special query rows), drop_mask uint32
+ * [H*nb, ceil(nb/32)] (bit j of row (h, i) set when block j is dropped).
+ * rounds in [0, 32]; rho in [0, 1]. */
+int ress_restore(const ress_dims* dims, const int32_t* c_h_host, int32_t rounds, float rho,
+                 void* ws, size_t ws_bytes, int32_t* row_ptr, int32_t* col_idx,
+                 int64_t col_capacity, float* J_best, uint32_t* drop_mask, void* stream);
+
+/* Sec. 3 step (3): for every head h, query block i and query token of that block,
+ * O = softmax(q K^T / 8) V over the tokens of the key blocks listed in row h*nb + i of the
+ * CSR (renormalised among them); keys past N are excluded.  Q, K, V: device bf16 [N, H, 64];
+ * O: device bf16 [N, H, 64].  Lists must hold ascending, distinct block indices < nb and be
+ * non-empty; entries past col_capacity or >= nb are skipped and flagged as RESS_EDEVICE in
+ * the status word.  Uses tcgen05 tensor cores with TMA-fed K/V tiles. */
+int ress_sparse_attn(const ress_dims* dims, const uint16_t* Q, const uint16_t* K,
+                     const uint16_t* V, const int32_t* row_ptr, const int32_t* col_idx,
+                     int64_t col_capacity, uint16_t* O, void* ws, size_t ws_bytes,
+                     void* stream);
+
+/* ress_score, ress_restore and ress_sparse_attn in order on one stream. */
+int ress_forward(const ress_dims* dims, const uint16_t* Q, const uint16_t* K, const uint16_t* V,
+                 const float* F, const int32_t* c_h_host, int32_t rounds, float rho, void* ws,
+                 size_t ws_bytes, int32_t* row_ptr, int32_t* col_idx, int64_t col_capacity,
+                 uint16_t* O, float* J_best, void* stream);
+
+/* Synchronises `stream`, returns the workspace status word as a ress_status_code
+ * (RESS_OK, RESS_ETIMEOUT or RESS_EDEVICE) and clears it. */
+int ress_status(void* ws, void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* RESS_H */

@@ -1,0 +1,538 @@
+// Block-sparse attention forward over the kept 64x64 blocks (Sec. 3 step (3)) on sm_103a.
+//
+// Work item = (head h, pair of adjacent query blocks 2p, 2p+1): their 128 query rows form
+// the M = 128 operand of tcgen05.mma, and the CTA walks the union of the two kept lists
+// (built by k_pairs, ascending).  Each union entry carries a 2-bit mask saying which of the
+// two query blocks keeps it; rows of a block that does not keep the tile get P = 0, so
+// every row sees exactly its own kept blocks (softmax renormalised among them).
+//
+// Warp roles (192 threads, 2 CTAs per SM):
+//   warp 0     TMA producer: Q tile (128 x 64) per item, K/V tiles (64 x 64) per entry into
+//              a 3-stage ring, 128-byte swizzled (UMMA K-major canonical layout).
+//   warp 1     TMEM owner and single-thread MMA issuer:
+//                S[g % 2] = Q K_g^T              (M128 N64 K64, both K-major)
+//                O       += P_{g-1} V_{g-1}       (M128 N64 K64, V MN-major)
+//              S is double-buffered in TMEM so that S_{g+1} runs while softmax works on S_g.
+//   warps 2-5  one query row per thread: tcgen05.ld of S, online softmax in the exp2 domain
+//              with lazy rescaling of the TMEM accumulator (only when the running max grows
+//              by more than 2^8), P as bf16 into a swizzled shared buffer, epilogue O / l.
+// Every mbarrier wait is bounded; a wait that gives up records RESS_ETIMEOUT in the status
+// word, makes the whole CTA leave its loops, drains in-flight copies and MMAs, frees TMEM
+// and returns.
+
+#include <climits>
+
+#include <cudaTypedefs.h>
+
+#include "ress_internal.cuh"
+#include "sm100_ptx.cuh"
+
+namespace ress {
+using namespace ptx;
+
+constexpr int kAttnThreads = 192;
+constexpr int kStages = 3;
+constexpr int kRows = 128;
+constexpr uint32_t kTmemCols = 256;
+constexpr uint32_t kColS0 = 0, kColO = 128;
+constexpr uint64_t kWaitNs = 2000000000ull;  // 2 s per wait
+constexpr uint64_t kDrainNs = 200000000ull;  // 0.2 s to drain after an abort
+constexpr int kFirst = 1, kLast = 2, kTerm = 4;
+constexpr uint32_t kTileBytes = 64 * 128;    // one 64 x 64 bf16 tile
+constexpr float kLazyThreshold = 8.0f;       // log2 units: rescale when max grows > 2^8
+
+struct TileInfo {
+  int j, mask, flags, item;
+};
+
+struct __align__(1024) AttnSmem {
+  uint8_t Q[kRows * 128];
+  uint8_t K[kStages][kTileBytes];
+  uint8_t V[kStages][kTileBytes];
+  uint8_t P[2][kRows * 128];
+  uint64_t kv_full[kStages], kv_empty[kStages];
+  uint64_t q_full, q_empty;
+  uint64_t s_full[2], p_full[2], p_empty[2];
+  uint64_t o_bar, drain;
+  TileInfo info[kStages];
+  uint32_t tmem_base;
+  int abort;
+};
+
+struct AttnParams {
+  int N, H, nb, npairs, nitems;
+  const int32_t* row_ptr;
+  const int32_t* plist;  // union lists: entry = j | mask << 16, at row_ptr[h*nb + 2p]
+  const int32_t* plen;   // [H * npairs]
+  uint16_t* O;
+  uint32_t* status;
+  uint32_t* counter;
+};
+
+__device__ __forceinline__ void give_up(AttnSmem& S, uint32_t* status) {
+  flag_status(status, kStatusTimeout);
+  *reinterpret_cast<volatile int*>(&S.abort) = 1;
+}
+
+// ------------------------------------------------------------------------------------
+// Union of the two kept lists of every query-block pair, via per-warp bitmaps.
+// One warp per pair; grid ceil(H * npairs / 8) x 256 threads.
+// ------------------------------------------------------------------------------------
+__global__ void __launch_bounds__(256) k_pairs(const int32_t* __restrict__ row_ptr,
+                                               const int32_t* __restrict__ col_idx,
+                                               int64_t cap, int64_t scratch_cap, int nb,
+                                               int npairs, int H, int32_t* __restrict__ plist,
+                                               int32_t* __restrict__ plen, uint32_t* status) {
+  __shared__ uint32_t bits[8][2][RESS_MAX_BLOCKS / 32];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int pair = blockIdx.x * 8 + warp;
+  if (pair >= H * npairs) return;
+  const int h = pair / npairs, p = pair % npairs;
+  const int words = (nb + 31) / 32;
+  uint32_t* bA = bits[warp][0];
+  uint32_t* bB = bits[warp][1];
+  for (int w = lane; w < words; w += 32) bA[w] = bB[w] = 0u;
+  const int64_t ra = (int64_t)h * nb + 2 * p;
+  const bool has_b = 2 * p + 1 < nb;
+  const int64_t sa = row_ptr[ra], ea = row_ptr[ra + 1];
+  const int64_t eb = has_b ? row_ptr[ra + 2] : ea;
+  const bool ok = sa >= 0 && sa <= ea && ea <= eb && eb <= cap && eb <= scratch_cap &&
+                  ea - sa <= nb && eb - ea <= nb;
+  __syncwarp();
+  if (!ok) {
+    if (lane == 0) {
+      flag_status(status, kStatusBadRow);
+      plen[pair] = 0;
+    }
+    return;
+  }
+  for (int64_t x = sa + lane; x < eb; x += 32) {
+    const int j = col_idx[x];
+    if (j < 0 || j >= nb) {
+      flag_status(status, kStatusBadIndex);
+      continue;
+    }
+    atomicOr((x < ea ? bA : bB) + (j >> 5), 1u << (j & 31));
+  }
+  __syncwarp();
+  // lane l owns words [4l, 4l + 4)
+  int cnt = 0;
+  for (int w = 4 * lane; w < min(words, 4 * lane + 4); ++w) cnt += __popc(bA[w] | bB[w]);
+  int incl = cnt;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const int v = __shfl_up_sync(0xffffffffu, incl, o);
+    if (lane >= o) incl += v;
+  }
+  int pos = incl - cnt;
+  for (int w = 4 * lane; w < min(words, 4 * lane + 4); ++w) {
+    const uint32_t a = bA[w], b = bB[w];
+    uint32_t u = a | b;
+    while (u) {
+      const int bit = __ffs(u) - 1;
+      u &= u - 1;
+      const int m = (int)((a >> bit) & 1u) | (int)(((b >> bit) & 1u) << 1);
+      plist[sa + pos] = (w * 32 + bit) | (m << 16);
+      ++pos;
+    }
+  }
+  if (lane == 31) plen[pair] = incl;
+}
+
+// ------------------------------------------------------------------------------------
+// main kernel
+// ------------------------------------------------------------------------------------
+__global__ void __launch_bounds__(kAttnThreads, 2)
+    k_attn(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
+           const __grid_constant__ CUtensorMap tmV, const AttnParams a) {
+  extern __shared__ uint8_t smem_raw[];
+  AttnSmem& S = *reinterpret_cast<AttnSmem*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
+                                             ~static_cast<uintptr_t>(1023));
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  volatile int* abort = &S.abort;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kStages; ++s) {
+      mbar_init(&S.kv_full[s], 1);
+      mbar_init(&S.kv_empty[s], 1);
+    }
+    mbar_init(&S.q_full, 1);
+    mbar_init(&S.q_empty, 1);
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(&S.s_full[b], 1);
+      mbar_init(&S.p_full[b], 4);
+      mbar_init(&S.p_empty[b], 1);
+    }
+    mbar_init(&S.o_bar, 1);
+    mbar_init(&S.drain, 1);
+    S.abort = 0;
+    fence_barrier_init();
+    prefetch_tensormap(&tmQ);
+    prefetch_tensormap(&tmK);
+    prefetch_tensormap(&tmV);
+  }
+  if (warp == 1) tmem_alloc(&S.tmem_base, kTmemCols);
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = S.tmem_base;
+
+  if (warp == 0) {
+    // =============================== producer ====================================
+    if (lane == 0) {
+      int g = 0, it = 0;
+      bool failed = false, q_loaded = false;
+      for (;;) {
+        const int item = (int)atomicAdd(a.counter, 1u);
+        if (item >= a.nitems) break;
+        const int p = a.npairs - 1 - item / a.H;  // pairs holding special query blocks first
+        const int h = item % a.H;
+        const int n = a.plen[h * a.npairs + p];
+        if (n <= 0) continue;
+        const int32_t* lst = a.plist + a.row_ptr[(int64_t)h * a.nb + 2 * p];
+        if (it > 0 && !mbar_wait(&S.q_empty, (it - 1) & 1, abort, kWaitNs)) {
+          failed = true;
+          break;
+        }
+        mbar_arrive_expect_tx(&S.q_full, kRows * 128);
+        tma_load_3d(S.Q, &tmQ, &S.q_full, 0, h, kRows * p);
+        q_loaded = true;
+        for (int e0 = 0; e0 < n && !failed; e0 += 32) {
+          int ent[32];
+#pragma unroll
+          for (int k = 0; k < 32; ++k) ent[k] = (e0 + k < n) ? lst[e0 + k] : 0;
+#pragma unroll 1
+          for (int k = 0; k < 32 && e0 + k < n; ++k) {
+            const int s = g % kStages, u = g / kStages;
+            if (u > 0 && !mbar_wait(&S.kv_empty[s], (u - 1) & 1, abort, kWaitNs)) {
+              failed = true;
+              break;
+            }
+            const int j = ent[k] & 0xffff;
+            int fl = 0;
+            if (e0 + k == 0) fl |= kFirst;
+            if (e0 + k == n - 1) fl |= kLast;
+            S.info[s] = TileInfo{j, ent[k] >> 16, fl, item};
+            mbar_arrive_expect_tx(&S.kv_full[s], 2 * kTileBytes);
+            tma_load_3d(S.K[s], &tmK, &S.kv_full[s], 0, h, 64 * j);
+            tma_load_3d(S.V[s], &tmV, &S.kv_full[s], 0, h, 64 * j);
+            ++g;
+          }
+        }
+        if (failed) break;
+        ++it;
+        q_loaded = false;
+      }
+      if (!failed) {
+        const int s = g % kStages, u = g / kStages;
+        if (u > 0 && !mbar_wait(&S.kv_empty[s], (u - 1) & 1, abort, kWaitNs)) {
+          failed = true;
+        } else {
+          S.info[s] = TileInfo{0, 0, kTerm, -1};
+          mbar_arrive(&S.kv_full[s]);
+        }
+      }
+      if (failed) {
+        give_up(S, a.status);
+        // let every copy already issued land before the CTA's shared memory goes away
+        for (int back = 1; back <= kStages && g - back >= 0; ++back) {
+          const int gg = g - back;
+          volatile int no_abort = 0;
+          mbar_wait(&S.kv_full[gg % kStages], (gg / kStages) & 1, &no_abort, kDrainNs);
+        }
+        if (q_loaded) {
+          volatile int no_abort = 0;
+          mbar_wait(&S.q_full, it & 1, &no_abort, kDrainNs);
+        }
+      }
+    }
+  } else if (warp == 1) {
+    // ================================ MMA issuer ===================================
+    if (lane == 0) {
+      const uint32_t idesc_qk = idesc_bf16_f32(kRows, 64, false);
+      const uint32_t idesc_pv = idesc_bf16_f32(kRows, 64, true);
+      const uint32_t q_addr = smem_u32(S.Q);
+      int g = 0, it = 0;
+      bool have_prev = false, prev_first = false, failed = false;
+      int prev_g = 0;
+      auto issue_pv = [&](int pg, bool first) -> bool {
+        const int pb = pg & 1, ps = pg % kStages;
+        if (!mbar_wait(&S.p_full[pb], (pg >> 1) & 1, abort, kWaitNs)) return false;
+        tc_fence_after();
+        const uint32_t p_addr = smem_u32(S.P[pb]);
+        const uint32_t v_addr = smem_u32(S.V[ps]);
+#pragma unroll
+        for (int k = 0; k < 4; ++k)
+          mma_bf16_ss(tmem + kColO, sdesc_sw128(p_addr + 32 * k), sdesc_sw128(v_addr + 2048 * k),
+                      idesc_pv, (k > 0 || !first) ? 1u : 0u);
+        mma_commit(&S.kv_empty[ps]);
+        mma_commit(&S.p_empty[pb]);
+        mma_commit(&S.o_bar);
+        return true;
+      };
+      for (;;) {
+        const int s = g % kStages;
+        if (!mbar_wait(&S.kv_full[s], (g / kStages) & 1, abort, kWaitNs)) {
+          failed = true;
+          break;
+        }
+        const TileInfo info = S.info[s];
+        if (info.flags & kTerm) break;
+        if ((info.flags & kFirst) && !mbar_wait(&S.q_full, it & 1, abort, kWaitNs)) {
+          failed = true;
+          break;
+        }
+        tc_fence_after();
+        const int b = g & 1;
+        const uint32_t k_addr = smem_u32(S.K[s]);
+#pragma unroll
+        for (int k = 0; k < 4; ++k)
+          mma_bf16_ss(tmem + kColS0 + 64 * b, sdesc_sw128(q_addr + 32 * k),
+                      sdesc_sw128(k_addr + 32 * k), idesc_qk, k > 0 ? 1u : 0u);
+        mma_commit(&S.s_full[b]);
+        if (info.flags & kLast) mma_commit(&S.q_empty);
+        if (have_prev && !issue_pv(prev_g, prev_first)) {
+          failed = true;
+          break;
+        }
+        if (info.flags & kLast) {
+          if (!issue_pv(g, (info.flags & kFirst) != 0)) {
+            failed = true;
+            break;
+          }
+          have_prev = false;
+          ++it;
+        } else {
+          have_prev = true;
+          prev_g = g;
+          prev_first = (info.flags & kFirst) != 0;
+        }
+        ++g;
+      }
+      if (failed) give_up(S, a.status);
+      // wait for every MMA issued so far before TMEM is released
+      mma_commit(&S.drain);
+      volatile int no_abort = 0;
+      mbar_wait(&S.drain, 0, &no_abort, kDrainNs);
+    }
+  } else {
+    // ================================ softmax =====================================
+    const int quarter = warp & 3;
+    const int r = quarter * 32 + lane;  // query row within the 128-row tile
+    const int half = r >> 6;
+    const uint32_t lane_base = (uint32_t)(quarter * 32) << 16;
+    const float kScale = 1.4426950408889634f * 0.125f;  // log2(e) / sqrt(64)
+    uint8_t* prow_base[2] = {S.P[0] + r * 128, S.P[1] + r * 128};
+    int g = 0;
+    float m_use = -INFINITY, l = 0.f;
+    int tile_in_item = 0;
+    for (;;) {
+      const int s = g % kStages;
+      if (!mbar_wait(&S.kv_full[s], (g / kStages) & 1, abort, kWaitNs)) {
+        give_up(S, a.status);
+        break;
+      }
+      const TileInfo info = S.info[s];
+      if (info.flags & kTerm) break;
+      if (info.flags & kFirst) {
+        m_use = -INFINITY;
+        l = 0.f;
+        tile_in_item = 0;
+      }
+      const int b = g & 1;
+      if (g >= 2 && !mbar_wait(&S.p_empty[b], ((g >> 1) - 1) & 1, abort, kWaitNs)) {
+        give_up(S, a.status);
+        break;
+      }
+      if (!mbar_wait(&S.s_full[b], (g >> 1) & 1, abort, kWaitNs)) {
+        give_up(S, a.status);
+        break;
+      }
+      tc_fence_after();
+      const bool active = (info.mask >> half) & 1;  // warp-uniform
+      uint4* prow = reinterpret_cast<uint4*>(prow_base[b]);
+      if (active) {
+        float x[64];
+        {
+          uint32_t v[32];
+          RESS_TMEM_LD32(tmem + lane_base + kColS0 + 64 * b, v);
+#pragma unroll
+          for (int c = 0; c < 32; ++c) x[c] = __uint_as_float(v[c]) * kScale;
+          RESS_TMEM_LD32(tmem + lane_base + kColS0 + 64 * b + 32, v);
+#pragma unroll
+          for (int c = 0; c < 32; ++c) x[32 + c] = __uint_as_float(v[c]) * kScale;
+        }
+        if (info.j == a.nb - 1) {  // ragged last key block: keys past N do not exist
+          const int valid = a.N - 64 * info.j;
+#pragma unroll
+          for (int c = 0; c < 64; ++c)
+            if (c >= valid) x[c] = -INFINITY;
+        }
+        float mt = x[0];
+#pragma unroll
+        for (int c = 1; c < 64; ++c) mt = fmaxf(mt, x[c]);
+        float alpha = 1.f;
+        bool rescale = false;
+        if (m_use == -INFINITY) {
+          m_use = mt;  // first kept tile of this row: O row is still zero
+        } else if (mt > m_use + kLazyThreshold) {
+          alpha = ex2(m_use - mt);
+          m_use = mt;
+          rescale = true;
+        }
+        if (__any_sync(0xffffffffu, rescale)) {
+          // the previous P V must have landed before the accumulator row is rescaled
+          if (!mbar_wait(&S.o_bar, (g - 1) & 1, abort, kWaitNs)) {
+            give_up(S, a.status);
+            break;
+          }
+          tc_fence_after();
+#pragma unroll
+          for (int hc = 0; hc < 2; ++hc) {
+            uint32_t v[32];
+            RESS_TMEM_LD32(tmem + lane_base + kColO + 32 * hc, v);
+#pragma unroll
+            for (int c = 0; c < 32; ++c) v[c] = __float_as_uint(__uint_as_float(v[c]) * alpha);
+            RESS_TMEM_ST32(tmem + lane_base + kColO + 32 * hc, v);
+          }
+        }
+        float rs = 0.f;
+#pragma unroll
+        for (int ch = 0; ch < 8; ++ch) {
+          uint32_t w[4];
+#pragma unroll
+          for (int e = 0; e < 4; ++e) {
+            const float p0 = ex2(x[ch * 8 + 2 * e] - m_use);
+            const float p1 = ex2(x[ch * 8 + 2 * e + 1] - m_use);
+            w[e] = pack_bf16x2(p0, p1);
+            rs += __uint_as_float(w[e] << 16) + __uint_as_float(w[e] & 0xffff0000u);
+          }
+          prow[ch ^ (r & 7)] = make_uint4(w[0], w[1], w[2], w[3]);
+        }
+        l = l * alpha + rs;
+      } else {
+#pragma unroll
+        for (int ch = 0; ch < 8; ++ch) prow[ch] = make_uint4(0u, 0u, 0u, 0u);
+      }
+      fence_proxy_async_smem();
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&S.p_full[b]);
+      ++tile_in_item;
+
+      if (info.flags & kLast) {
+        // epilogue: O / l for this row once the last P V has landed
+        if (!mbar_wait(&S.o_bar, g & 1, abort, kWaitNs)) {
+          give_up(S, a.status);
+          break;
+        }
+        tc_fence_after();
+        const int item = info.item;
+        const int p = a.npairs - 1 - item / a.H, h = item % a.H;
+        const int token = kRows * p + r;
+        const bool row_exists = (2 * p + half) < a.nb && token < a.N;
+        uint32_t o[2][32];
+        RESS_TMEM_LD32(tmem + lane_base + kColO, o[0]);
+        RESS_TMEM_LD32(tmem + lane_base + kColO + 32, o[1]);
+        if (row_exists) {
+          if (!(l > 0.f)) flag_status(a.status, kStatusBadRow);
+          const float inv = l > 0.f ? 1.0f / l : 0.f;
+          uint4* dst = reinterpret_cast<uint4*>(a.O + ((int64_t)token * a.H + h) * 64);
+#pragma unroll
+          for (int ch = 0; ch < 8; ++ch) {
+            uint32_t w[4];
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+              const int c = ch * 8 + 2 * e;
+              w[e] = pack_bf16x2(__uint_as_float(o[c >> 5][c & 31]) * inv,
+                                 __uint_as_float(o[(c + 1) >> 5][(c + 1) & 31]) * inv);
+            }
+            dst[ch] = make_uint4(w[0], w[1], w[2], w[3]);
+          }
+        }
+        tc_fence_before();
+      }
+      ++g;
+    }
+  }
+
+  __syncwarp();
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc(tmem, kTmemCols);
+  }
+}
+
+// ------------------------------------------------------------------------------------
+// host side
+// ------------------------------------------------------------------------------------
+static PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  if (!fn) {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault,
+                                         &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  }
+  return fn;
+}
+
+// [N, H, 64] bf16 viewed as a 3-D tensor {64, H, N}; box {64, 1, rows}, 128-byte swizzle.
+static bool make_map(CUtensorMap* m, const void* base, int N, int H, int rows) {
+  auto fn = encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[3] = {64, (cuuint64_t)H, (cuuint64_t)N};
+  cuuint64_t strides[2] = {128, (cuuint64_t)H * 128};
+  cuuint32_t box[3] = {64, 1, (cuuint32_t)rows};
+  cuuint32_t estr[3] = {1, 1, 1};
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides, box,
+            estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+static int sm_count() {
+  int dev = 0, n = 0;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev);
+  return n > 0 ? n : 1;
+}
+
+cudaError_t launch_sparse_attn(const AttnArgs& x, cudaStream_t st) {
+  const Shape& s = x.s;
+  CUtensorMap tq, tk, tv;
+  if (!make_map(&tq, x.Q, s.N, s.H, kRows) || !make_map(&tk, x.K, s.N, s.H, 64) ||
+      !make_map(&tv, x.V, s.N, s.H, 64))
+    return cudaErrorInvalidValue;
+  const int npairs = (s.nb + 1) / 2;
+  const int pairs = s.H * npairs;
+  k_pairs<<<(pairs + 7) / 8, 256, 0, st>>>(x.row_ptr, x.col_idx, x.col_capacity, x.scratch_cap,
+                                           s.nb, npairs, s.H, x.plist, x.plen, x.status);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  e = cudaMemsetAsync(x.counter, 0, sizeof(uint32_t), st);
+  if (e != cudaSuccess) return e;
+  AttnParams p;
+  p.N = s.N;
+  p.H = s.H;
+  p.nb = s.nb;
+  p.npairs = npairs;
+  p.nitems = pairs;
+  p.row_ptr = x.row_ptr;
+  p.plist = x.plist;
+  p.plen = x.plen;
+  p.O = x.O;
+  p.status = x.status;
+  p.counter = x.counter;
+  const size_t smem = sizeof(AttnSmem) + 1024;
+  e = cudaFuncSetAttribute(k_attn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e != cudaSuccess) return e;
+  const int grid = min(pairs, 2 * sm_count());
+  k_attn<<<grid, kAttnThreads, smem, st>>>(tq, tk, tv, p);
+  return cudaGetLastError();
+}
+
+}  // namespace ress

@@ -1,0 +1,744 @@
+// ReSS block selection on sm_103a: pooling, pooled attention map, drift scoring, initial
+// top-c selection and the restoration rounds (Sec. 4.1-4.3 of the paper).
+//
+// Arithmetic is float32 with fixed-order reductions (deterministic, Appendix B.4).  The
+// per-head Gram matrix M_h = W_O^h^T W_O^h (Eq. 8) enters through its Cholesky factor F_h
+// (F_h^T F_h = M_h), so every quadratic form of the method is a squared norm in the
+// 64-dimensional "F space":
+//   z~_j = F_h V_j,  y~_i = F_h v_bar_i = sum_j P_ij z~_j            (Eq. 1)
+//   q_ij = ||y~_i - z~_j||^2 = e_ij^T M_h e_ij                     (Eq. 9, never negative)
+//   g~   = F_h g = sum_{j in D} P_ij (y~_i - z~_j) = -sum_{j not in D} P_ij (y~_i - z~_j)
+//   G    = ||g~||^2,  d_ik^T M_h g = P_ik (y~_i - z~_k) . g~        (Eq. 12, 14, 15)
+// The last identity for g~ holds because sum_{j in B} P_ij (y~_i - z~_j) = 0: the net drift
+// of the drop set is minus that of the kept set, which is the smaller one at high sparsity.
+
+#include <math.h>
+
+#include "ress_internal.cuh"
+
+namespace ress {
+
+constexpr int kThreads = 256;
+constexpr int RT = 32;    // query rows per CTA (score and round kernels)
+constexpr int BN = 128;   // key blocks per staged chunk
+constexpr int LDA = 68;   // padded float stride of a staged 64-vector (17 x 16 B)
+constexpr unsigned kFull = 0xffffffffu;
+
+// ------------------------------------------------------------------------------------
+// Eq. 8: M_h = W_O^h^T W_O^h in float64, then its Cholesky factor F_h = L^T.
+// ------------------------------------------------------------------------------------
+__global__ void __launch_bounds__(kThreads) k_prepare_wo(const uint16_t* __restrict__ W,
+                                                          int d_model, int H,
+                                                          float* __restrict__ F) {
+  __shared__ double M[64][65];
+  __shared__ double Wc[16][64];
+  __shared__ double piv_s;
+  const int h = blockIdx.x, t = threadIdx.x;
+  const int a = t >> 2;  // row of M owned by this thread
+  double acc[16];
+#pragma unroll
+  for (int k = 0; k < 16; ++k) acc[k] = 0.0;
+  const int64_t ldw = (int64_t)H * kHeadDim;
+  for (int r0 = 0; r0 < d_model; r0 += 16) {
+    for (int f = t; f < 16 * 64; f += kThreads) {
+      const int rr = f >> 6, c = f & 63;
+      double v = 0.0;
+      if (r0 + rr < d_model) {
+        const uint16_t b = W[(int64_t)(r0 + rr) * ldw + h * kHeadDim + c];
+        v = (double)__uint_as_float((uint32_t)b << 16);
+      }
+      Wc[rr][c] = v;
+    }
+    __syncthreads();
+    for (int rr = 0; rr < 16; ++rr) {
+      const double wa = Wc[rr][a];
+#pragma unroll
+      for (int k = 0; k < 16; ++k) acc[k] += wa * Wc[rr][(t & 3) + 4 * k];
+    }
+    __syncthreads();
+  }
+#pragma unroll
+  for (int k = 0; k < 16; ++k) M[a][(t & 3) + 4 * k] = acc[k];
+  __syncthreads();
+  // pivot tolerance relative to the largest diagonal entry
+  if (t == 0) {
+    double mx = 0.0;
+    for (int k = 0; k < 64; ++k) mx = fmax(mx, M[k][k]);
+    piv_s = mx * 1e-13;
+  }
+  __syncthreads();
+  const double tol = piv_s;
+  for (int k = 0; k < 64; ++k) {
+    if (t == 0) {
+      const double d = M[k][k];
+      M[k][k] = d > tol ? sqrt(d) : 0.0;
+    }
+    __syncthreads();
+    const double p = M[k][k];
+    for (int i = k + 1 + t; i < 64; i += kThreads) M[i][k] = p > 0.0 ? M[i][k] / p : 0.0;
+    __syncthreads();
+    const int n = 63 - k;
+    for (int idx = t; idx < n * n; idx += kThreads) {
+      const int i = k + 1 + idx / n, j = k + 1 + idx % n;
+      if (j <= i) M[i][j] -= M[i][k] * M[j][k];
+    }
+    __syncthreads();
+  }
+  // F[a][b] = L[b][a] for b >= a (upper triangular)
+  for (int f = t; f < 64 * 64; f += kThreads) {
+    const int r = f >> 6, c = f & 63;
+    F[(int64_t)h * 4096 + f] = c >= r ? (float)M[c][r] : 0.0f;
+  }
+}
+
+// ------------------------------------------------------------------------------------
+// Sec. 3 step (1): block means of Q, K and V over the valid tokens of each block.
+// grid (nb, 3); one token is H*64 bf16 = 8H 16-byte chunks (H <= 32).
+// ------------------------------------------------------------------------------------
+__global__ void __launch_bounds__(kThreads) k_pool(const uint16_t* __restrict__ Q,
+                                                    const uint16_t* __restrict__ K,
+                                                    const uint16_t* __restrict__ V, int N,
+                                                    int H, int nb, float* __restrict__ qbar,
+                                                    float* __restrict__ kbar,
+                                                    float* __restrict__ vbar) {
+  __shared__ float part[kThreads * 8];
+  const int j = blockIdx.x, which = blockIdx.y;
+  const uint16_t* X = which == 0 ? Q : (which == 1 ? K : V);
+  float* out = which == 0 ? qbar : (which == 1 ? kbar : vbar);
+  const int C = 8 * H;
+  const int tpp = kThreads / C;
+  const int tok0 = j * kBlock;
+  const int valid = min(kBlock, N - tok0);
+  const int c = threadIdx.x % C, slot = threadIdx.x / C;
+  float acc[8];
+#pragma unroll
+  for (int e = 0; e < 8; ++e) acc[e] = 0.f;
+  if (slot < tpp) {
+    const uint4* base = reinterpret_cast<const uint4*>(X + (int64_t)tok0 * H * kHeadDim) + c;
+#pragma unroll 4
+    for (int tk = slot; tk < valid; tk += tpp) {
+      const uint4 v = ld_stream(base + (int64_t)tk * C);
+      acc[0] += bf16_lo(v.x); acc[1] += bf16_hi(v.x);
+      acc[2] += bf16_lo(v.y); acc[3] += bf16_hi(v.y);
+      acc[4] += bf16_lo(v.z); acc[5] += bf16_hi(v.z);
+      acc[6] += bf16_lo(v.w); acc[7] += bf16_hi(v.w);
+    }
+#pragma unroll
+    for (int e = 0; e < 8; ++e) part[slot * C * 8 + c * 8 + e] = acc[e];
+  }
+  __syncthreads();
+  const float inv = 1.0f / (float)valid;
+  for (int f = threadIdx.x; f < C * 8; f += kThreads) {
+    float s = 0.f;
+    for (int sl = 0; sl < tpp; ++sl) s += part[sl * C * 8 + f];
+    const int h = f >> 6, d = f & 63;
+    out[((int64_t)h * nb + j) * kHeadDim + d] = s * inv;
+  }
+}
+
+// ------------------------------------------------------------------------------------
+// z~_j = F_h V_j.  grid (ceil(nb/64), H).
+// ------------------------------------------------------------------------------------
+__global__ void __launch_bounds__(kThreads) k_zproj(const float* __restrict__ F,
+                                                     const float* __restrict__ vbar, int nb,
+                                                     float* __restrict__ ztil) {
+  __shared__ float Fs[64][65];
+  __shared__ float Vs[64][65];
+  const int h = blockIdx.y, j0 = blockIdx.x * 64, t = threadIdx.x;
+  for (int f = t; f < 4096; f += kThreads) {
+    const int r = f >> 6, c = f & 63;
+    Fs[r][c] = F[(int64_t)h * 4096 + f];
+    Vs[r][c] = (j0 + r < nb) ? vbar[((int64_t)h * nb + j0 + r) * 64 + c] : 0.f;
+  }
+  __syncthreads();
+  const int jj = t >> 2, a0 = (t & 3) * 16;
+  if (j0 + jj >= nb) return;
+  for (int a = a0; a < a0 + 16; ++a) {
+    float s = 0.f;
+    for (int b = 0; b < 64; ++b) s = fmaf(Fs[a][b], Vs[jj][b], s);
+    ztil[((int64_t)h * nb + j0 + jj) * 64 + a] = s;
+  }
+}
+
+// ------------------------------------------------------------------------------------
+// Shared pieces of the score and round kernels.
+// ------------------------------------------------------------------------------------
+struct SelSmem {
+  float A[RT][LDA];      // per-row 64-vectors: q_bar, then y~
+  float Gv[RT][LDA];     // per-row g~ (round kernel)
+  float B[BN][LDA];      // staged chunk of per-block 64-vectors (k_bar or z~)
+  float Pc[RT][BN + 4];  // staged chunk of P (score kernel)
+  float rowm[RT], rowiz[RT];
+};
+
+struct SelPtrs {
+  int nb, ncand, words, ld;
+  const float *qbar, *kbar, *ztil;
+  float *ytil, *gtil, *P, *q, *t, *K, *G, *J, *Jbest, *J0;
+  uint32_t *dmask, *bmask;
+};
+
+__host__ __device__ inline SelPtrs sel_ptrs(const Shape& s, char* ws, const ress_ws_layout& L) {
+  SelPtrs p;
+  p.nb = s.nb;
+  p.ncand = s.ncand;
+  p.words = s.words;
+  p.ld = s.ld;
+  p.qbar = (const float*)(ws + L.qbar);
+  p.kbar = (const float*)(ws + L.kbar);
+  p.ztil = (const float*)(ws + L.ztil);
+  p.ytil = (float*)(ws + L.ytil);
+  p.gtil = (float*)(ws + L.gtil);
+  p.P = (float*)(ws + L.P);
+  p.q = (float*)(ws + L.q);
+  p.t = (float*)(ws + L.t);
+  p.K = (float*)(ws + L.K);
+  p.G = (float*)(ws + L.G);
+  p.J = (float*)(ws + L.J);
+  p.Jbest = (float*)(ws + L.Jbest);
+  p.J0 = (float*)(ws + L.J0);
+  p.dmask = (uint32_t*)(ws + L.dmask);
+  p.bmask = (uint32_t*)(ws + L.bmask);
+  return p;
+}
+
+// Stage rows [j0, j0+BN) of a [nb, 64] float matrix into B (zeros past nb).
+__device__ __forceinline__ void stage_blocks(float (*B)[LDA], const float* __restrict__ src,
+                                             int j0, int nb) {
+  for (int f = threadIdx.x; f < BN * 16; f += kThreads) {
+    const int jj = f >> 4, d4 = (f & 15) << 2;
+    float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (j0 + jj < nb) v = *reinterpret_cast<const float4*>(src + (int64_t)(j0 + jj) * 64 + d4);
+    *reinterpret_cast<float4*>(&B[jj][d4]) = v;
+  }
+}
+
+// Stage RT per-row 64-vectors (rows past `nrows` are zero).
+__device__ __forceinline__ void stage_rows(float (*A)[LDA], const float* __restrict__ src,
+                                           int nrows) {
+  for (int f = threadIdx.x; f < RT * 16; f += kThreads) {
+    const int r = f >> 4, d4 = (f & 15) << 2;
+    float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (r < nrows) v = *reinterpret_cast<const float4*>(src + (int64_t)r * 64 + d4);
+    *reinterpret_cast<float4*>(&A[r][d4]) = v;
+  }
+}
+
+enum { kOpDot = 0, kOpDist = 1, kOpGain = 2 };
+
+// Warp tile of 8 rows (8*rg ..) x 2 staged blocks (jb, jb + 32), reduced over the 64
+// channels in ascending order:
+//   kOpDot  : sum_d A[r][d] B[j][d]
+//   kOpDist : sum_d (A[r][d] - B[j][d])^2
+//   kOpGain : sum_d (A[r][d] - B[j][d]) Gv[r][d]
+template <int OP>
+__device__ __forceinline__ void tile8x2(const SelSmem& S, int rg, int jb, float acc[8][2]) {
+#pragma unroll
+  for (int x = 0; x < 8; ++x) acc[x][0] = acc[x][1] = 0.f;
+#pragma unroll 2
+  for (int d = 0; d < 64; d += 4) {
+    const float4 b0 = *reinterpret_cast<const float4*>(&S.B[jb][d]);
+    const float4 b1 = *reinterpret_cast<const float4*>(&S.B[jb + 32][d]);
+#pragma unroll
+    for (int x = 0; x < 8; ++x) {
+      const float4 a = *reinterpret_cast<const float4*>(&S.A[rg * 8 + x][d]);
+      if (OP == kOpDot) {
+        acc[x][0] = fmaf(a.x, b0.x, acc[x][0]); acc[x][0] = fmaf(a.y, b0.y, acc[x][0]);
+        acc[x][0] = fmaf(a.z, b0.z, acc[x][0]); acc[x][0] = fmaf(a.w, b0.w, acc[x][0]);
+        acc[x][1] = fmaf(a.x, b1.x, acc[x][1]); acc[x][1] = fmaf(a.y, b1.y, acc[x][1]);
+        acc[x][1] = fmaf(a.z, b1.z, acc[x][1]); acc[x][1] = fmaf(a.w, b1.w, acc[x][1]);
+      } else if (OP == kOpDist) {
+        float e;
+        e = a.x - b0.x; acc[x][0] = fmaf(e, e, acc[x][0]);
+        e = a.y - b0.y; acc[x][0] = fmaf(e, e, acc[x][0]);
+        e = a.z - b0.z; acc[x][0] = fmaf(e, e, acc[x][0]);
+        e = a.w - b0.w; acc[x][0] = fmaf(e, e, acc[x][0]);
+        e = a.x - b1.x; acc[x][1] = fmaf(e, e, acc[x][1]);
+        e = a.y - b1.y; acc[x][1] = fmaf(e, e, acc[x][1]);
+        e = a.z - b1.z; acc[x][1] = fmaf(e, e, acc[x][1]);
+        e = a.w - b1.w; acc[x][1] = fmaf(e, e, acc[x][1]);
+      } else {
+        const float4 g = *reinterpret_cast<const float4*>(&S.Gv[rg * 8 + x][d]);
+        acc[x][0] = fmaf(a.x - b0.x, g.x, acc[x][0]); acc[x][0] = fmaf(a.y - b0.y, g.y, acc[x][0]);
+        acc[x][0] = fmaf(a.z - b0.z, g.z, acc[x][0]); acc[x][0] = fmaf(a.w - b0.w, g.w, acc[x][0]);
+        acc[x][1] = fmaf(a.x - b1.x, g.x, acc[x][1]); acc[x][1] = fmaf(a.y - b1.y, g.y, acc[x][1]);
+        acc[x][1] = fmaf(a.z - b1.z, g.z, acc[x][1]); acc[x][1] = fmaf(a.w - b1.w, g.w, acc[x][1]);
+      }
+    }
+  }
+}
+
+// Order-preserving map of a float to uint32; every non-NaN value maps above 0, so 0 can
+// mark "not a candidate".  -0 is folded onto +0; NaN maps to the lowest candidate value.
+__device__ __forceinline__ uint32_t order_key(float x) {
+  x = x + 0.0f;
+  const uint32_t b = __float_as_uint(x);
+  if (x != x) return 1u;
+  return (b & 0x80000000u) ? ~b : (b | 0x80000000u);
+}
+
+// Exact top-m of kb[0..n) for one warp: the m largest keys, ties to the lower index
+// (requires m <= number of nonzero keys).  Result: bitmask sel[words] in shared memory.
+__device__ void warp_topm(const uint32_t* kb, int n, int m, uint32_t* sel, int words) {
+  const int lane = threadIdx.x & 31;
+  uint32_t lo = 0;
+  if (m > 0) {
+    for (int bit = 31; bit >= 0; --bit) {
+      const uint32_t cand = lo | (1u << bit);
+      int cnt = 0;
+      for (int j = lane; j < n; j += 32) cnt += kb[j] >= cand ? 1 : 0;
+      cnt = __reduce_add_sync(kFull, cnt);
+      if (cnt >= m) {
+        lo = cand;
+        if (cnt == m) break;
+      }
+    }
+  }
+  int gt = 0;
+  for (int j = lane; j < n; j += 32) gt += kb[j] > lo ? 1 : 0;
+  gt = __reduce_add_sync(kFull, gt);
+  const int need = m - gt;
+  int taken = 0;
+  for (int w = 0; w < words; ++w) {
+    const int j = w * 32 + lane;
+    const uint32_t v = j < n ? kb[j] : 0u;
+    const bool is_gt = m > 0 && v > lo;
+    const bool is_eq = m > 0 && j < n && v == lo && v != 0u;
+    const uint32_t eqb = __ballot_sync(kFull, is_eq);
+    const int rank = taken + __popc(eqb & ((1u << lane) - 1u));
+    const uint32_t sb = __ballot_sync(kFull, is_gt || (is_eq && rank < need));
+    if (lane == 0) sel[w] = sb;
+    taken += __popc(eqb);
+  }
+  __syncwarp();
+}
+
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(kFull, v, o);
+  return v;
+}
+
+// Bits of word w that are valid key blocks (< nb).
+__device__ __forceinline__ uint32_t valid_bits(int w, int n) {
+  const int rem = n - w * 32;
+  return rem >= 32 ? kFull : (rem <= 0 ? 0u : ((1u << rem) - 1u));
+}
+
+// g~ = sum_{j not in D} P_ij (z~_j - y~_i) and K = sum_{j not in D} P_ij for one row, by
+// one warp (lane owns channels 2*lane, 2*lane+1).  D: bitmask words in shared memory.
+__device__ __forceinline__ void kept_drift(const uint32_t* D, const SelPtrs& p,
+                                           const float* __restrict__ Prow,
+                                           const float* __restrict__ zt, float y0, float y1,
+                                           float& g0, float& g1, float& K) {
+  const int lane = threadIdx.x & 31;
+  g0 = g1 = K = 0.f;
+  for (int w = 0; w < p.words; ++w) {
+    uint32_t keep = ~D[w] & valid_bits(w, p.nb);
+    while (keep) {
+      const int j = w * 32 + __ffs(keep) - 1;
+      keep &= keep - 1;
+      const float pj = Prow[j];
+      const float2 z = *reinterpret_cast<const float2*>(zt + (int64_t)j * 64 + 2 * lane);
+      g0 = fmaf(pj, z.x - y0, g0);
+      g1 = fmaf(pj, z.y - y1, g1);
+      K += pj;
+    }
+  }
+}
+
+// ------------------------------------------------------------------------------------
+// Score kernel: Sec. 4.1-4.2 and the initial state of Sec. 4.3 for RT query rows of one
+// head.  grid (ceil(ncand / RT), H).
+// ------------------------------------------------------------------------------------
+struct Budgets {
+  int c[RESS_MAX_HEADS];
+};
+
+__global__ void __launch_bounds__(kThreads, 2) k_score(SelPtrs p, Budgets bud) {
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  SelSmem& S = *reinterpret_cast<SelSmem*>(smem_raw);
+  uint32_t* kb_all = reinterpret_cast<uint32_t*>(smem_raw + sizeof(SelSmem));
+  uint32_t* sel_all = kb_all + 8 * p.ld;
+  const int h = blockIdx.y, i0 = blockIdx.x * RT;
+  const int nrows = min(RT, p.ncand - i0);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int rg = warp & 3, jb = (warp >> 2) * 64 + lane;
+  const int64_t hrow = (int64_t)h * p.nb;
+  float* Pbase = p.P + (hrow + i0) * p.ld;
+  float* qbase = p.q + (hrow + i0) * p.ld;
+  const float* kb_h = p.kbar + hrow * 64;
+  const float* zt_h = p.ztil + hrow * 64;
+
+  // ---- pass 1: pooled logits q_bar_i . k_bar_j / sqrt(64) into P (as logits) --------
+  stage_rows(S.A, p.qbar + (hrow + i0) * 64, nrows);
+  for (int j0 = 0; j0 < p.nb; j0 += BN) {
+    stage_blocks(S.B, kb_h, j0, p.nb);
+    __syncthreads();
+    float acc[8][2];
+    tile8x2<kOpDot>(S, rg, jb, acc);
+#pragma unroll
+    for (int x = 0; x < 8; ++x) {
+      const int r = rg * 8 + x;
+      if (r < nrows) {
+        if (j0 + jb < p.nb) Pbase[(int64_t)r * p.ld + j0 + jb] = acc[x][0] * 0.125f;
+        if (j0 + jb + 32 < p.nb) Pbase[(int64_t)r * p.ld + j0 + jb + 32] = acc[x][1] * 0.125f;
+      }
+    }
+    __syncthreads();
+  }
+
+  // ---- softmax statistics per row (max and normaliser, fixed order) ------------------
+  for (int r = warp; r < nrows; r += 8) {
+    const float* row = Pbase + (int64_t)r * p.ld;
+    float m = -INFINITY, z = 0.f;
+    for (int j = lane; j < p.nb; j += 32) {
+      const float x = row[j];
+      if (x > m) {
+        z = z * expf(m - x) + 1.f;
+        m = x;
+      } else {
+        z += expf(x - m);
+      }
+    }
+    float mall = m;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) mall = fmaxf(mall, __shfl_xor_sync(kFull, mall, o));
+    z = (m == -INFINITY) ? 0.f : z * expf(m - mall);
+    z = warp_sum(z);
+    if (lane == 0) {
+      S.rowm[r] = mall;
+      S.rowiz[r] = 1.0f / z;
+    }
+  }
+  __syncthreads();
+
+  // ---- pass 2: P_ij = softmax, y~_i = sum_j P_ij z~_j (Eq. 1 in F space) -----------
+  float ya[4][2];
+#pragma unroll
+  for (int x = 0; x < 4; ++x) ya[x][0] = ya[x][1] = 0.f;
+  for (int j0 = 0; j0 < p.nb; j0 += BN) {
+    stage_blocks(S.B, zt_h, j0, p.nb);
+    for (int f = threadIdx.x; f < RT * (BN / 4); f += kThreads) {
+      const int r = f / (BN / 4), c4 = (f % (BN / 4)) * 4;
+      float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+      if (r < nrows) {
+        float* src = Pbase + (int64_t)r * p.ld + j0 + c4;
+        const float m = S.rowm[r], iz = S.rowiz[r];
+        float e[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          e[u] = 0.f;
+          if (j0 + c4 + u < p.nb) {
+            e[u] = expf(src[u] - m) * iz;
+            src[u] = e[u];
+          }
+        }
+        v = make_float4(e[0], e[1], e[2], e[3]);
+      }
+      *reinterpret_cast<float4*>(&S.Pc[r][c4]) = v;
+    }
+    __syncthreads();
+#pragma unroll 2
+    for (int jj = 0; jj < BN; jj += 4) {
+      float4 pv[4];
+#pragma unroll
+      for (int x = 0; x < 4; ++x) pv[x] = *reinterpret_cast<const float4*>(&S.Pc[warp * 4 + x][jj]);
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const float2 z = *reinterpret_cast<const float2*>(&S.B[jj + u][2 * lane]);
+#pragma unroll
+        for (int x = 0; x < 4; ++x) {
+          const float pu = u == 0 ? pv[x].x : (u == 1 ? pv[x].y : (u == 2 ? pv[x].z : pv[x].w));
+          ya[x][0] = fmaf(pu, z.x, ya[x][0]);
+          ya[x][1] = fmaf(pu, z.y, ya[x][1]);
+        }
+      }
+    }
+    __syncthreads();
+  }
+#pragma unroll
+  for (int x = 0; x < 4; ++x) {
+    const int r = warp * 4 + x;
+    S.A[r][2 * lane] = ya[x][0];
+    S.A[r][2 * lane + 1] = ya[x][1];
+    if (r < nrows)
+      *reinterpret_cast<float2*>(p.ytil + (hrow + i0 + r) * 64 + 2 * lane) =
+          make_float2(ya[x][0], ya[x][1]);
+  }
+  __syncthreads();
+
+  // ---- pass 3: q_ij = ||y~_i - z~_j||^2 (Eq. 9) --------------------------------------
+  for (int j0 = 0; j0 < p.nb; j0 += BN) {
+    stage_blocks(S.B, zt_h, j0, p.nb);
+    __syncthreads();
+    float acc[8][2];
+    tile8x2<kOpDist>(S, rg, jb, acc);
+#pragma unroll
+    for (int x = 0; x < 8; ++x) {
+      const int r = rg * 8 + x;
+      if (r < nrows) {
+        if (j0 + jb < p.nb) qbase[(int64_t)r * p.ld + j0 + jb] = acc[x][0];
+        if (j0 + jb + 32 < p.nb) qbase[(int64_t)r * p.ld + j0 + jb + 32] = acc[x][1];
+      }
+    }
+    __syncthreads();
+  }
+
+  // ---- initial selection (Eq. 7) and the state of Eq. 10-12, one warp per row --------
+  uint32_t* kb = kb_all + warp * p.ld;
+  uint32_t* sel = sel_all + warp * p.words;
+  const int c = bud.c[h];
+  for (int r = warp; r < nrows; r += 8) {
+    const int i = i0 + r;
+    const float* Prow = Pbase + (int64_t)r * p.ld;
+    const float* qrow = qbase + (int64_t)r * p.ld;
+    for (int j = lane; j < p.ncand; j += 32) {
+      const float pj = Prow[j];
+      const float key = pj * sqrtf(qrow[j]) / fmaxf(1.0f - pj, kEps);
+      kb[j] = order_key(key);
+    }
+    __syncwarp();
+    warp_topm(kb, p.ncand, c, sel, p.words);  // sel = kept candidates
+    // drop set D0 = candidates not kept
+    for (int w = lane; w < p.words; w += 32) {
+      const uint32_t d = valid_bits(w, p.ncand) & ~sel[w];
+      sel[w] = d;
+      p.dmask[(hrow + i) * p.words + w] = d;
+      p.bmask[(hrow + i) * p.words + w] = d;
+    }
+    __syncwarp();
+    float g0, g1, K;
+    kept_drift(sel, p, Prow, zt_h, S.A[r][2 * lane], S.A[r][2 * lane + 1], g0, g1, K);
+    const float G = warp_sum(g0 * g0 + g1 * g1);
+    const float Kc = fmaxf(K, kEps);
+    const float J = G / (Kc * Kc);
+    *reinterpret_cast<float2*>(p.gtil + (hrow + i) * 64 + 2 * lane) = make_float2(g0, g1);
+    if (lane == 0) {
+      p.K[hrow + i] = K;
+      p.G[hrow + i] = G;
+      p.J[hrow + i] = J;
+      p.Jbest[hrow + i] = J;
+      p.J0[hrow + i] = J;
+    }
+    __syncwarp();
+  }
+}
+
+// Exact decrease of J (Eq. 16) when G changes by dG and K by u, with the denominators
+// clamped at eps as in Eq. 7.  When no clamp applies the two fractions are combined over
+// one denominator so that the result carries no cancellation of J-sized terms.
+__device__ __forceinline__ float delta_J(float G, float K, float dG, float u) {
+  const float K2 = K + u;
+  if (K >= kEps && K2 >= kEps) {
+    const float num = fmaf(G * u, 2.0f * K + u, -dG * (K * K));
+    return num / ((K * K) * (K2 * K2));
+  }
+  const float Kc = fmaxf(K, kEps), K2c = fmaxf(K2, kEps);
+  return G / (Kc * Kc) - (G + dG) / (K2c * K2c);
+}
+
+// ------------------------------------------------------------------------------------
+// Restoration round r (Sec. 4.3, Eq. 13-17) for RT rows of one head.
+// grid (ceil(ncand / RT), H).
+// ------------------------------------------------------------------------------------
+__global__ void __launch_bounds__(kThreads, 2) k_round(SelPtrs p, Budgets bud, int round,
+                                                       float rho) {
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  SelSmem& S = *reinterpret_cast<SelSmem*>(smem_raw);
+  uint32_t* kb_all = reinterpret_cast<uint32_t*>(smem_raw + sizeof(SelSmem));
+  uint32_t* sel_all = kb_all + 8 * p.ld;
+  const int h = blockIdx.y, i0 = blockIdx.x * RT;
+  const int c = bud.c[h];
+  // Eq. 17: m_r = floor(rho c_h / 2^(r+1)), capped by |D| and |P \ D|
+  int m = (int)floor((double)rho * (double)c / (double)(1ull << (round + 1)));
+  m = min(m, min(p.ncand - c, c));
+  if (m <= 0) return;
+  const int nrows = min(RT, p.ncand - i0);
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int rg = warp & 3, jb = (warp >> 2) * 64 + lane;
+  const int64_t hrow = (int64_t)h * p.nb;
+  const float* zt_h = p.ztil + hrow * 64;
+  float* tbase = p.t + (hrow + i0) * p.ld;
+
+  // ---- gains: t_ij = (y~_i - z~_j) . g~_i  (Eq. 14/15 without the P_ij factor) -------
+  stage_rows(S.A, p.ytil + (hrow + i0) * 64, nrows);
+  stage_rows(S.Gv, p.gtil + (hrow + i0) * 64, nrows);
+  for (int j0 = 0; j0 < p.ncand; j0 += BN) {
+    stage_blocks(S.B, zt_h, j0, p.ncand);
+    __syncthreads();
+    float acc[8][2];
+    tile8x2<kOpGain>(S, rg, jb, acc);
+#pragma unroll
+    for (int x = 0; x < 8; ++x) {
+      const int r = rg * 8 + x;
+      if (r < nrows) {
+        if (j0 + jb < p.ncand) tbase[(int64_t)r * p.ld + j0 + jb] = acc[x][0];
+        if (j0 + jb + 32 < p.ncand) tbase[(int64_t)r * p.ld + j0 + jb + 32] = acc[x][1];
+      }
+    }
+    __syncthreads();
+  }
+
+  // ---- per row: exact top-m restores and drops, update, track-best ------------------
+  uint32_t* kb = kb_all + warp * p.ld;
+  uint32_t* sel = sel_all + warp * (3 * p.words);
+  uint32_t* Dw = sel;                // current drop set
+  uint32_t* Rw = sel + p.words;      // chosen restores
+  uint32_t* Xw = sel + 2 * p.words;  // chosen drops
+  for (int r = warp; r < nrows; r += 8) {
+    const int i = i0 + r;
+    const int64_t ri = hrow + i;
+    const float* Prow = p.P + ri * p.ld;
+    const float* qrow = p.q + ri * p.ld;
+    const float* trow = tbase + (int64_t)r * p.ld;
+    for (int w = lane; w < p.words; w += 32) Dw[w] = p.dmask[ri * p.words + w];
+    const float K = p.K[ri], G = p.G[ri];
+    __syncwarp();
+    // restore candidates k in D: u = +P_k, dG = -2 P_k t_k + P_k^2 q_k (Eq. 13, 14)
+    for (int j = lane; j < p.ncand; j += 32) {
+      uint32_t key = 0u;
+      if ((Dw[j >> 5] >> (j & 31)) & 1u) {
+        const float pj = Prow[j];
+        const float dG = fmaf(pj * pj, qrow[j], -2.0f * pj * trow[j]);
+        key = order_key(delta_J(G, K, dG, pj));
+      }
+      kb[j] = key;
+    }
+    __syncwarp();
+    warp_topm(kb, p.ncand, m, Rw, p.words);
+    // drop candidates k in P \ D: u = -P_k, dG = +2 P_k t_k + P_k^2 q_k (Eq. 15)
+    for (int j = lane; j < p.ncand; j += 32) {
+      uint32_t key = 0u;
+      if (!((Dw[j >> 5] >> (j & 31)) & 1u)) {
+        const float pj = Prow[j];
+        const float dG = fmaf(pj * pj, qrow[j], 2.0f * pj * trow[j]);
+        key = order_key(delta_J(G, K, dG, -pj));
+      }
+      kb[j] = key;
+    }
+    __syncwarp();
+    warp_topm(kb, p.ncand, m, Xw, p.words);
+    for (int w = lane; w < p.words; w += 32) Dw[w] = (Dw[w] & ~Rw[w]) | Xw[w];
+    __syncwarp();
+    // exact state of the new set (Eq. 10-12)
+    const float y0 = p.ytil[ri * 64 + 2 * lane], y1 = p.ytil[ri * 64 + 2 * lane + 1];
+    float g0, g1, Kn;
+    kept_drift(Dw, p, Prow, zt_h, y0, y1, g0, g1, Kn);
+    const float Gn = warp_sum(g0 * g0 + g1 * g1);
+    const float Kc = fmaxf(Kn, kEps);
+    const float Jn = Gn / (Kc * Kc);
+    const bool better = Jn < p.Jbest[ri];
+    for (int w = lane; w < p.words; w += 32) {
+      p.dmask[ri * p.words + w] = Dw[w];
+      if (better) p.bmask[ri * p.words + w] = Dw[w];
+    }
+    *reinterpret_cast<float2*>(p.gtil + ri * 64 + 2 * lane) = make_float2(g0, g1);
+    __syncwarp();
+    if (lane == 0) {
+      p.K[ri] = Kn;
+      p.G[ri] = Gn;
+      p.J[ri] = Jn;
+      if (better) p.Jbest[ri] = Jn;
+    }
+    __syncwarp();
+  }
+}
+
+// ------------------------------------------------------------------------------------
+// Kept-block lists (CSR) from the best drop sets; special query rows keep everything.
+// grid (nb, H), one warp per row.
+// ------------------------------------------------------------------------------------
+struct CsrBases {
+  int64_t base[RESS_MAX_HEADS + 1];
+};
+
+__global__ void k_csr(SelPtrs p, Budgets bud, CsrBases cb, int H, int32_t* __restrict__ row_ptr,
+                      int32_t* __restrict__ col_idx, int64_t cap, float* __restrict__ J_best,
+                      uint32_t* __restrict__ drop_mask, uint32_t* status) {
+  const int i = blockIdx.x, h = blockIdx.y, lane = threadIdx.x;
+  const int64_t ri = (int64_t)h * p.nb + i;
+  const int c = bud.c[h];
+  const int ns = p.nb - p.ncand;
+  const bool dense = i >= p.ncand;
+  const int64_t off = cb.base[h] + (dense ? (int64_t)p.ncand * (c + ns) + (int64_t)(i - p.ncand) * p.nb
+                                          : (int64_t)i * (c + ns));
+  const int expect = dense ? p.nb : c + ns;
+  int pos = 0;
+  for (int w = 0; w < p.words; ++w) {
+    const uint32_t dm = dense ? 0u : p.bmask[ri * p.words + w];
+    const uint32_t keep = ~dm & valid_bits(w, p.nb);
+    if (drop_mask && lane == 0) drop_mask[ri * p.words + w] = dm;
+    const int j = w * 32 + lane;
+    const bool k = (keep >> lane) & 1u;
+    const int at = pos + __popc(keep & ((1u << lane) - 1u));
+    if (k && at < expect && off + at < cap) col_idx[off + at] = j;
+    pos += __popc(keep);
+  }
+  if (lane == 0) {
+    if (pos != expect) flag_status(status, kStatusBadRow);
+    row_ptr[ri] = (int32_t)off;
+    if (h == H - 1 && i == p.nb - 1) row_ptr[(int64_t)H * p.nb] = (int32_t)cb.base[H];
+    if (J_best) J_best[ri] = dense ? 0.f : p.Jbest[ri];
+  }
+}
+
+// ------------------------------------------------------------------------------------
+// launchers
+// ------------------------------------------------------------------------------------
+static size_t sel_smem_bytes(const Shape& s, int words_per_warp) {
+  return sizeof(SelSmem) + (size_t)8 * s.ld * 4 + (size_t)8 * words_per_warp * 4;
+}
+
+cudaError_t launch_prepare_wo(const Shape& s, const uint16_t* W_o, float* F, cudaStream_t st) {
+  k_prepare_wo<<<s.H, kThreads, 0, st>>>(W_o, s.d_model, s.H, F);
+  return cudaGetLastError();
+}
+
+static Budgets budgets_of(const SelectArgs& a) {
+  Budgets b;
+  for (int h = 0; h < RESS_MAX_HEADS; ++h) b.c[h] = a.c[h];
+  return b;
+}
+
+cudaError_t launch_score(const SelectArgs& a, cudaStream_t st) {
+  const Shape& s = a.s;
+  SelPtrs p = sel_ptrs(s, a.ws, a.L);
+  float* qbar = (float*)(a.ws + a.L.qbar);
+  float* kbar = (float*)(a.ws + a.L.kbar);
+  float* vbar = (float*)(a.ws + a.L.vbar);
+  float* ztil = (float*)(a.ws + a.L.ztil);
+  k_pool<<<dim3(s.nb, 3), kThreads, 0, st>>>(a.Q, a.K, a.V, s.N, s.H, s.nb, qbar, kbar, vbar);
+  k_zproj<<<dim3((s.nb + 63) / 64, s.H), kThreads, 0, st>>>(a.F, vbar, s.nb, ztil);
+  if (s.ncand <= 0) return cudaGetLastError();
+  const size_t smem = sel_smem_bytes(s, s.words);
+  cudaError_t e = cudaFuncSetAttribute(k_score, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e != cudaSuccess) return e;
+  k_score<<<dim3((s.ncand + RT - 1) / RT, s.H), kThreads, smem, st>>>(p, budgets_of(a));
+  return cudaGetLastError();
+}
+
+cudaError_t launch_round(const SelectArgs& a, int round, float rho, cudaStream_t st) {
+  const Shape& s = a.s;
+  if (s.ncand <= 0) return cudaSuccess;
+  SelPtrs p = sel_ptrs(s, a.ws, a.L);
+  const size_t smem = sel_smem_bytes(s, 3 * s.words);
+  cudaError_t e = cudaFuncSetAttribute(k_round, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e != cudaSuccess) return e;
+  k_round<<<dim3((s.ncand + RT - 1) / RT, s.H), kThreads, smem, st>>>(p, budgets_of(a), round, rho);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_csr(const SelectArgs& a, const int64_t* head_base, int32_t* row_ptr,
+                       int32_t* col_idx, int64_t col_capacity, float* J_best,
+                       uint32_t* drop_mask, cudaStream_t st) {
+  const Shape& s = a.s;
+  SelPtrs p = sel_ptrs(s, a.ws, a.L);
+  CsrBases cb;
+  for (int h = 0; h <= s.H; ++h) cb.base[h] = head_base[h];
+  k_csr<<<dim3(s.nb, s.H), 32, 0, st>>>(p, budgets_of(a), cb, s.H, row_ptr, col_idx, col_capacity,
+                                        J_best, drop_mask, (uint32_t*)(a.ws + a.L.status));
+  return cudaGetLastError();
+}
+
+}  // namespace ress

@@ -1,0 +1,271 @@
+// C ABI of the ReSS hot path: host-side validation, workspace layout and launch order.
+// Every check happens before the first launch; nothing here allocates device memory.
+
+#include <stdarg.h>
+#include <stdio.h>
+#include <string.h>
+
+#include "ress_internal.cuh"
+
+namespace {
+
+thread_local char g_err[512] = "";
+
+int fail(int code, const char* fmt, ...) {
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(g_err, sizeof(g_err), fmt, ap);
+  va_end(ap);
+  return code;
+}
+
+int ok() {
+  g_err[0] = '\0';
+  return RESS_OK;
+}
+
+int check_dims(const ress_dims* d) {
+  if (!d) return fail(RESS_EINVAL, "dims is NULL");
+  if (d->head_dim != RESS_HEAD_DIM)
+    return fail(RESS_EUNSUPPORTED, "head_dim %d unsupported (must be 64)", d->head_dim);
+  if (d->block != RESS_BLOCK) return fail(RESS_EUNSUPPORTED, "block %d unsupported (must be 64)", d->block);
+  if (d->n_heads < 1 || d->n_heads > RESS_MAX_HEADS)
+    return fail(RESS_EUNSUPPORTED, "n_heads %d outside 1..%d", d->n_heads, RESS_MAX_HEADS);
+  if (d->n_tokens < 1) return fail(RESS_EINVAL, "n_tokens %d < 1", d->n_tokens);
+  if (d->n_special < 0 || d->n_special >= d->n_tokens)
+    return fail(RESS_EINVAL, "n_special %d outside 0..n_tokens-1", d->n_special);
+  if (d->d_model < 1) return fail(RESS_EINVAL, "d_model %d < 1", d->d_model);
+  const int64_t nb = ((int64_t)d->n_tokens + RESS_BLOCK - 1) / RESS_BLOCK;
+  if (nb > RESS_MAX_BLOCKS)
+    return fail(RESS_EUNSUPPORTED, "%lld blocks exceed the limit of %d", (long long)nb, RESS_MAX_BLOCKS);
+  return RESS_OK;
+}
+
+int check_ptr(const void* p, size_t align, const char* name) {
+  if (!p) return fail(RESS_EINVAL, "%s is NULL", name);
+  if (reinterpret_cast<uintptr_t>(p) % align)
+    return fail(RESS_EINVAL, "%s is not %zu-byte aligned", name, align);
+  return RESS_OK;
+}
+
+int check_budgets(const ress::Shape& s, const int32_t* c) {
+  if (!c) return fail(RESS_EINVAL, "c_h_host is NULL");
+  for (int h = 0; h < s.H; ++h) {
+    if (s.ncand > 0 && (c[h] < 1 || c[h] > s.ncand))
+      return fail(RESS_EINVAL, "c_h[%d] = %d outside 1..|P| = %d", h, c[h], s.ncand);
+    if (s.ncand == 0 && c[h] != 0)
+      return fail(RESS_EINVAL, "c_h[%d] = %d but there are no candidate blocks", h, c[h]);
+  }
+  return RESS_OK;
+}
+
+int check_ws(const ress::Shape& s, void* ws, size_t ws_bytes, ress_ws_layout* L) {
+  int e = check_ptr(ws, 256, "ws");
+  if (e) return e;
+  *L = ress::make_layout(s);
+  if ((int64_t)ws_bytes < L->total)
+    return fail(RESS_EWORKSPACE, "workspace has %zu bytes, needs %lld", ws_bytes, (long long)L->total);
+  return RESS_OK;
+}
+
+int cuda_fail(cudaError_t e, const char* where) {
+  return fail(RESS_ECUDA, "%s: %s", where, cudaGetErrorString(e));
+}
+
+int64_t head_rows(const ress::Shape& s, int c) {
+  const int ns = s.nb - s.ncand;
+  return (int64_t)s.ncand * (c + ns) + (int64_t)ns * s.nb;
+}
+
+void head_bases(const ress::Shape& s, const int32_t* c, int64_t* base) {
+  base[0] = 0;
+  for (int h = 0; h < s.H; ++h) base[h + 1] = base[h] + head_rows(s, c[h]);
+}
+
+ress::SelectArgs select_args(const ress::Shape& s, const uint16_t* Q, const uint16_t* K,
+                             const uint16_t* V, const float* F, const int32_t* c, void* ws,
+                             const ress_ws_layout& L) {
+  ress::SelectArgs a;
+  a.s = s;
+  a.Q = Q;
+  a.K = K;
+  a.V = V;
+  a.F = F;
+  a.ws = static_cast<char*>(ws);
+  a.L = L;
+  for (int h = 0; h < RESS_MAX_HEADS; ++h) a.c[h] = (c && h < s.H) ? c[h] : 0;
+  return a;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char* ress_last_error(void) { return g_err; }
+
+int32_t ress_abi_version(void) { return RESS_ABI_VERSION; }
+
+int32_t ress_num_blocks(const ress_dims* d) {
+  if (check_dims(d)) return -1;
+  return ress::make_shape(*d).nb;
+}
+
+int32_t ress_num_candidates(const ress_dims* d) {
+  if (check_dims(d)) return -1;
+  return ress::make_shape(*d).ncand;
+}
+
+size_t ress_workspace_bytes(const ress_dims* d) {
+  if (check_dims(d)) return 0;
+  return (size_t)ress::make_layout(ress::make_shape(*d)).total;
+}
+
+int ress_workspace_layout(const ress_dims* d, ress_ws_layout* out) {
+  int e = check_dims(d);
+  if (e) return e;
+  if (!out) return fail(RESS_EINVAL, "out is NULL");
+  *out = ress::make_layout(ress::make_shape(*d));
+  return ok();
+}
+
+int64_t ress_csr_capacity(const ress_dims* d, const int32_t* c) {
+  if (check_dims(d)) return -1;
+  const ress::Shape s = ress::make_shape(*d);
+  if (check_budgets(s, c)) return -1;
+  int64_t base[RESS_MAX_HEADS + 1];
+  head_bases(s, c, base);
+  return base[s.H];
+}
+
+int ress_prepare_wo(const ress_dims* d, const uint16_t* W_o, float* F, void* stream) {
+  int e = check_dims(d);
+  if (e) return e;
+  if ((e = check_ptr(W_o, 2, "W_o")) || (e = check_ptr(F, 16, "F"))) return e;
+  const ress::Shape s = ress::make_shape(*d);
+  cudaError_t ce = ress::launch_prepare_wo(s, W_o, F, static_cast<cudaStream_t>(stream));
+  if (ce != cudaSuccess) return cuda_fail(ce, "ress_prepare_wo");
+  return ok();
+}
+
+int ress_score(const ress_dims* d, const uint16_t* Q, const uint16_t* K, const uint16_t* V,
+               const float* F, const int32_t* c_h, void* ws, size_t ws_bytes, void* stream) {
+  int e = check_dims(d);
+  if (e) return e;
+  if ((e = check_ptr(Q, 16, "Q")) || (e = check_ptr(K, 16, "K")) || (e = check_ptr(V, 16, "V")) ||
+      (e = check_ptr(F, 16, "F")))
+    return e;
+  const ress::Shape s = ress::make_shape(*d);
+  if ((e = check_budgets(s, c_h))) return e;
+  ress_ws_layout L;
+  if ((e = check_ws(s, ws, ws_bytes, &L))) return e;
+  const ress::SelectArgs a = select_args(s, Q, K, V, F, c_h, ws, L);
+  cudaError_t ce = ress::launch_score(a, static_cast<cudaStream_t>(stream));
+  if (ce != cudaSuccess) return cuda_fail(ce, "ress_score");
+  return ok();
+}
+
+int ress_restore(const ress_dims* d, const int32_t* c_h, int32_t rounds, float rho, void* ws,
+                 size_t ws_bytes, int32_t* row_ptr, int32_t* col_idx, int64_t col_capacity,
+                 float* J_best, uint32_t* drop_mask, void* stream) {
+  int e = check_dims(d);
+  if (e) return e;
+  const ress::Shape s = ress::make_shape(*d);
+  if ((e = check_budgets(s, c_h))) return e;
+  if (rounds < 0 || rounds > 32) return fail(RESS_EINVAL, "rounds %d outside 0..32", rounds);
+  if (!(rho >= 0.0f && rho <= 1.0f)) return fail(RESS_EINVAL, "rho %g outside [0, 1]", (double)rho);
+  ress_ws_layout L;
+  if ((e = check_ws(s, ws, ws_bytes, &L))) return e;
+  if ((e = check_ptr(row_ptr, 4, "row_ptr")) || (e = check_ptr(col_idx, 4, "col_idx"))) return e;
+  if (J_best && (e = check_ptr(J_best, 4, "J_best"))) return e;
+  if (drop_mask && (e = check_ptr(drop_mask, 4, "drop_mask"))) return e;
+  int64_t base[RESS_MAX_HEADS + 1];
+  head_bases(s, c_h, base);
+  if (col_capacity < base[s.H])
+    return fail(RESS_EWORKSPACE, "col_capacity %lld < %lld", (long long)col_capacity, (long long)base[s.H]);
+  if (base[s.H] > INT32_MAX) return fail(RESS_EUNSUPPORTED, "CSR larger than 2^31 entries");
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  const ress::SelectArgs a = select_args(s, nullptr, nullptr, nullptr, nullptr, c_h, ws, L);
+  for (int r = 0; r < rounds; ++r) {
+    cudaError_t ce = ress::launch_round(a, r, rho, st);
+    if (ce != cudaSuccess) return cuda_fail(ce, "ress_restore round");
+  }
+  cudaError_t ce = ress::launch_csr(a, base, row_ptr, col_idx, col_capacity, J_best, drop_mask, st);
+  if (ce != cudaSuccess) return cuda_fail(ce, "ress_restore csr");
+  return ok();
+}
+
+int ress_sparse_attn(const ress_dims* d, const uint16_t* Q, const uint16_t* K, const uint16_t* V,
+                     const int32_t* row_ptr, const int32_t* col_idx, int64_t col_capacity,
+                     uint16_t* O, void* ws, size_t ws_bytes, void* stream) {
+  int e = check_dims(d);
+  if (e) return e;
+  if ((e = check_ptr(Q, 16, "Q")) || (e = check_ptr(K, 16, "K")) || (e = check_ptr(V, 16, "V")) ||
+      (e = check_ptr(O, 16, "O")) || (e = check_ptr(row_ptr, 4, "row_ptr")) ||
+      (e = check_ptr(col_idx, 4, "col_idx")))
+    return e;
+  if (col_capacity < 0) return fail(RESS_EINVAL, "col_capacity %lld < 0", (long long)col_capacity);
+  const ress::Shape s = ress::make_shape(*d);
+  ress_ws_layout L;
+  if ((e = check_ws(s, ws, ws_bytes, &L))) return e;
+  char* w = static_cast<char*>(ws);
+  ress::AttnArgs a;
+  a.s = s;
+  a.Q = Q;
+  a.K = K;
+  a.V = V;
+  a.row_ptr = row_ptr;
+  a.col_idx = col_idx;
+  a.col_capacity = col_capacity;
+  a.O = O;
+  a.status = reinterpret_cast<uint32_t*>(w + L.status);
+  a.counter = reinterpret_cast<uint32_t*>(w + L.counter);
+  a.plist = reinterpret_cast<int32_t*>(w + L.t);  // the gains buffer is free during attention
+  a.plen = reinterpret_cast<int32_t*>(w + L.plen);
+  a.scratch_cap = (int64_t)s.H * s.nb * s.ld;
+  cudaError_t ce = ress::launch_sparse_attn(a, static_cast<cudaStream_t>(stream));
+  if (ce != cudaSuccess) return cuda_fail(ce, "ress_sparse_attn");
+  return ok();
+}
+
+int ress_forward(const ress_dims* d, const uint16_t* Q, const uint16_t* K, const uint16_t* V,
+                 const float* F, const int32_t* c_h, int32_t rounds, float rho, void* ws,
+                 size_t ws_bytes, int32_t* row_ptr, int32_t* col_idx, int64_t col_capacity,
+                 uint16_t* O, float* J_best, void* stream) {
+  // validate everything the three stages need before the first launch
+  int e = check_dims(d);
+  if (e) return e;
+  if ((e = check_ptr(O, 16, "O"))) return e;
+  const ress::Shape s = ress::make_shape(*d);
+  if ((e = check_budgets(s, c_h))) return e;
+  if (rounds < 0 || rounds > 32) return fail(RESS_EINVAL, "rounds %d outside 0..32", rounds);
+  if (!(rho >= 0.0f && rho <= 1.0f)) return fail(RESS_EINVAL, "rho %g outside [0, 1]", (double)rho);
+  if ((e = check_ptr(row_ptr, 4, "row_ptr")) || (e = check_ptr(col_idx, 4, "col_idx"))) return e;
+  if (J_best && (e = check_ptr(J_best, 4, "J_best"))) return e;
+  int64_t base[RESS_MAX_HEADS + 1];
+  head_bases(s, c_h, base);
+  if (col_capacity < base[s.H])
+    return fail(RESS_EWORKSPACE, "col_capacity %lld < %lld", (long long)col_capacity, (long long)base[s.H]);
+  if ((e = ress_score(d, Q, K, V, F, c_h, ws, ws_bytes, stream))) return e;
+  if ((e = ress_restore(d, c_h, rounds, rho, ws, ws_bytes, row_ptr, col_idx, col_capacity, J_best,
+                        nullptr, stream)))
+    return e;
+  return ress_sparse_attn(d, Q, K, V, row_ptr, col_idx, col_capacity, O, ws, ws_bytes, stream);
+}
+
+int ress_status(void* ws, void* stream) {
+  int e = check_ptr(ws, 256, "ws");
+  if (e) return e;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  cudaError_t ce = cudaStreamSynchronize(st);
+  if (ce != cudaSuccess) return cuda_fail(ce, "ress_status sync");
+  uint32_t word = 0;
+  ce = cudaMemcpy(&word, ws, sizeof(word), cudaMemcpyDeviceToHost);
+  if (ce != cudaSuccess) return cuda_fail(ce, "ress_status read");
+  ce = cudaMemset(ws, 0, sizeof(word));
+  if (ce != cudaSuccess) return cuda_fail(ce, "ress_status clear");
+  if (word == 0) return ok();
+  if (word == ress::kStatusTimeout) return fail(RESS_ETIMEOUT, "a bounded device wait gave up");
+  return fail(RESS_EDEVICE, "device-side argument check failed (code %u)", word);
+}
+
+}  // extern "C"

@@ -1,0 +1,125 @@
+// Internal definitions shared by the ReSS CUDA translation units (not part of the ABI).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "../../include/ress.h"
+
+namespace ress {
+
+constexpr int kHeadDim = RESS_HEAD_DIM;  // d_h
+constexpr int kBlock = RESS_BLOCK;       // 64x64 block grid
+constexpr float kEps = 1e-4f;            // Eq. 7
+
+// Device status word values (first error wins; read back by ress_status).
+constexpr uint32_t kStatusTimeout = 1;
+constexpr uint32_t kStatusBadIndex = 2;
+constexpr uint32_t kStatusBadRow = 3;
+
+// Derived sizes of one layer.
+struct Shape {
+  int N, H, nb, ncand, nspecial_blocks, words, ld, d_model;
+};
+
+inline Shape make_shape(const ress_dims& d) {
+  Shape s;
+  s.N = d.n_tokens;
+  s.H = d.n_heads;
+  s.nb = (d.n_tokens + kBlock - 1) / kBlock;
+  s.ncand = (d.n_tokens - d.n_special) / kBlock;
+  s.nspecial_blocks = s.nb - s.ncand;
+  s.words = (s.nb + 31) / 32;
+  s.ld = (s.nb + 31) / 32 * 32;
+  s.d_model = d.d_model;
+  return s;
+}
+
+inline int64_t align256(int64_t x) { return (x + 255) / 256 * 256; }
+
+inline ress_ws_layout make_layout(const Shape& s) {
+  ress_ws_layout L;
+  int64_t off = 0;
+  auto take = [&](int64_t bytes) {
+    int64_t o = off;
+    off = align256(off + bytes);
+    return o;
+  };
+  const int64_t vec = (int64_t)s.H * s.nb * kHeadDim * 4;
+  const int64_t mat = (int64_t)s.H * s.nb * s.ld * 4;
+  const int64_t row = (int64_t)s.H * s.nb * 4;
+  const int64_t msk = (int64_t)s.H * s.nb * s.words * 4;
+  L.status = take(64);
+  L.counter = take(64);
+  L.qbar = take(vec);
+  L.kbar = take(vec);
+  L.vbar = take(vec);
+  L.ztil = take(vec);
+  L.ytil = take(vec);
+  L.gtil = take(vec);
+  L.P = take(mat);
+  L.q = take(mat);
+  L.t = take(mat);
+  L.K = take(row);
+  L.G = take(row);
+  L.J = take(row);
+  L.Jbest = take(row);
+  L.J0 = take(row);
+  L.dmask = take(msk);
+  L.bmask = take(msk);
+  L.plen = take((int64_t)s.H * ((s.nb + 1) / 2) * 4);
+  L.ld = s.ld;
+  L.words = s.words;
+  L.total = off;
+  return L;
+}
+
+// Record the first device-side failure in the workspace status word.
+__device__ __forceinline__ void flag_status(uint32_t* status, uint32_t code) {
+  atomicCAS(status, 0u, code);
+}
+
+__device__ __forceinline__ float bf16_lo(uint32_t v) { return __uint_as_float(v << 16); }
+__device__ __forceinline__ float bf16_hi(uint32_t v) { return __uint_as_float(v & 0xffff0000u); }
+
+// Streaming 16-byte load that bypasses L1 allocation (read-once inputs).
+__device__ __forceinline__ uint4 ld_stream(const uint4* p) {
+  uint4 r;
+  asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0,%1,%2,%3}, [%4];"
+               : "=r"(r.x), "=r"(r.y), "=r"(r.z), "=r"(r.w)
+               : "l"(p));
+  return r;
+}
+
+// Kernel launchers (defined in k_select.cu / k_attn.cu); each returns a cudaError_t.
+struct SelectArgs {
+  Shape s;
+  const uint16_t *Q, *K, *V;
+  const float* F;
+  char* ws;
+  ress_ws_layout L;
+  int c[RESS_MAX_HEADS];
+};
+
+cudaError_t launch_prepare_wo(const Shape& s, const uint16_t* W_o, float* F, cudaStream_t st);
+cudaError_t launch_score(const SelectArgs& a, cudaStream_t st);
+cudaError_t launch_round(const SelectArgs& a, int round, float rho, cudaStream_t st);
+cudaError_t launch_csr(const SelectArgs& a, const int64_t* head_base, int32_t* row_ptr,
+                       int32_t* col_idx, int64_t col_capacity, float* J_best,
+                       uint32_t* drop_mask, cudaStream_t st);
+
+struct AttnArgs {
+  Shape s;
+  const uint16_t *Q, *K, *V;
+  const int32_t *row_ptr, *col_idx;
+  int64_t col_capacity;
+  uint16_t* O;
+  uint32_t* status;
+  uint32_t* counter;
+  int32_t* plist;       // scratch: union lists of query-block pairs (>= scratch_cap entries)
+  int32_t* plen;        // scratch: [H * ceil(nb / 2)] union lengths
+  int64_t scratch_cap;
+};
+cudaError_t launch_sparse_attn(const AttnArgs& a, cudaStream_t st);
+
+}  // namespace ress

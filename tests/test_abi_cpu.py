@@ -1,0 +1,121 @@
+"""The C-ABI library loads, exports every function include/ress.h declares, and validates its
+arguments on the host before any launch (no GPU needed: every call below fails validation
+or only computes sizes)."""
+import ctypes
+
+import numpy as np
+import pytest
+
+import oracle as O
+import synth
+from paper_2609_35593_gb300 import build as _build
+
+_build.build()
+import paper_2609_35593_gb300 as ress  # noqa: E402
+
+EINVAL, EWORKSPACE, EUNSUPPORTED = -1, -2, -3
+
+
+def test_every_declared_function_is_exported():
+    names = ress.exported_names_in_header()
+    assert len(names) >= 12
+    for n in names:
+        assert hasattr(ress._lib, n), n
+    for n in ("ress_score", "ress_restore", "ress_sparse_attn", "ress_forward"):
+        assert n in names
+    assert ress._lib.ress_abi_version() == 1
+
+
+@pytest.mark.parametrize("name", list(synth.WORKLOADS))
+def test_shape_helpers_match_the_oracle(name):
+    wl = synth.WORKLOADS[name]
+    d = ress.dims(wl.n_tokens, wl.heads, wl.n_special, wl.d_model)
+    assert ress.num_blocks(d) == O.n_blocks(wl.n_tokens)
+    assert ress.num_candidates(d) == O.n_candidates(wl.n_tokens, wl.n_special)
+    c = wl.budgets()
+    nb, nc = wl.n_blocks, wl.n_candidates
+    expect = wl.heads * (nc * (int(c[0]) + nb - nc) + (nb - nc) * nb)
+    assert ress.csr_capacity(d, c) == expect
+    L = ress.workspace_layout(d)
+    assert L.total == ress.workspace_bytes(d)
+    offs = sorted(getattr(L, f[0]) for f in ress.WsLayout._fields_[:19])
+    assert all(o % 256 == 0 for o in offs) and len(set(offs)) == len(offs)
+    assert L.ld >= nb and L.ld % 32 == 0 and L.words == -(-nb // 32)
+
+
+def test_csr_capacity_matches_oracle_lists():
+    X = {k: synth.bf16_to_f32(v).astype(np.float64) for k, v in synth.make_random_layer(778, 2, 128, 1).items()}
+    pooled = O.pool(X["Q"], X["K"], X["V"], 10)
+    c = [3, 7]
+    sel = O.ress_select(pooled, X["W_o"], c, 1)
+    rp, ci = O.csr_from_selection(sel, 2, pooled.nb)
+    assert ress.csr_capacity(ress.dims(778, 2, 10, 128), c) == ci.size
+
+
+@pytest.mark.parametrize("field,value,code", [
+    ("head_dim", 128, EUNSUPPORTED), ("block", 128, EUNSUPPORTED), ("n_heads", 0, EUNSUPPORTED),
+    ("n_heads", 33, EUNSUPPORTED), ("n_tokens", 0, EINVAL), ("n_special", -1, EINVAL),
+    ("d_model", 0, EINVAL), ("n_tokens", 64 * 4096 + 1, EUNSUPPORTED)])
+def test_invalid_dims_are_rejected(field, value, code):
+    d = ress.dims(2748, 4, 10, 256)
+    setattr(d, field, value)
+    assert ress._lib.ress_workspace_bytes(ctypes.byref(d)) == 0
+    L = ress.WsLayout()
+    assert ress._lib.ress_workspace_layout(ctypes.byref(d), ctypes.byref(L)) == code
+    assert ress._lib.ress_last_error()
+
+
+def _fake(addr):
+    return ctypes.c_void_p(addr)
+
+
+def test_score_validation_happens_before_launch():
+    d = ress.dims(2748, 4, 10, 256)
+    c = (ctypes.c_int32 * 4)(21, 21, 21, 21)
+    ws_n = ress.workspace_bytes(d)
+    A = 1 << 40  # never dereferenced: every call below fails validation
+    lib = ress._lib
+    args = lambda Q=A, c=c, ws=A, n=ws_n: (ctypes.byref(d), _fake(Q), _fake(A), _fake(A), _fake(A),
+                                           ctypes.cast(c, ctypes.c_void_p), _fake(ws), n, None)
+    assert lib.ress_score(*args(Q=0)) == EINVAL                  # NULL
+    assert lib.ress_score(*args(Q=A + 2)) == EINVAL              # not 16-byte aligned
+    assert lib.ress_score(*args(ws=A + 16)) == EINVAL            # workspace not 256-aligned
+    assert lib.ress_score(*args(n=ws_n - 1)) == EWORKSPACE
+    bad = (ctypes.c_int32 * 4)(21, 0, 21, 21)
+    assert lib.ress_score(*args(c=bad)) == EINVAL                # c_h < 1
+    big = (ctypes.c_int32 * 4)(21, 43, 21, 21)
+    assert lib.ress_score(*args(c=big)) == EINVAL                # c_h > |P| = 42
+    assert b"c_h[1]" in lib.ress_last_error()
+
+
+def test_restore_and_attention_validation():
+    d = ress.dims(2748, 4, 10, 256)
+    c = (ctypes.c_int32 * 4)(21, 21, 21, 21)
+    cp = ctypes.cast(c, ctypes.c_void_p)
+    ws_n = ress.workspace_bytes(d)
+    cap = ress.csr_capacity(d, [21] * 4)
+    A = 1 << 40
+    lib = ress._lib
+    assert lib.ress_restore(ctypes.byref(d), cp, -1, 0.5, _fake(A), ws_n, _fake(A), _fake(A), cap,
+                            None, None, None) == EINVAL
+    assert lib.ress_restore(ctypes.byref(d), cp, 3, 1.5, _fake(A), ws_n, _fake(A), _fake(A), cap,
+                            None, None, None) == EINVAL
+    assert lib.ress_restore(ctypes.byref(d), cp, 3, 0.5, _fake(A), ws_n, _fake(A), _fake(A), cap - 1,
+                            None, None, None) == EWORKSPACE
+    assert lib.ress_restore(ctypes.byref(d), cp, 3, 0.5, _fake(A), ws_n, _fake(A), _fake(A + 2), cap,
+                            None, None, None) == EINVAL
+    assert lib.ress_sparse_attn(ctypes.byref(d), _fake(A), _fake(A), _fake(A), _fake(A), _fake(A), cap,
+                                _fake(0), _fake(A), ws_n, None) == EINVAL
+    assert lib.ress_sparse_attn(ctypes.byref(d), _fake(A), _fake(A), _fake(A), _fake(A), _fake(A), -1,
+                                _fake(A), _fake(A), ws_n, None) == EINVAL
+    assert lib.ress_forward(ctypes.byref(d), _fake(A), _fake(A), _fake(A), _fake(A), cp, 3, 0.5,
+                            _fake(A), ws_n, _fake(A), _fake(A), cap - 1, _fake(A), None, None) == EWORKSPACE
+
+
+def test_binding_refuses_host_tensors():
+    torch = pytest.importorskip("torch")
+    d = ress.dims(2748, 4, 10, 256)
+    x = torch.zeros(2748, 4, 64, dtype=torch.bfloat16)
+    with pytest.raises(ValueError):
+        ress.sparse_attn(d, x, x, x, torch.zeros(3, dtype=torch.int32), torch.zeros(3, dtype=torch.int32),
+                         x, torch.zeros(8, dtype=torch.uint8))

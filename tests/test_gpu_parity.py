@@ -1,0 +1,211 @@
+"""GPU parity of every stage of the hot path against the CPU oracle (needs a GB300)."""
+import numpy as np
+import pytest
+
+import oracle as O
+import synth
+
+pytestmark = pytest.mark.gpu
+
+torch = pytest.importorskip("torch")
+if not torch.cuda.is_available():  # collected on CPU machines only to be deselected
+    pytest.skip("no CUDA device", allow_module_level=True)
+
+import gpu_harness as G  # noqa: E402
+
+
+def layer_for(name, **kw):
+    wl = synth.WORKLOADS[name].with_(**kw) if kw else synth.WORKLOADS[name]
+    return G.Layer(synth.make_inputs(wl), wl.n_special, wl.budgets(), wl.rounds, wl.rho), wl
+
+
+@pytest.fixture(scope="module")
+def tiny():
+    layer, _ = layer_for("tiny_v2")
+    return layer.run()
+
+
+@pytest.fixture(scope="module")
+def v8():
+    layer, _ = layer_for("vggt_v8")
+    return layer.run()
+
+
+def test_prepare_wo_factor(tiny):
+    F = tiny.buf.F.cpu().numpy().astype(np.float64)
+    W = tiny.W_o()
+    for h in range(tiny.H):
+        Wh = O.head_projection(W, h, 64)
+        M = Wh.T @ Wh
+        np.testing.assert_allclose(F[h].T @ F[h], M, rtol=2e-5, atol=2e-6 * np.abs(M).max())
+        assert np.allclose(np.tril(F[h], -1), 0)
+
+
+def test_pooling(tiny):
+    p = tiny.pooled()
+    H, nb = tiny.H, tiny.nb
+    for name, ref in (("qbar", p.Qb), ("kbar", p.Kb), ("vbar", p.Vb)):
+        got = tiny.ws(name, shape=(H, nb, 64))
+        np.testing.assert_allclose(got, ref, rtol=1e-5, atol=1e-6)
+
+
+def test_pooled_map_and_scores(tiny):
+    p = tiny.pooled()
+    L = tiny.buf.layout
+    P = tiny.ws("P", shape=(tiny.H, tiny.nb, L.ld))
+    q = tiny.ws("q", shape=(tiny.H, tiny.nb, L.ld))
+    W = tiny.W_o()
+    for h in range(tiny.H):
+        for i in range(0, tiny.ncand, 5):
+            P_i, vbar = O.row_quantities(p, h, i)
+            np.testing.assert_allclose(P[h, i, :tiny.nb], P_i, rtol=2e-5, atol=1e-9)
+            e, _, _ = O.residual_contributions(P_i, vbar, p.Vb[h], O.head_projection(W, h, 64))
+            Wh = O.head_projection(W, h, 64)
+            q_ref = ((e @ Wh.T) ** 2).sum(1)
+            np.testing.assert_allclose(q[h, i, :tiny.nb], q_ref, rtol=5e-4, atol=1e-6 * q_ref.max())
+
+
+def test_initial_objective(tiny):
+    """J of the initial selection (Eq. 7 then Eq. 12) on rows decided away from any tie."""
+    sel = tiny.oracle_select()
+    J0 = tiny.ws("J0", shape=(tiny.H, tiny.nb))
+    D = tiny.drop_sets()
+    checked = 0
+    for (h, i), s in sel.items():
+        if s.dense or s.near_threshold or not (D[h, i] == s.D_best).all():
+            continue
+        assert J0[h, i] == pytest.approx(s.J0, rel=G.DRIFT_REL)
+        checked += 1
+    assert checked > 0
+
+
+@pytest.mark.parametrize("fixture", ["tiny", "v8"])
+def test_drop_sets_and_drift(fixture, request):
+    layer = request.getfixturevalue(fixture)
+    sel = layer.oracle_select()
+    r = G.compare_selection(layer, sel)
+    print(fixture, r)
+    assert r["mismatched"] == 0, r
+    assert r["exact"] >= 0.95 * (r["exact"] + r["near"])
+    assert r["worst_row_rel"] <= G.DRIFT_REL
+    assert r["sum_rel_gpu_vs_ref"] <= G.DRIFT_REL
+    assert r["sum_rel_gpu_vs_oracle"] <= G.DRIFT_REL
+
+
+@pytest.mark.parametrize("fixture", ["tiny", "v8"])
+def test_csr_structure(fixture, request):
+    layer = request.getfixturevalue(fixture)
+    rp, ci = layer.csr()
+    nb, nc = layer.nb, layer.ncand
+    D = layer.drop_sets()
+    assert rp[0] == 0 and rp[-1] == ci.size
+    for h in range(layer.H):
+        for i in range(nb):
+            k = ci[rp[h * nb + i]:rp[h * nb + i + 1]]
+            assert np.all(np.diff(k) > 0)
+            if i >= nc:
+                assert k.tolist() == list(range(nb))
+            else:
+                assert k.size == layer.c_h[h] + nb - nc
+                assert np.array_equal(k, np.nonzero(~D[h, i])[0])
+
+
+@pytest.mark.parametrize("fixture", ["tiny", "v8"])
+def test_attention(fixture, request):
+    layer = request.getfixturevalue(fixture)
+    rng = np.random.default_rng(0)
+    rows = [(h, i) for h in range(layer.H) for i in range(layer.nb)]
+    if len(rows) > 400:
+        idx = rng.choice(len(rows), 400, replace=False)
+        rows = [rows[k] for k in sorted(idx)] + [(0, layer.nb - 1), (layer.H - 1, layer.nb - 2)]
+    r = G.compare_attention(layer, rows)
+    print(fixture, r)
+    assert r["max_abs"] <= G.ATT_MAX_ABS and r["mean_rel"] <= G.ATT_MEAN_REL, r
+
+
+def test_forward_equals_staged_calls(tiny):
+    layer, _ = layer_for("tiny_v2")
+    layer.run_forward()
+    assert np.array_equal(layer.csr()[1], tiny.csr()[1])
+    assert np.array_equal(layer.output(), tiny.output())
+    assert np.array_equal(layer.buf.J_best.cpu().numpy(), tiny.buf.J_best.cpu().numpy())
+
+
+def test_deterministic_bits():
+    a, _ = layer_for("tiny_v2")
+    b, _ = layer_for("tiny_v2")
+    a.run()
+    b.run()
+    assert np.array_equal(a.csr()[1], b.csr()[1])
+    assert torch.equal(a.buf.O.view(torch.int16), b.buf.O.view(torch.int16))
+    assert torch.equal(a.buf.J_best, b.buf.J_best)
+
+
+@pytest.mark.parametrize("N,H,ns,c,R", [
+    (65, 1, 0, 1, 2),          # two blocks, one candidate, ragged tail
+    (64 * 7, 1, 0, 3, 3),      # no special tokens, no ragged tail, odd block count
+    (64 * 10 + 17, 3, 5, 4, 2),  # three heads, ragged tail with special tokens
+    (1000, 2, 40, 1, 1),       # budget of one block
+    (1300, 2, 7, 20, 3),       # c_h = |P|: nothing dropped (0% sparsity)
+])
+def test_edge_shapes(N, H, ns, c, R):
+    inp = synth.make_random_layer(N, H, 64 * H, seed=N + H)
+    nc = O.n_candidates(N, ns)
+    c = min(c, nc)
+    layer = G.Layer(inp, ns, [c] * H, R).run()
+    sel = layer.oracle_select()
+    r = G.compare_selection(layer, sel)
+    assert r["mismatched"] == 0, r
+    rows = [(h, i) for h in range(H) for i in range(layer.nb)]
+    a = G.compare_attention(layer, rows)
+    assert a["max_abs"] <= G.ATT_MAX_ABS and a["mean_rel"] <= G.ATT_MEAN_REL, a
+
+
+def test_dense_csr_is_dense_attention(tiny):
+    """A CSR that keeps every block gives dense attention (same kernel, no dropped tiles)."""
+    H, nb = tiny.H, tiny.nb
+    rp = torch.arange(0, H * nb * nb + 1, nb, dtype=torch.int32, device="cuda")
+    ci = torch.arange(nb, dtype=torch.int32, device="cuda").repeat(H * nb)
+    O_ = torch.empty_like(tiny.buf.O)
+    tiny.ress.sparse_attn(tiny.d, tiny.Q, tiny.K, tiny.V, rp, ci, O_, tiny.buf.ws)
+    tiny.ress.status(tiny.buf.ws)
+    q, k, v = (t.float().permute(1, 0, 2) for t in (tiny.Q, tiny.K, tiny.V))
+    ref = torch.nn.functional.scaled_dot_product_attention(q, k, v).permute(1, 0, 2)
+    diff = (O_.float() - ref).abs()
+    assert diff.max().item() <= G.ATT_MAX_ABS
+    assert diff.sum().item() / ref.abs().sum().item() <= G.ATT_MEAN_REL
+
+
+def test_bad_csr_index_is_reported_not_faulted(tiny):
+    import paper_2609_35593_gb300 as ress
+    rp = tiny.buf.row_ptr.clone()
+    ci = tiny.buf.col_idx.clone()
+    ci[5] = tiny.nb + 100
+    O_ = torch.empty_like(tiny.buf.O)
+    ress.sparse_attn(tiny.d, tiny.Q, tiny.K, tiny.V, rp, ci, O_, tiny.buf.ws)
+    with pytest.raises(ress.RessError) as e:
+        ress.status(tiny.buf.ws)
+    assert e.value.code == -6
+    ress.status(tiny.buf.ws)  # cleared
+
+
+def test_headline_shape_sampled():
+    """32 views, 16 heads, 90% sparsity, R = 3: sampled rows against the oracle, and
+    properties that hold at any size on every row."""
+    layer, wl = layer_for("vggt_v32")
+    layer.run()
+    rng = np.random.default_rng(1)
+    rows = [(int(h), int(i)) for h, i in zip(rng.integers(0, wl.heads, 24), rng.integers(0, wl.n_candidates, 24))]
+    sel = layer.oracle_select(rows)
+    r = G.compare_selection(layer, sel)
+    print(r)
+    assert r["mismatched"] == 0, r
+    J0 = layer.ws("J0", shape=(layer.H, layer.nb))
+    Jb = layer.buf.J_best.cpu().numpy().reshape(layer.H, layer.nb)
+    assert np.all(Jb[:, :layer.ncand] <= J0[:, :layer.ncand])
+    rp, ci = layer.csr()
+    assert rp[-1] == ci.size
+    arows = rows[:8] + [(0, layer.nb - 1), (5, layer.nb - 2)]
+    a = G.compare_attention(layer, arows)
+    print(a)
+    assert a["max_abs"] <= G.ATT_MAX_ABS and a["mean_rel"] <= G.ATT_MEAN_REL, a
