@@ -8,9 +8,9 @@ import pytest
 
 import oracle as O
 import synth
-from paper_2609_35593_gb300 import build as _build
+import __graft_entry__
 
-_build.build()
+__graft_entry__._build_module().build()
 import paper_2609_35593_gb300 as ress  # noqa: E402
 
 EINVAL, EWORKSPACE, EUNSUPPORTED = -1, -2, -3
