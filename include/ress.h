@@ -144,6 +144,14 @@ int ress_sparse_attn(const ress_dims* dims, const uint16_t* Q, const uint16_t* K
                      int64_t col_capacity, uint16_t* O, void* ws, size_t ws_bytes,
                      void* stream);
 
+/* ress_sparse_attn with a float32 output O [N, H, 64] (16-byte aligned): the same kernel
+ * and the same arithmetic; the bf16 output of ress_sparse_attn is this result rounded to
+ * nearest-even.  For callers that keep the attention output in float32 and for checking
+ * the kernel against a float32 reference without the bf16 output rounding. */
+int ress_sparse_attn_f32(const ress_dims* dims, const uint16_t* Q, const uint16_t* K,
+                         const uint16_t* V, const int32_t* row_ptr, const int32_t* col_idx,
+                         int64_t col_capacity, float* O, void* ws, size_t ws_bytes, void* stream);
+
 /* ress_score, ress_restore and ress_sparse_attn in order on one stream. */
 int ress_forward(const ress_dims* dims, const uint16_t* Q, const uint16_t* K, const uint16_t* V,
                  const float* F, const int32_t* c_h_host, int32_t rounds, float rho, void* ws,

@@ -65,6 +65,8 @@ _SIGS = {
                                 _P, _P, _c.c_int64, _P, _P, _P]),
     "ress_sparse_attn": (_c.c_int, [_c.POINTER(Dims), _P, _P, _P, _P, _P, _c.c_int64, _P, _P,
                                     _c.c_size_t, _P]),
+    "ress_sparse_attn_f32": (_c.c_int, [_c.POINTER(Dims), _P, _P, _P, _P, _P, _c.c_int64, _P, _P,
+                                        _c.c_size_t, _P]),
     "ress_forward": (_c.c_int, [_c.POINTER(Dims), _P, _P, _P, _P, _P, _c.c_int32, _c.c_float, _P,
                                 _c.c_size_t, _P, _P, _c.c_int64, _P, _P, _P]),
     "ress_status": (_c.c_int, [_P, _P]),
@@ -189,6 +191,16 @@ def sparse_attn(d: Dims, Q, K, V, row_ptr, col_idx, O, ws, stream=None):
                                  _dev(col_idx, (torch.int32,), "col_idx"), col_idx.numel(),
                                  _dev(O, _bf16(), "O"), _dev(ws, None, "ws"),
                                  ws.numel() * ws.element_size(), _stream(stream)))
+
+
+def sparse_attn_f32(d: Dims, Q, K, V, row_ptr, col_idx, O, ws, stream=None):
+    """ress_sparse_attn with a float32 output tensor O [N, H, 64]."""
+    torch = _torch()
+    _check(_lib.ress_sparse_attn_f32(_c.byref(d), _dev(Q, _bf16(), "Q"), _dev(K, _bf16(), "K"),
+                                     _dev(V, _bf16(), "V"), _dev(row_ptr, (torch.int32,), "row_ptr"),
+                                     _dev(col_idx, (torch.int32,), "col_idx"), col_idx.numel(),
+                                     _dev(O, (torch.float32,), "O"), _dev(ws, None, "ws"),
+                                     ws.numel() * ws.element_size(), _stream(stream)))
 
 
 def forward(d: Dims, Q, K, V, F, c_h, rounds: int, rho: float, ws, row_ptr, col_idx, O,

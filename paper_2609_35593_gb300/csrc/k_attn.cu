@@ -53,7 +53,7 @@ struct __align__(1024) AttnSmem {
   uint64_t kv_full[kStages], kv_empty[kStages];
   uint64_t q_full, q_empty;
   uint64_t s_full[2], p_full[2], p_empty[2];
-  uint64_t o_bar, drain;
+  uint64_t o_bar[2], drain;  // o_bar[k & 1] completes when P_k V_k has landed
   TileInfo info[kStages];
   uint32_t tmem_base;
   int abort;
@@ -64,7 +64,7 @@ struct AttnParams {
   const int32_t* row_ptr;
   const int32_t* plist;  // union lists: entry = j | mask << 16, at row_ptr[h*nb + 2p]
   const int32_t* plen;   // [H * npairs]
-  uint16_t* O;
+  void* O;               // bf16 or float32 [N, H, 64]
   uint32_t* status;
   uint32_t* counter;
 };
@@ -142,6 +142,7 @@ __global__ void __launch_bounds__(256) k_pairs(const int32_t* __restrict__ row_p
 // ------------------------------------------------------------------------------------
 // main kernel
 // ------------------------------------------------------------------------------------
+template <bool kOutF32>
 __global__ void __launch_bounds__(kAttnThreads, 2)
     k_attn(const __grid_constant__ CUtensorMap tmQ, const __grid_constant__ CUtensorMap tmK,
            const __grid_constant__ CUtensorMap tmV, const AttnParams a) {
@@ -163,7 +164,8 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
       mbar_init(&S.p_full[b], 4);
       mbar_init(&S.p_empty[b], 1);
     }
-    mbar_init(&S.o_bar, 1);
+    mbar_init(&S.o_bar[0], 1);
+    mbar_init(&S.o_bar[1], 1);
     mbar_init(&S.drain, 1);
     S.abort = 0;
     fence_barrier_init();
@@ -267,7 +269,7 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
                       idesc_pv, (k > 0 || !first) ? 1u : 0u);
         mma_commit(&S.kv_empty[ps]);
         mma_commit(&S.p_empty[pb]);
-        mma_commit(&S.o_bar);
+        mma_commit(&S.o_bar[pg & 1]);
         return true;
       };
       for (;;) {
@@ -382,7 +384,7 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
         }
         if (__any_sync(0xffffffffu, rescale)) {
           // the previous P V must have landed before the accumulator row is rescaled
-          if (!mbar_wait(&S.o_bar, (g - 1) & 1, abort, kWaitNs)) {
+          if (!mbar_wait(&S.o_bar[(g - 1) & 1], ((g - 1) >> 1) & 1, abort, kWaitNs)) {
             give_up(S, a.status);
             break;
           }
@@ -422,7 +424,7 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
 
       if (info.flags & kLast) {
         // epilogue: O / l for this row once the last P V has landed
-        if (!mbar_wait(&S.o_bar, g & 1, abort, kWaitNs)) {
+        if (!mbar_wait(&S.o_bar[g & 1], (g >> 1) & 1, abort, kWaitNs)) {
           give_up(S, a.status);
           break;
         }
@@ -437,17 +439,30 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
         if (row_exists) {
           if (!(l > 0.f)) flag_status(a.status, kStatusBadRow);
           const float inv = l > 0.f ? 1.0f / l : 0.f;
-          uint4* dst = reinterpret_cast<uint4*>(a.O + ((int64_t)token * a.H + h) * 64);
+          const int64_t off = ((int64_t)token * a.H + h) * 64;
+          if (kOutF32) {
+            float4* dst = reinterpret_cast<float4*>(static_cast<float*>(a.O) + off);
 #pragma unroll
-          for (int ch = 0; ch < 8; ++ch) {
-            uint32_t w[4];
-#pragma unroll
-            for (int e = 0; e < 4; ++e) {
-              const int c = ch * 8 + 2 * e;
-              w[e] = pack_bf16x2(__uint_as_float(o[c >> 5][c & 31]) * inv,
-                                 __uint_as_float(o[(c + 1) >> 5][(c + 1) & 31]) * inv);
+            for (int ch = 0; ch < 16; ++ch) {
+              const int c = ch * 4;
+              dst[ch] = make_float4(__uint_as_float(o[c >> 5][c & 31]) * inv,
+                                    __uint_as_float(o[(c + 1) >> 5][(c + 1) & 31]) * inv,
+                                    __uint_as_float(o[(c + 2) >> 5][(c + 2) & 31]) * inv,
+                                    __uint_as_float(o[(c + 3) >> 5][(c + 3) & 31]) * inv);
             }
-            dst[ch] = make_uint4(w[0], w[1], w[2], w[3]);
+          } else {
+            uint4* dst = reinterpret_cast<uint4*>(static_cast<uint16_t*>(a.O) + off);
+#pragma unroll
+            for (int ch = 0; ch < 8; ++ch) {
+              uint32_t w[4];
+#pragma unroll
+              for (int e = 0; e < 4; ++e) {
+                const int c = ch * 8 + 2 * e;
+                w[e] = pack_bf16x2(__uint_as_float(o[c >> 5][c & 31]) * inv,
+                                   __uint_as_float(o[(c + 1) >> 5][(c + 1) & 31]) * inv);
+              }
+              dst[ch] = make_uint4(w[0], w[1], w[2], w[3]);
+            }
           }
         }
         tc_fence_before();
@@ -528,10 +543,11 @@ cudaError_t launch_sparse_attn(const AttnArgs& x, cudaStream_t st) {
   p.status = x.status;
   p.counter = x.counter;
   const size_t smem = sizeof(AttnSmem) + 1024;
-  e = cudaFuncSetAttribute(k_attn, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  auto kern = x.out_f32 ? k_attn<true> : k_attn<false>;
+  e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   const int grid = min(pairs, 2 * sm_count());
-  k_attn<<<grid, kAttnThreads, smem, st>>>(tq, tk, tv, p);
+  kern<<<grid, kAttnThreads, smem, st>>>(tq, tk, tv, p);
   return cudaGetLastError();
 }
 

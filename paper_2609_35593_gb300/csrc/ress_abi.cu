@@ -194,9 +194,10 @@ int ress_restore(const ress_dims* d, const int32_t* c_h, int32_t rounds, float r
   return ok();
 }
 
-int ress_sparse_attn(const ress_dims* d, const uint16_t* Q, const uint16_t* K, const uint16_t* V,
-                     const int32_t* row_ptr, const int32_t* col_idx, int64_t col_capacity,
-                     uint16_t* O, void* ws, size_t ws_bytes, void* stream) {
+static int sparse_attn_impl(const ress_dims* d, const uint16_t* Q, const uint16_t* K,
+                            const uint16_t* V, const int32_t* row_ptr, const int32_t* col_idx,
+                            int64_t col_capacity, void* O, bool out_f32, void* ws, size_t ws_bytes,
+                            void* stream) {
   int e = check_dims(d);
   if (e) return e;
   if ((e = check_ptr(Q, 16, "Q")) || (e = check_ptr(K, 16, "K")) || (e = check_ptr(V, 16, "V")) ||
@@ -217,6 +218,7 @@ int ress_sparse_attn(const ress_dims* d, const uint16_t* Q, const uint16_t* K, c
   a.col_idx = col_idx;
   a.col_capacity = col_capacity;
   a.O = O;
+  a.out_f32 = out_f32;
   a.status = reinterpret_cast<uint32_t*>(w + L.status);
   a.counter = reinterpret_cast<uint32_t*>(w + L.counter);
   a.plist = reinterpret_cast<int32_t*>(w + L.t);  // the gains buffer is free during attention
@@ -225,6 +227,18 @@ int ress_sparse_attn(const ress_dims* d, const uint16_t* Q, const uint16_t* K, c
   cudaError_t ce = ress::launch_sparse_attn(a, static_cast<cudaStream_t>(stream));
   if (ce != cudaSuccess) return cuda_fail(ce, "ress_sparse_attn");
   return ok();
+}
+
+int ress_sparse_attn(const ress_dims* d, const uint16_t* Q, const uint16_t* K, const uint16_t* V,
+                     const int32_t* row_ptr, const int32_t* col_idx, int64_t col_capacity,
+                     uint16_t* O, void* ws, size_t ws_bytes, void* stream) {
+  return sparse_attn_impl(d, Q, K, V, row_ptr, col_idx, col_capacity, O, false, ws, ws_bytes, stream);
+}
+
+int ress_sparse_attn_f32(const ress_dims* d, const uint16_t* Q, const uint16_t* K,
+                         const uint16_t* V, const int32_t* row_ptr, const int32_t* col_idx,
+                         int64_t col_capacity, float* O, void* ws, size_t ws_bytes, void* stream) {
+  return sparse_attn_impl(d, Q, K, V, row_ptr, col_idx, col_capacity, O, true, ws, ws_bytes, stream);
 }
 
 int ress_forward(const ress_dims* d, const uint16_t* Q, const uint16_t* K, const uint16_t* V,

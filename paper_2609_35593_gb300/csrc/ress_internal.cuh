@@ -113,7 +113,8 @@ struct AttnArgs {
   const uint16_t *Q, *K, *V;
   const int32_t *row_ptr, *col_idx;
   int64_t col_capacity;
-  uint16_t* O;
+  void* O;              // bf16, or float32 when out_f32
+  bool out_f32;
   uint32_t* status;
   uint32_t* counter;
   int32_t* plist;       // scratch: union lists of query-block pairs (>= scratch_cap entries)

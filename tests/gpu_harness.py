@@ -3,7 +3,10 @@
 Tolerances (from the task's acceptance rules, written here once):
   * drop sets: identical on every row whose oracle decision margin is >= 1e-3 (relative);
   * attention: max |O_gpu - O_ref| <= 2e-2 and sum|O_gpu - O_ref| / sum|O_ref| <= 5e-3,
-    O_ref = oracle attention (float64) over the GPU's kept lists;
+    O_ref = oracle attention (float64) over the GPU's kept lists and O_gpu the kernel's
+    float32 result (ress_sparse_attn_f32); the bf16 output of ress_sparse_attn must be
+    exactly that result rounded to nearest-even (bf16 storage alone can be 3e-2 off for
+    |O| in [8, 16), so the bound applies before the storage rounding);
   * realised drift: |J_gpu - J_ref| <= 1e-3 J_ref per row and for the sum.
 """
 from __future__ import annotations
@@ -46,6 +49,7 @@ class Layer:
         self.V = bits_to_device(inputs["V"])
         self.W = bits_to_device(inputs["W_o"])
         self.buf = ress.Buffers(self.d, self.c_h)
+        self.O32 = torch.zeros(self.N, self.H, 64, dtype=torch.float32, device="cuda")
         self.nb = self.buf.nb
         self.ncand = ress.num_candidates(self.d)
 
@@ -57,6 +61,7 @@ class Layer:
         r.restore(self.d, self.c_h, self.rounds, self.rho, b.ws, b.row_ptr, b.col_idx, b.J_best)
         if attention:
             r.sparse_attn(self.d, self.Q, self.K, self.V, b.row_ptr, b.col_idx, b.O, b.ws)
+            r.sparse_attn_f32(self.d, self.Q, self.K, self.V, b.row_ptr, b.col_idx, self.O32, b.ws)
         r.status(b.ws)
         torch.cuda.synchronize()
         return self
@@ -66,6 +71,7 @@ class Layer:
         r.prepare_wo(self.d, self.W, b.F)
         r.forward(self.d, self.Q, self.K, self.V, b.F, self.c_h, self.rounds, self.rho, b.ws,
                   b.row_ptr, b.col_idx, b.O, b.J_best)
+        r.sparse_attn_f32(self.d, self.Q, self.K, self.V, b.row_ptr, b.col_idx, self.O32, b.ws)
         r.status(b.ws)
         torch.cuda.synchronize()
         return self
@@ -89,6 +95,10 @@ class Layer:
                 for h in range(self.H) for i in range(self.nb)}
 
     def output(self) -> np.ndarray:
+        """The kernel's float32 attention output."""
+        return self.O32.cpu().numpy()
+
+    def output_bf16(self) -> np.ndarray:
         return self.buf.O.float().cpu().numpy()
 
     # ---- oracle --------------------------------------------------------------------

@@ -123,10 +123,17 @@ def test_attention(fixture, request):
     assert r["max_abs"] <= G.ATT_MAX_ABS and r["mean_rel"] <= G.ATT_MEAN_REL, r
 
 
+@pytest.mark.parametrize("fixture", ["tiny", "v8"])
+def test_bf16_output_is_rounded_f32_output(fixture, request):
+    layer = request.getfixturevalue(fixture)
+    assert torch.equal(layer.O32.to(torch.bfloat16).view(torch.int16), layer.buf.O.view(torch.int16))
+
+
 def test_forward_equals_staged_calls(tiny):
     layer, _ = layer_for("tiny_v2")
     layer.run_forward()
     assert np.array_equal(layer.csr()[1], tiny.csr()[1])
+    assert np.array_equal(layer.output_bf16(), tiny.output_bf16())
     assert np.array_equal(layer.output(), tiny.output())
     assert np.array_equal(layer.buf.J_best.cpu().numpy(), tiny.buf.J_best.cpu().numpy())
 
@@ -166,8 +173,8 @@ def test_dense_csr_is_dense_attention(tiny):
     H, nb = tiny.H, tiny.nb
     rp = torch.arange(0, H * nb * nb + 1, nb, dtype=torch.int32, device="cuda")
     ci = torch.arange(nb, dtype=torch.int32, device="cuda").repeat(H * nb)
-    O_ = torch.empty_like(tiny.buf.O)
-    tiny.ress.sparse_attn(tiny.d, tiny.Q, tiny.K, tiny.V, rp, ci, O_, tiny.buf.ws)
+    O_ = torch.empty_like(tiny.O32)
+    tiny.ress.sparse_attn_f32(tiny.d, tiny.Q, tiny.K, tiny.V, rp, ci, O_, tiny.buf.ws)
     tiny.ress.status(tiny.buf.ws)
     q, k, v = (t.float().permute(1, 0, 2) for t in (tiny.Q, tiny.K, tiny.V))
     ref = torch.nn.functional.scaled_dot_product_attention(q, k, v).permute(1, 0, 2)
