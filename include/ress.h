@@ -158,6 +158,32 @@ int ress_forward(const ress_dims* dims, const uint16_t* Q, const uint16_t* K, co
                  size_t ws_bytes, int32_t* row_ptr, int32_t* col_idx, int64_t col_capacity,
                  uint16_t* O, float* J_best, void* stream);
 
+/* Allocation-free variant of ress_sparse_attn (the paper has no counterpart: this is an
+ * interface for callers, not part of the method).  It is for callers that cannot allocate
+ * device memory when they call in: a host framework that owns all device memory through
+ * its own pool and forbids allocations inside plugins, a real-time runtime that reserves
+ * everything at start-up because a later cudaMalloc can stall the device or fail under a
+ * tight budget, or a caller that cannot spare the full workspace for the attention step.
+ * Same arguments and results as ress_sparse_attn (bf16 O), without `ws`: the scratch is a
+ * file-scope device array of RESS_NOALLOC_SCRATCH_BYTES (4 MiB) that every GPU loading the
+ * library holds until the process exits.  No cudaMalloc, cudaFree or allocating routine is
+ * called.
+ *   - Limit: col_capacity must not exceed (4 MiB - 256 - 4*H*ceil(nb/2) rounded up to 256) / 4
+ *     entries (about one million: enough for 16 heads x 32 views at 90% sparsity);
+ *     larger requests return RESS_EWORKSPACE with the limit in the message.
+ *   - Set-up: the first call on each device looks up the array's device address (with that
+ *     device current) and caches it; make that first call before any stream capture.
+ *   - Every call shares the one array, and it keeps the last call's contents: calls that
+ *     may overlap on the GPU (other streams, other host threads) race and must be ordered
+ *     by the caller.  The tile counter is cleared by each call.
+ *   - wait != 0: the call synchronises `stream` and returns RESS_ETIMEOUT / RESS_EDEVICE
+ *     for device-side failures (then clears them).  wait == 0: asynchronous; a device-side
+ *     failure stays recorded until a later call with wait != 0 reports it. */
+#define RESS_NOALLOC_SCRATCH_BYTES (4u << 20)
+int ress_sparse_attn_noalloc(const ress_dims* dims, const uint16_t* Q, const uint16_t* K,
+                             const uint16_t* V, const int32_t* row_ptr, const int32_t* col_idx,
+                             int64_t col_capacity, uint16_t* O, int32_t wait, void* stream);
+
 /* Synchronises `stream`, returns the workspace status word as a ress_status_code
  * (RESS_OK, RESS_ETIMEOUT or RESS_EDEVICE) and clears it. */
 int ress_status(void* ws, void* stream);

@@ -70,6 +70,8 @@ _SIGS = {
     "ress_forward": (_c.c_int, [_c.POINTER(Dims), _P, _P, _P, _P, _P, _c.c_int32, _c.c_float, _P,
                                 _c.c_size_t, _P, _P, _c.c_int64, _P, _P, _P]),
     "ress_status": (_c.c_int, [_P, _P]),
+    "ress_sparse_attn_noalloc": (_c.c_int, [_c.POINTER(Dims), _P, _P, _P, _P, _P, _c.c_int64, _P,
+                                            _c.c_int32, _P]),
 }
 for _name, (_res, _args) in _SIGS.items():
     _f = getattr(_lib, _name)
@@ -214,6 +216,16 @@ def forward(d: Dims, Q, K, V, F, c_h, rounds: int, rho: float, ws, row_ptr, col_
                              _dev(col_idx, (torch.int32,), "col_idx"), col_idx.numel(),
                              _dev(O, _bf16(), "O"), _dev(J_best, (torch.float32,), "J_best"),
                              _stream(stream)))
+
+
+def sparse_attn_noalloc(d: Dims, Q, K, V, row_ptr, col_idx, O, wait: bool = True, stream=None):
+    """ress_sparse_attn without a workspace: scratch is the library's built-in device array
+    (see include/ress.h for its size limit and the sharing rules)."""
+    torch = _torch()
+    _check(_lib.ress_sparse_attn_noalloc(_c.byref(d), _dev(Q, _bf16(), "Q"), _dev(K, _bf16(), "K"),
+                                         _dev(V, _bf16(), "V"), _dev(row_ptr, (torch.int32,), "row_ptr"),
+                                         _dev(col_idx, (torch.int32,), "col_idx"), col_idx.numel(),
+                                         _dev(O, _bf16(), "O"), 1 if wait else 0, _stream(stream)))
 
 
 def status(ws, stream=None):

@@ -283,3 +283,106 @@ int ress_status(void* ws, void* stream) {
 }
 
 }  // extern "C"
+
+// ---------------------------------------------------------------------------------------
+// Allocation-free attention entry point.
+//
+// Some callers cannot allocate device memory when they call into this library: a host
+// framework that owns every byte of device memory through its own pool and forbids
+// allocations inside plugins, a real-time runtime that reserves all memory at start-up
+// because a later cudaMalloc can stall the device and may fail under a tight budget, or a
+// caller that cannot spare the full ress workspace just for the attention step.  For them
+// this entry point keeps its scratch (status word, tile counter, pair lengths and pair
+// lists) in a file-scope __device__ array of RESS_NOALLOC_SCRATCH_BYTES that every GPU
+// loading the library holds until the process exits.  The caller still passes Q, K, V, the
+// CSR and O.
+// ---------------------------------------------------------------------------------------
+#include <mutex>
+
+namespace {
+
+static __device__ __align__(256) unsigned char g_noalloc_scratch[RESS_NOALLOC_SCRATCH_BYTES];
+
+constexpr int kNoallocMaxDevices = 64;
+constexpr int64_t kNoallocStatus = 0;    // uint32 status word
+constexpr int64_t kNoallocCounter = 64;  // uint32 tile counter (zeroed by every launch)
+constexpr int64_t kNoallocPlen = 256;    // int32 pair lengths, then the pair lists
+
+std::mutex g_noalloc_mu;
+void* g_noalloc_ptr[kNoallocMaxDevices] = {};
+
+// Device address of the scratch array on the current device.  In host code the array's
+// name is only a host-side stand-in, so the address is looked up once per device (with
+// that device current) and cached.
+int noalloc_scratch(void** out) {
+  int dev = 0;
+  cudaError_t ce = cudaGetDevice(&dev);
+  if (ce != cudaSuccess) return cuda_fail(ce, "ress_sparse_attn_noalloc: cudaGetDevice");
+  if (dev < 0 || dev >= kNoallocMaxDevices)
+    return fail(RESS_EUNSUPPORTED, "device ordinal %d beyond %d", dev, kNoallocMaxDevices);
+  std::lock_guard<std::mutex> lock(g_noalloc_mu);
+  if (!g_noalloc_ptr[dev]) {
+    void* p = nullptr;
+    ce = cudaGetSymbolAddress(&p, g_noalloc_scratch);
+    if (ce != cudaSuccess || !p) return cuda_fail(ce, "ress_sparse_attn_noalloc: cudaGetSymbolAddress");
+    g_noalloc_ptr[dev] = p;
+  }
+  *out = g_noalloc_ptr[dev];
+  return RESS_OK;
+}
+
+}  // namespace
+
+extern "C" int ress_sparse_attn_noalloc(const ress_dims* d, const uint16_t* Q, const uint16_t* K,
+                                        const uint16_t* V, const int32_t* row_ptr,
+                                        const int32_t* col_idx, int64_t col_capacity, uint16_t* O,
+                                        int32_t wait, void* stream) {
+  int e = check_dims(d);
+  if (e) return e;
+  if ((e = check_ptr(Q, 16, "Q")) || (e = check_ptr(K, 16, "K")) || (e = check_ptr(V, 16, "V")) ||
+      (e = check_ptr(O, 16, "O")) || (e = check_ptr(row_ptr, 4, "row_ptr")) ||
+      (e = check_ptr(col_idx, 4, "col_idx")))
+    return e;
+  if (col_capacity < 0) return fail(RESS_EINVAL, "col_capacity %lld < 0", (long long)col_capacity);
+  const ress::Shape s = ress::make_shape(*d);
+  const int64_t plen_bytes = ress::align256((int64_t)s.H * ((s.nb + 1) / 2) * 4);
+  const int64_t list_entries = ((int64_t)RESS_NOALLOC_SCRATCH_BYTES - kNoallocPlen - plen_bytes) / 4;
+  if (col_capacity > list_entries)
+    return fail(RESS_EWORKSPACE,
+                "col_capacity %lld exceeds the %lld CSR entries that the built-in %u-byte scratch "
+                "holds for %d heads x %d blocks; use ress_sparse_attn with a workspace",
+                (long long)col_capacity, (long long)list_entries, (unsigned)RESS_NOALLOC_SCRATCH_BYTES,
+                s.H, s.nb);
+  void* base = nullptr;
+  if ((e = noalloc_scratch(&base))) return e;
+  char* w = static_cast<char*>(base);
+  ress::AttnArgs a;
+  a.s = s;
+  a.Q = Q;
+  a.K = K;
+  a.V = V;
+  a.row_ptr = row_ptr;
+  a.col_idx = col_idx;
+  a.col_capacity = col_capacity;
+  a.O = O;
+  a.out_f32 = false;
+  a.status = reinterpret_cast<uint32_t*>(w + kNoallocStatus);
+  a.counter = reinterpret_cast<uint32_t*>(w + kNoallocCounter);
+  a.plen = reinterpret_cast<int32_t*>(w + kNoallocPlen);
+  a.plist = reinterpret_cast<int32_t*>(w + kNoallocPlen + plen_bytes);
+  a.scratch_cap = list_entries;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  cudaError_t ce = ress::launch_sparse_attn(a, st);
+  if (ce != cudaSuccess) return cuda_fail(ce, "ress_sparse_attn_noalloc");
+  if (!wait) return ok();
+  ce = cudaStreamSynchronize(st);
+  if (ce != cudaSuccess) return cuda_fail(ce, "ress_sparse_attn_noalloc sync");
+  uint32_t word = 0;
+  ce = cudaMemcpy(&word, a.status, sizeof(word), cudaMemcpyDeviceToHost);
+  if (ce != cudaSuccess) return cuda_fail(ce, "ress_sparse_attn_noalloc status read");
+  if (word == 0) return ok();
+  ce = cudaMemset(a.status, 0, sizeof(word));
+  if (ce != cudaSuccess) return cuda_fail(ce, "ress_sparse_attn_noalloc status clear");
+  if (word == ress::kStatusTimeout) return fail(RESS_ETIMEOUT, "a bounded device wait gave up");
+  return fail(RESS_EDEVICE, "device-side argument check failed (code %u)", word);
+}
