@@ -61,6 +61,7 @@ struct __align__(1024) AttnSmem {
 
 struct AttnParams {
   int N, H, nb, npairs, nitems;
+  int nsparse;           // pairs 0..nsparse-1 of a head hold only candidate query blocks
   const int32_t* row_ptr;
   const int32_t* plist;  // union lists: entry = j | mask << 16, at row_ptr[h*nb + 2p]
   const int32_t* plen;   // [H * npairs]
@@ -68,6 +69,27 @@ struct AttnParams {
   uint32_t* status;
   uint32_t* counter;
 };
+
+// Work order: the pairs that hold special (dense) query blocks of every head first (they
+// are the longest), then the remaining pairs head by head, so that the CTAs running at the
+// same time share one head's K and V in L2.
+__device__ __forceinline__ void item_pair(const AttnParams& a, int item, int& h, int& p) {
+  const int ndense = a.npairs - a.nsparse;
+  const int first = a.H * ndense;
+  if (item < first) {
+    h = item / ndense;
+    p = a.nsparse + item % ndense;
+  } else {
+    h = (item - first) / a.nsparse;
+    p = (item - first) % a.nsparse;
+  }
+}
+
+// Bounded wait taken by every lane of a warp, with one verdict for the whole warp so that
+// no lane leaves a loop that its neighbours stay in (the warp runs .sync.aligned code).
+__device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, volatile int* abort) {
+  return __all_sync(0xffffffffu, mbar_wait(bar, parity, abort, kWaitNs));
+}
 
 __device__ __forceinline__ void give_up(AttnSmem& S, uint32_t* status) {
   flag_status(status, kStatusTimeout);
@@ -181,71 +203,76 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
 
   if (warp == 0) {
     // =============================== producer ====================================
-    if (lane == 0) {
-      int g = 0, it = 0;
-      bool failed = false, q_loaded = false;
-      for (;;) {
-        const int item = (int)atomicAdd(a.counter, 1u);
-        if (item >= a.nitems) break;
-        const int p = a.npairs - 1 - item / a.H;  // pairs holding special query blocks first
-        const int h = item % a.H;
-        const int n = a.plen[h * a.npairs + p];
-        if (n <= 0) continue;
-        const int32_t* lst = a.plist + a.row_ptr[(int64_t)h * a.nb + 2 * p];
-        if (it > 0 && !mbar_wait(&S.q_empty, (it - 1) & 1, abort, kWaitNs)) {
-          failed = true;
-          break;
-        }
+    // All lanes walk the list together (32 entries per coalesced load, broadcast by
+    // shuffle); lane 0 issues the barrier operations and the TMA copies.
+    int g = 0, it = 0;
+    bool failed = false, q_loaded = false;
+    for (;;) {
+      int item = 0;
+      if (lane == 0) item = (int)atomicAdd(a.counter, 1u);
+      item = __shfl_sync(0xffffffffu, item, 0);
+      if (item >= a.nitems) break;
+      int h, p;
+      item_pair(a, item, h, p);
+      const int n = a.plen[h * a.npairs + p];
+      if (n <= 0) continue;
+      const int32_t* lst = a.plist + a.row_ptr[(int64_t)h * a.nb + 2 * p];
+      if (it > 0 && !warp_wait(&S.q_empty, (it - 1) & 1, abort)) {
+        failed = true;
+        break;
+      }
+      if (lane == 0) {
         mbar_arrive_expect_tx(&S.q_full, kRows * 128);
         tma_load_3d(S.Q, &tmQ, &S.q_full, 0, h, kRows * p);
-        q_loaded = true;
-        for (int e0 = 0; e0 < n && !failed; e0 += 32) {
-          int ent[32];
-#pragma unroll
-          for (int k = 0; k < 32; ++k) ent[k] = (e0 + k < n) ? lst[e0 + k] : 0;
-#pragma unroll 1
-          for (int k = 0; k < 32 && e0 + k < n; ++k) {
-            const int s = g % kStages, u = g / kStages;
-            if (u > 0 && !mbar_wait(&S.kv_empty[s], (u - 1) & 1, abort, kWaitNs)) {
-              failed = true;
-              break;
-            }
-            const int j = ent[k] & 0xffff;
+      }
+      q_loaded = true;
+      for (int e0 = 0; e0 < n && !failed; e0 += 32) {
+        const int mine = (e0 + lane < n) ? lst[e0 + lane] : 0;
+        const int cnt = min(32, n - e0);
+        for (int k = 0; k < cnt; ++k) {
+          const int ent = __shfl_sync(0xffffffffu, mine, k);
+          const int s = g % kStages, u = g / kStages;
+          if (u > 0 && !warp_wait(&S.kv_empty[s], (u - 1) & 1, abort)) {
+            failed = true;
+            break;
+          }
+          if (lane == 0) {
+            const int j = ent & 0xffff;
             int fl = 0;
             if (e0 + k == 0) fl |= kFirst;
             if (e0 + k == n - 1) fl |= kLast;
-            S.info[s] = TileInfo{j, ent[k] >> 16, fl, item};
+            S.info[s] = TileInfo{j, ent >> 16, fl, item};
             mbar_arrive_expect_tx(&S.kv_full[s], 2 * kTileBytes);
             tma_load_3d(S.K[s], &tmK, &S.kv_full[s], 0, h, 64 * j);
             tma_load_3d(S.V[s], &tmV, &S.kv_full[s], 0, h, 64 * j);
-            ++g;
           }
-        }
-        if (failed) break;
-        ++it;
-        q_loaded = false;
-      }
-      if (!failed) {
-        const int s = g % kStages, u = g / kStages;
-        if (u > 0 && !mbar_wait(&S.kv_empty[s], (u - 1) & 1, abort, kWaitNs)) {
-          failed = true;
-        } else {
-          S.info[s] = TileInfo{0, 0, kTerm, -1};
-          mbar_arrive(&S.kv_full[s]);
+          ++g;
         }
       }
-      if (failed) {
-        give_up(S, a.status);
-        // let every copy already issued land before the CTA's shared memory goes away
-        for (int back = 1; back <= kStages && g - back >= 0; ++back) {
-          const int gg = g - back;
-          volatile int no_abort = 0;
-          mbar_wait(&S.kv_full[gg % kStages], (gg / kStages) & 1, &no_abort, kDrainNs);
-        }
-        if (q_loaded) {
-          volatile int no_abort = 0;
-          mbar_wait(&S.q_full, it & 1, &no_abort, kDrainNs);
-        }
+      if (failed) break;
+      ++it;
+      q_loaded = false;
+    }
+    if (!failed) {
+      const int s = g % kStages, u = g / kStages;
+      if (u > 0 && !warp_wait(&S.kv_empty[s], (u - 1) & 1, abort)) {
+        failed = true;
+      } else if (lane == 0) {
+        S.info[s] = TileInfo{0, 0, kTerm, -1};
+        mbar_arrive(&S.kv_full[s]);
+      }
+    }
+    if (failed && lane == 0) {
+      give_up(S, a.status);
+      // let every copy already issued land before the CTA's shared memory goes away
+      for (int back = 1; back <= kStages && g - back >= 0; ++back) {
+        const int gg = g - back;
+        volatile int no_abort = 0;
+        mbar_wait(&S.kv_full[gg % kStages], (gg / kStages) & 1, &no_abort, kDrainNs);
+      }
+      if (q_loaded) {
+        volatile int no_abort = 0;
+        mbar_wait(&S.q_full, it & 1, &no_abort, kDrainNs);
       }
     }
   } else if (warp == 1) {
@@ -330,7 +357,7 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
     int tile_in_item = 0;
     for (;;) {
       const int s = g % kStages;
-      if (!mbar_wait(&S.kv_full[s], (g / kStages) & 1, abort, kWaitNs)) {
+      if (!warp_wait(&S.kv_full[s], (g / kStages) & 1, abort)) {
         give_up(S, a.status);
         break;
       }
@@ -342,11 +369,11 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
         tile_in_item = 0;
       }
       const int b = g & 1;
-      if (g >= 2 && !mbar_wait(&S.p_empty[b], ((g >> 1) - 1) & 1, abort, kWaitNs)) {
+      if (g >= 2 && !warp_wait(&S.p_empty[b], ((g >> 1) - 1) & 1, abort)) {
         give_up(S, a.status);
         break;
       }
-      if (!mbar_wait(&S.s_full[b], (g >> 1) & 1, abort, kWaitNs)) {
+      if (!warp_wait(&S.s_full[b], (g >> 1) & 1, abort)) {
         give_up(S, a.status);
         break;
       }
@@ -359,10 +386,10 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
           uint32_t v[32];
           RESS_TMEM_LD32(tmem + lane_base + kColS0 + 64 * b, v);
 #pragma unroll
-          for (int c = 0; c < 32; ++c) x[c] = __uint_as_float(v[c]) * kScale;
+          for (int c = 0; c < 32; ++c) x[c] = __uint_as_float(v[c]);
           RESS_TMEM_LD32(tmem + lane_base + kColS0 + 64 * b + 32, v);
 #pragma unroll
-          for (int c = 0; c < 32; ++c) x[32 + c] = __uint_as_float(v[c]) * kScale;
+          for (int c = 0; c < 32; ++c) x[32 + c] = __uint_as_float(v[c]);
         }
         if (info.j == a.nb - 1) {  // ragged last key block: keys past N do not exist
           const int valid = a.N - 64 * info.j;
@@ -370,9 +397,12 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
           for (int c = 0; c < 64; ++c)
             if (c >= valid) x[c] = -INFINITY;
         }
-        float mt = x[0];
+        // row max of the raw scores (the scale is positive), three operands at a time
+        float mr = fmax3(x[0], x[1], x[2]);
 #pragma unroll
-        for (int c = 1; c < 64; ++c) mt = fmaxf(mt, x[c]);
+        for (int c = 3; c < 63; c += 2) mr = fmax3(mr, x[c], x[c + 1]);
+        mr = fmaxf(mr, x[63]);
+        const float mt = mr * kScale;
         float alpha = 1.f;
         bool rescale = false;
         if (m_use == -INFINITY) {
@@ -384,7 +414,7 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
         }
         if (__any_sync(0xffffffffu, rescale)) {
           // the previous P V must have landed before the accumulator row is rescaled
-          if (!mbar_wait(&S.o_bar[(g - 1) & 1], ((g - 1) >> 1) & 1, abort, kWaitNs)) {
+          if (!warp_wait(&S.o_bar[(g - 1) & 1], ((g - 1) >> 1) & 1, abort)) {
             give_up(S, a.status);
             break;
           }
@@ -398,20 +428,23 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
             RESS_TMEM_ST32(tmem + lane_base + kColO + 32 * hc, v);
           }
         }
-        float rs = 0.f;
+        // p = 2^(s * log2(e)/8 - m), two columns per packed FMA; row sum in float32
+        const float nm = -m_use;
+        float rs0 = 0.f, rs1 = 0.f;
 #pragma unroll
         for (int ch = 0; ch < 8; ++ch) {
           uint32_t w[4];
 #pragma unroll
           for (int e = 0; e < 4; ++e) {
-            const float p0 = ex2(x[ch * 8 + 2 * e] - m_use);
-            const float p1 = ex2(x[ch * 8 + 2 * e + 1] - m_use);
+            float t0, t1;
+            fma2(t0, t1, x[ch * 8 + 2 * e], x[ch * 8 + 2 * e + 1], kScale, kScale, nm, nm);
+            const float p0 = ex2(t0), p1 = ex2(t1);
+            add2(rs0, rs1, rs0, rs1, p0, p1);
             w[e] = pack_bf16x2(p0, p1);
-            rs += __uint_as_float(w[e] << 16) + __uint_as_float(w[e] & 0xffff0000u);
           }
           prow[ch ^ (r & 7)] = make_uint4(w[0], w[1], w[2], w[3]);
         }
-        l = l * alpha + rs;
+        l = l * alpha + (rs0 + rs1);
       } else {
 #pragma unroll
         for (int ch = 0; ch < 8; ++ch) prow[ch] = make_uint4(0u, 0u, 0u, 0u);
@@ -424,13 +457,13 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
 
       if (info.flags & kLast) {
         // epilogue: O / l for this row once the last P V has landed
-        if (!mbar_wait(&S.o_bar[g & 1], (g >> 1) & 1, abort, kWaitNs)) {
+        if (!warp_wait(&S.o_bar[g & 1], (g >> 1) & 1, abort)) {
           give_up(S, a.status);
           break;
         }
         tc_fence_after();
-        const int item = info.item;
-        const int p = a.npairs - 1 - item / a.H, h = item % a.H;
+        int h, p;
+        item_pair(a, info.item, h, p);
         const int token = kRows * p + r;
         const bool row_exists = (2 * p + half) < a.nb && token < a.N;
         uint32_t o[2][32];
@@ -535,6 +568,7 @@ cudaError_t launch_sparse_attn(const AttnArgs& x, cudaStream_t st) {
   p.H = s.H;
   p.nb = s.nb;
   p.npairs = npairs;
+  p.nsparse = s.ncand / 2;
   p.nitems = pairs;
   p.row_ptr = x.row_ptr;
   p.plist = x.plist;

@@ -277,16 +277,23 @@ __device__ __forceinline__ uint32_t order_key(float x) {
   return (b & 0x80000000u) ? ~b : (b | 0x80000000u);
 }
 
-// Exact top-m of kb[0..n) for one warp: the m largest keys, ties to the lower index
-// (requires m <= number of nonzero keys).  Result: bitmask sel[words] in shared memory.
-__device__ void warp_topm(const uint32_t* kb, int n, int m, uint32_t* sel, int words) {
+// Exact top-m of kb[0..n) for one warp: the m largest keys, ties to the lower index.
+// With `member` set, only positions j whose bit in member[] equals `want` take part.
+// Requires m <= number of participating positions.  Result: bitmask sel[words].
+__device__ __forceinline__ bool takes_part(const uint32_t* member, bool want, int j) {
+  return member == nullptr || (((member[j >> 5] >> (j & 31)) & 1u) != 0) == want;
+}
+
+__device__ void warp_topm(const uint32_t* kb, int n, int m, uint32_t* sel, int words,
+                          const uint32_t* member = nullptr, bool want = true) {
   const int lane = threadIdx.x & 31;
   uint32_t lo = 0;
   if (m > 0) {
     for (int bit = 31; bit >= 0; --bit) {
       const uint32_t cand = lo | (1u << bit);
       int cnt = 0;
-      for (int j = lane; j < n; j += 32) cnt += kb[j] >= cand ? 1 : 0;
+#pragma unroll 4
+      for (int j = lane; j < n; j += 32) cnt += (kb[j] >= cand && takes_part(member, want, j)) ? 1 : 0;
       cnt = __reduce_add_sync(kFull, cnt);
       if (cnt >= m) {
         lo = cand;
@@ -295,15 +302,17 @@ __device__ void warp_topm(const uint32_t* kb, int n, int m, uint32_t* sel, int w
     }
   }
   int gt = 0;
-  for (int j = lane; j < n; j += 32) gt += kb[j] > lo ? 1 : 0;
+#pragma unroll 4
+  for (int j = lane; j < n; j += 32) gt += (kb[j] > lo && takes_part(member, want, j)) ? 1 : 0;
   gt = __reduce_add_sync(kFull, gt);
   const int need = m - gt;
   int taken = 0;
   for (int w = 0; w < words; ++w) {
     const int j = w * 32 + lane;
-    const uint32_t v = j < n ? kb[j] : 0u;
-    const bool is_gt = m > 0 && v > lo;
-    const bool is_eq = m > 0 && j < n && v == lo && v != 0u;
+    const bool part = j < n && takes_part(member, want, j);
+    const uint32_t v = part ? kb[j] : 0u;
+    const bool is_gt = m > 0 && part && v > lo;
+    const bool is_eq = m > 0 && part && v == lo;
     const uint32_t eqb = __ballot_sync(kFull, is_eq);
     const int rank = taken + __popc(eqb & ((1u << lane) - 1u));
     const uint32_t sb = __ballot_sync(kFull, is_gt || (is_eq && rank < need));
@@ -326,25 +335,43 @@ __device__ __forceinline__ uint32_t valid_bits(int w, int n) {
 }
 
 // g~ = sum_{j not in D} P_ij (z~_j - y~_i) and K = sum_{j not in D} P_ij for one row, by
-// one warp (lane owns channels 2*lane, 2*lane+1).  D: bitmask words in shared memory.
+// one warp (lane owns channels 2*lane, 2*lane+1), in ascending j.  The kept blocks are
+// first compacted into idx[] (per-warp shared memory, >= nb entries) so that the loads of
+// eight blocks are in flight together.
 __device__ __forceinline__ void kept_drift(const uint32_t* D, const SelPtrs& p,
                                            const float* __restrict__ Prow,
                                            const float* __restrict__ zt, float y0, float y1,
-                                           float& g0, float& g1, float& K) {
+                                           uint32_t* idx, float& g0, float& g1, float& K) {
   const int lane = threadIdx.x & 31;
-  g0 = g1 = K = 0.f;
+  int n = 0;
   for (int w = 0; w < p.words; ++w) {
-    uint32_t keep = ~D[w] & valid_bits(w, p.nb);
-    while (keep) {
-      const int j = w * 32 + __ffs(keep) - 1;
-      keep &= keep - 1;
-      const float pj = Prow[j];
-      const float2 z = *reinterpret_cast<const float2*>(zt + (int64_t)j * 64 + 2 * lane);
-      g0 = fmaf(pj, z.x - y0, g0);
-      g1 = fmaf(pj, z.y - y1, g1);
-      K += pj;
+    const uint32_t keep = ~D[w] & valid_bits(w, p.nb);
+    if ((keep >> lane) & 1u) idx[n + __popc(keep & ((1u << lane) - 1u))] = w * 32 + lane;
+    n += __popc(keep);
+  }
+  __syncwarp();
+  g0 = g1 = K = 0.f;
+  for (int k0 = 0; k0 < n; k0 += 8) {
+    float pj[8];
+    float2 z[8];
+#pragma unroll
+    for (int u = 0; u < 8; ++u) {
+      if (k0 + u < n) {
+        const int j = idx[k0 + u];
+        pj[u] = Prow[j];
+        z[u] = *reinterpret_cast<const float2*>(zt + (int64_t)j * 64 + 2 * lane);
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < 8; ++u) {
+      if (k0 + u < n) {
+        g0 = fmaf(pj[u], z[u].x - y0, g0);
+        g1 = fmaf(pj[u], z[u].y - y1, g1);
+        K += pj[u];
+      }
     }
   }
+  __syncwarp();
 }
 
 // ------------------------------------------------------------------------------------
@@ -392,6 +419,7 @@ __global__ void __launch_bounds__(kThreads, 2) k_score(SelPtrs p, Budgets bud) {
   for (int r = warp; r < nrows; r += 8) {
     const float* row = Pbase + (int64_t)r * p.ld;
     float m = -INFINITY, z = 0.f;
+#pragma unroll 4
     for (int j = lane; j < p.nb; j += 32) {
       const float x = row[j];
       if (x > m) {
@@ -493,6 +521,7 @@ __global__ void __launch_bounds__(kThreads, 2) k_score(SelPtrs p, Budgets bud) {
     const int i = i0 + r;
     const float* Prow = Pbase + (int64_t)r * p.ld;
     const float* qrow = qbase + (int64_t)r * p.ld;
+#pragma unroll 4
     for (int j = lane; j < p.ncand; j += 32) {
       const float pj = Prow[j];
       const float key = pj * sqrtf(qrow[j]) / fmaxf(1.0f - pj, kEps);
@@ -509,7 +538,7 @@ __global__ void __launch_bounds__(kThreads, 2) k_score(SelPtrs p, Budgets bud) {
     }
     __syncwarp();
     float g0, g1, K;
-    kept_drift(sel, p, Prow, zt_h, S.A[r][2 * lane], S.A[r][2 * lane + 1], g0, g1, K);
+    kept_drift(sel, p, Prow, zt_h, S.A[r][2 * lane], S.A[r][2 * lane + 1], kb, g0, g1, K);
     const float G = warp_sum(g0 * g0 + g1 * g1);
     const float Kc = fmaxf(K, kEps);
     const float J = G / (Kc * Kc);
@@ -595,36 +624,26 @@ __global__ void __launch_bounds__(kThreads, 2) k_round(SelPtrs p, Budgets bud, i
     for (int w = lane; w < p.words; w += 32) Dw[w] = p.dmask[ri * p.words + w];
     const float K = p.K[ri], G = p.G[ri];
     __syncwarp();
-    // restore candidates k in D: u = +P_k, dG = -2 P_k t_k + P_k^2 q_k (Eq. 13, 14)
+    // one pass over the candidates: a block k in D is a restore candidate (u = +P_k,
+    // dG = -2 P_k t_k + P_k^2 q_k, Eq. 13-14), a kept candidate a drop candidate (u = -P_k,
+    // dG = +2 P_k t_k + P_k^2 q_k, Eq. 15); the key is the exact decrease of J (Eq. 16)
+#pragma unroll 4
     for (int j = lane; j < p.ncand; j += 32) {
-      uint32_t key = 0u;
-      if ((Dw[j >> 5] >> (j & 31)) & 1u) {
-        const float pj = Prow[j];
-        const float dG = fmaf(pj * pj, qrow[j], -2.0f * pj * trow[j]);
-        key = order_key(delta_J(G, K, dG, pj));
-      }
-      kb[j] = key;
+      const float pj = Prow[j], qj = qrow[j], tj = trow[j];
+      const bool inD = (Dw[j >> 5] >> (j & 31)) & 1u;
+      const float s2 = pj * pj * qj;
+      const float dG = inD ? fmaf(-2.0f * pj, tj, s2) : fmaf(2.0f * pj, tj, s2);
+      kb[j] = order_key(delta_J(G, K, dG, inD ? pj : -pj));
     }
     __syncwarp();
-    warp_topm(kb, p.ncand, m, Rw, p.words);
-    // drop candidates k in P \ D: u = -P_k, dG = +2 P_k t_k + P_k^2 q_k (Eq. 15)
-    for (int j = lane; j < p.ncand; j += 32) {
-      uint32_t key = 0u;
-      if (!((Dw[j >> 5] >> (j & 31)) & 1u)) {
-        const float pj = Prow[j];
-        const float dG = fmaf(pj * pj, qrow[j], 2.0f * pj * trow[j]);
-        key = order_key(delta_J(G, K, dG, -pj));
-      }
-      kb[j] = key;
-    }
-    __syncwarp();
-    warp_topm(kb, p.ncand, m, Xw, p.words);
+    warp_topm(kb, p.ncand, m, Rw, p.words, Dw, true);
+    warp_topm(kb, p.ncand, m, Xw, p.words, Dw, false);
     for (int w = lane; w < p.words; w += 32) Dw[w] = (Dw[w] & ~Rw[w]) | Xw[w];
     __syncwarp();
     // exact state of the new set (Eq. 10-12)
     const float y0 = p.ytil[ri * 64 + 2 * lane], y1 = p.ytil[ri * 64 + 2 * lane + 1];
     float g0, g1, Kn;
-    kept_drift(Dw, p, Prow, zt_h, y0, y1, g0, g1, Kn);
+    kept_drift(Dw, p, Prow, zt_h, y0, y1, kb, g0, g1, Kn);
     const float Gn = warp_sum(g0 * g0 + g1 * g1);
     const float Kc = fmaxf(Kn, kEps);
     const float Jn = Gn / (Kc * Kc);
