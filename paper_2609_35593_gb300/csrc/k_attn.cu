@@ -428,7 +428,7 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
             RESS_TMEM_ST32(tmem + lane_base + kColO + 32 * hc, v);
           }
         }
-        // p = 2^(s * log2(e)/8 - m), two columns per packed FMA; row sum in float32
+        // p = 2^(s * log2(e)/8 - m), two columns per packed FMA
         const float nm = -m_use;
         float rs0 = 0.f, rs1 = 0.f;
 #pragma unroll
@@ -438,9 +438,10 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
           for (int e = 0; e < 4; ++e) {
             float t0, t1;
             fma2(t0, t1, x[ch * 8 + 2 * e], x[ch * 8 + 2 * e + 1], kScale, kScale, nm, nm);
-            const float p0 = ex2(t0), p1 = ex2(t1);
-            add2(rs0, rs1, rs0, rs1, p0, p1);
-            w[e] = pack_bf16x2(p0, p1);
+            w[e] = pack_bf16x2(ex2(t0), ex2(t1));
+            // sum the bf16 values the MMA multiplies, so that a row dominated by one key
+            // keeps O = V exactly up to the accumulation (p reaches 2^8 between rescales)
+            add2(rs0, rs1, rs0, rs1, __uint_as_float(w[e] << 16), __uint_as_float(w[e] & 0xffff0000u));
           }
           prow[ch ^ (r & 7)] = make_uint4(w[0], w[1], w[2], w[3]);
         }
