@@ -8,14 +8,18 @@
 //
 // Warp roles (192 threads, 2 CTAs per SM):
 //   warp 0     TMA producer: Q tile (128 x 64) per item, K/V tiles (64 x 64) per entry into
-//              a 3-stage ring, 128-byte swizzled (UMMA K-major canonical layout).
+//              a 5-stage ring, 128-byte swizzled (UMMA canonical layouts).
 //   warp 1     TMEM owner and single-thread MMA issuer:
-//                S[g % 2] = Q K_g^T              (M128 N64 K64, both K-major)
-//                O       += P_{g-1} V_{g-1}       (M128 N64 K64, V MN-major)
-//              S is double-buffered in TMEM so that S_{g+1} runs while softmax works on S_g.
+//                S[g % 2] = Q K_g^T              (M128 N64 K64, Q and K from shared memory)
+//                O       += P_{g-1} V_{g-1}       (M128 N64 K64, P from TMEM, V MN-major)
+//              S is double-buffered in TMEM so that S_{g+1} runs while softmax works on S_g;
+//              P_g (bf16) is written over the first half of S_g's columns and read from
+//              there as the A operand, which keeps it off the shared-memory bus.  MMAs
+//              issued by one thread run in issue order, so S_{g+2} overwrites P_g only after
+//              P_g V_g has read it.
 //   warps 2-5  one query row per thread: tcgen05.ld of S, online softmax in the exp2 domain
 //              with lazy rescaling of the TMEM accumulator (only when the running max grows
-//              by more than 2^8), P as bf16 into a swizzled shared buffer, epilogue O / l.
+//              by more than 2^8), tcgen05.st of P, epilogue O / l.
 // Every mbarrier wait is bounded; a wait that gives up records RESS_ETIMEOUT in the status
 // word, makes the whole CTA leave its loops, drains in-flight copies and MMAs, frees TMEM
 // and returns.
@@ -31,7 +35,7 @@ namespace ress {
 using namespace ptx;
 
 constexpr int kAttnThreads = 192;
-constexpr int kStages = 3;
+constexpr int kStages = 5;
 constexpr int kRows = 128;
 constexpr uint32_t kTmemCols = 256;
 constexpr uint32_t kColS0 = 0, kColO = 128;
@@ -49,10 +53,9 @@ struct __align__(1024) AttnSmem {
   uint8_t Q[kRows * 128];
   uint8_t K[kStages][kTileBytes];
   uint8_t V[kStages][kTileBytes];
-  uint8_t P[2][kRows * 128];
   uint64_t kv_full[kStages], kv_empty[kStages];
   uint64_t q_full, q_empty;
-  uint64_t s_full[2], p_full[2], p_empty[2];
+  uint64_t s_full[2], p_full[2];
   uint64_t o_bar[2], drain;  // o_bar[k & 1] completes when P_k V_k has landed
   TileInfo info[kStages];
   uint32_t tmem_base;
@@ -85,10 +88,16 @@ __device__ __forceinline__ void item_pair(const AttnParams& a, int item, int& h,
   }
 }
 
-// Bounded wait taken by every lane of a warp, with one verdict for the whole warp so that
-// no lane leaves a loop that its neighbours stay in (the warp runs .sync.aligned code).
+// Bounded wait for a whole warp: lane 0 polls (one poller per warp keeps the barrier traffic
+// low), the verdict is broadcast so that no lane leaves a loop its neighbours stay in (the
+// warp runs .sync.aligned code), and __syncwarp orders the other lanes' later reads after
+// lane 0's acquire.
 __device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, volatile int* abort) {
-  return __all_sync(0xffffffffu, mbar_wait(bar, parity, abort, kWaitNs));
+  int ok = 1;
+  if ((threadIdx.x & 31) == 0) ok = mbar_wait(bar, parity, abort, kWaitNs) ? 1 : 0;
+  ok = __shfl_sync(0xffffffffu, ok, 0);
+  __syncwarp();
+  return ok != 0;
 }
 
 __device__ __forceinline__ void give_up(AttnSmem& S, uint32_t* status) {
@@ -184,7 +193,6 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
     for (int b = 0; b < 2; ++b) {
       mbar_init(&S.s_full[b], 1);
       mbar_init(&S.p_full[b], 4);
-      mbar_init(&S.p_empty[b], 1);
     }
     mbar_init(&S.o_bar[0], 1);
     mbar_init(&S.o_bar[1], 1);
@@ -288,14 +296,12 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
         const int pb = pg & 1, ps = pg % kStages;
         if (!mbar_wait(&S.p_full[pb], (pg >> 1) & 1, abort, kWaitNs)) return false;
         tc_fence_after();
-        const uint32_t p_addr = smem_u32(S.P[pb]);
         const uint32_t v_addr = smem_u32(S.V[ps]);
 #pragma unroll
         for (int k = 0; k < 4; ++k)
-          mma_bf16_ss(tmem + kColO, sdesc_sw128(p_addr + 32 * k), sdesc_sw128(v_addr + 2048 * k),
+          mma_bf16_ts(tmem + kColO, tmem + kColS0 + 64 * pb + 8 * k, sdesc_sw128(v_addr + 2048 * k),
                       idesc_pv, (k > 0 || !first) ? 1u : 0u);
         mma_commit(&S.kv_empty[ps]);
-        mma_commit(&S.p_empty[pb]);
         mma_commit(&S.o_bar[pg & 1]);
         return true;
       };
@@ -351,7 +357,6 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
     const int half = r >> 6;
     const uint32_t lane_base = (uint32_t)(quarter * 32) << 16;
     const float kScale = 1.4426950408889634f * 0.125f;  // log2(e) / sqrt(64)
-    uint8_t* prow_base[2] = {S.P[0] + r * 128, S.P[1] + r * 128};
     int g = 0;
     float m_use = -INFINITY, l = 0.f;
     int tile_in_item = 0;
@@ -369,25 +374,22 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
         tile_in_item = 0;
       }
       const int b = g & 1;
-      if (g >= 2 && !warp_wait(&S.p_empty[b], ((g >> 1) - 1) & 1, abort)) {
-        give_up(S, a.status);
-        break;
-      }
+      // S_g complete implies every earlier MMA complete, P_{g-2} V_{g-2} included
       if (!warp_wait(&S.s_full[b], (g >> 1) & 1, abort)) {
         give_up(S, a.status);
         break;
       }
       tc_fence_after();
       const bool active = (info.mask >> half) & 1;  // warp-uniform
-      uint4* prow = reinterpret_cast<uint4*>(prow_base[b]);
+      const uint32_t tS = tmem + lane_base + kColS0 + 64 * b;
       if (active) {
         float x[64];
         {
           uint32_t v[32];
-          RESS_TMEM_LD32(tmem + lane_base + kColS0 + 64 * b, v);
+          RESS_TMEM_LD32(tS, v);
 #pragma unroll
           for (int c = 0; c < 32; ++c) x[c] = __uint_as_float(v[c]);
-          RESS_TMEM_LD32(tmem + lane_base + kColS0 + 64 * b + 32, v);
+          RESS_TMEM_LD32(tS + 32, v);
 #pragma unroll
           for (int c = 0; c < 32; ++c) x[32 + c] = __uint_as_float(v[c]);
         }
@@ -431,26 +433,24 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
         // p = 2^(s * log2(e)/8 - m), two columns per packed FMA
         const float nm = -m_use;
         float rs0 = 0.f, rs1 = 0.f;
+        uint32_t w[32];
 #pragma unroll
-        for (int ch = 0; ch < 8; ++ch) {
-          uint32_t w[4];
-#pragma unroll
-          for (int e = 0; e < 4; ++e) {
-            float t0, t1;
-            fma2(t0, t1, x[ch * 8 + 2 * e], x[ch * 8 + 2 * e + 1], kScale, kScale, nm, nm);
-            w[e] = pack_bf16x2(ex2(t0), ex2(t1));
-            // sum the bf16 values the MMA multiplies, so that a row dominated by one key
-            // keeps O = V exactly up to the accumulation (p reaches 2^8 between rescales)
-            add2(rs0, rs1, rs0, rs1, __uint_as_float(w[e] << 16), __uint_as_float(w[e] & 0xffff0000u));
-          }
-          prow[ch ^ (r & 7)] = make_uint4(w[0], w[1], w[2], w[3]);
+        for (int e = 0; e < 32; ++e) {
+          float t0, t1;
+          fma2(t0, t1, x[2 * e], x[2 * e + 1], kScale, kScale, nm, nm);
+          w[e] = pack_bf16x2(ex2(t0), ex2(t1));
+          // sum the bf16 values the MMA multiplies, so that a row dominated by one key
+          // keeps O = V exactly up to the accumulation (p reaches 2^8 between rescales)
+          add2(rs0, rs1, rs0, rs1, __uint_as_float(w[e] << 16), __uint_as_float(w[e] & 0xffff0000u));
         }
+        RESS_TMEM_ST32(tS, w);  // P_g over the first 32 columns of S_g
         l = l * alpha + (rs0 + rs1);
       } else {
+        uint32_t w[32];
 #pragma unroll
-        for (int ch = 0; ch < 8; ++ch) prow[ch] = make_uint4(0u, 0u, 0u, 0u);
+        for (int e = 0; e < 32; ++e) w[e] = 0u;
+        RESS_TMEM_ST32(tS, w);
       }
-      fence_proxy_async_smem();
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&S.p_full[b]);
