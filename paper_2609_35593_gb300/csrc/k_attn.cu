@@ -6,7 +6,7 @@
 // two query blocks keeps it; rows of a block that does not keep the tile get P = 0, so
 // every row sees exactly its own kept blocks (softmax renormalised among them).
 //
-// Warp roles (320 threads, 2 CTAs per SM):
+// Warp roles (192 threads, 2 CTAs per SM):
 //   warp 0     TMA producer: Q tile (128 x 64) per item, K/V tiles (64 x 64) per entry into
 //              a 5-stage ring, 128-byte swizzled (UMMA canonical layouts).
 //   warp 1     TMEM owner and single-thread MMA issuer:
@@ -17,7 +17,7 @@
 //              there as the A operand, which keeps it off the shared-memory bus.  MMAs
 //              issued by one thread run in issue order, so S_{g+2} overwrites P_g only after
 //              P_g V_g has read it.
-//   warps 2-9  two threads per query row (32 columns each): tcgen05.ld of S, online softmax in the exp2 domain
+//   warps 2-5  one query row per thread: tcgen05.ld of S, online softmax in the exp2 domain
 //              with lazy rescaling of the TMEM accumulator (only when the running max grows
 //              by more than 2^8), tcgen05.st of P, epilogue O / l.
 // Every mbarrier wait is bounded; a wait that gives up records RESS_ETIMEOUT in the status
@@ -34,7 +34,7 @@
 namespace ress {
 using namespace ptx;
 
-constexpr int kAttnThreads = 320;  // producer, MMA, 8 softmax warps
+constexpr int kAttnThreads = 192;
 constexpr int kStages = 5;
 constexpr int kRows = 128;
 constexpr uint32_t kTmemCols = 256;
@@ -56,11 +56,8 @@ struct __align__(1024) AttnSmem {
   uint64_t kv_full[kStages], kv_empty[kStages];
   uint64_t q_full, q_empty;
   uint64_t s_full[2], p_full[2];
-  uint64_t o_bar[2], drain;
-  uint64_t pair_bar[4];  // the two softmax warps of one TMEM lane quarter meet here  // o_bar[k & 1] completes when P_k V_k has landed
+  uint64_t o_bar[2], drain;  // o_bar[k & 1] completes when P_k V_k has landed
   TileInfo info[kStages];
-  float pmax[2][2][kRows];  // [tile parity][column group][row] partial row maxima
-  float psum[2][2][kRows];  // [tile parity][column group][row] partial row sums (epilogue)
   uint32_t tmem_base;
   int abort;
 };
@@ -195,12 +192,11 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
     mbar_init(&S.q_empty, 1);
     for (int b = 0; b < 2; ++b) {
       mbar_init(&S.s_full[b], 1);
-      mbar_init(&S.p_full[b], 8);
+      mbar_init(&S.p_full[b], 4);
     }
     mbar_init(&S.o_bar[0], 1);
     mbar_init(&S.o_bar[1], 1);
     mbar_init(&S.drain, 1);
-    for (int q = 0; q < 4; ++q) mbar_init(&S.pair_bar[q], 2);
     S.abort = 0;
     fence_barrier_init();
     prefetch_tensormap(&tmQ);
@@ -356,29 +352,14 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
     }
   } else {
     // ================================ softmax =====================================
-    // Two threads per query row: warps 2-5 own columns 0-31 of every 64-key tile, warps 6-9
-    // columns 32-63, for the same TMEM lane quarter (warp & 3).  The two halves of a row
-    // agree on the row maximum through shared memory and a named barrier per warp pair.
     const int quarter = warp & 3;
-    const int cg = (warp - 2) >> 2;     // column group of this warp
     const int r = quarter * 32 + lane;  // query row within the 128-row tile
-    const int half = r >> 6;            // query block of the pair this row belongs to
-    uint64_t* pair_bar = &S.pair_bar[quarter];
-    int pair_phase = 0;
-    // Both warps of the pair arrive, then wait (bounded) for the other one.
-    auto pair_sync = [&]() -> bool {
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(pair_bar);
-      const bool ok = warp_wait(pair_bar, pair_phase & 1, abort);
-      ++pair_phase;
-      tc_fence_after();
-      return ok;
-    };
+    const int half = r >> 6;
     const uint32_t lane_base = (uint32_t)(quarter * 32) << 16;
     const float kScale = 1.4426950408889634f * 0.125f;  // log2(e) / sqrt(64)
     int g = 0;
     float m_use = -INFINITY, l = 0.f;
+    int tile_in_item = 0;
     for (;;) {
       const int s = g % kStages;
       if (!warp_wait(&S.kv_full[s], (g / kStages) & 1, abort)) {
@@ -390,6 +371,7 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
       if (info.flags & kFirst) {
         m_use = -INFINITY;
         l = 0.f;
+        tile_in_item = 0;
       }
       const int b = g & 1;
       // S_g complete implies every earlier MMA complete, P_{g-2} V_{g-2} included
@@ -398,36 +380,30 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
         break;
       }
       tc_fence_after();
-      const bool active = (info.mask >> half) & 1;  // the same for both warps of the pair
+      const bool active = (info.mask >> half) & 1;  // warp-uniform
       const uint32_t tS = tmem + lane_base + kColS0 + 64 * b;
       if (active) {
-        float x[32];
+        float x[64];
         {
           uint32_t v[32];
-          RESS_TMEM_LD32(tS + 32 * cg, v);
+          RESS_TMEM_LD32(tS, v);
 #pragma unroll
           for (int c = 0; c < 32; ++c) x[c] = __uint_as_float(v[c]);
+          RESS_TMEM_LD32(tS + 32, v);
+#pragma unroll
+          for (int c = 0; c < 32; ++c) x[32 + c] = __uint_as_float(v[c]);
         }
         if (info.j == a.nb - 1) {  // ragged last key block: keys past N do not exist
-          const int valid = a.N - 64 * info.j - 32 * cg;
+          const int valid = a.N - 64 * info.j;
 #pragma unroll
-          for (int c = 0; c < 32; ++c)
+          for (int c = 0; c < 64; ++c)
             if (c >= valid) x[c] = -INFINITY;
         }
-        // row max of the raw scores (the scale is positive): own half, then the partner's
-        float m0 = fmax3(x[0], x[1], x[2]), m1 = fmax3(x[3], x[4], x[5]);
+        // row max of the raw scores (the scale is positive), three operands at a time
+        float mr = fmax3(x[0], x[1], x[2]);
 #pragma unroll
-        for (int c = 6; c < 30; c += 4) {
-          m0 = fmax3(m0, x[c], x[c + 1]);
-          m1 = fmax3(m1, x[c + 2], x[c + 3]);
-        }
-        float mr = fmax3(m0, m1, fmaxf(x[30], x[31]));
-        S.pmax[b][cg][r] = mr;
-        if (!pair_sync()) {  // both halves of S_g read, both partial maxima written
-          give_up(S, a.status);
-          break;
-        }
-        mr = fmaxf(mr, S.pmax[b][cg ^ 1][r]);
+        for (int c = 3; c < 63; c += 2) mr = fmax3(mr, x[c], x[c + 1]);
+        mr = fmaxf(mr, x[63]);
         const float mt = mr * kScale;
         float alpha = 1.f;
         bool rescale = false;
@@ -445,48 +421,43 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
             break;
           }
           tc_fence_after();
-          uint32_t v[32];
-          RESS_TMEM_LD32(tmem + lane_base + kColO + 32 * cg, v);
 #pragma unroll
-          for (int c = 0; c < 32; ++c) v[c] = __float_as_uint(__uint_as_float(v[c]) * alpha);
-          RESS_TMEM_ST32(tmem + lane_base + kColO + 32 * cg, v);
+          for (int hc = 0; hc < 2; ++hc) {
+            uint32_t v[32];
+            RESS_TMEM_LD32(tmem + lane_base + kColO + 32 * hc, v);
+#pragma unroll
+            for (int c = 0; c < 32; ++c) v[c] = __float_as_uint(__uint_as_float(v[c]) * alpha);
+            RESS_TMEM_ST32(tmem + lane_base + kColO + 32 * hc, v);
+          }
         }
         // p = 2^(s * log2(e)/8 - m), two columns per packed FMA
         const float nm = -m_use;
-        float rs0 = 0.f, rs1 = 0.f, rs2 = 0.f, rs3 = 0.f;
-        uint32_t w[16];
+        float rs0 = 0.f, rs1 = 0.f;
+        uint32_t w[32];
 #pragma unroll
-        for (int e = 0; e < 16; ++e) {
+        for (int e = 0; e < 32; ++e) {
           float t0, t1;
           fma2(t0, t1, x[2 * e], x[2 * e + 1], kScale, kScale, nm, nm);
           w[e] = pack_bf16x2(ex2(t0), ex2(t1));
           // sum the bf16 values the MMA multiplies, so that a row dominated by one key
           // keeps O = V exactly up to the accumulation (p reaches 2^8 between rescales)
-          if (e & 1)
-            add2(rs2, rs3, rs2, rs3, __uint_as_float(w[e] << 16), __uint_as_float(w[e] & 0xffff0000u));
-          else
-            add2(rs0, rs1, rs0, rs1, __uint_as_float(w[e] << 16), __uint_as_float(w[e] & 0xffff0000u));
+          add2(rs0, rs1, rs0, rs1, __uint_as_float(w[e] << 16), __uint_as_float(w[e] & 0xffff0000u));
         }
-        RESS_TMEM_ST16(tS + 16 * cg, w);  // P_g over the first 32 columns of S_g
-        l = l * alpha + ((rs0 + rs1) + (rs2 + rs3));
+        RESS_TMEM_ST32(tS, w);  // P_g over the first 32 columns of S_g
+        l = l * alpha + (rs0 + rs1);
       } else {
-        uint32_t w[16];
+        uint32_t w[32];
 #pragma unroll
-        for (int e = 0; e < 16; ++e) w[e] = 0u;
-        RESS_TMEM_ST16(tS + 16 * cg, w);
+        for (int e = 0; e < 32; ++e) w[e] = 0u;
+        RESS_TMEM_ST32(tS, w);
       }
       tc_fence_before();
       __syncwarp();
       if (lane == 0) mbar_arrive(&S.p_full[b]);
+      ++tile_in_item;
 
       if (info.flags & kLast) {
         // epilogue: O / l for this row once the last P V has landed
-        S.psum[b][cg][r] = l;
-        if (!pair_sync()) {
-          give_up(S, a.status);
-          break;
-        }
-        const float lt = l + S.psum[b][cg ^ 1][r];
         if (!warp_wait(&S.o_bar[g & 1], (g >> 1) & 1, abort)) {
           give_up(S, a.status);
           break;
@@ -496,27 +467,34 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
         item_pair(a, info.item, h, p);
         const int token = kRows * p + r;
         const bool row_exists = (2 * p + half) < a.nb && token < a.N;
-        uint32_t o[32];
-        RESS_TMEM_LD32(tmem + lane_base + kColO + 32 * cg, o);
+        uint32_t o[2][32];
+        RESS_TMEM_LD32(tmem + lane_base + kColO, o[0]);
+        RESS_TMEM_LD32(tmem + lane_base + kColO + 32, o[1]);
         if (row_exists) {
-          if (!(lt > 0.f)) flag_status(a.status, kStatusBadRow);
-          const float inv = lt > 0.f ? 1.0f / lt : 0.f;
-          const int64_t off = ((int64_t)token * a.H + h) * 64 + 32 * cg;
+          if (!(l > 0.f)) flag_status(a.status, kStatusBadRow);
+          const float inv = l > 0.f ? 1.0f / l : 0.f;
+          const int64_t off = ((int64_t)token * a.H + h) * 64;
           if (kOutF32) {
             float4* dst = reinterpret_cast<float4*>(static_cast<float*>(a.O) + off);
 #pragma unroll
-            for (int ch = 0; ch < 8; ++ch)
-              dst[ch] = make_float4(__uint_as_float(o[4 * ch]) * inv, __uint_as_float(o[4 * ch + 1]) * inv,
-                                    __uint_as_float(o[4 * ch + 2]) * inv, __uint_as_float(o[4 * ch + 3]) * inv);
+            for (int ch = 0; ch < 16; ++ch) {
+              const int c = ch * 4;
+              dst[ch] = make_float4(__uint_as_float(o[c >> 5][c & 31]) * inv,
+                                    __uint_as_float(o[(c + 1) >> 5][(c + 1) & 31]) * inv,
+                                    __uint_as_float(o[(c + 2) >> 5][(c + 2) & 31]) * inv,
+                                    __uint_as_float(o[(c + 3) >> 5][(c + 3) & 31]) * inv);
+            }
           } else {
             uint4* dst = reinterpret_cast<uint4*>(static_cast<uint16_t*>(a.O) + off);
 #pragma unroll
-            for (int ch = 0; ch < 4; ++ch) {
+            for (int ch = 0; ch < 8; ++ch) {
               uint32_t w[4];
 #pragma unroll
-              for (int e = 0; e < 4; ++e)
-                w[e] = pack_bf16x2(__uint_as_float(o[8 * ch + 2 * e]) * inv,
-                                   __uint_as_float(o[8 * ch + 2 * e + 1]) * inv);
+              for (int e = 0; e < 4; ++e) {
+                const int c = ch * 8 + 2 * e;
+                w[e] = pack_bf16x2(__uint_as_float(o[c >> 5][c & 31]) * inv,
+                                   __uint_as_float(o[(c + 1) >> 5][(c + 1) & 31]) * inv);
+              }
               dst[ch] = make_uint4(w[0], w[1], w[2], w[3]);
             }
           }
