@@ -10,8 +10,11 @@
 //   warp 0     TMA producer: Q tile (128 x 64) per item, K/V tiles (64 x 64) per entry into
 //              a 5-stage ring, 128-byte swizzled (UMMA canonical layouts).
 //   warp 1     TMEM owner and single-thread MMA issuer:
-//                S[g % 2] = Q K_g^T              (M128 N64 K64, Q and K from shared memory)
+//                S[g % 2] = Q K_g^T              (M128 N64 K64, Q from TMEM, K from shared memory)
 //                O       += P_{g-1} V_{g-1}       (M128 N64 K64, P from TMEM, V MN-major)
+//              Q is copied once per item from its TMA staging buffer into TMEM (tcgen05.cp),
+//              so that neither A operand is read from shared memory, whose bandwidth the
+//              N = 64 MMAs would otherwise saturate together with the TMA writes.
 //              S is double-buffered in TMEM so that S_{g+1} runs while softmax works on S_g;
 //              P_g (bf16) is written over the first half of S_g's columns and read from
 //              there as the A operand, which keeps it off the shared-memory bus.  MMAs
@@ -38,7 +41,7 @@ constexpr int kAttnThreads = 192;
 constexpr int kStages = 5;
 constexpr int kRows = 128;
 constexpr uint32_t kTmemCols = 256;
-constexpr uint32_t kColS0 = 0, kColO = 128;
+constexpr uint32_t kColS0 = 0, kColO = 128, kColQ = 192;  // TMEM columns: S/P x2, O, Q
 constexpr uint64_t kWaitNs = 2000000000ull;  // 2 s per wait
 constexpr uint64_t kDrainNs = 200000000ull;  // 0.2 s to drain after an abort
 constexpr int kFirst = 1, kLast = 2, kTerm = 4;
@@ -313,19 +316,27 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
         }
         const TileInfo info = S.info[s];
         if (info.flags & kTerm) break;
-        if ((info.flags & kFirst) && !mbar_wait(&S.q_full, it & 1, abort, kWaitNs)) {
-          failed = true;
-          break;
+        if (info.flags & kFirst) {
+          if (!mbar_wait(&S.q_full, it & 1, abort, kWaitNs)) {
+            failed = true;
+            break;
+          }
+          tc_fence_after();
+          // Q (128 x 64) into TMEM, one K16 slice (8 columns) per copy; the staging buffer
+          // is free again once the copies have completed.  Copies and MMAs issued by this
+          // thread run in order, so earlier S MMAs have read the previous Q by then.
+#pragma unroll
+          for (int k = 0; k < 4; ++k) tmem_cp_128x256b(tmem + kColQ + 8 * k, sdesc_sw128(q_addr + 32 * k));
+          mma_commit(&S.q_empty);
         }
         tc_fence_after();
         const int b = g & 1;
         const uint32_t k_addr = smem_u32(S.K[s]);
 #pragma unroll
         for (int k = 0; k < 4; ++k)
-          mma_bf16_ss(tmem + kColS0 + 64 * b, sdesc_sw128(q_addr + 32 * k),
-                      sdesc_sw128(k_addr + 32 * k), idesc_qk, k > 0 ? 1u : 0u);
+          mma_bf16_ts(tmem + kColS0 + 64 * b, tmem + kColQ + 8 * k, sdesc_sw128(k_addr + 32 * k),
+                      idesc_qk, k > 0 ? 1u : 0u);
         mma_commit(&S.s_full[b]);
-        if (info.flags & kLast) mma_commit(&S.q_empty);
         if (have_prev && !issue_pv(prev_g, prev_first)) {
           failed = true;
           break;

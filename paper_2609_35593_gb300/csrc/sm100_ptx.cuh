@@ -135,6 +135,13 @@ __device__ __forceinline__ void mma_bf16_ts(uint32_t d_tmem, uint32_t a_tmem, ui
       : "memory");
 }
 
+// Copy a 128-row x 256-bit slice of a shared-memory matrix (matrix descriptor) into TMEM:
+// row i to lane i, 8 columns.  With a K-major 128B-swizzled bf16 descriptor advanced by 32 B
+// per slice this lays a 128 x 64 tile out as the A operand of mma_bf16_ts.
+__device__ __forceinline__ void tmem_cp_128x256b(uint32_t taddr, uint64_t sdesc) {
+  asm volatile("tcgen05.cp.cta_group::1.128x256b [%0], %1;" ::"r"(taddr), "l"(sdesc) : "memory");
+}
+
 // Arrive (once) on the mbarrier when every tcgen05 operation issued so far by this thread
 // has completed.
 __device__ __forceinline__ void mma_commit(uint64_t* bar) {
