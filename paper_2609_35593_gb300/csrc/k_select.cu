@@ -277,48 +277,135 @@ __device__ __forceinline__ uint32_t order_key(float x) {
   return (b & 0x80000000u) ? ~b : (b | 0x80000000u);
 }
 
-// Exact top-m of kb[0..n) for one warp: the m largest keys, ties to the lower index.
-// With `member` set, only positions j whose bit in member[] equals `want` take part.
-// Requires m <= number of participating positions.  Result: bitmask sel[words].
-__device__ __forceinline__ bool takes_part(const uint32_t* member, bool want, int j) {
-  return member == nullptr || (((member[j >> 5] >> (j & 31)) & 1u) != 0) == want;
+// ------------------------------------------------------------------------------------
+// Exact top-m for one warp over a compact list of (key, block index) pairs held in shared
+// memory in ascending index order: the m largest keys, ties to the lower index (the order
+// the oracle uses).  Result: the chosen blocks' bits set in sel[words] (cleared first).
+//
+// 1. lower bound: the m-th largest value among every lane's local top-ceil(m/32) keys is
+//    <= the m-th largest key overall (those 32 ceil(m/32) values include m list entries);
+// 2. survivors: the entries >= that bound (usually about 1.5 m of them) are compacted into
+//    a short list, still in index order;
+// 3. the m-th largest survivor value T is found bit by bit (count of survivors >= T),
+//    and the survivors > T plus the lowest-index ones == T are chosen.
+// When m needs more than kTopK candidates per lane, or too many survivors tie at the
+// bound, step 3 runs on the whole list instead (same result, slower).
+// ------------------------------------------------------------------------------------
+constexpr int kTopK = 4;          // lane-local candidates: fast path for m <= 128
+constexpr int kSurvivors = 256;   // capacity of the survivor list
+
+// m-th largest of the values v[] (n of them per lane, up to N), bit by bit with early exit.
+template <int N>
+__device__ __forceinline__ uint32_t mth_largest(const uint32_t (&v)[N], int m) {
+  uint32_t lo = 0;
+  for (int bit = 31; bit >= 0; --bit) {
+    const uint32_t cand = lo | (1u << bit);
+    int cnt = 0;
+#pragma unroll
+    for (int k = 0; k < N; ++k) cnt += v[k] >= cand ? 1 : 0;
+    cnt = __reduce_add_sync(kFull, cnt);
+    if (cnt >= m) {
+      lo = cand;
+      if (cnt == m) break;
+    }
+  }
+  return lo;
 }
 
-__device__ void warp_topm(const uint32_t* kb, int n, int m, uint32_t* sel, int words,
-                          const uint32_t* member = nullptr, bool want = true) {
+// Exact selection on a list in shared memory (keys kk[0..n), indices ki[0..n)).
+__device__ void select_on_list(const uint32_t* kk, const uint16_t* ki, int n, int m, uint32_t* sel) {
   const int lane = threadIdx.x & 31;
   uint32_t lo = 0;
-  if (m > 0) {
-    for (int bit = 31; bit >= 0; --bit) {
-      const uint32_t cand = lo | (1u << bit);
-      int cnt = 0;
+  for (int bit = 31; bit >= 0; --bit) {
+    const uint32_t cand = lo | (1u << bit);
+    int cnt = 0;
 #pragma unroll 4
-      for (int j = lane; j < n; j += 32) cnt += (kb[j] >= cand && takes_part(member, want, j)) ? 1 : 0;
-      cnt = __reduce_add_sync(kFull, cnt);
-      if (cnt >= m) {
-        lo = cand;
-        if (cnt == m) break;
-      }
+    for (int x = lane; x < n; x += 32) cnt += kk[x] >= cand ? 1 : 0;
+    cnt = __reduce_add_sync(kFull, cnt);
+    if (cnt >= m) {
+      lo = cand;
+      if (cnt == m) break;
     }
   }
   int gt = 0;
 #pragma unroll 4
-  for (int j = lane; j < n; j += 32) gt += (kb[j] > lo && takes_part(member, want, j)) ? 1 : 0;
+  for (int x = lane; x < n; x += 32) gt += kk[x] > lo ? 1 : 0;
   gt = __reduce_add_sync(kFull, gt);
   const int need = m - gt;
   int taken = 0;
-  for (int w = 0; w < words; ++w) {
-    const int j = w * 32 + lane;
-    const bool part = j < n && takes_part(member, want, j);
-    const uint32_t v = part ? kb[j] : 0u;
-    const bool is_gt = m > 0 && part && v > lo;
-    const bool is_eq = m > 0 && part && v == lo;
+  for (int x0 = 0; x0 < n; x0 += 32) {
+    const int x = x0 + lane;
+    const uint32_t v = x < n ? kk[x] : 0u;
+    const bool is_eq = x < n && v == lo;
     const uint32_t eqb = __ballot_sync(kFull, is_eq);
     const int rank = taken + __popc(eqb & ((1u << lane) - 1u));
-    const uint32_t sb = __ballot_sync(kFull, is_gt || (is_eq && rank < need));
-    if (lane == 0) sel[w] = sb;
+    if ((x < n && v > lo) || (is_eq && rank < need)) {
+      const int j = ki[x];
+      atomicOr(&sel[j >> 5], 1u << (j & 31));
+    }
     taken += __popc(eqb);
   }
+}
+
+// kk/ki: the candidate list (n entries, ascending index, every key nonzero);
+// sk/si: survivor scratch of kSurvivors entries.  Requires 0 <= m <= n.
+__device__ void warp_topm(const uint32_t* kk, const uint16_t* ki, int n, int m, uint32_t* sel,
+                          int words, uint32_t* sk, uint16_t* si) {
+  const int lane = threadIdx.x & 31;
+  for (int w = lane; w < words; w += 32) sel[w] = 0u;
+  __syncwarp();
+  if (m <= 0) return;
+  if (m >= n) {  // everything is chosen
+    for (int x = lane; x < n; x += 32) atomicOr(&sel[ki[x] >> 5], 1u << (ki[x] & 31));
+    __syncwarp();
+    return;
+  }
+  const int K = (m + 31) / 32;
+  if (K > kTopK) {
+    select_on_list(kk, ki, n, m, sel);
+    __syncwarp();
+    return;
+  }
+  // 1. lane-local top-kTopK (descending), then the lower bound
+  uint32_t top[kTopK];
+#pragma unroll
+  for (int k = 0; k < kTopK; ++k) top[k] = 0u;
+  for (int x = lane; x < n; x += 32) {
+    uint32_t v = kk[x];
+#pragma unroll
+    for (int k = 0; k < kTopK; ++k) {
+      const uint32_t hi = max(top[k], v);
+      v = min(top[k], v);
+      top[k] = hi;
+    }
+  }
+  if (K < kTopK) {
+#pragma unroll
+    for (int k = 0; k < kTopK; ++k)
+      if (k >= K) top[k] = 0u;
+  }
+  const uint32_t bound = mth_largest(top, m);
+  // 2. survivors (>= bound), compacted in list order
+  int cnt = 0;
+  bool overflow = false;
+  for (int x0 = 0; x0 < n; x0 += 32) {
+    const int x = x0 + lane;
+    const bool keep = x < n && kk[x] >= bound;
+    const uint32_t b = __ballot_sync(kFull, keep);
+    const int pos = cnt + __popc(b & ((1u << lane) - 1u));
+    if (keep && pos < kSurvivors) {
+      sk[pos] = kk[x];
+      si[pos] = ki[x];
+    }
+    cnt += __popc(b);
+  }
+  overflow = cnt > kSurvivors;
+  __syncwarp();
+  // 3. exact selection on the survivors (or on the whole list if they did not fit)
+  if (overflow)
+    select_on_list(kk, ki, n, m, sel);
+  else
+    select_on_list(sk, si, cnt, m, sel);
   __syncwarp();
 }
 
@@ -337,7 +424,7 @@ __device__ __forceinline__ uint32_t valid_bits(int w, int n) {
 // g~ = sum_{j not in D} P_ij (z~_j - y~_i) and K = sum_{j not in D} P_ij for one row, by
 // one warp (lane owns channels 2*lane, 2*lane+1), in ascending j.  The kept blocks are
 // first compacted into idx[] (per-warp shared memory, >= nb entries) so that the loads of
-// eight blocks are in flight together.
+// sixteen blocks are in flight together.
 __device__ __forceinline__ void kept_drift(const uint32_t* D, const SelPtrs& p,
                                            const float* __restrict__ Prow,
                                            const float* __restrict__ zt, float y0, float y1,
@@ -351,11 +438,11 @@ __device__ __forceinline__ void kept_drift(const uint32_t* D, const SelPtrs& p,
   }
   __syncwarp();
   g0 = g1 = K = 0.f;
-  for (int k0 = 0; k0 < n; k0 += 8) {
-    float pj[8];
-    float2 z[8];
+  for (int k0 = 0; k0 < n; k0 += 16) {
+    float pj[16];
+    float2 z[16];
 #pragma unroll
-    for (int u = 0; u < 8; ++u) {
+    for (int u = 0; u < 16; ++u) {
       if (k0 + u < n) {
         const int j = idx[k0 + u];
         pj[u] = Prow[j];
@@ -363,7 +450,7 @@ __device__ __forceinline__ void kept_drift(const uint32_t* D, const SelPtrs& p,
       }
     }
 #pragma unroll
-    for (int u = 0; u < 8; ++u) {
+    for (int u = 0; u < 16; ++u) {
       if (k0 + u < n) {
         g0 = fmaf(pj[u], z[u].x - y0, g0);
         g1 = fmaf(pj[u], z[u].y - y1, g1);
@@ -372,6 +459,31 @@ __device__ __forceinline__ void kept_drift(const uint32_t* D, const SelPtrs& p,
     }
   }
   __syncwarp();
+}
+
+// Per-warp scratch after SelSmem: keys [ld] u32, indices [ld] u16, survivor keys
+// [kSurvivors] u32, survivor indices [kSurvivors] u16, bitmask words.
+__host__ __device__ constexpr size_t warp_scratch_words(int ld, int words_per_warp) {
+  return (size_t)ld + ld / 2 + kSurvivors + kSurvivors / 2 + words_per_warp;
+}
+
+struct WarpScratch {
+  uint32_t* kk;
+  uint16_t* ki;
+  uint32_t* sk;
+  uint16_t* si;
+  uint32_t* words;
+};
+
+__device__ __forceinline__ WarpScratch warp_scratch(unsigned char* base, int warp, int ld, int wpw) {
+  uint32_t* w0 = reinterpret_cast<uint32_t*>(base) + (size_t)warp * warp_scratch_words(ld, wpw);
+  WarpScratch ws;
+  ws.kk = w0;
+  ws.ki = reinterpret_cast<uint16_t*>(w0 + ld);
+  ws.sk = w0 + ld + ld / 2;
+  ws.si = reinterpret_cast<uint16_t*>(ws.sk + kSurvivors);
+  ws.words = ws.sk + kSurvivors + kSurvivors / 2;
+  return ws;
 }
 
 // ------------------------------------------------------------------------------------
@@ -385,8 +497,6 @@ struct Budgets {
 __global__ void __launch_bounds__(kThreads, 2) k_score(SelPtrs p, Budgets bud) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
   SelSmem& S = *reinterpret_cast<SelSmem*>(smem_raw);
-  uint32_t* kb_all = reinterpret_cast<uint32_t*>(smem_raw + sizeof(SelSmem));
-  uint32_t* sel_all = kb_all + 8 * p.ld;
   const int h = blockIdx.y, i0 = blockIdx.x * RT;
   const int nrows = min(RT, p.ncand - i0);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -514,8 +624,8 @@ __global__ void __launch_bounds__(kThreads, 2) k_score(SelPtrs p, Budgets bud) {
   }
 
   // ---- initial selection (Eq. 7) and the state of Eq. 10-12, one warp per row --------
-  uint32_t* kb = kb_all + warp * p.ld;
-  uint32_t* sel = sel_all + warp * p.words;
+  WarpScratch W = warp_scratch(smem_raw + sizeof(SelSmem), warp, p.ld, p.words);
+  uint32_t* sel = W.words;
   const int c = bud.c[h];
   for (int r = warp; r < nrows; r += 8) {
     const int i = i0 + r;
@@ -525,10 +635,11 @@ __global__ void __launch_bounds__(kThreads, 2) k_score(SelPtrs p, Budgets bud) {
     for (int j = lane; j < p.ncand; j += 32) {
       const float pj = Prow[j];
       const float key = pj * sqrtf(qrow[j]) / fmaxf(1.0f - pj, kEps);
-      kb[j] = order_key(key);
+      W.kk[j] = order_key(key);
+      W.ki[j] = (uint16_t)j;
     }
     __syncwarp();
-    warp_topm(kb, p.ncand, c, sel, p.words);  // sel = kept candidates
+    warp_topm(W.kk, W.ki, p.ncand, c, sel, p.words, W.sk, W.si);  // sel = kept candidates
     // drop set D0 = candidates not kept
     for (int w = lane; w < p.words; w += 32) {
       const uint32_t d = valid_bits(w, p.ncand) & ~sel[w];
@@ -538,7 +649,7 @@ __global__ void __launch_bounds__(kThreads, 2) k_score(SelPtrs p, Budgets bud) {
     }
     __syncwarp();
     float g0, g1, K;
-    kept_drift(sel, p, Prow, zt_h, S.A[r][2 * lane], S.A[r][2 * lane + 1], kb, g0, g1, K);
+    kept_drift(sel, p, Prow, zt_h, S.A[r][2 * lane], S.A[r][2 * lane + 1], W.kk, g0, g1, K);
     const float G = warp_sum(g0 * g0 + g1 * g1);
     const float Kc = fmaxf(K, kEps);
     const float J = G / (Kc * Kc);
@@ -561,7 +672,7 @@ __device__ __forceinline__ float delta_J(float G, float K, float dG, float u) {
   const float K2 = K + u;
   if (K >= kEps && K2 >= kEps) {
     const float num = fmaf(G * u, 2.0f * K + u, -dG * (K * K));
-    return num / ((K * K) * (K2 * K2));
+    return __fdividef(num, (K * K) * (K2 * K2));
   }
   const float Kc = fmaxf(K, kEps), K2c = fmaxf(K2, kEps);
   return G / (Kc * Kc) - (G + dG) / (K2c * K2c);
@@ -575,8 +686,6 @@ __global__ void __launch_bounds__(kThreads, 2) k_round(SelPtrs p, Budgets bud, i
                                                        float rho) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
   SelSmem& S = *reinterpret_cast<SelSmem*>(smem_raw);
-  uint32_t* kb_all = reinterpret_cast<uint32_t*>(smem_raw + sizeof(SelSmem));
-  uint32_t* sel_all = kb_all + 8 * p.ld;
   const int h = blockIdx.y, i0 = blockIdx.x * RT;
   const int c = bud.c[h];
   // Eq. 17: m_r = floor(rho c_h / 2^(r+1)), capped by |D| and |P \ D|
@@ -610,11 +719,11 @@ __global__ void __launch_bounds__(kThreads, 2) k_round(SelPtrs p, Budgets bud, i
   }
 
   // ---- per row: exact top-m restores and drops, update, track-best ------------------
-  uint32_t* kb = kb_all + warp * p.ld;
-  uint32_t* sel = sel_all + warp * (3 * p.words);
-  uint32_t* Dw = sel;                // current drop set
-  uint32_t* Rw = sel + p.words;      // chosen restores
-  uint32_t* Xw = sel + 2 * p.words;  // chosen drops
+  WarpScratch W = warp_scratch(smem_raw + sizeof(SelSmem), warp, p.ld, 3 * p.words);
+  uint32_t* Dw = W.words;            // current drop set
+  uint32_t* Rw = W.words + p.words;  // chosen restores
+  uint32_t* Xw = Rw + p.words;       // chosen drops
+  const int base_drop = p.ncand - c; // |D|: the restore list fills [0, |D|), drops follow
   for (int r = warp; r < nrows; r += 8) {
     const int i = i0 + r;
     const int64_t ri = hrow + i;
@@ -626,24 +735,45 @@ __global__ void __launch_bounds__(kThreads, 2) k_round(SelPtrs p, Budgets bud, i
     __syncwarp();
     // one pass over the candidates: a block k in D is a restore candidate (u = +P_k,
     // dG = -2 P_k t_k + P_k^2 q_k, Eq. 13-14), a kept candidate a drop candidate (u = -P_k,
-    // dG = +2 P_k t_k + P_k^2 q_k, Eq. 15); the key is the exact decrease of J (Eq. 16)
-#pragma unroll 4
-    for (int j = lane; j < p.ncand; j += 32) {
-      const float pj = Prow[j], qj = qrow[j], tj = trow[j];
-      const bool inD = (Dw[j >> 5] >> (j & 31)) & 1u;
-      const float s2 = pj * pj * qj;
-      const float dG = inD ? fmaf(-2.0f * pj, tj, s2) : fmaf(2.0f * pj, tj, s2);
-      kb[j] = order_key(delta_J(G, K, dG, inD ? pj : -pj));
+    // dG = +2 P_k t_k + P_k^2 q_k, Eq. 15); the key is the exact decrease of J (Eq. 16).
+    // The two kinds go to two lists, each in ascending block order.
+    int nr = 0, nd = 0;
+#pragma unroll 2
+    for (int j0 = 0; j0 < p.ncand; j0 += 32) {
+      const int j = j0 + lane;
+      const bool valid = j < p.ncand;
+      const bool inD = valid && ((Dw[j >> 5] >> (j & 31)) & 1u);
+      uint32_t key = 0u;
+      if (valid) {
+        const float pj = Prow[j], qj = qrow[j], tj = trow[j];
+        const float s2 = pj * pj * qj;
+        const float dG = inD ? fmaf(-2.0f * pj, tj, s2) : fmaf(2.0f * pj, tj, s2);
+        key = order_key(delta_J(G, K, dG, inD ? pj : -pj));
+      }
+      const uint32_t br = __ballot_sync(kFull, inD);
+      const uint32_t bd = __ballot_sync(kFull, valid && !inD);
+      const uint32_t lt = (1u << lane) - 1u;
+      if (inD) {
+        const int pos = nr + __popc(br & lt);
+        W.kk[pos] = key;
+        W.ki[pos] = (uint16_t)j;
+      } else if (valid) {
+        const int pos = base_drop + nd + __popc(bd & lt);
+        W.kk[pos] = key;
+        W.ki[pos] = (uint16_t)j;
+      }
+      nr += __popc(br);
+      nd += __popc(bd);
     }
     __syncwarp();
-    warp_topm(kb, p.ncand, m, Rw, p.words, Dw, true);
-    warp_topm(kb, p.ncand, m, Xw, p.words, Dw, false);
+    warp_topm(W.kk, W.ki, nr, m, Rw, p.words, W.sk, W.si);
+    warp_topm(W.kk + base_drop, W.ki + base_drop, nd, m, Xw, p.words, W.sk, W.si);
     for (int w = lane; w < p.words; w += 32) Dw[w] = (Dw[w] & ~Rw[w]) | Xw[w];
     __syncwarp();
     // exact state of the new set (Eq. 10-12)
     const float y0 = p.ytil[ri * 64 + 2 * lane], y1 = p.ytil[ri * 64 + 2 * lane + 1];
     float g0, g1, Kn;
-    kept_drift(Dw, p, Prow, zt_h, y0, y1, kb, g0, g1, Kn);
+    kept_drift(Dw, p, Prow, zt_h, y0, y1, W.kk, g0, g1, Kn);
     const float Gn = warp_sum(g0 * g0 + g1 * g1);
     const float Kc = fmaxf(Kn, kEps);
     const float Jn = Gn / (Kc * Kc);
@@ -706,7 +836,7 @@ __global__ void k_csr(SelPtrs p, Budgets bud, CsrBases cb, int H, int32_t* __res
 // launchers
 // ------------------------------------------------------------------------------------
 static size_t sel_smem_bytes(const Shape& s, int words_per_warp) {
-  return sizeof(SelSmem) + (size_t)8 * s.ld * 4 + (size_t)8 * words_per_warp * 4;
+  return sizeof(SelSmem) + (size_t)8 * warp_scratch_words(s.ld, words_per_warp) * 4;
 }
 
 cudaError_t launch_prepare_wo(const Shape& s, const uint16_t* W_o, float* F, cudaStream_t st) {
