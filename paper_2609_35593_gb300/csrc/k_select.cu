@@ -13,6 +13,7 @@
 // of the drop set is minus that of the kept set, which is the smaller one at high sparsity.
 
 #include <math.h>
+#include <stddef.h>
 
 #include "ress_internal.cuh"
 
@@ -278,23 +279,28 @@ __device__ __forceinline__ uint32_t order_key(float x) {
 }
 
 // ------------------------------------------------------------------------------------
-// Exact top-m for one warp over a compact list of (key, block index) pairs held in shared
-// memory in ascending index order: the m largest keys, ties to the lower index (the order
-// the oracle uses).  Result: the chosen blocks' bits set in sel[words] (cleared first).
+// Exact top-m for one warp over keys kk[0..n) in shared memory (block j has key kk[j]):
+// the m largest keys, ties to the lower block index (the order the oracle uses).  With
+// `member` set, only blocks whose bit in member[] equals `want` take part.  Result: the
+// chosen blocks' bits in sel[words] (cleared first).
 //
 // 1. lower bound: the m-th largest value among every lane's local top-ceil(m/32) keys is
-//    <= the m-th largest key overall (those 32 ceil(m/32) values include m list entries);
-// 2. survivors: the entries >= that bound (usually about 1.5 m of them) are compacted into
-//    a short list, still in index order;
-// 3. the m-th largest survivor value T is found bit by bit (count of survivors >= T),
-//    and the survivors > T plus the lowest-index ones == T are chosen.
-// When m needs more than kTopK candidates per lane, or too many survivors tie at the
-// bound, step 3 runs on the whole list instead (same result, slower).
+//    <= the m-th largest key overall (those 32 ceil(m/32) values include m entries);
+// 2. survivors: the participating keys >= that bound (usually about 1.5 m of them) are
+//    compacted, in block order, into a short list;
+// 3. the m-th largest survivor T is found bit by bit (count of survivors >= T), and the
+//    survivors > T plus the lowest-index ones == T are chosen.
+// When m needs more than kTopK candidates per lane, or too many keys tie at the bound,
+// step 3 runs on all participating keys instead (same result, slower).
 // ------------------------------------------------------------------------------------
 constexpr int kTopK = 4;          // lane-local candidates: fast path for m <= 128
 constexpr int kSurvivors = 256;   // capacity of the survivor list
 
-// m-th largest of the values v[] (n of them per lane, up to N), bit by bit with early exit.
+__device__ __forceinline__ bool takes_part(const uint32_t* member, bool want, int j) {
+  return member == nullptr || (((member[j >> 5] >> (j & 31)) & 1u) != 0) == want;
+}
+
+// m-th largest of the values v[] (up to N per lane), bit by bit with early exit.
 template <int N>
 __device__ __forceinline__ uint32_t mth_largest(const uint32_t (&v)[N], int m) {
   uint32_t lo = 0;
@@ -312,15 +318,18 @@ __device__ __forceinline__ uint32_t mth_largest(const uint32_t (&v)[N], int m) {
   return lo;
 }
 
-// Exact selection on a list in shared memory (keys kk[0..n), indices ki[0..n)).
-__device__ void select_on_list(const uint32_t* kk, const uint16_t* ki, int n, int m, uint32_t* sel) {
+// Exact selection over a list of n (key, index) pairs in ascending index order; with `member`
+// the list is kk itself (index = position) filtered by membership, otherwise (sk, si).
+__device__ void select_exact(const uint32_t* keys, const uint16_t* idx, int n, int m,
+                             const uint32_t* member, bool want, uint32_t* sel) {
   const int lane = threadIdx.x & 31;
+  auto part = [&](int x) { return idx != nullptr || takes_part(member, want, x); };
   uint32_t lo = 0;
   for (int bit = 31; bit >= 0; --bit) {
     const uint32_t cand = lo | (1u << bit);
     int cnt = 0;
 #pragma unroll 4
-    for (int x = lane; x < n; x += 32) cnt += kk[x] >= cand ? 1 : 0;
+    for (int x = lane; x < n; x += 32) cnt += (keys[x] >= cand && part(x)) ? 1 : 0;
     cnt = __reduce_add_sync(kFull, cnt);
     if (cnt >= m) {
       lo = cand;
@@ -329,49 +338,46 @@ __device__ void select_on_list(const uint32_t* kk, const uint16_t* ki, int n, in
   }
   int gt = 0;
 #pragma unroll 4
-  for (int x = lane; x < n; x += 32) gt += kk[x] > lo ? 1 : 0;
+  for (int x = lane; x < n; x += 32) gt += (keys[x] > lo && part(x)) ? 1 : 0;
   gt = __reduce_add_sync(kFull, gt);
   const int need = m - gt;
   int taken = 0;
   for (int x0 = 0; x0 < n; x0 += 32) {
     const int x = x0 + lane;
-    const uint32_t v = x < n ? kk[x] : 0u;
-    const bool is_eq = x < n && v == lo;
+    const bool in = x < n && part(x);
+    const uint32_t v = in ? keys[x] : 0u;
+    const bool is_eq = in && v == lo;
     const uint32_t eqb = __ballot_sync(kFull, is_eq);
     const int rank = taken + __popc(eqb & ((1u << lane) - 1u));
-    if ((x < n && v > lo) || (is_eq && rank < need)) {
-      const int j = ki[x];
+    if ((in && v > lo) || (is_eq && rank < need)) {
+      const int j = idx ? (int)idx[x] : x;
       atomicOr(&sel[j >> 5], 1u << (j & 31));
     }
     taken += __popc(eqb);
   }
 }
 
-// kk/ki: the candidate list (n entries, ascending index, every key nonzero);
-// sk/si: survivor scratch of kSurvivors entries.  Requires 0 <= m <= n.
-__device__ void warp_topm(const uint32_t* kk, const uint16_t* ki, int n, int m, uint32_t* sel,
-                          int words, uint32_t* sk, uint16_t* si) {
+// Requires m <= number of participating blocks.  sk/si: survivor scratch (kSurvivors).
+__device__ void warp_topm(const uint32_t* kk, int n, int m, uint32_t* sel, int words,
+                          uint32_t* sk, uint16_t* si, const uint32_t* member = nullptr,
+                          bool want = true) {
   const int lane = threadIdx.x & 31;
   for (int w = lane; w < words; w += 32) sel[w] = 0u;
   __syncwarp();
   if (m <= 0) return;
-  if (m >= n) {  // everything is chosen
-    for (int x = lane; x < n; x += 32) atomicOr(&sel[ki[x] >> 5], 1u << (ki[x] & 31));
-    __syncwarp();
-    return;
-  }
   const int K = (m + 31) / 32;
   if (K > kTopK) {
-    select_on_list(kk, ki, n, m, sel);
+    select_exact(kk, nullptr, n, m, member, want, sel);
     __syncwarp();
     return;
   }
-  // 1. lane-local top-kTopK (descending), then the lower bound
+  // 1. lane-local top-kTopK (descending) of the participating keys, then the lower bound
   uint32_t top[kTopK];
 #pragma unroll
   for (int k = 0; k < kTopK; ++k) top[k] = 0u;
+#pragma unroll 2
   for (int x = lane; x < n; x += 32) {
-    uint32_t v = kk[x];
+    uint32_t v = takes_part(member, want, x) ? kk[x] : 0u;
 #pragma unroll
     for (int k = 0; k < kTopK; ++k) {
       const uint32_t hi = max(top[k], v);
@@ -379,33 +385,29 @@ __device__ void warp_topm(const uint32_t* kk, const uint16_t* ki, int n, int m, 
       top[k] = hi;
     }
   }
-  if (K < kTopK) {
 #pragma unroll
-    for (int k = 0; k < kTopK; ++k)
-      if (k >= K) top[k] = 0u;
-  }
+  for (int k = 0; k < kTopK; ++k)
+    if (k >= K) top[k] = 0u;
   const uint32_t bound = mth_largest(top, m);
-  // 2. survivors (>= bound), compacted in list order
+  // 2. survivors (participating, >= bound), compacted in block order
   int cnt = 0;
-  bool overflow = false;
   for (int x0 = 0; x0 < n; x0 += 32) {
     const int x = x0 + lane;
-    const bool keep = x < n && kk[x] >= bound;
+    const bool keep = x < n && kk[x] >= bound && takes_part(member, want, x);
     const uint32_t b = __ballot_sync(kFull, keep);
     const int pos = cnt + __popc(b & ((1u << lane) - 1u));
     if (keep && pos < kSurvivors) {
       sk[pos] = kk[x];
-      si[pos] = ki[x];
+      si[pos] = (uint16_t)x;
     }
     cnt += __popc(b);
   }
-  overflow = cnt > kSurvivors;
   __syncwarp();
-  // 3. exact selection on the survivors (or on the whole list if they did not fit)
-  if (overflow)
-    select_on_list(kk, ki, n, m, sel);
+  // 3. exact selection on the survivors (or on every participating key if they overflowed)
+  if (cnt > kSurvivors)
+    select_exact(kk, nullptr, n, m, member, want, sel);
   else
-    select_on_list(sk, si, cnt, m, sel);
+    select_exact(sk, si, cnt, m, nullptr, true, sel);
   __syncwarp();
 }
 
@@ -461,29 +463,42 @@ __device__ __forceinline__ void kept_drift(const uint32_t* D, const SelPtrs& p,
   __syncwarp();
 }
 
-// Per-warp scratch after SelSmem: keys [ld] u32, indices [ld] u16, survivor keys
-// [kSurvivors] u32, survivor indices [kSurvivors] u16, bitmask words.
+// Per-warp scratch of the per-row phase: keys [ld] u32, survivor keys [kSurvivors] u32,
+// survivor indices [kSurvivors] u16, bitmask words.  It reuses the GEMM staging area (B,
+// Pc), which the per-row phase no longer needs, when that area is large enough.
 __host__ __device__ constexpr size_t warp_scratch_words(int ld, int words_per_warp) {
-  return (size_t)ld + ld / 2 + kSurvivors + kSurvivors / 2 + words_per_warp;
+  return (size_t)ld + kSurvivors + kSurvivors / 2 + words_per_warp;
 }
 
 struct WarpScratch {
   uint32_t* kk;
-  uint16_t* ki;
   uint32_t* sk;
   uint16_t* si;
   uint32_t* words;
 };
 
-__device__ __forceinline__ WarpScratch warp_scratch(unsigned char* base, int warp, int ld, int wpw) {
-  uint32_t* w0 = reinterpret_cast<uint32_t*>(base) + (size_t)warp * warp_scratch_words(ld, wpw);
+// Offset of the per-warp scratch from the start of SelSmem.
+__host__ __device__ inline size_t scratch_offset(int ld, int wpw) {
+  const size_t need = (size_t)8 * warp_scratch_words(ld, wpw) * 4;
+  const size_t staged = sizeof(SelSmem) - offsetof(SelSmem, B);
+  return need <= staged ? offsetof(SelSmem, B) : sizeof(SelSmem);
+}
+
+__device__ __forceinline__ WarpScratch warp_scratch(unsigned char* smem, int warp, int ld, int wpw) {
+  uint32_t* w0 = reinterpret_cast<uint32_t*>(smem + scratch_offset(ld, wpw)) +
+                 (size_t)warp * warp_scratch_words(ld, wpw);
   WarpScratch ws;
   ws.kk = w0;
-  ws.ki = reinterpret_cast<uint16_t*>(w0 + ld);
-  ws.sk = w0 + ld + ld / 2;
+  ws.sk = w0 + ld;
   ws.si = reinterpret_cast<uint16_t*>(ws.sk + kSurvivors);
   ws.words = ws.sk + kSurvivors + kSurvivors / 2;
   return ws;
+}
+
+static size_t sel_smem_bytes(const Shape& s, int words_per_warp) {
+  const size_t end = scratch_offset(s.ld, words_per_warp) +
+                     (size_t)8 * warp_scratch_words(s.ld, words_per_warp) * 4;
+  return end > sizeof(SelSmem) ? end : sizeof(SelSmem);
 }
 
 // ------------------------------------------------------------------------------------
@@ -624,7 +639,7 @@ __global__ void __launch_bounds__(kThreads, 2) k_score(SelPtrs p, Budgets bud) {
   }
 
   // ---- initial selection (Eq. 7) and the state of Eq. 10-12, one warp per row --------
-  WarpScratch W = warp_scratch(smem_raw + sizeof(SelSmem), warp, p.ld, p.words);
+  WarpScratch W = warp_scratch(smem_raw, warp, p.ld, p.words);
   uint32_t* sel = W.words;
   const int c = bud.c[h];
   for (int r = warp; r < nrows; r += 8) {
@@ -636,10 +651,9 @@ __global__ void __launch_bounds__(kThreads, 2) k_score(SelPtrs p, Budgets bud) {
       const float pj = Prow[j];
       const float key = pj * sqrtf(qrow[j]) / fmaxf(1.0f - pj, kEps);
       W.kk[j] = order_key(key);
-      W.ki[j] = (uint16_t)j;
     }
     __syncwarp();
-    warp_topm(W.kk, W.ki, p.ncand, c, sel, p.words, W.sk, W.si);  // sel = kept candidates
+    warp_topm(W.kk, p.ncand, c, sel, p.words, W.sk, W.si);  // sel = kept candidates
     // drop set D0 = candidates not kept
     for (int w = lane; w < p.words; w += 32) {
       const uint32_t d = valid_bits(w, p.ncand) & ~sel[w];
@@ -719,11 +733,10 @@ __global__ void __launch_bounds__(kThreads, 2) k_round(SelPtrs p, Budgets bud, i
   }
 
   // ---- per row: exact top-m restores and drops, update, track-best ------------------
-  WarpScratch W = warp_scratch(smem_raw + sizeof(SelSmem), warp, p.ld, 3 * p.words);
+  WarpScratch W = warp_scratch(smem_raw, warp, p.ld, 3 * p.words);
   uint32_t* Dw = W.words;            // current drop set
   uint32_t* Rw = W.words + p.words;  // chosen restores
   uint32_t* Xw = Rw + p.words;       // chosen drops
-  const int base_drop = p.ncand - c; // |D|: the restore list fills [0, |D|), drops follow
   for (int r = warp; r < nrows; r += 8) {
     const int i = i0 + r;
     const int64_t ri = hrow + i;
@@ -735,39 +748,18 @@ __global__ void __launch_bounds__(kThreads, 2) k_round(SelPtrs p, Budgets bud, i
     __syncwarp();
     // one pass over the candidates: a block k in D is a restore candidate (u = +P_k,
     // dG = -2 P_k t_k + P_k^2 q_k, Eq. 13-14), a kept candidate a drop candidate (u = -P_k,
-    // dG = +2 P_k t_k + P_k^2 q_k, Eq. 15); the key is the exact decrease of J (Eq. 16).
-    // The two kinds go to two lists, each in ascending block order.
-    int nr = 0, nd = 0;
-#pragma unroll 2
-    for (int j0 = 0; j0 < p.ncand; j0 += 32) {
-      const int j = j0 + lane;
-      const bool valid = j < p.ncand;
-      const bool inD = valid && ((Dw[j >> 5] >> (j & 31)) & 1u);
-      uint32_t key = 0u;
-      if (valid) {
-        const float pj = Prow[j], qj = qrow[j], tj = trow[j];
-        const float s2 = pj * pj * qj;
-        const float dG = inD ? fmaf(-2.0f * pj, tj, s2) : fmaf(2.0f * pj, tj, s2);
-        key = order_key(delta_J(G, K, dG, inD ? pj : -pj));
-      }
-      const uint32_t br = __ballot_sync(kFull, inD);
-      const uint32_t bd = __ballot_sync(kFull, valid && !inD);
-      const uint32_t lt = (1u << lane) - 1u;
-      if (inD) {
-        const int pos = nr + __popc(br & lt);
-        W.kk[pos] = key;
-        W.ki[pos] = (uint16_t)j;
-      } else if (valid) {
-        const int pos = base_drop + nd + __popc(bd & lt);
-        W.kk[pos] = key;
-        W.ki[pos] = (uint16_t)j;
-      }
-      nr += __popc(br);
-      nd += __popc(bd);
+    // dG = +2 P_k t_k + P_k^2 q_k, Eq. 15); the key is the exact decrease of J (Eq. 16)
+#pragma unroll 4
+    for (int j = lane; j < p.ncand; j += 32) {
+      const float pj = Prow[j], qj = qrow[j], tj = trow[j];
+      const bool inD = (Dw[j >> 5] >> (j & 31)) & 1u;
+      const float s2 = pj * pj * qj;
+      const float dG = inD ? fmaf(-2.0f * pj, tj, s2) : fmaf(2.0f * pj, tj, s2);
+      W.kk[j] = order_key(delta_J(G, K, dG, inD ? pj : -pj));
     }
     __syncwarp();
-    warp_topm(W.kk, W.ki, nr, m, Rw, p.words, W.sk, W.si);
-    warp_topm(W.kk + base_drop, W.ki + base_drop, nd, m, Xw, p.words, W.sk, W.si);
+    warp_topm(W.kk, p.ncand, m, Rw, p.words, W.sk, W.si, Dw, true);
+    warp_topm(W.kk, p.ncand, m, Xw, p.words, W.sk, W.si, Dw, false);
     for (int w = lane; w < p.words; w += 32) Dw[w] = (Dw[w] & ~Rw[w]) | Xw[w];
     __syncwarp();
     // exact state of the new set (Eq. 10-12)
@@ -835,9 +827,6 @@ __global__ void k_csr(SelPtrs p, Budgets bud, CsrBases cb, int H, int32_t* __res
 // ------------------------------------------------------------------------------------
 // launchers
 // ------------------------------------------------------------------------------------
-static size_t sel_smem_bytes(const Shape& s, int words_per_warp) {
-  return sizeof(SelSmem) + (size_t)8 * warp_scratch_words(s.ld, words_per_warp) * 4;
-}
 
 cudaError_t launch_prepare_wo(const Shape& s, const uint16_t* W_o, float* F, cudaStream_t st) {
   k_prepare_wo<<<s.H, kThreads, 0, st>>>(W_o, s.d_model, s.H, F);
