@@ -495,11 +495,6 @@ __device__ __forceinline__ WarpScratch warp_scratch(unsigned char* smem, int war
   return ws;
 }
 
-static size_t sel_smem_bytes(const Shape& s, int words_per_warp) {
-  const size_t end = scratch_offset(s.ld, words_per_warp) +
-                     (size_t)8 * warp_scratch_words(s.ld, words_per_warp) * 4;
-  return end > sizeof(SelSmem) ? end : sizeof(SelSmem);
-}
 
 // ------------------------------------------------------------------------------------
 // Score kernel: Sec. 4.1-4.2 and the initial state of Sec. 4.3 for RT query rows of one
@@ -638,45 +633,6 @@ __global__ void __launch_bounds__(kThreads, 2) k_score(SelPtrs p, Budgets bud) {
     __syncthreads();
   }
 
-  // ---- initial selection (Eq. 7) and the state of Eq. 10-12, one warp per row --------
-  WarpScratch W = warp_scratch(smem_raw, warp, p.ld, p.words);
-  uint32_t* sel = W.words;
-  const int c = bud.c[h];
-  for (int r = warp; r < nrows; r += 8) {
-    const int i = i0 + r;
-    const float* Prow = Pbase + (int64_t)r * p.ld;
-    const float* qrow = qbase + (int64_t)r * p.ld;
-#pragma unroll 4
-    for (int j = lane; j < p.ncand; j += 32) {
-      const float pj = Prow[j];
-      const float key = pj * sqrtf(qrow[j]) / fmaxf(1.0f - pj, kEps);
-      W.kk[j] = order_key(key);
-    }
-    __syncwarp();
-    warp_topm(W.kk, p.ncand, c, sel, p.words, W.sk, W.si);  // sel = kept candidates
-    // drop set D0 = candidates not kept
-    for (int w = lane; w < p.words; w += 32) {
-      const uint32_t d = valid_bits(w, p.ncand) & ~sel[w];
-      sel[w] = d;
-      p.dmask[(hrow + i) * p.words + w] = d;
-      p.bmask[(hrow + i) * p.words + w] = d;
-    }
-    __syncwarp();
-    float g0, g1, K;
-    kept_drift(sel, p, Prow, zt_h, S.A[r][2 * lane], S.A[r][2 * lane + 1], W.kk, g0, g1, K);
-    const float G = warp_sum(g0 * g0 + g1 * g1);
-    const float Kc = fmaxf(K, kEps);
-    const float J = G / (Kc * Kc);
-    *reinterpret_cast<float2*>(p.gtil + (hrow + i) * 64 + 2 * lane) = make_float2(g0, g1);
-    if (lane == 0) {
-      p.K[hrow + i] = K;
-      p.G[hrow + i] = G;
-      p.J[hrow + i] = J;
-      p.Jbest[hrow + i] = J;
-      p.J0[hrow + i] = J;
-    }
-    __syncwarp();
-  }
 }
 
 // Exact decrease of J (Eq. 16) when G changes by dG and K by u, with the denominators
@@ -692,20 +648,93 @@ __device__ __forceinline__ float delta_J(float G, float K, float dG, float u) {
   return G / (Kc * Kc) - (G + dG) / (K2c * K2c);
 }
 
+
 // ------------------------------------------------------------------------------------
-// Restoration round r (Sec. 4.3, Eq. 13-17) for RT rows of one head.
-// grid (ceil(ncand / RT), H).
+// Per-row kernels: one warp per candidate query row, 4 rows per CTA.  They hold few
+// registers so that many warps share an SM and hide the latency of the row's loads.
+// ------------------------------------------------------------------------------------
+constexpr int kRowWarps = 4;
+
+// Candidate keys of one row, four blocks per lane and load (rows are 16-byte aligned and
+// padded to a multiple of 32 entries).
+template <typename KeyFn>
+__device__ __forceinline__ void row_keys(int n, uint32_t* kk, KeyFn key_of) {
+  const int lane = threadIdx.x & 31;
+#pragma unroll 2
+  for (int j4 = 4 * lane; j4 < n; j4 += 128) {
+    uint32_t k4[4];
+    key_of(j4, k4);
+#pragma unroll
+    for (int u = 0; u < 4; ++u)
+      if (j4 + u < n) kk[j4 + u] = k4[u];
+  }
+  __syncwarp();
+}
+
+// Initial selection (Eq. 7) and the state of Eq. 10-12.  grid (ceil(|P| / 4), H).
+__global__ void __launch_bounds__(32 * kRowWarps, 8) k_score_rows(SelPtrs p, Budgets bud) {
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int h = blockIdx.y, i = blockIdx.x * kRowWarps + warp;
+  if (i >= p.ncand) return;
+  const int64_t ri = (int64_t)h * p.nb + i;
+  const float* Prow = p.P + ri * p.ld;
+  const float* qrow = p.q + ri * p.ld;
+  const float* zt_h = p.ztil + (int64_t)h * p.nb * 64;
+  uint32_t* base = reinterpret_cast<uint32_t*>(smem_raw) + (size_t)warp * warp_scratch_words(p.ld, p.words);
+  uint32_t* kk = base;
+  uint32_t* sk = base + p.ld;
+  uint16_t* si = reinterpret_cast<uint16_t*>(sk + kSurvivors);
+  uint32_t* sel = sk + kSurvivors + kSurvivors / 2;
+  row_keys(p.ncand, kk, [&](int j, uint32_t (&k4)[4]) {
+    const float4 P4 = *reinterpret_cast<const float4*>(Prow + j);
+    const float4 q4 = *reinterpret_cast<const float4*>(qrow + j);
+    const float pv[4] = {P4.x, P4.y, P4.z, P4.w}, qv[4] = {q4.x, q4.y, q4.z, q4.w};
+#pragma unroll
+    for (int u = 0; u < 4; ++u)  // s_ij / max(1 - P_ij, eps), s_ij = P_ij sqrt(q_ij)
+      k4[u] = order_key(pv[u] * sqrtf(qv[u]) / fmaxf(1.0f - pv[u], kEps));
+  });
+  warp_topm(kk, p.ncand, bud.c[h], sel, p.words, sk, si);  // sel = kept candidates
+  // drop set D0 = candidates not kept
+  for (int w = lane; w < p.words; w += 32) {
+    const uint32_t d = valid_bits(w, p.ncand) & ~sel[w];
+    sel[w] = d;
+    p.dmask[ri * p.words + w] = d;
+    p.bmask[ri * p.words + w] = d;
+  }
+  __syncwarp();
+  const float2 y = *reinterpret_cast<const float2*>(p.ytil + ri * 64 + 2 * lane);
+  float g0, g1, K;
+  kept_drift(sel, p, Prow, zt_h, y.x, y.y, kk, g0, g1, K);
+  const float G = warp_sum(g0 * g0 + g1 * g1);
+  const float Kc = fmaxf(K, kEps);
+  const float J = G / (Kc * Kc);
+  *reinterpret_cast<float2*>(p.gtil + ri * 64 + 2 * lane) = make_float2(g0, g1);
+  if (lane == 0) {
+    p.K[ri] = K;
+    p.G[ri] = G;
+    p.J[ri] = J;
+    p.Jbest[ri] = J;
+    p.J0[ri] = J;
+  }
+}
+
+// Swap count of round r (Eq. 17): floor(rho c_h / 2^(r+1)), capped by |D| and |P \ D|.
+__device__ __forceinline__ int swap_count(int c, int ncand, int round, float rho) {
+  const int m = (int)floor((double)rho * (double)c / (double)(1ull << (round + 1)));
+  return min(m, min(ncand - c, c));
+}
+
+// ------------------------------------------------------------------------------------
+// Restoration round r (Sec. 4.3, Eq. 13-17), first half: the gain inner products
+// t_ij = (y~_i - z~_j) . g~_i for RT rows of one head.  grid (ceil(ncand / RT), H).
 // ------------------------------------------------------------------------------------
 __global__ void __launch_bounds__(kThreads, 2) k_round(SelPtrs p, Budgets bud, int round,
                                                        float rho) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
   SelSmem& S = *reinterpret_cast<SelSmem*>(smem_raw);
   const int h = blockIdx.y, i0 = blockIdx.x * RT;
-  const int c = bud.c[h];
-  // Eq. 17: m_r = floor(rho c_h / 2^(r+1)), capped by |D| and |P \ D|
-  int m = (int)floor((double)rho * (double)c / (double)(1ull << (round + 1)));
-  m = min(m, min(p.ncand - c, c));
-  if (m <= 0) return;
+  if (swap_count(bud.c[h], p.ncand, round, rho) <= 0) return;
   const int nrows = min(RT, p.ncand - i0);
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int rg = warp & 3, jb = (warp >> 2) * 64 + lane;
@@ -732,57 +761,72 @@ __global__ void __launch_bounds__(kThreads, 2) k_round(SelPtrs p, Budgets bud, i
     __syncthreads();
   }
 
-  // ---- per row: exact top-m restores and drops, update, track-best ------------------
-  WarpScratch W = warp_scratch(smem_raw, warp, p.ld, 3 * p.words);
-  uint32_t* Dw = W.words;            // current drop set
-  uint32_t* Rw = W.words + p.words;  // chosen restores
-  uint32_t* Xw = Rw + p.words;       // chosen drops
-  for (int r = warp; r < nrows; r += 8) {
-    const int i = i0 + r;
-    const int64_t ri = hrow + i;
-    const float* Prow = p.P + ri * p.ld;
-    const float* qrow = p.q + ri * p.ld;
-    const float* trow = tbase + (int64_t)r * p.ld;
-    for (int w = lane; w < p.words; w += 32) Dw[w] = p.dmask[ri * p.words + w];
-    const float K = p.K[ri], G = p.G[ri];
-    __syncwarp();
-    // one pass over the candidates: a block k in D is a restore candidate (u = +P_k,
-    // dG = -2 P_k t_k + P_k^2 q_k, Eq. 13-14), a kept candidate a drop candidate (u = -P_k,
-    // dG = +2 P_k t_k + P_k^2 q_k, Eq. 15); the key is the exact decrease of J (Eq. 16)
-#pragma unroll 4
-    for (int j = lane; j < p.ncand; j += 32) {
-      const float pj = Prow[j], qj = qrow[j], tj = trow[j];
-      const bool inD = (Dw[j >> 5] >> (j & 31)) & 1u;
-      const float s2 = pj * pj * qj;
-      const float dG = inD ? fmaf(-2.0f * pj, tj, s2) : fmaf(2.0f * pj, tj, s2);
-      W.kk[j] = order_key(delta_J(G, K, dG, inD ? pj : -pj));
+}
+
+// Restoration round r, per row: exact top-m restores and drops from the round-start state,
+// update, track-best.  grid (ceil(|P| / 4), H).
+__global__ void __launch_bounds__(32 * kRowWarps, 8) k_round_rows(SelPtrs p, Budgets bud,
+                                                                  int round, float rho) {
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int h = blockIdx.y, i = blockIdx.x * kRowWarps + warp;
+  const int m = swap_count(bud.c[h], p.ncand, round, rho);
+  if (m <= 0 || i >= p.ncand) return;
+  const int64_t ri = (int64_t)h * p.nb + i;
+  const float* Prow = p.P + ri * p.ld;
+  const float* qrow = p.q + ri * p.ld;
+  const float* trow = p.t + ri * p.ld;
+  const float* zt_h = p.ztil + (int64_t)h * p.nb * 64;
+  uint32_t* base = reinterpret_cast<uint32_t*>(smem_raw) + (size_t)warp * warp_scratch_words(p.ld, 3 * p.words);
+  uint32_t* kk = base;
+  uint32_t* sk = base + p.ld;
+  uint16_t* si = reinterpret_cast<uint16_t*>(sk + kSurvivors);
+  uint32_t* Dw = sk + kSurvivors + kSurvivors / 2;  // current drop set
+  uint32_t* Rw = Dw + p.words;                       // chosen restores
+  uint32_t* Xw = Rw + p.words;                       // chosen drops
+  for (int w = lane; w < p.words; w += 32) Dw[w] = p.dmask[ri * p.words + w];
+  const float K = p.K[ri], G = p.G[ri];
+  __syncwarp();
+  // one pass over the candidates: a block k in D is a restore candidate (u = +P_k,
+  // dG = -2 P_k t_k + P_k^2 q_k, Eq. 13-14), a kept candidate a drop candidate (u = -P_k,
+  // dG = +2 P_k t_k + P_k^2 q_k, Eq. 15); the key is the exact decrease of J (Eq. 16)
+  row_keys(p.ncand, kk, [&](int j, uint32_t (&k4)[4]) {
+    const float4 P4 = *reinterpret_cast<const float4*>(Prow + j);
+    const float4 q4 = *reinterpret_cast<const float4*>(qrow + j);
+    const float4 t4 = *reinterpret_cast<const float4*>(trow + j);
+    const float pv[4] = {P4.x, P4.y, P4.z, P4.w}, qv[4] = {q4.x, q4.y, q4.z, q4.w},
+                tv[4] = {t4.x, t4.y, t4.z, t4.w};
+    const uint32_t dword = Dw[j >> 5] >> (j & 31);
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const bool inD = (dword >> u) & 1u;
+      const float s2 = pv[u] * pv[u] * qv[u];
+      const float dG = inD ? fmaf(-2.0f * pv[u], tv[u], s2) : fmaf(2.0f * pv[u], tv[u], s2);
+      k4[u] = order_key(delta_J(G, K, dG, inD ? pv[u] : -pv[u]));
     }
-    __syncwarp();
-    warp_topm(W.kk, p.ncand, m, Rw, p.words, W.sk, W.si, Dw, true);
-    warp_topm(W.kk, p.ncand, m, Xw, p.words, W.sk, W.si, Dw, false);
-    for (int w = lane; w < p.words; w += 32) Dw[w] = (Dw[w] & ~Rw[w]) | Xw[w];
-    __syncwarp();
-    // exact state of the new set (Eq. 10-12)
-    const float y0 = p.ytil[ri * 64 + 2 * lane], y1 = p.ytil[ri * 64 + 2 * lane + 1];
-    float g0, g1, Kn;
-    kept_drift(Dw, p, Prow, zt_h, y0, y1, W.kk, g0, g1, Kn);
-    const float Gn = warp_sum(g0 * g0 + g1 * g1);
-    const float Kc = fmaxf(Kn, kEps);
-    const float Jn = Gn / (Kc * Kc);
-    const bool better = Jn < p.Jbest[ri];
-    for (int w = lane; w < p.words; w += 32) {
-      p.dmask[ri * p.words + w] = Dw[w];
-      if (better) p.bmask[ri * p.words + w] = Dw[w];
-    }
-    *reinterpret_cast<float2*>(p.gtil + ri * 64 + 2 * lane) = make_float2(g0, g1);
-    __syncwarp();
-    if (lane == 0) {
-      p.K[ri] = Kn;
-      p.G[ri] = Gn;
-      p.J[ri] = Jn;
-      if (better) p.Jbest[ri] = Jn;
-    }
-    __syncwarp();
+  });
+  warp_topm(kk, p.ncand, m, Rw, p.words, sk, si, Dw, true);
+  warp_topm(kk, p.ncand, m, Xw, p.words, sk, si, Dw, false);
+  for (int w = lane; w < p.words; w += 32) Dw[w] = (Dw[w] & ~Rw[w]) | Xw[w];
+  __syncwarp();
+  // exact state of the new set (Eq. 10-12)
+  const float2 y = *reinterpret_cast<const float2*>(p.ytil + ri * 64 + 2 * lane);
+  float g0, g1, Kn;
+  kept_drift(Dw, p, Prow, zt_h, y.x, y.y, kk, g0, g1, Kn);
+  const float Gn = warp_sum(g0 * g0 + g1 * g1);
+  const float Kc = fmaxf(Kn, kEps);
+  const float Jn = Gn / (Kc * Kc);
+  const bool better = Jn < p.Jbest[ri];
+  for (int w = lane; w < p.words; w += 32) {
+    p.dmask[ri * p.words + w] = Dw[w];
+    if (better) p.bmask[ri * p.words + w] = Dw[w];
+  }
+  *reinterpret_cast<float2*>(p.gtil + ri * 64 + 2 * lane) = make_float2(g0, g1);
+  if (lane == 0) {
+    p.K[ri] = Kn;
+    p.G[ri] = Gn;
+    p.J[ri] = Jn;
+    if (better) p.Jbest[ri] = Jn;
   }
 }
 
@@ -849,10 +893,15 @@ cudaError_t launch_score(const SelectArgs& a, cudaStream_t st) {
   k_pool<<<dim3(s.nb, 3), kThreads, 0, st>>>(a.Q, a.K, a.V, s.N, s.H, s.nb, qbar, kbar, vbar);
   k_zproj<<<dim3((s.nb + 63) / 64, s.H), kThreads, 0, st>>>(a.F, vbar, s.nb, ztil);
   if (s.ncand <= 0) return cudaGetLastError();
-  const size_t smem = sel_smem_bytes(s, s.words);
+  const size_t smem = sizeof(SelSmem);
   cudaError_t e = cudaFuncSetAttribute(k_score, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   k_score<<<dim3((s.ncand + RT - 1) / RT, s.H), kThreads, smem, st>>>(p, budgets_of(a));
+  const size_t rsmem = (size_t)kRowWarps * warp_scratch_words(s.ld, s.words) * 4;
+  e = cudaFuncSetAttribute(k_score_rows, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)rsmem);
+  if (e != cudaSuccess) return e;
+  k_score_rows<<<dim3((s.ncand + kRowWarps - 1) / kRowWarps, s.H), 32 * kRowWarps, rsmem, st>>>(
+      p, budgets_of(a));
   return cudaGetLastError();
 }
 
@@ -860,10 +909,15 @@ cudaError_t launch_round(const SelectArgs& a, int round, float rho, cudaStream_t
   const Shape& s = a.s;
   if (s.ncand <= 0) return cudaSuccess;
   SelPtrs p = sel_ptrs(s, a.ws, a.L);
-  const size_t smem = sel_smem_bytes(s, 3 * s.words);
+  const size_t smem = sizeof(SelSmem);
   cudaError_t e = cudaFuncSetAttribute(k_round, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   k_round<<<dim3((s.ncand + RT - 1) / RT, s.H), kThreads, smem, st>>>(p, budgets_of(a), round, rho);
+  const size_t rsmem = (size_t)kRowWarps * warp_scratch_words(s.ld, 3 * s.words) * 4;
+  e = cudaFuncSetAttribute(k_round_rows, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)rsmem);
+  if (e != cudaSuccess) return e;
+  k_round_rows<<<dim3((s.ncand + kRowWarps - 1) / kRowWarps, s.H), 32 * kRowWarps, rsmem, st>>>(
+      p, budgets_of(a), round, rho);
   return cudaGetLastError();
 }
 
