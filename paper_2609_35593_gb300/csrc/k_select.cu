@@ -138,27 +138,33 @@ __global__ void __launch_bounds__(kThreads) k_pool(const uint16_t* __restrict__ 
 }
 
 // ------------------------------------------------------------------------------------
-// z~_j = F_h V_j.  grid (ceil(nb/64), H).
+// z~_j = F_h V_j.  grid (ceil(nb/16), H); thread (block jj, channels 4a..4a+3).
 // ------------------------------------------------------------------------------------
 __global__ void __launch_bounds__(kThreads) k_zproj(const float* __restrict__ F,
                                                      const float* __restrict__ vbar, int nb,
                                                      float* __restrict__ ztil) {
-  __shared__ float Fs[64][65];
-  __shared__ float Vs[64][65];
-  const int h = blockIdx.y, j0 = blockIdx.x * 64, t = threadIdx.x;
-  for (int f = t; f < 4096; f += kThreads) {
+  __shared__ __align__(16) float Ft[64][64];  // Ft[b][a] = F[a][b]
+  __shared__ float Vs[16][65];
+  const int h = blockIdx.y, j0 = blockIdx.x * 16, t = threadIdx.x;
+  for (int f = t; f < 4096; f += kThreads) Ft[f & 63][f >> 6] = F[(int64_t)h * 4096 + f];
+  for (int f = t; f < 16 * 64; f += kThreads) {
     const int r = f >> 6, c = f & 63;
-    Fs[r][c] = F[(int64_t)h * 4096 + f];
     Vs[r][c] = (j0 + r < nb) ? vbar[((int64_t)h * nb + j0 + r) * 64 + c] : 0.f;
   }
   __syncthreads();
-  const int jj = t >> 2, a0 = (t & 3) * 16;
+  const int jj = t >> 4, a4 = (t & 15) * 4;
   if (j0 + jj >= nb) return;
-  for (int a = a0; a < a0 + 16; ++a) {
-    float s = 0.f;
-    for (int b = 0; b < 64; ++b) s = fmaf(Fs[a][b], Vs[jj][b], s);
-    ztil[((int64_t)h * nb + j0 + jj) * 64 + a] = s;
+  float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll 8
+  for (int b = 0; b < 64; ++b) {
+    const float v = Vs[jj][b];
+    const float4 f = *reinterpret_cast<const float4*>(&Ft[b][a4]);
+    acc.x = fmaf(f.x, v, acc.x);
+    acc.y = fmaf(f.y, v, acc.y);
+    acc.z = fmaf(f.z, v, acc.z);
+    acc.w = fmaf(f.w, v, acc.w);
   }
+  *reinterpret_cast<float4*>(ztil + ((int64_t)h * nb + j0 + jj) * 64 + a4) = acc;
 }
 
 // ------------------------------------------------------------------------------------
@@ -227,45 +233,65 @@ __device__ __forceinline__ void stage_rows(float (*A)[LDA], const float* __restr
 
 enum { kOpDot = 0, kOpDist = 1, kOpGain = 2 };
 
+// Packed pairs of floats (two fp32 lanes of one 64-bit register) for the f32x2 FMA path.
+__device__ __forceinline__ uint64_t ffma2(uint64_t a, uint64_t b, uint64_t c) {
+  uint64_t d;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
+  return d;
+}
+__device__ __forceinline__ uint64_t fsub2(uint64_t a, uint64_t b) {
+  uint64_t d;
+  asm("sub.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
+  return d;
+}
+__device__ __forceinline__ float hsum2(uint64_t v) {
+  float lo, hi;
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(v));
+  return lo + hi;
+}
+
 // Warp tile of 8 rows (8*rg ..) x 2 staged blocks (jb, jb + 32), reduced over the 64
-// channels in ascending order:
+// channels; each accumulator is a pair (even channels, odd channels) updated by packed
+// f32x2 instructions straight from the float4 operands, the halves added at the end:
 //   kOpDot  : sum_d A[r][d] B[j][d]
 //   kOpDist : sum_d (A[r][d] - B[j][d])^2
 //   kOpGain : sum_d (A[r][d] - B[j][d]) Gv[r][d]
 template <int OP>
-__device__ __forceinline__ void tile8x2(const SelSmem& S, int rg, int jb, float acc[8][2]) {
+__device__ __forceinline__ void tile8x2(const SelSmem& S, int rg, int jb, float out[8][2]) {
+  uint64_t acc[8][2];
 #pragma unroll
-  for (int x = 0; x < 8; ++x) acc[x][0] = acc[x][1] = 0.f;
+  for (int x = 0; x < 8; ++x) acc[x][0] = acc[x][1] = 0ull;
 #pragma unroll 2
   for (int d = 0; d < 64; d += 4) {
-    const float4 b0 = *reinterpret_cast<const float4*>(&S.B[jb][d]);
-    const float4 b1 = *reinterpret_cast<const float4*>(&S.B[jb + 32][d]);
+    const ulonglong2 b0 = *reinterpret_cast<const ulonglong2*>(&S.B[jb][d]);
+    const ulonglong2 b1 = *reinterpret_cast<const ulonglong2*>(&S.B[jb + 32][d]);
 #pragma unroll
     for (int x = 0; x < 8; ++x) {
-      const float4 a = *reinterpret_cast<const float4*>(&S.A[rg * 8 + x][d]);
+      const ulonglong2 a = *reinterpret_cast<const ulonglong2*>(&S.A[rg * 8 + x][d]);
       if (OP == kOpDot) {
-        acc[x][0] = fmaf(a.x, b0.x, acc[x][0]); acc[x][0] = fmaf(a.y, b0.y, acc[x][0]);
-        acc[x][0] = fmaf(a.z, b0.z, acc[x][0]); acc[x][0] = fmaf(a.w, b0.w, acc[x][0]);
-        acc[x][1] = fmaf(a.x, b1.x, acc[x][1]); acc[x][1] = fmaf(a.y, b1.y, acc[x][1]);
-        acc[x][1] = fmaf(a.z, b1.z, acc[x][1]); acc[x][1] = fmaf(a.w, b1.w, acc[x][1]);
+        acc[x][0] = ffma2(a.x, b0.x, acc[x][0]);
+        acc[x][0] = ffma2(a.y, b0.y, acc[x][0]);
+        acc[x][1] = ffma2(a.x, b1.x, acc[x][1]);
+        acc[x][1] = ffma2(a.y, b1.y, acc[x][1]);
       } else if (OP == kOpDist) {
-        float e;
-        e = a.x - b0.x; acc[x][0] = fmaf(e, e, acc[x][0]);
-        e = a.y - b0.y; acc[x][0] = fmaf(e, e, acc[x][0]);
-        e = a.z - b0.z; acc[x][0] = fmaf(e, e, acc[x][0]);
-        e = a.w - b0.w; acc[x][0] = fmaf(e, e, acc[x][0]);
-        e = a.x - b1.x; acc[x][1] = fmaf(e, e, acc[x][1]);
-        e = a.y - b1.y; acc[x][1] = fmaf(e, e, acc[x][1]);
-        e = a.z - b1.z; acc[x][1] = fmaf(e, e, acc[x][1]);
-        e = a.w - b1.w; acc[x][1] = fmaf(e, e, acc[x][1]);
+        uint64_t e;
+        e = fsub2(a.x, b0.x); acc[x][0] = ffma2(e, e, acc[x][0]);
+        e = fsub2(a.y, b0.y); acc[x][0] = ffma2(e, e, acc[x][0]);
+        e = fsub2(a.x, b1.x); acc[x][1] = ffma2(e, e, acc[x][1]);
+        e = fsub2(a.y, b1.y); acc[x][1] = ffma2(e, e, acc[x][1]);
       } else {
-        const float4 g = *reinterpret_cast<const float4*>(&S.Gv[rg * 8 + x][d]);
-        acc[x][0] = fmaf(a.x - b0.x, g.x, acc[x][0]); acc[x][0] = fmaf(a.y - b0.y, g.y, acc[x][0]);
-        acc[x][0] = fmaf(a.z - b0.z, g.z, acc[x][0]); acc[x][0] = fmaf(a.w - b0.w, g.w, acc[x][0]);
-        acc[x][1] = fmaf(a.x - b1.x, g.x, acc[x][1]); acc[x][1] = fmaf(a.y - b1.y, g.y, acc[x][1]);
-        acc[x][1] = fmaf(a.z - b1.z, g.z, acc[x][1]); acc[x][1] = fmaf(a.w - b1.w, g.w, acc[x][1]);
+        const ulonglong2 g = *reinterpret_cast<const ulonglong2*>(&S.Gv[rg * 8 + x][d]);
+        acc[x][0] = ffma2(fsub2(a.x, b0.x), g.x, acc[x][0]);
+        acc[x][0] = ffma2(fsub2(a.y, b0.y), g.y, acc[x][0]);
+        acc[x][1] = ffma2(fsub2(a.x, b1.x), g.x, acc[x][1]);
+        acc[x][1] = ffma2(fsub2(a.y, b1.y), g.y, acc[x][1]);
       }
     }
+  }
+#pragma unroll
+  for (int x = 0; x < 8; ++x) {
+    out[x][0] = hsum2(acc[x][0]);
+    out[x][1] = hsum2(acc[x][1]);
   }
 }
 
@@ -426,7 +452,7 @@ __device__ __forceinline__ uint32_t valid_bits(int w, int n) {
 // g~ = sum_{j not in D} P_ij (z~_j - y~_i) and K = sum_{j not in D} P_ij for one row, by
 // one warp (lane owns channels 2*lane, 2*lane+1), in ascending j.  The kept blocks are
 // first compacted into idx[] (per-warp shared memory, >= nb entries) so that the loads of
-// sixteen blocks are in flight together.
+// eight blocks are in flight together.
 __device__ __forceinline__ void kept_drift(const uint32_t* D, const SelPtrs& p,
                                            const float* __restrict__ Prow,
                                            const float* __restrict__ zt, float y0, float y1,
@@ -440,11 +466,11 @@ __device__ __forceinline__ void kept_drift(const uint32_t* D, const SelPtrs& p,
   }
   __syncwarp();
   g0 = g1 = K = 0.f;
-  for (int k0 = 0; k0 < n; k0 += 16) {
-    float pj[16];
-    float2 z[16];
+  for (int k0 = 0; k0 < n; k0 += 8) {
+    float pj[8];
+    float2 z[8];
 #pragma unroll
-    for (int u = 0; u < 16; ++u) {
+    for (int u = 0; u < 8; ++u) {
       if (k0 + u < n) {
         const int j = idx[k0 + u];
         pj[u] = Prow[j];
@@ -452,7 +478,7 @@ __device__ __forceinline__ void kept_drift(const uint32_t* D, const SelPtrs& p,
       }
     }
 #pragma unroll
-    for (int u = 0; u < 16; ++u) {
+    for (int u = 0; u < 8; ++u) {
       if (k0 + u < n) {
         g0 = fmaf(pj[u], z[u].x - y0, g0);
         g1 = fmaf(pj[u], z[u].y - y1, g1);
@@ -891,7 +917,7 @@ cudaError_t launch_score(const SelectArgs& a, cudaStream_t st) {
   float* vbar = (float*)(a.ws + a.L.vbar);
   float* ztil = (float*)(a.ws + a.L.ztil);
   k_pool<<<dim3(s.nb, 3), kThreads, 0, st>>>(a.Q, a.K, a.V, s.N, s.H, s.nb, qbar, kbar, vbar);
-  k_zproj<<<dim3((s.nb + 63) / 64, s.H), kThreads, 0, st>>>(a.F, vbar, s.nb, ztil);
+  k_zproj<<<dim3((s.nb + 15) / 16, s.H), kThreads, 0, st>>>(a.F, vbar, s.nb, ztil);
   if (s.ncand <= 0) return cudaGetLastError();
   const size_t smem = sizeof(SelSmem);
   cudaError_t e = cudaFuncSetAttribute(k_score, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
