@@ -16,8 +16,8 @@
 //              so that neither A operand is read from shared memory, whose bandwidth the
 //              N = 64 MMAs would otherwise saturate together with the TMA writes.
 //              S is double-buffered in TMEM and a buffer is handed back as soon as the
-//              softmax has loaded it, so S_{g+2} is issued before P_g V_g and both S_{g+1}
-//              and S_{g+2} run while the softmax works on S_g.  P (bf16) has its own 32 TMEM columns and is read from
+//              softmax has loaded it, so S_{g+1} is issued before P_g V_g and runs while the
+//              softmax works on S_g.  P (bf16) has its own 32 TMEM columns and is read from
 //              there as the A operand of P V, which keeps it off the shared-memory bus.
 //              TMEM per CTA: S0 | S1 | O | Q | P = 64 + 64 + 64 + 32 + 32 columns.
 //   warps 2-5  one query row per thread: tcgen05.ld of S, online softmax in the exp2 domain
@@ -289,8 +289,8 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
     }
   } else if (warp == 1) {
     // ================================ MMA issuer ===================================
-    // Order per step g: S_{g+2} (as soon as K_{g+2} has landed and the softmax has read
-    // S_g out of that buffer), then P_g V_g (once P_g is in TMEM): S runs two tiles ahead.
+    // Order per step g: S_{g+1} (as soon as K_{g+1} has landed and the softmax has read
+    // S_{g-1} out of that buffer), then P_g V_g (once P_g is in TMEM).
     if (lane == 0) {
       const uint32_t idesc_qk = idesc_bf16_f32(kRows, 64, false);
       const uint32_t idesc_pv = idesc_bf16_f32(kRows, 64, true);
@@ -342,31 +342,24 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
         mma_commit(&S.o_bar[t & 1]);
         return true;
       };
-      // window of tile infos: ti[t % 3] for steps g, g+1, g+2; have[] marks real tiles
-      TileInfo ti[3];
-      bool have[3] = {false, false, false};
-      have[0] = fetch(0, ti[0]);
-      if (have[0] && !failed) {
-        if (!issue_s(0, ti[0])) failed = true;
-        if (!failed) {
-          have[1] = fetch(1, ti[1]);
-          if (have[1] && !failed && !issue_s(1, ti[1])) failed = true;
+      TileInfo cur, nxt;
+      if (fetch(0, cur) && issue_s(0, cur)) {
+        for (int g = 0;; ++g) {
+          const bool more = fetch(g + 1, nxt);
+          if (failed) break;
+          if (more && !issue_s(g + 1, nxt)) {
+            failed = true;
+            break;
+          }
+          if (!issue_pv(g, cur)) {
+            failed = true;
+            break;
+          }
+          if (!more) break;
+          cur = nxt;
         }
-      }
-      for (int g = 0; have[g % 3] && !failed; ++g) {
-        const int c = g % 3, n1 = (g + 1) % 3, n2 = (g + 2) % 3;
-        // S_{g+2} into the buffer S_g leaves once the softmax has loaded S_g
-        have[n2] = have[n1] && fetch(g + 2, ti[n2]);
-        if (failed) break;
-        if (have[n2] && !issue_s(g + 2, ti[n2])) {
-          failed = true;
-          break;
-        }
-        if (!issue_pv(g, ti[c])) {
-          failed = true;
-          break;
-        }
-        have[c] = false;
+      } else if (!failed && !(cur.flags & kTerm)) {
+        failed = true;
       }
       if (failed) give_up(S, a.status);
       // wait for every MMA issued so far before TMEM is released
