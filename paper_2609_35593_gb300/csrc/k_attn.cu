@@ -15,11 +15,11 @@
 //              Q is copied once per item from its TMA staging buffer into TMEM (tcgen05.cp),
 //              so that neither A operand is read from shared memory, whose bandwidth the
 //              N = 64 MMAs would otherwise saturate together with the TMA writes.
-//              S is double-buffered in TMEM and a buffer is handed back as soon as the
-//              softmax has loaded it, so S_{g+1} is issued before P_g V_g and runs while the
-//              softmax works on S_g.  P (bf16) has its own 32 TMEM columns and is read from
-//              there as the A operand of P V, which keeps it off the shared-memory bus.
-//              TMEM per CTA: S0 | S1 | O | Q | P = 64 + 64 + 64 + 32 + 32 columns.
+//              S is double-buffered in TMEM so that S_{g+1} runs while softmax works on S_g;
+//              P_g (bf16) is written over the first half of S_g's columns and read from
+//              there as the A operand, which keeps it off the shared-memory bus.  MMAs
+//              issued by one thread run in issue order, so S_{g+2} overwrites P_g only after
+//              P_g V_g has read it.
 //   warps 2-5  one query row per thread: tcgen05.ld of S, online softmax in the exp2 domain
 //              with lazy rescaling of the TMEM accumulator (only when the running max grows
 //              by more than 2^8), tcgen05.st of P, epilogue O / l.
@@ -41,7 +41,7 @@ constexpr int kAttnThreads = 192;
 constexpr int kStages = 5;
 constexpr int kRows = 128;
 constexpr uint32_t kTmemCols = 256;
-constexpr uint32_t kColS0 = 0, kColO = 128, kColQ = 192, kColP = 224;  // TMEM: S x2, O, Q, P
+constexpr uint32_t kColS0 = 0, kColO = 128, kColQ = 192;  // TMEM columns: S/P x2, O, Q
 constexpr uint64_t kWaitNs = 2000000000ull;  // 2 s per wait
 constexpr uint64_t kDrainNs = 200000000ull;  // 0.2 s to drain after an abort
 constexpr int kFirst = 1, kLast = 2, kTerm = 4;
@@ -58,7 +58,7 @@ struct __align__(1024) AttnSmem {
   uint8_t V[kStages][kTileBytes];
   uint64_t kv_full[kStages], kv_empty[kStages];
   uint64_t q_full, q_empty;
-  uint64_t s_full[2], s_free[2], p_full;
+  uint64_t s_full[2], p_full[2];
   uint64_t o_bar[2], drain;  // o_bar[k & 1] completes when P_k V_k has landed
   TileInfo info[kStages];
   uint32_t tmem_base;
@@ -195,9 +195,8 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
     mbar_init(&S.q_empty, 1);
     for (int b = 0; b < 2; ++b) {
       mbar_init(&S.s_full[b], 1);
-      mbar_init(&S.s_free[b], 4);
+      mbar_init(&S.p_full[b], 4);
     }
-    mbar_init(&S.p_full, 4);
     mbar_init(&S.o_bar[0], 1);
     mbar_init(&S.o_bar[1], 1);
     mbar_init(&S.drain, 1);
@@ -289,26 +288,39 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
     }
   } else if (warp == 1) {
     // ================================ MMA issuer ===================================
-    // Order per step g: S_{g+1} (as soon as K_{g+1} has landed and the softmax has read
-    // S_{g-1} out of that buffer), then P_g V_g (once P_g is in TMEM).
     if (lane == 0) {
       const uint32_t idesc_qk = idesc_bf16_f32(kRows, 64, false);
       const uint32_t idesc_pv = idesc_bf16_f32(kRows, 64, true);
       const uint32_t q_addr = smem_u32(S.Q);
-      int it = 0;
-      bool failed = false;
-      // tile info of step t once its K/V stage has landed; false at the end marker
-      auto fetch = [&](int t, TileInfo& info) -> bool {
-        if (!mbar_wait(&S.kv_full[t % kStages], (t / kStages) & 1, abort, kWaitNs)) {
-          failed = true;
-          return false;
-        }
-        info = S.info[t % kStages];
-        return !(info.flags & kTerm);
+      int g = 0, it = 0;
+      bool have_prev = false, prev_first = false, failed = false;
+      int prev_g = 0;
+      auto issue_pv = [&](int pg, bool first) -> bool {
+        const int pb = pg & 1, ps = pg % kStages;
+        if (!mbar_wait(&S.p_full[pb], (pg >> 1) & 1, abort, kWaitNs)) return false;
+        tc_fence_after();
+        const uint32_t v_addr = smem_u32(S.V[ps]);
+#pragma unroll
+        for (int k = 0; k < 4; ++k)
+          mma_bf16_ts(tmem + kColO, tmem + kColS0 + 64 * pb + 8 * k, sdesc_sw128(v_addr + 2048 * k),
+                      idesc_pv, (k > 0 || !first) ? 1u : 0u);
+        mma_commit(&S.kv_empty[ps]);
+        mma_commit(&S.o_bar[pg & 1]);
+        return true;
       };
-      auto issue_s = [&](int t, const TileInfo& info) -> bool {
+      for (;;) {
+        const int s = g % kStages;
+        if (!mbar_wait(&S.kv_full[s], (g / kStages) & 1, abort, kWaitNs)) {
+          failed = true;
+          break;
+        }
+        const TileInfo info = S.info[s];
+        if (info.flags & kTerm) break;
         if (info.flags & kFirst) {
-          if (!mbar_wait(&S.q_full, it & 1, abort, kWaitNs)) return false;
+          if (!mbar_wait(&S.q_full, it & 1, abort, kWaitNs)) {
+            failed = true;
+            break;
+          }
           tc_fence_after();
           // Q (128 x 64) into TMEM, one K16 slice (8 columns) per copy; the staging buffer
           // is free again once the copies have completed.  Copies and MMAs issued by this
@@ -316,50 +328,32 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
 #pragma unroll
           for (int k = 0; k < 4; ++k) tmem_cp_128x256b(tmem + kColQ + 8 * k, sdesc_sw128(q_addr + 32 * k));
           mma_commit(&S.q_empty);
-          ++it;
         }
-        const int b = t & 1;
-        if (t >= 2 && !mbar_wait(&S.s_free[b], ((t - 2) >> 1) & 1, abort, kWaitNs)) return false;
         tc_fence_after();
-        const uint32_t k_addr = smem_u32(S.K[t % kStages]);
+        const int b = g & 1;
+        const uint32_t k_addr = smem_u32(S.K[s]);
 #pragma unroll
         for (int k = 0; k < 4; ++k)
           mma_bf16_ts(tmem + kColS0 + 64 * b, tmem + kColQ + 8 * k, sdesc_sw128(k_addr + 32 * k),
                       idesc_qk, k > 0 ? 1u : 0u);
         mma_commit(&S.s_full[b]);
-        return true;
-      };
-      auto issue_pv = [&](int t, const TileInfo& info) -> bool {
-        if (!mbar_wait(&S.p_full, t & 1, abort, kWaitNs)) return false;
-        tc_fence_after();
-        const uint32_t v_addr = smem_u32(S.V[t % kStages]);
-        const bool first = (info.flags & kFirst) != 0;
-#pragma unroll
-        for (int k = 0; k < 4; ++k)
-          mma_bf16_ts(tmem + kColO, tmem + kColP + 8 * k, sdesc_sw128(v_addr + 2048 * k), idesc_pv,
-                      (k > 0 || !first) ? 1u : 0u);
-        mma_commit(&S.kv_empty[t % kStages]);
-        mma_commit(&S.o_bar[t & 1]);
-        return true;
-      };
-      TileInfo cur, nxt;
-      if (fetch(0, cur) && issue_s(0, cur)) {
-        for (int g = 0;; ++g) {
-          const bool more = fetch(g + 1, nxt);
-          if (failed) break;
-          if (more && !issue_s(g + 1, nxt)) {
-            failed = true;
-            break;
-          }
-          if (!issue_pv(g, cur)) {
-            failed = true;
-            break;
-          }
-          if (!more) break;
-          cur = nxt;
+        if (have_prev && !issue_pv(prev_g, prev_first)) {
+          failed = true;
+          break;
         }
-      } else if (!failed && !(cur.flags & kTerm)) {
-        failed = true;
+        if (info.flags & kLast) {
+          if (!issue_pv(g, (info.flags & kFirst) != 0)) {
+            failed = true;
+            break;
+          }
+          have_prev = false;
+          ++it;
+        } else {
+          have_prev = true;
+          prev_g = g;
+          prev_first = (info.flags & kFirst) != 0;
+        }
+        ++g;
       }
       if (failed) give_up(S, a.status);
       // wait for every MMA issued so far before TMEM is released
@@ -376,6 +370,7 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
     const float kScale = 1.4426950408889634f * 0.125f;  // log2(e) / sqrt(64)
     int g = 0;
     float m_use = -INFINITY, l = 0.f;
+    int tile_in_item = 0;
     for (;;) {
       const int s = g % kStages;
       if (!warp_wait(&S.kv_full[s], (g / kStages) & 1, abort)) {
@@ -387,8 +382,10 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
       if (info.flags & kFirst) {
         m_use = -INFINITY;
         l = 0.f;
+        tile_in_item = 0;
       }
       const int b = g & 1;
+      // S_g complete implies every earlier MMA complete, P_{g-2} V_{g-2} included
       if (!warp_wait(&S.s_full[b], (g >> 1) & 1, abort)) {
         give_up(S, a.status);
         break;
@@ -396,43 +393,31 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
       tc_fence_after();
       const bool active = (info.mask >> half) & 1;  // warp-uniform
       const uint32_t tS = tmem + lane_base + kColS0 + 64 * b;
-      float x[64];
       if (active) {
-        uint32_t v[32];
-        RESS_TMEM_LD32(tS, v);
+        float x[64];
+        {
+          uint32_t v[32];
+          RESS_TMEM_LD32(tS, v);
 #pragma unroll
-        for (int c = 0; c < 32; ++c) x[c] = __uint_as_float(v[c]);
-        RESS_TMEM_LD32(tS + 32, v);
+          for (int c = 0; c < 32; ++c) x[c] = __uint_as_float(v[c]);
+          RESS_TMEM_LD32(tS + 32, v);
 #pragma unroll
-        for (int c = 0; c < 32; ++c) x[32 + c] = __uint_as_float(v[c]);
-      }
-      // S_g is in registers: its TMEM buffer can take S_{g+2}
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&S.s_free[b]);
-
-      float alpha = 1.f;
-      bool rescale = false;
-      uint32_t w[32];
-      float rsum = 0.f;
-      if (active) {
+          for (int c = 0; c < 32; ++c) x[32 + c] = __uint_as_float(v[c]);
+        }
         if (info.j == a.nb - 1) {  // ragged last key block: keys past N do not exist
           const int valid = a.N - 64 * info.j;
 #pragma unroll
           for (int c = 0; c < 64; ++c)
             if (c >= valid) x[c] = -INFINITY;
         }
-        // row max of the raw scores (the scale is positive) as a tree of 3-input maxima
-        float m1[22];
+        // row max of the raw scores (the scale is positive), three operands at a time
+        float mr = fmax3(x[0], x[1], x[2]);
 #pragma unroll
-        for (int k = 0; k < 21; ++k) m1[k] = fmax3(x[3 * k], x[3 * k + 1], x[3 * k + 2]);
-        m1[21] = x[63];
-        float m2[8];
-#pragma unroll
-        for (int k = 0; k < 7; ++k) m2[k] = fmax3(m1[3 * k], m1[3 * k + 1], m1[3 * k + 2]);
-        m2[7] = m1[21];
-        const float mr = fmax3(fmax3(m2[0], m2[1], m2[2]), fmax3(m2[3], m2[4], m2[5]), fmaxf(m2[6], m2[7]));
+        for (int c = 3; c < 63; c += 2) mr = fmax3(mr, x[c], x[c + 1]);
+        mr = fmaxf(mr, x[63]);
         const float mt = mr * kScale;
+        float alpha = 1.f;
+        bool rescale = false;
         if (m_use == -INFINITY) {
           m_use = mt;  // first kept tile of this row: O row is still zero
         } else if (mt > m_use + kLazyThreshold) {
@@ -440,47 +425,47 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
           m_use = mt;
           rescale = true;
         }
-        // p = 2^(s * log2(e)/8 - m), two columns per packed FMA; the row sum adds the bf16
-        // values the MMA multiplies, so that a row dominated by one key keeps O = V exactly
-        // up to the accumulation (p reaches 2^8 between rescales)
-        const float nm = -m_use;
-        float rs[8];
+        if (__any_sync(0xffffffffu, rescale)) {
+          // the previous P V must have landed before the accumulator row is rescaled
+          if (!warp_wait(&S.o_bar[(g - 1) & 1], ((g - 1) >> 1) & 1, abort)) {
+            give_up(S, a.status);
+            break;
+          }
+          tc_fence_after();
 #pragma unroll
-        for (int k = 0; k < 8; ++k) rs[k] = 0.f;
+          for (int hc = 0; hc < 2; ++hc) {
+            uint32_t v[32];
+            RESS_TMEM_LD32(tmem + lane_base + kColO + 32 * hc, v);
+#pragma unroll
+            for (int c = 0; c < 32; ++c) v[c] = __float_as_uint(__uint_as_float(v[c]) * alpha);
+            RESS_TMEM_ST32(tmem + lane_base + kColO + 32 * hc, v);
+          }
+        }
+        // p = 2^(s * log2(e)/8 - m), two columns per packed FMA
+        const float nm = -m_use;
+        float rs0 = 0.f, rs1 = 0.f;
+        uint32_t w[32];
 #pragma unroll
         for (int e = 0; e < 32; ++e) {
           float t0, t1;
           fma2(t0, t1, x[2 * e], x[2 * e + 1], kScale, kScale, nm, nm);
           w[e] = pack_bf16x2(ex2(t0), ex2(t1));
-          add2(rs[2 * (e & 3)], rs[2 * (e & 3) + 1], rs[2 * (e & 3)], rs[2 * (e & 3) + 1],
-               __uint_as_float(w[e] << 16), __uint_as_float(w[e] & 0xffff0000u));
+          // sum the bf16 values the MMA multiplies, so that a row dominated by one key
+          // keeps O = V exactly up to the accumulation (p reaches 2^8 between rescales)
+          add2(rs0, rs1, rs0, rs1, __uint_as_float(w[e] << 16), __uint_as_float(w[e] & 0xffff0000u));
         }
-        rsum = ((rs[0] + rs[1]) + (rs[2] + rs[3])) + ((rs[4] + rs[5]) + (rs[6] + rs[7]));
+        RESS_TMEM_ST32(tS, w);  // P_g over the first 32 columns of S_g
+        l = l * alpha + (rs0 + rs1);
       } else {
+        uint32_t w[32];
 #pragma unroll
         for (int e = 0; e < 32; ++e) w[e] = 0u;
+        RESS_TMEM_ST32(tS, w);
       }
-      // P_{g-1} V_{g-1} must have read the P buffer (and updated O) before P_g replaces it
-      if (g >= 1 && !warp_wait(&S.o_bar[(g - 1) & 1], ((g - 1) >> 1) & 1, abort)) {
-        give_up(S, a.status);
-        break;
-      }
-      tc_fence_after();
-      if (__any_sync(0xffffffffu, rescale)) {
-        uint32_t v[32];
-#pragma unroll
-        for (int hc = 0; hc < 2; ++hc) {
-          RESS_TMEM_LD32(tmem + lane_base + kColO + 32 * hc, v);
-#pragma unroll
-          for (int c = 0; c < 32; ++c) v[c] = __float_as_uint(__uint_as_float(v[c]) * alpha);
-          RESS_TMEM_ST32(tmem + lane_base + kColO + 32 * hc, v);
-        }
-      }
-      RESS_TMEM_ST32(tmem + lane_base + kColP, w);
-      l = l * alpha + rsum;
       tc_fence_before();
       __syncwarp();
-      if (lane == 0) mbar_arrive(&S.p_full);
+      if (lane == 0) mbar_arrive(&S.p_full[b]);
+      ++tile_in_item;
 
       if (info.flags & kLast) {
         // epilogue: O / l for this row once the last P V has landed
@@ -514,14 +499,14 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
             uint4* dst = reinterpret_cast<uint4*>(static_cast<uint16_t*>(a.O) + off);
 #pragma unroll
             for (int ch = 0; ch < 8; ++ch) {
-              uint32_t q4[4];
+              uint32_t w[4];
 #pragma unroll
               for (int e = 0; e < 4; ++e) {
                 const int c = ch * 8 + 2 * e;
-                q4[e] = pack_bf16x2(__uint_as_float(o[c >> 5][c & 31]) * inv,
-                                    __uint_as_float(o[(c + 1) >> 5][(c + 1) & 31]) * inv);
+                w[e] = pack_bf16x2(__uint_as_float(o[c >> 5][c & 31]) * inv,
+                                   __uint_as_float(o[(c + 1) >> 5][(c + 1) & 31]) * inv);
               }
-              dst[ch] = make_uint4(q4[0], q4[1], q4[2], q4[3]);
+              dst[ch] = make_uint4(w[0], w[1], w[2], w[3]);
             }
           }
         }
