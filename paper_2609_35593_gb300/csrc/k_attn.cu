@@ -11,7 +11,10 @@
 //              a 5-stage ring, 128-byte swizzled (UMMA canonical layouts).
 //   warp 1     TMEM owner and single-thread MMA issuer:
 //                S[g % 2] = Q K_g^T              (M128 N64 K64, Q from TMEM, K from shared memory)
-//                O       += P_{g-1} V_{g-1}       (M128 N64 K64, P from TMEM, V MN-major)
+//                O       += P_{g-1} [V_{g-1} | 1]  (M128 N80 K64, P from TMEM, V MN-major)
+//              The second 64-column atom of that B operand is a constant shared tile whose
+//              first column is 1, so O's column 64 accumulates the row sum of exactly the bf16
+//              P values the MMA multiplies, in fp32, and follows every rescale of O for free.
 //              Q is copied once per item from its TMA staging buffer into TMEM (tcgen05.cp),
 //              so that neither A operand is read from shared memory, whose bandwidth the
 //              N = 64 MMAs would otherwise saturate together with the TMA writes.
@@ -41,7 +44,8 @@ constexpr int kAttnThreads = 192;
 constexpr int kStages = 5;
 constexpr int kRows = 128;
 constexpr uint32_t kTmemCols = 256;
-constexpr uint32_t kColS0 = 0, kColO = 128, kColQ = 192;  // TMEM columns: S/P x2, O, Q
+constexpr uint32_t kColS0 = 0, kColO = 128, kColQ = 208;  // TMEM columns: S/P x2, O (80), Q
+constexpr int kNO = 80;  // O columns: 64 output channels, the row sum, 15 unused
 constexpr uint64_t kWaitNs = 2000000000ull;  // 2 s per wait
 constexpr uint64_t kDrainNs = 200000000ull;  // 0.2 s to drain after an abort
 constexpr int kFirst = 1, kLast = 2, kTerm = 4;
@@ -56,6 +60,7 @@ struct __align__(1024) AttnSmem {
   uint8_t Q[kRows * 128];
   uint8_t K[kStages][kTileBytes];
   uint8_t V[kStages][kTileBytes];
+  uint8_t ONES[kTileBytes];  // B operand columns 64..127 of P V: column 64 all ones
   uint64_t kv_full[kStages], kv_empty[kStages];
   uint64_t q_full, q_empty;
   uint64_t s_full[2], p_full[2];
@@ -206,6 +211,12 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
     prefetch_tensormap(&tmK);
     prefetch_tensormap(&tmV);
   }
+  for (int f = threadIdx.x; f < kTileBytes / 16; f += blockDim.x)
+    reinterpret_cast<uint4*>(S.ONES)[f] = make_uint4(0u, 0u, 0u, 0u);
+  __syncthreads();
+  if (threadIdx.x < 64)  // key row k: element 0 of its 128-byte swizzled row = bf16 1.0
+    *reinterpret_cast<uint16_t*>(S.ONES + threadIdx.x * 128 + ((threadIdx.x & 7) << 4)) = 0x3F80;
+  fence_proxy_async_smem();
   if (warp == 1) tmem_alloc(&S.tmem_base, kTmemCols);
   tc_fence_before();
   __syncthreads();
@@ -290,7 +301,8 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
     // ================================ MMA issuer ===================================
     if (lane == 0) {
       const uint32_t idesc_qk = idesc_bf16_f32(kRows, 64, false);
-      const uint32_t idesc_pv = idesc_bf16_f32(kRows, 64, true);
+      const uint32_t idesc_pv = idesc_bf16_f32(kRows, kNO, true);
+      const uint32_t ones_addr = smem_u32(S.ONES);
       const uint32_t q_addr = smem_u32(S.Q);
       int g = 0, it = 0;
       bool have_prev = false, prev_first = false, failed = false;
@@ -300,10 +312,13 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
         if (!mbar_wait(&S.p_full[pb], (pg >> 1) & 1, abort, kWaitNs)) return false;
         tc_fence_after();
         const uint32_t v_addr = smem_u32(S.V[ps]);
+        // the N = 80 B operand: atom 0 = V (channels), atom 1 = ONES, LBO bytes after it
+        const uint64_t lbo = (uint64_t)(((ones_addr - v_addr) >> 4) & 0x3FFFu) << 16;
 #pragma unroll
         for (int k = 0; k < 4; ++k)
-          mma_bf16_ts(tmem + kColO, tmem + kColS0 + 64 * pb + 8 * k, sdesc_sw128(v_addr + 2048 * k),
-                      idesc_pv, (k > 0 || !first) ? 1u : 0u);
+          mma_bf16_ts(tmem + kColO, tmem + kColS0 + 64 * pb + 8 * k,
+                      (sdesc_sw128(v_addr + 2048 * k) & ~(0x3FFFull << 16)) | lbo, idesc_pv,
+                      (k > 0 || !first) ? 1u : 0u);
         mma_commit(&S.kv_empty[ps]);
         mma_commit(&S.o_bar[pg & 1]);
         return true;
@@ -369,7 +384,7 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
     const uint32_t lane_base = (uint32_t)(quarter * 32) << 16;
     const float kScale = 1.4426950408889634f * 0.125f;  // log2(e) / sqrt(64)
     int g = 0;
-    float m_use = -INFINITY, l = 0.f;
+    float m_use = -INFINITY;
     int tile_in_item = 0;
     for (;;) {
       const int s = g % kStages;
@@ -381,7 +396,6 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
       if (info.flags & kTerm) break;
       if (info.flags & kFirst) {
         m_use = -INFINITY;
-        l = 0.f;
         tile_in_item = 0;
       }
       const int b = g & 1;
@@ -410,11 +424,17 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
           for (int c = 0; c < 64; ++c)
             if (c >= valid) x[c] = -INFINITY;
         }
-        // row max of the raw scores (the scale is positive), three operands at a time
-        float mr = fmax3(x[0], x[1], x[2]);
+        // row max of the raw scores (the scale is positive) as a tree of 3-input maxima
+        float m1[22];
 #pragma unroll
-        for (int c = 3; c < 63; c += 2) mr = fmax3(mr, x[c], x[c + 1]);
-        mr = fmaxf(mr, x[63]);
+        for (int k = 0; k < 21; ++k) m1[k] = fmax3(x[3 * k], x[3 * k + 1], x[3 * k + 2]);
+        m1[21] = x[63];
+        float m2[8];
+#pragma unroll
+        for (int k = 0; k < 7; ++k) m2[k] = fmax3(m1[3 * k], m1[3 * k + 1], m1[3 * k + 2]);
+        m2[7] = m1[21];
+        const float mr =
+            fmax3(fmax3(m2[0], m2[1], m2[2]), fmax3(m2[3], m2[4], m2[5]), fmaxf(m2[6], m2[7]));
         const float mt = mr * kScale;
         float alpha = 1.f;
         bool rescale = false;
@@ -440,22 +460,24 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
             for (int c = 0; c < 32; ++c) v[c] = __float_as_uint(__uint_as_float(v[c]) * alpha);
             RESS_TMEM_ST32(tmem + lane_base + kColO + 32 * hc, v);
           }
+          {  // the row sum (column 64) and the unused columns after it
+            uint32_t v[16];
+            RESS_TMEM_LD16(tmem + lane_base + kColO + 64, v);
+#pragma unroll
+            for (int c = 0; c < 16; ++c) v[c] = __float_as_uint(__uint_as_float(v[c]) * alpha);
+            RESS_TMEM_ST16(tmem + lane_base + kColO + 64, v);
+          }
         }
         // p = 2^(s * log2(e)/8 - m), two columns per packed FMA
         const float nm = -m_use;
-        float rs0 = 0.f, rs1 = 0.f;
         uint32_t w[32];
 #pragma unroll
         for (int e = 0; e < 32; ++e) {
           float t0, t1;
           fma2(t0, t1, x[2 * e], x[2 * e + 1], kScale, kScale, nm, nm);
           w[e] = pack_bf16x2(ex2(t0), ex2(t1));
-          // sum the bf16 values the MMA multiplies, so that a row dominated by one key
-          // keeps O = V exactly up to the accumulation (p reaches 2^8 between rescales)
-          add2(rs0, rs1, rs0, rs1, __uint_as_float(w[e] << 16), __uint_as_float(w[e] & 0xffff0000u));
         }
         RESS_TMEM_ST32(tS, w);  // P_g over the first 32 columns of S_g
-        l = l * alpha + (rs0 + rs1);
       } else {
         uint32_t w[32];
 #pragma unroll
@@ -478,9 +500,11 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
         item_pair(a, info.item, h, p);
         const int token = kRows * p + r;
         const bool row_exists = (2 * p + half) < a.nb && token < a.N;
-        uint32_t o[2][32];
+        uint32_t o[2][32], ls[16];
         RESS_TMEM_LD32(tmem + lane_base + kColO, o[0]);
         RESS_TMEM_LD32(tmem + lane_base + kColO + 32, o[1]);
+        RESS_TMEM_LD16(tmem + lane_base + kColO + 64, ls);
+        const float l = __uint_as_float(ls[0]);  // row sum of the bf16 probabilities
         if (row_exists) {
           if (!(l > 0.f)) flag_status(a.status, kStatusBadRow);
           const float inv = l > 0.f ? 1.0f / l : 0.f;
