@@ -25,7 +25,8 @@
 //              P_g V_g has read it.
 //   warps 2-5  one query row per thread: tcgen05.ld of S, online softmax in the exp2 domain
 //              with lazy rescaling of the TMEM accumulator (only when the running max grows
-//              by more than 2^8), tcgen05.st of P, epilogue O / l.
+//              by more than 2^20, done after P is written so that the exponentials overlap
+//              the previous P V), tcgen05.st of P, epilogue O / l.
 // Every mbarrier wait is bounded; a wait that gives up records RESS_ETIMEOUT in the status
 // word, makes the whole CTA leave its loops, drains in-flight copies and MMAs, frees TMEM
 // and returns.
@@ -50,7 +51,10 @@ constexpr uint64_t kWaitNs = 2000000000ull;  // 2 s per wait
 constexpr uint64_t kDrainNs = 200000000ull;  // 0.2 s to drain after an abort
 constexpr int kFirst = 1, kLast = 2, kTerm = 4;
 constexpr uint32_t kTileBytes = 64 * 128;    // one 64 x 64 bf16 tile
-constexpr float kLazyThreshold = 8.0f;       // log2 units: rescale when max grows > 2^8
+// log2 units: rescale only when the running max grows by more than 2^20.  P is bf16 and O
+// and its row sum accumulate in fp32, so p <= 2^20 over at most 2^18 keys stays far from
+// overflow; a stale max changes no result, the scale cancels in O / l.
+constexpr float kLazyThreshold = 20.0f;
 
 struct TileInfo {
   int j, mask, flags, item;
@@ -64,7 +68,7 @@ struct __align__(1024) AttnSmem {
   uint64_t kv_full[kStages], kv_empty[kStages];
   uint64_t q_full, q_empty;
   uint64_t s_full[2], p_full[2];
-  uint64_t o_bar[2], drain;  // o_bar[k & 1] completes when P_k V_k has landed
+  uint64_t drain;
   TileInfo info[kStages];
   uint32_t tmem_base;
   int abort;
@@ -202,8 +206,6 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
       mbar_init(&S.s_full[b], 1);
       mbar_init(&S.p_full[b], 4);
     }
-    mbar_init(&S.o_bar[0], 1);
-    mbar_init(&S.o_bar[1], 1);
     mbar_init(&S.drain, 1);
     S.abort = 0;
     fence_barrier_init();
@@ -319,8 +321,7 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
           mma_bf16_ts(tmem + kColO, tmem + kColS0 + 64 * pb + 8 * k,
                       (sdesc_sw128(v_addr + 2048 * k) & ~(0x3FFFull << 16)) | lbo, idesc_pv,
                       (k > 0 || !first) ? 1u : 0u);
-        mma_commit(&S.kv_empty[ps]);
-        mma_commit(&S.o_bar[pg & 1]);
+        mma_commit(&S.kv_empty[ps]);  // also tells the softmax warps that P V has landed
         return true;
       };
       for (;;) {
@@ -344,7 +345,8 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
           for (int k = 0; k < 4; ++k) tmem_cp_128x256b(tmem + kColQ + 8 * k, sdesc_sw128(q_addr + 32 * k));
           mma_commit(&S.q_empty);
         }
-        tc_fence_after();
+        // no thread-sync fence here: S_g overwrites what softmax read for tile g-2, and the
+        // fence after waiting for P_{g-2} already orders every later tcgen05 operation
         const int b = g & 1;
         const uint32_t k_addr = smem_u32(S.K[s]);
 #pragma unroll
@@ -445,9 +447,20 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
           m_use = mt;
           rescale = true;
         }
+        // p = 2^(s * log2(e)/8 - m), two columns per packed FMA
+        const float nm = -m_use;
+        uint32_t w[32];
+#pragma unroll
+        for (int e = 0; e < 32; ++e) {
+          float t0, t1;
+          fma2(t0, t1, x[2 * e], x[2 * e + 1], kScale, kScale, nm, nm);
+          w[e] = pack_bf16x2(ex2(t0), ex2(t1));
+        }
+        RESS_TMEM_ST32(tS, w);  // P_g over the first 32 columns of S_g
         if (__any_sync(0xffffffffu, rescale)) {
-          // the previous P V must have landed before the accumulator row is rescaled
-          if (!warp_wait(&S.o_bar[(g - 1) & 1], ((g - 1) >> 1) & 1, abort)) {
+          // the previous P V must have landed before the accumulator row is rescaled; the
+          // exponentials above ran while it was in flight
+          if (!warp_wait(&S.kv_empty[(g - 1) % kStages], ((g - 1) / kStages) & 1, abort)) {
             give_up(S, a.status);
             break;
           }
@@ -468,16 +481,6 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
             RESS_TMEM_ST16(tmem + lane_base + kColO + 64, v);
           }
         }
-        // p = 2^(s * log2(e)/8 - m), two columns per packed FMA
-        const float nm = -m_use;
-        uint32_t w[32];
-#pragma unroll
-        for (int e = 0; e < 32; ++e) {
-          float t0, t1;
-          fma2(t0, t1, x[2 * e], x[2 * e + 1], kScale, kScale, nm, nm);
-          w[e] = pack_bf16x2(ex2(t0), ex2(t1));
-        }
-        RESS_TMEM_ST32(tS, w);  // P_g over the first 32 columns of S_g
       } else {
         uint32_t w[32];
 #pragma unroll
@@ -491,7 +494,7 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
 
       if (info.flags & kLast) {
         // epilogue: O / l for this row once the last P V has landed
-        if (!warp_wait(&S.o_bar[g & 1], (g >> 1) & 1, abort)) {
+        if (!warp_wait(&S.kv_empty[g % kStages], (g / kStages) & 1, abort)) {
           give_up(S, a.status);
           break;
         }
