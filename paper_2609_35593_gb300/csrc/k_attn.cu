@@ -301,83 +301,102 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
     }
   } else if (warp == 1) {
     // ================================ MMA issuer ===================================
-    if (lane == 0) {
-      const uint32_t idesc_qk = idesc_bf16_f32(kRows, 64, false);
-      const uint32_t idesc_pv = idesc_bf16_f32(kRows, kNO, true);
-      const uint32_t ones_addr = smem_u32(S.ONES);
-      const uint32_t q_addr = smem_u32(S.Q);
-      int g = 0, it = 0;
-      bool have_prev = false, prev_first = false, failed = false;
-      int prev_g = 0;
-      auto issue_pv = [&](int pg, bool first) -> bool {
-        const int pb = pg & 1, ps = pg % kStages;
-        if (!mbar_wait(&S.p_full[pb], (pg >> 1) & 1, abort, kWaitNs)) return false;
-        tc_fence_after();
-        const uint32_t v_addr = smem_u32(S.V[ps]);
-        // the N = 80 B operand: atom 0 = V (channels), atom 1 = ONES, LBO bytes after it
-        const uint64_t lbo = (uint64_t)(((ones_addr - v_addr) >> 4) & 0x3FFFu) << 16;
+    // The whole warp walks the pipeline (lane 0 polls each barrier and broadcasts the
+    // verdict) and one lane, chosen by elect.sync, issues every tcgen05 operation: issued
+    // from converged code the MMAs go out several times faster than from a lone thread.
+    const bool leader = elect_one();
+    bool failed = false;
+    if (__popc(__ballot_sync(0xffffffffu, leader)) != 1) {  // exactly one issuing lane
+      if (lane == 0) flag_status(a.status, kStatusBadRow);
+      failed = true;
+    }
+    const uint32_t idesc_qk = idesc_bf16_f32(kRows, 64, false);
+    const uint32_t idesc_pv = idesc_bf16_f32(kRows, kNO, true);
+    const uint32_t ones_addr = smem_u32(S.ONES);
+    const uint32_t q_addr = smem_u32(S.Q);
+    int g = 0, it = 0;
+    bool have_prev = false, prev_first = false;
+    int prev_g = 0;
+    auto issue_pv = [&](int pg, bool first) -> bool {
+      const int pb = pg & 1, ps = pg % kStages;
+      if (!warp_wait(&S.p_full[pb], (pg >> 1) & 1, abort)) return false;
+      tc_fence_after();
+      const uint32_t v_addr = smem_u32(S.V[ps]);
+      // the N = 80 B operand: atom 0 = V (channels), atom 1 = ONES, LBO bytes after it
+      const uint64_t lbo = (uint64_t)(((ones_addr - v_addr) >> 4) & 0x3FFFu) << 16;
+      if (leader) {
 #pragma unroll
         for (int k = 0; k < 4; ++k)
           mma_bf16_ts(tmem + kColO, tmem + kColS0 + 64 * pb + 8 * k,
                       (sdesc_sw128(v_addr + 2048 * k) & ~(0x3FFFull << 16)) | lbo, idesc_pv,
                       (k > 0 || !first) ? 1u : 0u);
         mma_commit(&S.kv_empty[ps]);  // also tells the softmax warps that P V has landed
-        return true;
-      };
-      for (;;) {
-        const int s = g % kStages;
-        if (!mbar_wait(&S.kv_full[s], (g / kStages) & 1, abort, kWaitNs)) {
+      }
+      __syncwarp();
+      return true;
+    };
+    while (!failed) {
+      const int s = g % kStages;
+      if (!warp_wait(&S.kv_full[s], (g / kStages) & 1, abort)) {
+        failed = true;
+        break;
+      }
+      const TileInfo info = S.info[s];
+      if (info.flags & kTerm) break;
+      if (info.flags & kFirst) {
+        if (!warp_wait(&S.q_full, it & 1, abort)) {
           failed = true;
           break;
         }
-        const TileInfo info = S.info[s];
-        if (info.flags & kTerm) break;
-        if (info.flags & kFirst) {
-          if (!mbar_wait(&S.q_full, it & 1, abort, kWaitNs)) {
-            failed = true;
-            break;
-          }
-          tc_fence_after();
-          // Q (128 x 64) into TMEM, one K16 slice (8 columns) per copy; the staging buffer
-          // is free again once the copies have completed.  Copies and MMAs issued by this
-          // thread run in order, so earlier S MMAs have read the previous Q by then.
+        tc_fence_after();
+        // Q (128 x 64) into TMEM, one K16 slice (8 columns) per copy; the staging buffer
+        // is free again once the copies have completed.  Copies and MMAs issued by this
+        // lane run in order, so earlier S MMAs have read the previous Q by then.
+        if (leader) {
 #pragma unroll
           for (int k = 0; k < 4; ++k) tmem_cp_128x256b(tmem + kColQ + 8 * k, sdesc_sw128(q_addr + 32 * k));
           mma_commit(&S.q_empty);
         }
-        // no thread-sync fence here: S_g overwrites what softmax read for tile g-2, and the
-        // fence after waiting for P_{g-2} already orders every later tcgen05 operation
-        const int b = g & 1;
-        const uint32_t k_addr = smem_u32(S.K[s]);
+        __syncwarp();
+      }
+      // no thread-sync fence here: S_g overwrites what softmax read for tile g-2, and the
+      // fence after waiting for P_{g-2} already orders every later tcgen05 operation
+      const int b = g & 1;
+      const uint32_t k_addr = smem_u32(S.K[s]);
+      if (leader) {
 #pragma unroll
         for (int k = 0; k < 4; ++k)
           mma_bf16_ts(tmem + kColS0 + 64 * b, tmem + kColQ + 8 * k, sdesc_sw128(k_addr + 32 * k),
                       idesc_qk, k > 0 ? 1u : 0u);
         mma_commit(&S.s_full[b]);
-        if (have_prev && !issue_pv(prev_g, prev_first)) {
+      }
+      __syncwarp();
+      if (have_prev && !issue_pv(prev_g, prev_first)) {
+        failed = true;
+        break;
+      }
+      if (info.flags & kLast) {
+        if (!issue_pv(g, (info.flags & kFirst) != 0)) {
           failed = true;
           break;
         }
-        if (info.flags & kLast) {
-          if (!issue_pv(g, (info.flags & kFirst) != 0)) {
-            failed = true;
-            break;
-          }
-          have_prev = false;
-          ++it;
-        } else {
-          have_prev = true;
-          prev_g = g;
-          prev_first = (info.flags & kFirst) != 0;
-        }
-        ++g;
+        have_prev = false;
+        ++it;
+      } else {
+        have_prev = true;
+        prev_g = g;
+        prev_first = (info.flags & kFirst) != 0;
       }
-      if (failed) give_up(S, a.status);
-      // wait for every MMA issued so far before TMEM is released
+      ++g;
+    }
+    if (failed && lane == 0) give_up(S, a.status);
+    // wait for every MMA issued so far before TMEM is released
+    if (leader) {
       mma_commit(&S.drain);
       volatile int no_abort = 0;
       mbar_wait(&S.drain, 0, &no_abort, kDrainNs);
     }
+    __syncwarp();
   } else {
     // ================================ softmax =====================================
     const int quarter = warp & 3;
