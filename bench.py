@@ -31,7 +31,7 @@ import numpy as np  # noqa: E402
 METRIC = "ReSS layer ms & kept-FLOP TFLOP/s at 32 views/90% sparsity; select overhead %"
 
 
-def parse():
+def parse(argv=None):
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=200)
@@ -41,7 +41,12 @@ def parse():
     ap.add_argument("--cpu-budget", type=float, default=15.0, help="seconds of oracle work")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--sweep", action="store_true", help="64-view sparsity x rounds sweep lines")
-    return ap.parse_args()
+    return ap.parse_args(argv)
+
+
+def workload(a):
+    import synth
+    return synth.WORKLOADS[a.workload]
 
 
 def peaks():
@@ -170,6 +175,21 @@ def _oracle_attn(args):
     t = time.perf_counter()
     O.block_sparse_attention(*_ORACLE["X"], kept, rows)
     return time.perf_counter() - t
+
+
+def job_totals(dist, ms, units, device="cpu"):
+    """Whole-job figures of N replicas: (the slowest rank's ms, the units all ranks processed).
+
+    `dist` is torch.distributed with an initialised process group, or None for one process.
+    The rate a line reports is units / ms of this pair, so every rank must call it."""
+    if dist is None:
+        return float(ms), float(units)
+    import torch
+    t_max = torch.tensor([float(ms)], dtype=torch.float64, device=device)
+    t_sum = torch.tensor([float(units)], dtype=torch.float64, device=device)
+    dist.all_reduce(t_max, op=dist.ReduceOp.MAX)
+    dist.all_reduce(t_sum, op=dist.ReduceOp.SUM)
+    return float(t_max.item()), float(t_sum.item())
 
 
 def attn_traffic():
@@ -354,12 +374,10 @@ def run_ours(a, wl):
             step()
         ev1.record(stream)
         torch.cuda.synchronize()
+    if dist:
+        dist.barrier()
     ms = ev0.elapsed_time(ev1) / a.steps
     ress.status(buf.ws)
-    if dist:
-        t = torch.tensor([ms], device="cuda")
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
 
     # ---- stage breakdown (same work, events between the three calls) ---------------
     nst = max(20, min(200, a.steps))
@@ -436,16 +454,19 @@ def run_ours(a, wl):
 
     sel_bytes = selection_bytes(N, H, nb, buf.layout.ld, wl.rounds, ci.size)
     sel_ms = score_ms + restore_ms
+    dev = "cuda" if dist and dist.get_backend() == "nccl" else "cpu"
+    ms_job, flops_job = job_totals(dist, ms, flops, dev)      # device-timed step
+    ems_job, eflops_job = job_totals(dist, ems, flops, dev)   # end to end, host buffers
     line = {
-        "metric": METRIC, "value": flops / ms / 1e9 * world, "unit": "TFLOP/s", "n_gpus": world,
-        "steps": a.steps, "warmup": a.warmup, "ms_per_step": ms, "higher_is_better": True,
+        "metric": METRIC, "value": flops_job / ms_job / 1e9, "unit": "TFLOP/s", "n_gpus": world,
+        "steps": a.steps, "warmup": a.warmup, "ms_per_step": ms_job, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
         "data": "synthetic (seeded VGGT-shaped Q/K/V and W_o; inputs 3x larger than L2, no flush)",
         "config": {"workload": wl.name, "views": wl.views, "heads": H, "tokens": N, "head_dim": 64,
                    "block": 64, "sparsity": wl.sparsity, "rounds": wl.rounds, "rho": wl.rho,
                    "c_h": int(c_h[0]), "parallelism": f"replicas{world}",
                    "l2": "inputs larger than L2 (270 MB Q/K/V at 32 views)"},
-        "layer_ms": ms, "stage_ms": {"score": score_ms, "restore": restore_ms, "attn": attn_ms},
+        "layer_ms": ms_job, "stage_ms": {"score": score_ms, "restore": restore_ms, "attn": attn_ms},
         "select_overhead_pct": 100.0 * sel_ms / (sel_ms + attn_ms),
         "attn_tflops": flops / attn_ms / 1e9,
         "selection": {"algorithmic_bytes": sel_bytes, "gbs": sel_bytes / sel_ms / 1e6,
@@ -461,7 +482,7 @@ def run_ours(a, wl):
         # per step: pooling, z-projection, score, score rows; two kernels per round; CSR;
         # pair unions and attention
         "gpu_launches": a.steps * (4 + 2 * wl.rounds + 1 + 2),
-        "e2e": {"value": flops / ems / 1e9 * world, "unit": "TFLOP/s", "ms_per_step": ems,
+        "e2e": {"value": eflops_job / ems_job / 1e9, "unit": "TFLOP/s", "ms_per_step": ems_job,
                 "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
         "clocks": clk.summary(),
     }
@@ -523,8 +544,7 @@ def sweep(a):
 
 def main():
     a = parse()
-    import synth
-    wl = synth.WORKLOADS[a.workload]
+    wl = workload(a)
     if a.impl == "reference":
         run_reference(a, wl)
     else:
