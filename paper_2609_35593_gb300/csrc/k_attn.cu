@@ -314,9 +314,8 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
     const uint32_t idesc_pv = idesc_bf16_f32(kRows, kNO, true);
     const uint32_t ones_addr = smem_u32(S.ONES);
     const uint32_t q_addr = smem_u32(S.Q);
-    int g = 0, it = 0;
-    bool have_prev = false, prev_first = false;
-    int prev_g = 0;
+    bool prev_first = false;
+    int it = 0;
     auto issue_pv = [&](int pg, bool first) -> bool {
       const int pb = pg & 1, ps = pg % kStages;
       if (!warp_wait(&S.p_full[pb], (pg >> 1) & 1, abort)) return false;
@@ -335,14 +334,18 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
       __syncwarp();
       return true;
     };
-    while (!failed) {
-      const int s = g % kStages;
-      if (!warp_wait(&S.kv_full[s], (g / kStages) & 1, abort)) {
-        failed = true;
-        break;
-      }
-      const TileInfo info = S.info[s];
-      if (info.flags & kTerm) break;
+    // the info of tile t once its K/V stage has landed
+    auto fetch = [&](int t, TileInfo& info) -> bool {
+      if (!warp_wait(&S.kv_full[t % kStages], (t / kStages) & 1, abort)) return false;
+      info = S.info[t % kStages];
+      return true;
+    };
+    // Order per tile g: S_g, then (with tile g+1 already landed and its info read, so that
+    // none of that sits between P_{g-1} and the next S) P_{g-1} V_{g-1}.  S_{g+1} overwrites
+    // the buffer of P_{g-1}, which P_{g-1} V_{g-1}, issued before it, has read by then.
+    TileInfo info;
+    if (!failed && !fetch(0, info)) failed = true;
+    for (int g = 0; !failed && !(info.flags & kTerm); ++g) {
       if (info.flags & kFirst) {
         if (!warp_wait(&S.q_full, it & 1, abort)) {
           failed = true;
@@ -358,10 +361,11 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
           mma_commit(&S.q_empty);
         }
         __syncwarp();
+        ++it;
       }
       // no thread-sync fence here: S_g overwrites what softmax read for tile g-2, and the
       // fence after waiting for P_{g-2} already orders every later tcgen05 operation
-      const int b = g & 1;
+      const int s = g % kStages, b = g & 1;
       const uint32_t k_addr = smem_u32(S.K[s]);
       if (leader) {
 #pragma unroll
@@ -371,23 +375,20 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
         mma_commit(&S.s_full[b]);
       }
       __syncwarp();
-      if (have_prev && !issue_pv(prev_g, prev_first)) {
+      const bool first = (info.flags & kFirst) != 0;
+      if (!fetch(g + 1, info)) {
         failed = true;
         break;
       }
-      if (info.flags & kLast) {
-        if (!issue_pv(g, (info.flags & kFirst) != 0)) {
-          failed = true;
-          break;
-        }
-        have_prev = false;
-        ++it;
-      } else {
-        have_prev = true;
-        prev_g = g;
-        prev_first = (info.flags & kFirst) != 0;
+      if (g > 0 && !issue_pv(g - 1, prev_first)) {
+        failed = true;
+        break;
       }
-      ++g;
+      prev_first = first;
+      if ((info.flags & kTerm) && !issue_pv(g, first)) {  // the CTA's last tile
+        failed = true;
+        break;
+      }
     }
     if (failed && lane == 0) give_up(S, a.status);
     // wait for every MMA issued so far before TMEM is released
