@@ -100,11 +100,14 @@ __device__ __forceinline__ void item_pair(const AttnParams& a, int item, int& h,
   }
 }
 
-// Bounded wait for a whole warp: lane 0 polls (one poller per warp keeps the barrier traffic
-// low), the verdict is broadcast so that no lane leaves a loop its neighbours stay in (the
-// warp runs .sync.aligned code), and __syncwarp orders the other lanes' later reads after
-// lane 0's acquire.
+// Bounded wait for a whole warp.  Fast path: every lane tests the barrier (one shared-memory
+// access for the warp, each lane acquiring for itself) and the warp leaves together if all
+// saw the phase complete.  Otherwise lane 0 polls (one poller per warp keeps the barrier
+// traffic low) and the verdict is broadcast, so that no lane leaves a loop its neighbours
+// stay in (the warp runs .sync.aligned code); __syncwarp orders the other lanes' later reads
+// after lane 0's acquire.
 __device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, volatile int* abort) {
+  if (__all_sync(0xffffffffu, mbar_try_wait(bar, parity))) return true;
   int ok = 1;
   if ((threadIdx.x & 31) == 0) ok = mbar_wait(bar, parity, abort, kWaitNs) ? 1 : 0;
   ok = __shfl_sync(0xffffffffu, ok, 0);
