@@ -216,3 +216,39 @@ def test_headline_shape_sampled():
     a = G.compare_attention(layer, arows)
     print(a)
     assert a["max_abs"] <= G.ATT_MAX_ABS and a["mean_rel"] <= G.ATT_MEAN_REL, a
+
+
+def test_attention_rescale_path():
+    """Logits that grow along every kept list by several times the lazy-rescale threshold
+    (2^20 in the exp2 domain), so the kernel rescales its accumulator several times per row;
+    the output must still match the oracle."""
+    N, H, ns, c, R = 64 * 24 + 5, 2, 5, 12, 2
+    inp = synth.make_random_layer(N, H, 64 * H, seed=11)
+    rng = np.random.default_rng(5)
+    q = synth.bf16_to_f32(inp["Q"])
+    k = synth.bf16_to_f32(inp["K"])
+    u = rng.standard_normal((H, 64)).astype(np.float32)
+    blk = np.minimum(np.arange(N) // 64, (N - ns) // 64).astype(np.float32)
+    q = q + 2.0 * u[None]                                  # every query leans along u
+    k = k + (0.3 * blk)[:, None, None] * u[None]           # keys along u grow with the block
+    inp = dict(inp, Q=synth.bf16_bits(q), K=synth.bf16_bits(k))
+    layer = G.Layer(inp, ns, [c] * H, R).run()
+    # the exp2-domain growth of the running block max along each kept list, from the
+    # inputs the kernel received: at least one rescale per sampled row must be needed
+    kq, kk = synth.bf16_to_f32(inp["Q"]), synth.bf16_to_f32(inp["K"])
+    kept = layer.kept()
+    scale = 1.4426950408889634 / 8.0
+    rescales = 0
+    rows = [(h, i) for h in range(H) for i in range(layer.nb)]
+    for (h, i) in rows:
+        qi = kq[64 * i:64 * i + 64, h]
+        m_use = None
+        for j in kept[(h, i)]:
+            mt = float((qi @ kk[64 * j:64 * j + 64, h].T).max(axis=1).min()) * scale
+            if m_use is None:
+                m_use = mt
+            elif mt > m_use + 20.0:
+                m_use, rescales = mt, rescales + 1
+    assert rescales > len(rows)  # several rescales per row on average
+    a = G.compare_attention(layer, rows)
+    assert a["max_abs"] <= G.ATT_MAX_ABS and a["mean_rel"] <= G.ATT_MEAN_REL, a
