@@ -72,12 +72,13 @@ def kept_flops(row_ptr, col_idx, N, H, nb):
 
 
 def selection_bytes(N, H, nb, ld, rounds, csr_entries):
-    """Algorithmic bytes of scoring + restoration: read Q, K, V once; write P and q; per
-    round read P, q, t and read/write the drop masks; write the CSR."""
+    """Algorithmic bytes of scoring + restoration, a fixed formula whatever the kernels move:
+    read Q, K, V once and write P and q (score); per round read P and q and read/write the
+    drop masks (one bit per pair); write the CSR (col_idx and row_ptr)."""
     mat = H * nb * nb * 4
     score = 3 * N * H * 64 * 2 + 2 * mat
-    per_round = 3 * mat + 2 * H * nb * math.ceil(nb / 32) * 4
-    return score + rounds * per_round + 4 * (csr_entries + H * nb + 1)
+    per_round = 2 * mat + 2 * H * nb * nb // 8
+    return score + rounds * per_round + 4 * csr_entries + 4 * (H * nb + 1)
 
 
 # ----------------------------------------------------------------------------------------
