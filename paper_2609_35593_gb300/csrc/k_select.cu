@@ -244,6 +244,16 @@ __device__ __forceinline__ uint64_t fsub2(uint64_t a, uint64_t b) {
   asm("sub.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
   return d;
 }
+__device__ __forceinline__ uint64_t pack2(float lo, float hi) {
+  uint64_t d;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(d) : "f"(lo), "f"(hi));
+  return d;
+}
+__device__ __forceinline__ float2 unpack2(uint64_t v) {
+  float2 r;
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(r.x), "=f"(r.y) : "l"(v));
+  return r;
+}
 __device__ __forceinline__ float hsum2(uint64_t v) {
   float lo, hi;
   asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(v));
@@ -588,9 +598,9 @@ __global__ void __launch_bounds__(kThreads, 2) k_score(SelPtrs p, Budgets bud) {
   __syncthreads();
 
   // ---- pass 2: P_ij = softmax, y~_i = sum_j P_ij z~_j (Eq. 1 in F space) -----------
-  float ya[4][2];
+  uint64_t ya[4];  // (channel 2 lane, channel 2 lane + 1) of 4 rows, packed f32x2
 #pragma unroll
-  for (int x = 0; x < 4; ++x) ya[x][0] = ya[x][1] = 0.f;
+  for (int x = 0; x < 4; ++x) ya[x] = 0ull;
   for (int j0 = 0; j0 < p.nb; j0 += BN) {
     stage_blocks(S.B, zt_h, j0, p.nb);
     for (int f = threadIdx.x; f < RT * (BN / 4); f += kThreads) {
@@ -620,12 +630,11 @@ __global__ void __launch_bounds__(kThreads, 2) k_score(SelPtrs p, Budgets bud) {
       for (int x = 0; x < 4; ++x) pv[x] = *reinterpret_cast<const float4*>(&S.Pc[warp * 4 + x][jj]);
 #pragma unroll
       for (int u = 0; u < 4; ++u) {
-        const float2 z = *reinterpret_cast<const float2*>(&S.B[jj + u][2 * lane]);
+        const uint64_t z = *reinterpret_cast<const uint64_t*>(&S.B[jj + u][2 * lane]);
 #pragma unroll
         for (int x = 0; x < 4; ++x) {
           const float pu = u == 0 ? pv[x].x : (u == 1 ? pv[x].y : (u == 2 ? pv[x].z : pv[x].w));
-          ya[x][0] = fmaf(pu, z.x, ya[x][0]);
-          ya[x][1] = fmaf(pu, z.y, ya[x][1]);
+          ya[x] = ffma2(pack2(pu, pu), z, ya[x]);  // each half an fma.rn, as fmaf
         }
       }
     }
@@ -634,11 +643,10 @@ __global__ void __launch_bounds__(kThreads, 2) k_score(SelPtrs p, Budgets bud) {
 #pragma unroll
   for (int x = 0; x < 4; ++x) {
     const int r = warp * 4 + x;
-    S.A[r][2 * lane] = ya[x][0];
-    S.A[r][2 * lane + 1] = ya[x][1];
-    if (r < nrows)
-      *reinterpret_cast<float2*>(p.ytil + (hrow + i0 + r) * 64 + 2 * lane) =
-          make_float2(ya[x][0], ya[x][1]);
+    const float2 y = unpack2(ya[x]);
+    S.A[r][2 * lane] = y.x;
+    S.A[r][2 * lane + 1] = y.y;
+    if (r < nrows) *reinterpret_cast<float2*>(p.ytil + (hrow + i0 + r) * 64 + 2 * lane) = y;
   }
   __syncthreads();
 
@@ -753,9 +761,11 @@ __device__ __forceinline__ int swap_count(int c, int ncand, int round, float rho
 
 // ------------------------------------------------------------------------------------
 // Restoration round r (Sec. 4.3, Eq. 13-17), first half: the gain inner products
-// t_ij = (y~_i - z~_j) . g~_i for RT rows of one head.  grid (ceil(ncand / RT), H).
+// t_ij = (y~_i - z~_j) . g~_i for RT rows of one head and one BN-block chunk of candidates.
+// grid (ceil(ncand / RT), H, ceil(ncand / BN)): small CTAs in many waves, so the last wave
+// leaves little of the GPU idle.
 // ------------------------------------------------------------------------------------
-__global__ void __launch_bounds__(kThreads, 2) k_round(SelPtrs p, Budgets bud, int round,
+__global__ void __launch_bounds__(kThreads, 3) k_round(SelPtrs p, Budgets bud, int round,
                                                        float rho) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
   SelSmem& S = *reinterpret_cast<SelSmem*>(smem_raw);
@@ -769,22 +779,20 @@ __global__ void __launch_bounds__(kThreads, 2) k_round(SelPtrs p, Budgets bud, i
   float* tbase = p.t + (hrow + i0) * p.ld;
 
   // ---- gains: t_ij = (y~_i - z~_j) . g~_i  (Eq. 14/15 without the P_ij factor) -------
+  const int j0 = blockIdx.z * BN;
   stage_rows(S.A, p.ytil + (hrow + i0) * 64, nrows);
   stage_rows(S.Gv, p.gtil + (hrow + i0) * 64, nrows);
-  for (int j0 = 0; j0 < p.ncand; j0 += BN) {
-    stage_blocks(S.B, zt_h, j0, p.ncand);
-    __syncthreads();
-    float acc[8][2];
-    tile8x2<kOpGain>(S, rg, jb, acc);
+  stage_blocks(S.B, zt_h, j0, p.ncand);
+  __syncthreads();
+  float acc[8][2];
+  tile8x2<kOpGain>(S, rg, jb, acc);
 #pragma unroll
-    for (int x = 0; x < 8; ++x) {
-      const int r = rg * 8 + x;
-      if (r < nrows) {
-        if (j0 + jb < p.ncand) tbase[(int64_t)r * p.ld + j0 + jb] = acc[x][0];
-        if (j0 + jb + 32 < p.ncand) tbase[(int64_t)r * p.ld + j0 + jb + 32] = acc[x][1];
-      }
+  for (int x = 0; x < 8; ++x) {
+    const int r = rg * 8 + x;
+    if (r < nrows) {
+      if (j0 + jb < p.ncand) tbase[(int64_t)r * p.ld + j0 + jb] = acc[x][0];
+      if (j0 + jb + 32 < p.ncand) tbase[(int64_t)r * p.ld + j0 + jb + 32] = acc[x][1];
     }
-    __syncthreads();
   }
 
 }
@@ -935,10 +943,11 @@ cudaError_t launch_round(const SelectArgs& a, int round, float rho, cudaStream_t
   const Shape& s = a.s;
   if (s.ncand <= 0) return cudaSuccess;
   SelPtrs p = sel_ptrs(s, a.ws, a.L);
-  const size_t smem = sizeof(SelSmem);
+  const size_t smem = offsetof(SelSmem, Pc);  // the gain pass stages no P chunk
   cudaError_t e = cudaFuncSetAttribute(k_round, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
-  k_round<<<dim3((s.ncand + RT - 1) / RT, s.H), kThreads, smem, st>>>(p, budgets_of(a), round, rho);
+  k_round<<<dim3((s.ncand + RT - 1) / RT, s.H, (s.ncand + BN - 1) / BN), kThreads, smem, st>>>(
+      p, budgets_of(a), round, rho);
   const size_t rsmem = (size_t)kRowWarps * warp_scratch_words(s.ld, 3 * s.words) * 4;
   e = cudaFuncSetAttribute(k_round_rows, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)rsmem);
   if (e != cudaSuccess) return e;
