@@ -540,7 +540,7 @@ struct Budgets {
   int c[RESS_MAX_HEADS];
 };
 
-__global__ void __launch_bounds__(kThreads, 2) k_score(SelPtrs p, Budgets bud) {
+__global__ void __launch_bounds__(kThreads, 3) k_score(SelPtrs p, Budgets bud) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
   SelSmem& S = *reinterpret_cast<SelSmem*>(smem_raw);
   const int h = blockIdx.y, i0 = blockIdx.x * RT;
