@@ -252,3 +252,31 @@ def test_attention_rescale_path():
     assert rescales > len(rows)  # several rescales per row on average
     a = G.compare_attention(layer, rows)
     assert a["max_abs"] <= G.ATT_MAX_ABS and a["mean_rel"] <= G.ATT_MEAN_REL, a
+
+
+@pytest.mark.parametrize("name,kw", [
+    ("vggt_v100", {}),                                  # 137400 tokens, cross-view term
+    ("vggt_v64", {"sparsity": 0.5, "rounds": 4}),       # sweep corners
+    ("vggt_v64", {"sparsity": 0.95, "rounds": 0}),
+])
+def test_large_shapes_sampled(name, kw):
+    """The long-view configuration and two corners of the 64-view sweep: sampled rows
+    against the oracle, and the properties that hold at any size on every row."""
+    layer, wl = layer_for(name, **kw)
+    layer.run()
+    rng = np.random.default_rng(2)
+    rows = [(int(h), int(i)) for h, i in zip(rng.integers(0, wl.heads, 10), rng.integers(0, wl.n_candidates, 10))]
+    r = G.compare_selection(layer, layer.oracle_select(rows))
+    print(name, kw, r)
+    assert r["mismatched"] == 0, r
+    J0 = layer.ws("J0", shape=(layer.H, layer.nb))
+    Jb = layer.buf.J_best.cpu().numpy().reshape(layer.H, layer.nb)
+    assert np.all(Jb[:, :layer.ncand] <= J0[:, :layer.ncand])
+    if wl.rounds == 0:
+        assert np.array_equal(Jb[:, :layer.ncand], J0[:, :layer.ncand])
+    rp, ci = layer.csr()
+    assert rp[-1] == ci.size
+    arows = rows[:6] + [(0, layer.nb - 1), (wl.heads - 1, layer.nb - 2)]
+    a = G.compare_attention(layer, arows)
+    print(a)
+    assert a["max_abs"] <= G.ATT_MAX_ABS and a["mean_rel"] <= G.ATT_MEAN_REL, a
