@@ -778,23 +778,30 @@ __global__ void __launch_bounds__(kThreads, 3) k_round(SelPtrs p, Budgets bud, i
   const float* zt_h = p.ztil + hrow * 64;
   float* tbase = p.t + (hrow + i0) * p.ld;
 
-  // ---- gains: t_ij = (y~_i - z~_j) . g~_i  (Eq. 14/15 without the P_ij factor) -------
+  // ---- gains: t_ij = (y~_i - z~_j) . g~_i  (Eq. 14/15 without the P_ij factor), as
+  // c_i - z~_j . g~_i with c_i = y~_i . g~_i: one packed FMA per channel pair -------------
   const int j0 = blockIdx.z * BN;
-  stage_rows(S.A, p.ytil + (hrow + i0) * 64, nrows);
-  stage_rows(S.Gv, p.gtil + (hrow + i0) * 64, nrows);
+  stage_rows(S.A, p.gtil + (hrow + i0) * 64, nrows);
+  stage_rows(S.Gv, p.ytil + (hrow + i0) * 64, nrows);
   stage_blocks(S.B, zt_h, j0, p.ncand);
   __syncthreads();
+  for (int r = warp; r < RT; r += kThreads / 32) {
+    const float c = warp_sum(S.A[r][2 * lane] * S.Gv[r][2 * lane] +
+                             S.A[r][2 * lane + 1] * S.Gv[r][2 * lane + 1]);
+    if (lane == 0) S.rowm[r] = c;
+  }
+  __syncthreads();
   float acc[8][2];
-  tile8x2<kOpGain>(S, rg, jb, acc);
+  tile8x2<kOpDot>(S, rg, jb, acc);
 #pragma unroll
   for (int x = 0; x < 8; ++x) {
     const int r = rg * 8 + x;
     if (r < nrows) {
-      if (j0 + jb < p.ncand) tbase[(int64_t)r * p.ld + j0 + jb] = acc[x][0];
-      if (j0 + jb + 32 < p.ncand) tbase[(int64_t)r * p.ld + j0 + jb + 32] = acc[x][1];
+      const float c = S.rowm[r];
+      if (j0 + jb < p.ncand) tbase[(int64_t)r * p.ld + j0 + jb] = c - acc[x][0];
+      if (j0 + jb + 32 < p.ncand) tbase[(int64_t)r * p.ld + j0 + jb + 32] = c - acc[x][1];
     }
   }
-
 }
 
 // Restoration round r, per row: exact top-m restores and drops from the round-start state,
@@ -943,7 +950,7 @@ cudaError_t launch_round(const SelectArgs& a, int round, float rho, cudaStream_t
   const Shape& s = a.s;
   if (s.ncand <= 0) return cudaSuccess;
   SelPtrs p = sel_ptrs(s, a.ws, a.L);
-  const size_t smem = offsetof(SelSmem, Pc);  // the gain pass stages no P chunk
+  const size_t smem = sizeof(SelSmem);
   cudaError_t e = cudaFuncSetAttribute(k_round, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   k_round<<<dim3((s.ncand + RT - 1) / RT, s.H, (s.ncand + BN - 1) / BN), kThreads, smem, st>>>(
