@@ -499,6 +499,48 @@ __device__ __forceinline__ void kept_drift(const uint32_t* D, const SelPtrs& p,
   __syncwarp();
 }
 
+// The state after a round from the one before it: the restored blocks R join the kept set
+// and the dropped blocks X leave it, so g~ += sum_R P_k (z~_k - y~) - sum_X P_k (z~_k - y~)
+// and K += sum_R P_k - sum_X P_k over the 2m swapped blocks (exactly the kept-set sums of
+// Eq. 10-11 in exact arithmetic).  Same lane layout and staging as kept_drift.
+__device__ __forceinline__ void swap_drift(const uint32_t* R, const uint32_t* X, const SelPtrs& p,
+                                           const float* __restrict__ Prow,
+                                           const float* __restrict__ zt, float y0, float y1,
+                                           uint32_t* idx, float& g0, float& g1, float& K) {
+  const int lane = threadIdx.x & 31;
+  int n = 0;
+  for (int w = 0; w < p.words; ++w) {
+    const uint32_t sw = R[w] | X[w];
+    if ((sw >> lane) & 1u)
+      idx[n + __popc(sw & ((1u << lane) - 1u))] = (w * 32 + lane) | (((X[w] >> lane) & 1u) << 31);
+    n += __popc(sw);
+  }
+  __syncwarp();
+  for (int k0 = 0; k0 < n; k0 += 8) {
+    float pj[8];
+    float2 z[8];
+#pragma unroll
+    for (int u = 0; u < 8; ++u) {
+      pj[u] = 0.f;
+      z[u] = make_float2(y0, y1);
+      if (k0 + u < n) {
+        const uint32_t e = idx[k0 + u];
+        const int j = (int)(e & 0x7fffffffu);
+        const float pv = Prow[j];
+        pj[u] = (e >> 31) ? -pv : pv;
+        z[u] = *reinterpret_cast<const float2*>(zt + (int64_t)j * 64 + 2 * lane);
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < 8; ++u) {
+      g0 = fmaf(pj[u], z[u].x - y0, g0);
+      g1 = fmaf(pj[u], z[u].y - y1, g1);
+      K += pj[u];
+    }
+  }
+  __syncwarp();
+}
+
 // Per-warp scratch of the per-row phase: keys [ld] u32, survivor keys [kSurvivors] u32,
 // survivor indices [kSurvivors] u16, bitmask words.  It reuses the GEMM staging area (B,
 // Pc), which the per-row phase no longer needs, when that area is large enough.
@@ -850,10 +892,11 @@ __global__ void __launch_bounds__(32 * kRowWarps, 8) k_round_rows(SelPtrs p, Bud
   warp_topm(kk, p.ncand, m, Xw, p.words, sk, si, Dw, false);
   for (int w = lane; w < p.words; w += 32) Dw[w] = (Dw[w] & ~Rw[w]) | Xw[w];
   __syncwarp();
-  // exact state of the new set (Eq. 10-12)
+  // state of the new set (Eq. 10-12): the swapped blocks update g~ and K
   const float2 y = *reinterpret_cast<const float2*>(p.ytil + ri * 64 + 2 * lane);
-  float g0, g1, Kn;
-  kept_drift(Dw, p, Prow, zt_h, y.x, y.y, kk, g0, g1, Kn);
+  const float2 gold = *reinterpret_cast<const float2*>(p.gtil + ri * 64 + 2 * lane);
+  float g0 = gold.x, g1 = gold.y, Kn = K;
+  swap_drift(Rw, Xw, p, Prow, zt_h, y.x, y.y, kk, g0, g1, Kn);
   const float Gn = warp_sum(g0 * g0 + g1 * g1);
   const float Kc = fmaxf(Kn, kEps);
   const float Jn = Gn / (Kc * Kc);
