@@ -435,13 +435,10 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
       if (active) {
         float x[64];
         {
-          uint32_t v[32];
-          RESS_TMEM_LD32(tS, v);
+          uint32_t v[64];
+          RESS_TMEM_LD64(tS, v);
 #pragma unroll
-          for (int c = 0; c < 32; ++c) x[c] = __uint_as_float(v[c]);
-          RESS_TMEM_LD32(tS + 32, v);
-#pragma unroll
-          for (int c = 0; c < 32; ++c) x[32 + c] = __uint_as_float(v[c]);
+          for (int c = 0; c < 64; ++c) x[c] = __uint_as_float(v[c]);
         }
         if (info.j == a.nb - 1) {  // ragged last key block: keys past N do not exist
           const int valid = a.N - 64 * info.j;
