@@ -152,6 +152,7 @@ __global__ void __launch_bounds__(256) k_pairs(const int32_t* __restrict__ row_p
     }
     return;
   }
+#pragma unroll 4
   for (int64_t x = sa + lane; x < eb; x += 32) {
     const int j = col_idx[x];
     if (j < 0 || j >= nb) {
@@ -161,28 +162,17 @@ __global__ void __launch_bounds__(256) k_pairs(const int32_t* __restrict__ row_p
     atomicOr((x < ea ? bA : bB) + (j >> 5), 1u << (j & 31));
   }
   __syncwarp();
-  // lane l owns words [4l, 4l + 4)
-  int cnt = 0;
-  for (int w = 4 * lane; w < min(words, 4 * lane + 4); ++w) cnt += __popc(bA[w] | bB[w]);
-  int incl = cnt;
-#pragma unroll
-  for (int o = 1; o < 32; o <<= 1) {
-    const int v = __shfl_up_sync(0xffffffffu, incl, o);
-    if (lane >= o) incl += v;
-  }
-  int pos = incl - cnt;
-  for (int w = 4 * lane; w < min(words, 4 * lane + 4); ++w) {
-    const uint32_t a = bA[w], b = bB[w];
-    uint32_t u = a | b;
-    while (u) {
-      const int bit = __ffs(u) - 1;
-      u &= u - 1;
-      const int m = (int)((a >> bit) & 1u) | (int)(((b >> bit) & 1u) << 1);
-      plist[sa + pos] = (w * 32 + bit) | (m << 16);
-      ++pos;
+  // union in ascending block order, 32 blocks per step: lane l looks at block 32 w + l
+  int pos = 0;
+  for (int w = 0; w < words; ++w) {
+    const uint32_t a = bA[w], b = bB[w], u = a | b;
+    if ((u >> lane) & 1u) {
+      const int m = (int)((a >> lane) & 1u) | (int)(((b >> lane) & 1u) << 1);
+      plist[sa + pos + __popc(u & ((1u << lane) - 1u))] = (w * 32 + lane) | (m << 16);
     }
+    pos += __popc(u);
   }
-  if (lane == 31) plen[pair] = incl;
+  if (lane == 0) plen[pair] = pos;
 }
 
 // ------------------------------------------------------------------------------------
