@@ -158,6 +158,23 @@ int ress_forward(const ress_dims* dims, const uint16_t* Q, const uint16_t* K, co
                  size_t ws_bytes, int32_t* row_ptr, int32_t* col_idx, int64_t col_capacity,
                  uint16_t* O, float* J_best, void* stream);
 
+/* ress_forward from host memory to host memory, for callers that keep a layer's Q, K, V
+ * and O on the host (the paper has no counterpart: an interface, not part of the method).
+ * Enqueued on `stream`, in order: host -> device copies of Q, K, V into the caller's device
+ * buffers Q_dev, K_dev, V_dev, then ress_forward on them, then the device -> host copy of
+ * O_dev into O_host; nothing waits for completion.  Host buffers should be page-locked (for
+ * example cudaHostAlloc) for the copies to overlap other work; every buffer belongs to the
+ * caller and must stay untouched until the stream has passed the call.  Two calls on two
+ * streams with separate device buffers, workspaces and CSR arrays overlap one layer's copies
+ * with another's compute.  Q_host, K_host, V_host, O_host: bf16 [N, H, 64]; the other
+ * arguments as ress_forward.  Returns as ress_forward, or RESS_ECUDA if a copy could not be
+ * enqueued; arguments are checked before anything is enqueued. */
+int ress_forward_host(const ress_dims* dims, const uint16_t* Q_host, const uint16_t* K_host,
+                      const uint16_t* V_host, uint16_t* O_host, uint16_t* Q_dev, uint16_t* K_dev,
+                      uint16_t* V_dev, uint16_t* O_dev, const float* F, const int32_t* c_h_host,
+                      int32_t rounds, float rho, void* ws, size_t ws_bytes, int32_t* row_ptr,
+                      int32_t* col_idx, int64_t col_capacity, float* J_best, void* stream);
+
 /* Allocation-free variant of ress_sparse_attn (the paper has no counterpart: this is an
  * interface for callers, not part of the method).  It is for callers that cannot allocate
  * device memory when they call in: a host framework that owns all device memory through

@@ -69,6 +69,9 @@ _SIGS = {
                                         _c.c_size_t, _P]),
     "ress_forward": (_c.c_int, [_c.POINTER(Dims), _P, _P, _P, _P, _P, _c.c_int32, _c.c_float, _P,
                                 _c.c_size_t, _P, _P, _c.c_int64, _P, _P, _P]),
+    "ress_forward_host": (_c.c_int, [_c.POINTER(Dims), _P, _P, _P, _P, _P, _P, _P, _P, _P, _P,
+                                     _c.c_int32, _c.c_float, _P, _c.c_size_t, _P, _P, _c.c_int64,
+                                     _P, _P]),
     "ress_status": (_c.c_int, [_P, _P]),
     "ress_sparse_attn_noalloc": (_c.c_int, [_c.POINTER(Dims), _P, _P, _P, _P, _P, _c.c_int64, _P,
                                             _c.c_int32, _P]),
@@ -149,6 +152,20 @@ def _dev(t, dtypes, name):
     return _c.c_void_p(t.data_ptr())
 
 
+def _host(t, dtypes, name):
+    """Host pointer of a contiguous CPU tensor (page-locked for asynchronous copies)."""
+    torch = _torch()
+    if not isinstance(t, torch.Tensor):
+        raise TypeError(f"{name} must be a torch.Tensor")
+    if t.device.type != "cpu":
+        raise ValueError(f"{name} must live in host memory")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    if dtypes is not None and t.dtype not in dtypes:
+        raise TypeError(f"{name} has dtype {t.dtype}, expected one of {dtypes}")
+    return _c.c_void_p(t.data_ptr())
+
+
 def _stream(stream):
     torch = _torch()
     s = torch.cuda.current_stream() if stream is None else stream
@@ -216,6 +233,24 @@ def forward(d: Dims, Q, K, V, F, c_h, rounds: int, rho: float, ws, row_ptr, col_
                              _dev(col_idx, (torch.int32,), "col_idx"), col_idx.numel(),
                              _dev(O, _bf16(), "O"), _dev(J_best, (torch.float32,), "J_best"),
                              _stream(stream)))
+
+
+def forward_host(d: Dims, Q_host, K_host, V_host, O_host, Q_dev, K_dev, V_dev, O_dev, F, c_h,
+                 rounds: int, rho: float, ws, row_ptr, col_idx, J_best=None, stream=None):
+    """ress_forward_host: copies of Q, K, V in, the forward, the copy of O out, all enqueued
+    on `stream` (host tensors should be pinned)."""
+    torch = _torch()
+    b = _bf16()
+    _check(_lib.ress_forward_host(_c.byref(d), _host(Q_host, b, "Q_host"), _host(K_host, b, "K_host"),
+                                  _host(V_host, b, "V_host"), _host(O_host, b, "O_host"),
+                                  _dev(Q_dev, b, "Q_dev"), _dev(K_dev, b, "K_dev"),
+                                  _dev(V_dev, b, "V_dev"), _dev(O_dev, b, "O_dev"),
+                                  _dev(F, (torch.float32,), "F"), _c.cast(_budget_array(c_h), _P),
+                                  int(rounds), float(rho), _dev(ws, None, "ws"),
+                                  ws.numel() * ws.element_size(),
+                                  _dev(row_ptr, (torch.int32,), "row_ptr"),
+                                  _dev(col_idx, (torch.int32,), "col_idx"), col_idx.numel(),
+                                  _dev(J_best, (torch.float32,), "J_best"), _stream(stream)))
 
 
 def sparse_attn_noalloc(d: Dims, Q, K, V, row_ptr, col_idx, O, wait: bool = True, stream=None):

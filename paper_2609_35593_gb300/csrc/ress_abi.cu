@@ -266,6 +266,48 @@ int ress_forward(const ress_dims* d, const uint16_t* Q, const uint16_t* K, const
   return ress_sparse_attn(d, Q, K, V, row_ptr, col_idx, col_capacity, O, ws, ws_bytes, stream);
 }
 
+int ress_forward_host(const ress_dims* d, const uint16_t* Q_host, const uint16_t* K_host,
+                      const uint16_t* V_host, uint16_t* O_host, uint16_t* Q_dev, uint16_t* K_dev,
+                      uint16_t* V_dev, uint16_t* O_dev, const float* F, const int32_t* c_h,
+                      int32_t rounds, float rho, void* ws, size_t ws_bytes, int32_t* row_ptr,
+                      int32_t* col_idx, int64_t col_capacity, float* J_best, void* stream) {
+  int e = check_dims(d);
+  if (e) return e;
+  if (!Q_host || !K_host || !V_host || !O_host) return fail(RESS_EINVAL, "null host buffer");
+  if ((e = check_ptr(Q_dev, 16, "Q_dev")) || (e = check_ptr(K_dev, 16, "K_dev")) ||
+      (e = check_ptr(V_dev, 16, "V_dev")) || (e = check_ptr(O_dev, 16, "O_dev")))
+    return e;
+  const size_t bytes = (size_t)d->n_tokens * (size_t)d->n_heads * 64 * sizeof(uint16_t);
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  // the forward's own checks run before any copy is enqueued: a dry validation first
+  {
+    const ress::Shape s = ress::make_shape(*d);
+    if ((e = check_budgets(s, c_h))) return e;
+    if (rounds < 0 || rounds > 32) return fail(RESS_EINVAL, "rounds %d outside 0..32", rounds);
+    if (!(rho >= 0.0f && rho <= 1.0f)) return fail(RESS_EINVAL, "rho %g outside [0, 1]", (double)rho);
+    if ((e = check_ptr(row_ptr, 4, "row_ptr")) || (e = check_ptr(col_idx, 4, "col_idx"))) return e;
+    if (J_best && (e = check_ptr(J_best, 4, "J_best"))) return e;
+    ress_ws_layout L;
+    if ((e = check_ws(s, ws, ws_bytes, &L))) return e;
+    int64_t base[RESS_MAX_HEADS + 1];
+    head_bases(s, c_h, base);
+    if (col_capacity < base[s.H])
+      return fail(RESS_EWORKSPACE, "col_capacity %lld < %lld", (long long)col_capacity, (long long)base[s.H]);
+  }
+  const uint16_t* src[3] = {Q_host, K_host, V_host};
+  uint16_t* dst[3] = {Q_dev, K_dev, V_dev};
+  for (int k = 0; k < 3; ++k) {  // one copy per tensor
+    cudaError_t ce = cudaMemcpyAsync(dst[k], src[k], bytes, cudaMemcpyHostToDevice, st);
+    if (ce != cudaSuccess) return cuda_fail(ce, "ress_forward_host input copy");
+  }
+  if ((e = ress_forward(d, Q_dev, K_dev, V_dev, F, c_h, rounds, rho, ws, ws_bytes, row_ptr, col_idx,
+                        col_capacity, O_dev, J_best, stream)))
+    return e;
+  cudaError_t ce = cudaMemcpyAsync(O_host, O_dev, bytes, cudaMemcpyDeviceToHost, st);
+  if (ce != cudaSuccess) return cuda_fail(ce, "ress_forward_host output copy");
+  return ok();
+}
+
 int ress_status(void* ws, void* stream) {
   int e = check_ptr(ws, 256, "ws");
   if (e) return e;

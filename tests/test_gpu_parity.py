@@ -280,3 +280,20 @@ def test_large_shapes_sampled(name, kw):
     a = G.compare_attention(layer, arows)
     print(a)
     assert a["max_abs"] <= G.ATT_MAX_ABS and a["mean_rel"] <= G.ATT_MEAN_REL, a
+
+
+def test_forward_host_equals_forward(tiny):
+    """ress_forward_host (copies in, forward, copy out, one stream) gives the bits of the
+    staged device calls."""
+    layer, _ = layer_for("tiny_v2")
+    r, b = layer.ress, layer.buf
+    r.prepare_wo(layer.d, layer.W, b.F)
+    Qh, Kh, Vh = (t.cpu().pin_memory() for t in (layer.Q, layer.K, layer.V))
+    Oh = torch.empty(b.O.shape, dtype=torch.bfloat16).pin_memory()
+    Qd, Kd, Vd, Od = (torch.empty_like(t) for t in (layer.Q, layer.K, layer.V, b.O))
+    r.forward_host(layer.d, Qh, Kh, Vh, Oh, Qd, Kd, Vd, Od, b.F, layer.c_h, layer.rounds,
+                   layer.rho, b.ws, b.row_ptr, b.col_idx, b.J_best)
+    r.status(b.ws)
+    torch.cuda.synchronize()
+    assert torch.equal(Oh.view(torch.int16), tiny.buf.O.cpu().view(torch.int16))
+    assert np.array_equal(layer.csr()[1], tiny.csr()[1])
