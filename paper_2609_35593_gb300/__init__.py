@@ -46,7 +46,8 @@ class WsLayout(ctypes.Structure):
     """ress_ws_layout: byte offsets of the workspace arrays."""
     _fields_ = [(n, ctypes.c_int64) for n in
                 ("status", "counter", "qbar", "kbar", "vbar", "ztil", "ytil", "gtil", "P", "q", "t",
-                 "K", "G", "J", "Jbest", "J0", "dmask", "bmask", "plen", "ld", "words", "total")]
+                 "K", "G", "J", "Jbest", "J0", "dmask", "bmask", "plen", "gsplit", "zsplit", "cdot",
+                 "ld", "words", "total")]
 
 
 _c = ctypes
@@ -291,7 +292,7 @@ class Buffers:
         L = self.layout
         names = [f[0] for f in WsLayout._fields_]
         off = getattr(L, name)
-        order = sorted(getattr(L, n) for n in names[:19])
+        order = sorted(getattr(L, n) for n in names[:names.index("ld")])
         nxt = min([o for o in order if o > off] + [L.total])
         dtype = dtype or torch.float32
         raw = self.ws[off:nxt]

@@ -142,7 +142,9 @@ __global__ void __launch_bounds__(kThreads) k_pool(const uint16_t* __restrict__ 
 // ------------------------------------------------------------------------------------
 __global__ void __launch_bounds__(kThreads) k_zproj(const float* __restrict__ F,
                                                      const float* __restrict__ vbar, int nb,
-                                                     float* __restrict__ ztil) {
+                                                     float* __restrict__ ztil,
+                                                     uint2* __restrict__ zsplit,
+                                                     int64_t term_stride) {
   __shared__ __align__(16) float Ft[64][64];  // Ft[b][a] = F[a][b]
   __shared__ float Vs[16][65];
   const int h = blockIdx.y, j0 = blockIdx.x * 16, t = threadIdx.x;
@@ -164,7 +166,15 @@ __global__ void __launch_bounds__(kThreads) k_zproj(const float* __restrict__ F,
     acc.z = fmaf(f.z, v, acc.z);
     acc.w = fmaf(f.w, v, acc.w);
   }
-  *reinterpret_cast<float4*>(ztil + ((int64_t)h * nb + j0 + jj) * 64 + a4) = acc;
+  const int64_t at = ((int64_t)h * nb + j0 + jj) * 64 + a4;
+  *reinterpret_cast<float4*>(ztil + at) = acc;
+  // the same vectors as three bf16 terms, the B operands of the tensor-core gains
+  uint2 hi, mid, lo;
+  split3_bf16x2(acc.x, acc.y, hi.x, mid.x, lo.x);
+  split3_bf16x2(acc.z, acc.w, hi.y, mid.y, lo.y);
+  zsplit[at / 4] = hi;
+  zsplit[at / 4 + term_stride] = mid;
+  zsplit[at / 4 + 2 * term_stride] = lo;
 }
 
 // ------------------------------------------------------------------------------------
@@ -172,7 +182,6 @@ __global__ void __launch_bounds__(kThreads) k_zproj(const float* __restrict__ F,
 // ------------------------------------------------------------------------------------
 struct SelSmem {
   float A[RT][LDA];      // per-row 64-vectors: q_bar, then y~
-  float Gv[RT][LDA];     // per-row g~ (round kernel)
   float B[BN][LDA];      // staged chunk of per-block 64-vectors (k_bar or z~)
   float Pc[RT][BN + 4];  // staged chunk of P (score kernel)
   float rowm[RT], rowiz[RT];
@@ -183,6 +192,9 @@ struct SelPtrs {
   const float *qbar, *kbar, *ztil;
   float *ytil, *gtil, *P, *q, *t, *K, *G, *J, *Jbest, *J0;
   uint32_t *dmask, *bmask;
+  uint32_t* gsplit;      // bf16x2 [3][H][nb][32]: g~ as three bf16 terms (tensor-core gains)
+  float* cdot;           // [H, nb] y~_i . g~_i
+  int64_t split_stride;  // H nb 32: uint32 words per term
 };
 
 __host__ __device__ inline SelPtrs sel_ptrs(const Shape& s, char* ws, const ress_ws_layout& L) {
@@ -206,6 +218,9 @@ __host__ __device__ inline SelPtrs sel_ptrs(const Shape& s, char* ws, const ress
   p.J0 = (float*)(ws + L.J0);
   p.dmask = (uint32_t*)(ws + L.dmask);
   p.bmask = (uint32_t*)(ws + L.bmask);
+  p.gsplit = (uint32_t*)(ws + L.gsplit);
+  p.cdot = (float*)(ws + L.cdot);
+  p.split_stride = (int64_t)s.H * s.nb * 32;
   return p;
 }
 
@@ -231,7 +246,7 @@ __device__ __forceinline__ void stage_rows(float (*A)[LDA], const float* __restr
   }
 }
 
-enum { kOpDot = 0, kOpDist = 1, kOpGain = 2 };
+enum { kOpDot = 0, kOpDist = 1 };
 
 // Packed pairs of floats (two fp32 lanes of one 64-bit register) for the f32x2 FMA path.
 __device__ __forceinline__ uint64_t ffma2(uint64_t a, uint64_t b, uint64_t c) {
@@ -265,7 +280,6 @@ __device__ __forceinline__ float hsum2(uint64_t v) {
 // f32x2 instructions straight from the float4 operands, the halves added at the end:
 //   kOpDot  : sum_d A[r][d] B[j][d]
 //   kOpDist : sum_d (A[r][d] - B[j][d])^2
-//   kOpGain : sum_d (A[r][d] - B[j][d]) Gv[r][d]
 template <int OP>
 __device__ __forceinline__ void tile8x2(const SelSmem& S, int rg, int jb, float out[8][2]) {
   uint64_t acc[8][2];
@@ -283,18 +297,12 @@ __device__ __forceinline__ void tile8x2(const SelSmem& S, int rg, int jb, float 
         acc[x][0] = ffma2(a.y, b0.y, acc[x][0]);
         acc[x][1] = ffma2(a.x, b1.x, acc[x][1]);
         acc[x][1] = ffma2(a.y, b1.y, acc[x][1]);
-      } else if (OP == kOpDist) {
+      } else {
         uint64_t e;
         e = fsub2(a.x, b0.x); acc[x][0] = ffma2(e, e, acc[x][0]);
         e = fsub2(a.y, b0.y); acc[x][0] = ffma2(e, e, acc[x][0]);
         e = fsub2(a.x, b1.x); acc[x][1] = ffma2(e, e, acc[x][1]);
         e = fsub2(a.y, b1.y); acc[x][1] = ffma2(e, e, acc[x][1]);
-      } else {
-        const ulonglong2 g = *reinterpret_cast<const ulonglong2*>(&S.Gv[rg * 8 + x][d]);
-        acc[x][0] = ffma2(fsub2(a.x, b0.x), g.x, acc[x][0]);
-        acc[x][0] = ffma2(fsub2(a.y, b0.y), g.y, acc[x][0]);
-        acc[x][1] = ffma2(fsub2(a.x, b1.x), g.x, acc[x][1]);
-        acc[x][1] = ffma2(fsub2(a.y, b1.y), g.y, acc[x][1]);
       }
     }
   }
@@ -454,6 +462,21 @@ __device__ __forceinline__ float warp_sum(float v) {
 }
 
 // Bits of word w that are valid key blocks (< nb).
+// g~ of row ri (this lane's channels 2 lane, 2 lane + 1), its three bf16 terms (the A
+// operands of the tensor-core gains) and c_i = y~_i . g~_i.
+__device__ __forceinline__ void store_gtil(const SelPtrs& p, int64_t ri, int lane, float2 y,
+                                           float g0, float g1) {
+  *reinterpret_cast<float2*>(p.gtil + ri * 64 + 2 * lane) = make_float2(g0, g1);
+  uint32_t hi, mid, lo;
+  split3_bf16x2(g0, g1, hi, mid, lo);
+  uint32_t* gs = p.gsplit + ri * 32 + lane;
+  gs[0] = hi;
+  gs[p.split_stride] = mid;
+  gs[2 * p.split_stride] = lo;
+  const float c = warp_sum(y.x * g0 + y.y * g1);
+  if (lane == 0) p.cdot[ri] = c;
+}
+
 __device__ __forceinline__ uint32_t valid_bits(int w, int n) {
   const int rem = n - w * 32;
   return rem >= 32 ? kFull : (rem <= 0 ? 0u : ((1u << rem) - 1u));
@@ -578,10 +601,6 @@ __device__ __forceinline__ WarpScratch warp_scratch(unsigned char* smem, int war
 // Score kernel: Sec. 4.1-4.2 and the initial state of Sec. 4.3 for RT query rows of one
 // head.  grid (ceil(ncand / RT), H).
 // ------------------------------------------------------------------------------------
-struct Budgets {
-  int c[RESS_MAX_HEADS];
-};
-
 __global__ void __launch_bounds__(kThreads, 3) k_score(SelPtrs p, Budgets bud) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
   SelSmem& S = *reinterpret_cast<SelSmem*>(smem_raw);
@@ -785,7 +804,7 @@ __global__ void __launch_bounds__(32 * kRowWarps, 8) k_score_rows(SelPtrs p, Bud
   const float G = warp_sum(g0 * g0 + g1 * g1);
   const float Kc = fmaxf(K, kEps);
   const float J = G / (Kc * Kc);
-  *reinterpret_cast<float2*>(p.gtil + ri * 64 + 2 * lane) = make_float2(g0, g1);
+  store_gtil(p, ri, lane, y, g0, g1);
   if (lane == 0) {
     p.K[ri] = K;
     p.G[ri] = G;
@@ -795,57 +814,10 @@ __global__ void __launch_bounds__(32 * kRowWarps, 8) k_score_rows(SelPtrs p, Bud
   }
 }
 
-// Swap count of round r (Eq. 17): floor(rho c_h / 2^(r+1)), capped by |D| and |P \ D|.
-__device__ __forceinline__ int swap_count(int c, int ncand, int round, float rho) {
-  const int m = (int)floor((double)rho * (double)c / (double)(1ull << (round + 1)));
-  return min(m, min(ncand - c, c));
-}
-
 // ------------------------------------------------------------------------------------
-// Restoration round r (Sec. 4.3, Eq. 13-17), first half: the gain inner products
-// t_ij = (y~_i - z~_j) . g~_i for RT rows of one head and one BN-block chunk of candidates.
-// grid (ceil(ncand / RT), H, ceil(ncand / BN)): small CTAs in many waves, so the last wave
-// leaves little of the GPU idle.
+// Restoration round r (Sec. 4.3, Eq. 13-17).  The gain inner products t_ij of the round
+// come from k_gain (tensor cores, k_gain.cu); the rest of the round runs per row here.
 // ------------------------------------------------------------------------------------
-__global__ void __launch_bounds__(kThreads, 3) k_round(SelPtrs p, Budgets bud, int round,
-                                                       float rho) {
-  extern __shared__ __align__(16) unsigned char smem_raw[];
-  SelSmem& S = *reinterpret_cast<SelSmem*>(smem_raw);
-  const int h = blockIdx.y, i0 = blockIdx.x * RT;
-  if (swap_count(bud.c[h], p.ncand, round, rho) <= 0) return;
-  const int nrows = min(RT, p.ncand - i0);
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int rg = warp & 3, jb = (warp >> 2) * 64 + lane;
-  const int64_t hrow = (int64_t)h * p.nb;
-  const float* zt_h = p.ztil + hrow * 64;
-  float* tbase = p.t + (hrow + i0) * p.ld;
-
-  // ---- gains: t_ij = (y~_i - z~_j) . g~_i  (Eq. 14/15 without the P_ij factor), as
-  // c_i - z~_j . g~_i with c_i = y~_i . g~_i: one packed FMA per channel pair -------------
-  const int j0 = blockIdx.z * BN;
-  stage_rows(S.A, p.gtil + (hrow + i0) * 64, nrows);
-  stage_rows(S.Gv, p.ytil + (hrow + i0) * 64, nrows);
-  stage_blocks(S.B, zt_h, j0, p.ncand);
-  __syncthreads();
-  for (int r = warp; r < RT; r += kThreads / 32) {
-    const float c = warp_sum(S.A[r][2 * lane] * S.Gv[r][2 * lane] +
-                             S.A[r][2 * lane + 1] * S.Gv[r][2 * lane + 1]);
-    if (lane == 0) S.rowm[r] = c;
-  }
-  __syncthreads();
-  float acc[8][2];
-  tile8x2<kOpDot>(S, rg, jb, acc);
-#pragma unroll
-  for (int x = 0; x < 8; ++x) {
-    const int r = rg * 8 + x;
-    if (r < nrows) {
-      const float c = S.rowm[r];
-      if (j0 + jb < p.ncand) tbase[(int64_t)r * p.ld + j0 + jb] = c - acc[x][0];
-      if (j0 + jb + 32 < p.ncand) tbase[(int64_t)r * p.ld + j0 + jb + 32] = c - acc[x][1];
-    }
-  }
-}
-
 // Restoration round r, per row: exact top-m restores and drops from the round-start state,
 // update, track-best.  grid (ceil(|P| / 4), H).
 __global__ void __launch_bounds__(32 * kRowWarps, 8) k_round_rows(SelPtrs p, Budgets bud,
@@ -905,7 +877,7 @@ __global__ void __launch_bounds__(32 * kRowWarps, 8) k_round_rows(SelPtrs p, Bud
     p.dmask[ri * p.words + w] = Dw[w];
     if (better) p.bmask[ri * p.words + w] = Dw[w];
   }
-  *reinterpret_cast<float2*>(p.gtil + ri * 64 + 2 * lane) = make_float2(g0, g1);
+  store_gtil(p, ri, lane, y, g0, g1);
   if (lane == 0) {
     p.K[ri] = Kn;
     p.G[ri] = Gn;
@@ -975,7 +947,8 @@ cudaError_t launch_score(const SelectArgs& a, cudaStream_t st) {
   float* vbar = (float*)(a.ws + a.L.vbar);
   float* ztil = (float*)(a.ws + a.L.ztil);
   k_pool<<<dim3(s.nb, 3), kThreads, 0, st>>>(a.Q, a.K, a.V, s.N, s.H, s.nb, qbar, kbar, vbar);
-  k_zproj<<<dim3((s.nb + 15) / 16, s.H), kThreads, 0, st>>>(a.F, vbar, s.nb, ztil);
+  k_zproj<<<dim3((s.nb + 15) / 16, s.H), kThreads, 0, st>>>(
+      a.F, vbar, s.nb, ztil, (uint2*)(a.ws + a.L.zsplit), p.split_stride / 2);
   if (s.ncand <= 0) return cudaGetLastError();
   const size_t smem = sizeof(SelSmem);
   cudaError_t e = cudaFuncSetAttribute(k_score, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
@@ -993,11 +966,8 @@ cudaError_t launch_round(const SelectArgs& a, int round, float rho, cudaStream_t
   const Shape& s = a.s;
   if (s.ncand <= 0) return cudaSuccess;
   SelPtrs p = sel_ptrs(s, a.ws, a.L);
-  const size_t smem = sizeof(SelSmem);
-  cudaError_t e = cudaFuncSetAttribute(k_round, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  cudaError_t e = launch_gain(a, round, rho, st);  // t_ij on the tensor cores
   if (e != cudaSuccess) return e;
-  k_round<<<dim3((s.ncand + RT - 1) / RT, s.H, (s.ncand + BN - 1) / BN), kThreads, smem, st>>>(
-      p, budgets_of(a), round, rho);
   const size_t rsmem = (size_t)kRowWarps * warp_scratch_words(s.ld, 3 * s.words) * 4;
   e = cudaFuncSetAttribute(k_round_rows, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)rsmem);
   if (e != cudaSuccess) return e;

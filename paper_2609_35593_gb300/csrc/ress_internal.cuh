@@ -2,6 +2,7 @@
 #pragma once
 
 #include <cuda_runtime.h>
+#include <math.h>
 #include <stdint.h>
 
 #include "../../include/ress.h"
@@ -68,6 +69,9 @@ inline ress_ws_layout make_layout(const Shape& s) {
   L.dmask = take(msk);
   L.bmask = take(msk);
   L.plen = take((int64_t)s.H * ((s.nb + 1) / 2) * 4);
+  L.gsplit = take(3 * (int64_t)s.H * s.nb * kHeadDim * 2);
+  L.zsplit = take(3 * (int64_t)s.H * s.nb * kHeadDim * 2);
+  L.cdot = take(row);
   L.ld = s.ld;
   L.words = s.words;
   L.total = off;
@@ -81,6 +85,34 @@ __device__ __forceinline__ void flag_status(uint32_t* status, uint32_t code) {
 
 __device__ __forceinline__ float bf16_lo(uint32_t v) { return __uint_as_float(v << 16); }
 __device__ __forceinline__ float bf16_hi(uint32_t v) { return __uint_as_float(v & 0xffff0000u); }
+
+// Per-head kept-block budgets c_h (Eq. 7), passed to kernels by value.
+struct Budgets {
+  int c[RESS_MAX_HEADS];
+};
+
+// Swap count of round r (Eq. 17): floor(rho c_h / 2^(r+1)), capped by |D| and |P \ D|.
+__host__ __device__ inline int swap_count(int c, int ncand, int round, float rho) {
+  const int m = (int)floor((double)rho * (double)c / (double)(1ull << (round + 1)));
+  return min(m, min(ncand - c, c));
+}
+
+// Two floats as sums of three bf16 terms each, every term rounded to nearest:
+// x = hi + mid + lo up to |x| 2^-24 or so (hi carries the top 8 significant bits, mid
+// the next 8, lo the rest; both subtractions are exact).  Packed bf16x2, x0 in the low half.
+__device__ __forceinline__ uint32_t cvt_bf16x2(float lo_elem, float hi_elem) {
+  uint32_t r;
+  asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(hi_elem), "f"(lo_elem));
+  return r;
+}
+__device__ __forceinline__ void split3_bf16x2(float x0, float x1, uint32_t& hi, uint32_t& mid,
+                                              uint32_t& lo) {
+  hi = cvt_bf16x2(x0, x1);
+  const float r0 = x0 - __uint_as_float(hi << 16), r1 = x1 - __uint_as_float(hi & 0xffff0000u);
+  mid = cvt_bf16x2(r0, r1);
+  const float s0 = r0 - __uint_as_float(mid << 16), s1 = r1 - __uint_as_float(mid & 0xffff0000u);
+  lo = cvt_bf16x2(s0, s1);
+}
 
 // Streaming 16-byte load that bypasses L1 allocation (read-once inputs).
 __device__ __forceinline__ uint4 ld_stream(const uint4* p) {
@@ -104,6 +136,7 @@ struct SelectArgs {
 cudaError_t launch_prepare_wo(const Shape& s, const uint16_t* W_o, float* F, cudaStream_t st);
 cudaError_t launch_score(const SelectArgs& a, cudaStream_t st);
 cudaError_t launch_round(const SelectArgs& a, int round, float rho, cudaStream_t st);
+cudaError_t launch_gain(const SelectArgs& a, int round, float rho, cudaStream_t st);
 cudaError_t launch_csr(const SelectArgs& a, const int64_t* head_base, int32_t* row_ptr,
                        int32_t* col_idx, int64_t col_capacity, float* J_best,
                        uint32_t* drop_mask, cudaStream_t st);

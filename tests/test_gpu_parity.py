@@ -297,3 +297,43 @@ def test_forward_host_equals_forward(tiny):
     torch.cuda.synchronize()
     assert torch.equal(Oh.view(torch.int16), tiny.buf.O.cpu().view(torch.int16))
     assert np.array_equal(layer.csr()[1], tiny.csr()[1])
+
+
+@pytest.mark.parametrize("fixture_name", ["tiny_v2", "vggt_v8"])
+def test_gain_products(fixture_name):
+    """Restoration gains t_ij = (y~_i - z~_j) . g~_i (Eq. 14/15), computed on the tensor
+    cores from three-term bf16 splits, against float64 products of the same float32 y~, z~
+    and g~ (the state after the initial selection, i.e. the start of round 0)."""
+    layer, wl = layer_for(fixture_name)
+    r, b = layer.ress, layer.buf
+    r.prepare_wo(layer.d, layer.W, b.F)
+    r.score(layer.d, layer.Q, layer.K, layer.V, b.F, layer.c_h, b.ws)
+    torch.cuda.synchronize()
+    H, nb, nc, L = layer.H, layer.nb, layer.ncand, b.layout
+    y = layer.ws("ytil", shape=(H, nb, 64)).astype(np.float64)
+    z = layer.ws("ztil", shape=(H, nb, 64)).astype(np.float64)
+    g = layer.ws("gtil", shape=(H, nb, 64)).astype(np.float64)
+    cdot = layer.ws("cdot", shape=(H, nb)).astype(np.float64)
+    for name, x, rows in (("gsplit", g, nc), ("zsplit", z, nb)):
+        terms = synth.bf16_to_f32(layer.ws(name, torch.int16, (3, H, nb, 64)).view(np.uint16))
+        hi, mid, lo = (terms[k].astype(np.float64)[:, :rows] for k in range(3))
+        xs = x[:, :rows]
+        assert np.all(np.abs(mid) <= 2.0 ** -8 * np.abs(xs) + 1e-30)
+        assert np.all(np.abs(hi + mid + lo - xs) <= 2.0 ** -23 * np.abs(xs) + 1e-30), name
+    yn, zn, gn = (np.linalg.norm(v, axis=2) for v in (y, z, g))
+    np.testing.assert_array_less(np.abs(cdot[:, :nc] - (y * g).sum(2)[:, :nc]),
+                                 1e-5 * (yn * gn)[:, :nc] + 1e-30)
+    r.restore(layer.d, layer.c_h, 1, layer.rho, b.ws, b.row_ptr, b.col_idx, b.J_best)
+    r.status(b.ws)
+    torch.cuda.synchronize()
+    t = layer.ws("t", shape=(H, nb, L.ld))
+    checked = 0
+    for h in range(H):
+        if min(O.swap_schedule(layer.c_h[h], 1, layer.rho)[0], nc - layer.c_h[h]) <= 0:
+            continue
+        ref = (y[h, :nc] * g[h, :nc]).sum(1)[:, None] - g[h, :nc] @ z[h, :nc].T
+        bound = 1e-5 * gn[h, :nc, None] * (yn[h, :nc, None] + zn[h, None, :nc]) + 1e-30
+        err = np.abs(t[h, :nc, :nc] - ref)
+        assert np.all(err <= bound), (h, float((err / bound).max()))
+        checked += 1
+    assert checked > 0
