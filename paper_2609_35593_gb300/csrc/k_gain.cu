@@ -15,7 +15,10 @@
 //   warp 0     converged MMA warp, one elected lane issues 6 x 4 tcgen05.mma M128 N128 K16
 //              (A = g~ terms, B = z~ terms, both K-major from shared memory) and commits;
 //   warps 0-3  epilogue: tcgen05.ld of the accumulator rows (warp w: rows 32w..32w+31),
-//              t = c_i - acc, 16-byte stores of row i's 128 gains.
+//              t = c_i - acc into shared memory (the operand tiles are free by then) as
+//              four 32-column boxes in the 128-byte-swizzled layout, which thread 0 writes
+//              to t with TMA bulk tensor stores (rows past nb and columns past the row
+//              stride are clipped by the copy; rows past |P| are never read).
 // Every mbarrier wait is bounded; a wait that gives up records RESS_ETIMEOUT, lets copies
 // and MMAs already issued finish (again bounded), frees TMEM and returns.
 
@@ -70,7 +73,7 @@ __device__ __forceinline__ bool gain_wait(uint64_t* bar, uint32_t parity, volati
 
 __global__ void __launch_bounds__(kGainThreads)
     k_gain(const __grid_constant__ CUtensorMap tmG, const __grid_constant__ CUtensorMap tmZ,
-           const GainParams p) {
+           const __grid_constant__ CUtensorMap tmT, const GainParams p) {
   const int h = blockIdx.z, i0 = blockIdx.y * kGainTile, j0 = blockIdx.x * kGainTile;
   if (swap_count(p.bud.c[h], p.ncand, p.round, p.rho) <= 0) return;
   extern __shared__ uint8_t smem_raw[];
@@ -86,6 +89,7 @@ __global__ void __launch_bounds__(kGainThreads)
     fence_barrier_init();
     prefetch_tensormap(&tmG);
     prefetch_tensormap(&tmZ);
+    prefetch_tensormap(&tmT);
   }
   if (warp == 0) tmem_alloc(&S.tmem_base, kGainCols);
   tc_fence_before();
@@ -146,24 +150,30 @@ __global__ void __launch_bounds__(kGainThreads)
   }
   if (ok) {
     tc_fence_after();
-    const int i = i0 + 32 * warp + lane;
-    const bool row_ok = i < p.ncand;
-    const float c = row_ok ? p.cdot[(int64_t)h * p.nb + i] : 0.f;
-    float* trow = p.t + ((int64_t)h * p.nb + (row_ok ? i : 0)) * p.ld;
+    const int r = 32 * warp + lane;  // row of the tile = TMEM lane
+    const int i = i0 + r;
+    const float c = i < p.nb ? p.cdot[(int64_t)h * p.nb + i] : 0.f;
+    uint8_t* stage = &S.A[0][0];  // 4 boxes of 128 rows x 32 fp32, 16 KB each
 #pragma unroll 1
     for (int q = 0; q < kGainTile / 32; ++q) {
-      const int jq = j0 + 32 * q;
-      if (jq >= p.ld) break;  // uniform: ld is a multiple of 32
-      uint32_t r[32];
-      RESS_TMEM_LD32(tmem + ((uint32_t)(32 * warp) << 16) + 32 * q, r);
-      if (row_ok) {
+      uint32_t v[32];
+      RESS_TMEM_LD32(tmem + ((uint32_t)(32 * warp) << 16) + 32 * q, v);
+      uint8_t* row = stage + q * 16384 + r * 128;
 #pragma unroll
-        for (int e = 0; e < 8; ++e)
-          *reinterpret_cast<float4*>(trow + jq + 4 * e) =
-              make_float4(c - __uint_as_float(r[4 * e]), c - __uint_as_float(r[4 * e + 1]),
-                          c - __uint_as_float(r[4 * e + 2]), c - __uint_as_float(r[4 * e + 3]));
-      }
+      for (int k = 0; k < 8; ++k)  // 16-byte chunk k of the row goes to chunk k ^ (r mod 8)
+        *reinterpret_cast<float4*>(row + ((k ^ (r & 7)) << 4)) =
+            make_float4(c - __uint_as_float(v[4 * k]), c - __uint_as_float(v[4 * k + 1]),
+                        c - __uint_as_float(v[4 * k + 2]), c - __uint_as_float(v[4 * k + 3]));
     }
+    fence_proxy_async_smem();
+  }
+  __syncthreads();
+  if (ok && threadIdx.x == 0) {
+#pragma unroll 1
+    for (int q = 0; q < kGainTile / 32; ++q)
+      if (j0 + 32 * q < p.ld) tma_store_3d(&tmT, &S.A[0][0] + q * 16384, j0 + 32 * q, i0, h);
+    bulk_commit();
+    bulk_wait_read_all();  // the boxes are read before the shared memory goes away
   }
   if (warp == 0 && issued && !ok) {  // MMAs still running: let them finish before the free
     volatile int no_abort = 0;
@@ -205,14 +215,28 @@ bool make_term_map(CUtensorMap* m, const void* base, int nb, int H) {
             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// t: fp32 [H][nb][ld] viewed as {ld, nb, H}; box {32, 128, 1}, 128-byte swizzle.
+bool make_gain_out_map(CUtensorMap* m, void* base, int nb, int H, int ld) {
+  auto fn = gain_encode_fn();
+  if (!fn) return false;
+  cuuint64_t dims[3] = {(cuuint64_t)ld, (cuuint64_t)nb, (cuuint64_t)H};
+  cuuint64_t strides[2] = {(cuuint64_t)ld * 4, (cuuint64_t)nb * ld * 4};
+  cuuint32_t box[3] = {32, (cuuint32_t)kGainTile, 1};
+  cuuint32_t estr[3] = {1, 1, 1};
+  return fn(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 3, base, dims, strides, box, estr,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 }  // namespace
 
 cudaError_t launch_gain(const SelectArgs& a, int round, float rho, cudaStream_t st) {
   const Shape& s = a.s;
   if (s.ncand <= 0) return cudaSuccess;
-  CUtensorMap tg, tz;
+  CUtensorMap tg, tz, tt;
   if (!make_term_map(&tg, a.ws + a.L.gsplit, s.nb, s.H) ||
-      !make_term_map(&tz, a.ws + a.L.zsplit, s.nb, s.H))
+      !make_term_map(&tz, a.ws + a.L.zsplit, s.nb, s.H) ||
+      !make_gain_out_map(&tt, a.ws + a.L.t, s.nb, s.H, s.ld))
     return cudaErrorInvalidValue;
   GainParams p;
   p.nb = s.nb;
@@ -228,7 +252,7 @@ cudaError_t launch_gain(const SelectArgs& a, int round, float rho, cudaStream_t 
   cudaError_t e = cudaFuncSetAttribute(k_gain, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   const int tiles = (s.ncand + kGainTile - 1) / kGainTile;
-  k_gain<<<dim3(tiles, tiles, s.H), kGainThreads, smem, st>>>(tg, tz, p);
+  k_gain<<<dim3(tiles, tiles, s.H), kGainThreads, smem, st>>>(tg, tz, tt, p);
   return cudaGetLastError();
 }
 

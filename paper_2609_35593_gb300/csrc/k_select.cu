@@ -455,13 +455,95 @@ __device__ void warp_topm(const uint32_t* kk, int n, int m, uint32_t* sel, int w
   __syncwarp();
 }
 
+// This lane's two largest keys on each side of a drop set, kept while the keys are written.
+struct LaneTop2 {
+  uint32_t d1 = 0, d2 = 0, b1 = 0, b2 = 0;  // in D: largest, second; outside D: same
+  __device__ __forceinline__ void add(uint32_t v, bool inD) {
+    uint32_t& a1 = inD ? d1 : b1;
+    uint32_t& a2 = inD ? d2 : b2;
+    a2 = max(a2, min(a1, v));
+    a1 = max(a1, v);
+  }
+};
+
+// Both selections of a restoration round at once, for m <= 64: the m largest keys among
+// the blocks in D (bit set in Dw) into selD and the m largest among the other candidates
+// into selB, ties to the lower block index.  `top` holds this lane's two largest keys on
+// each side (0 where it has none), taken while the keys were written, so the lane-local
+// pass of warp_topm is not needed: the m-th largest of the 64 lane values of a side bounds
+// that side's m-th key from below.  Both bounds come from one bit search (counts packed in
+// one reduction) and both survivor lists from one ballot pass; each side then selects
+// exactly.
+__device__ void warp_topm_pair(const uint32_t* kk, int n, int m, const uint32_t* Dw,
+                               const LaneTop2& top, uint32_t* selD, uint32_t* selB,
+                               int words, uint32_t* sk, uint16_t* si) {
+  const int lane = threadIdx.x & 31;
+  for (int w = lane; w < words; w += 32) selD[w] = selB[w] = 0u;
+  __syncwarp();
+  if (m <= 0) return;
+  uint32_t bD = 0, bB = 0;
+  bool doneD = false, doneB = false;
+  for (int bit = 31; bit >= 0 && !(doneD && doneB); --bit) {
+    const uint32_t cD = bD | (1u << bit), cB = bB | (1u << bit);
+    int c = 0;
+    if (!doneD) c += (top.d1 >= cD ? 1 : 0) + (top.d2 >= cD ? 1 : 0);
+    if (!doneB) c += (top.b1 >= cB ? 1 << 16 : 0) + (top.b2 >= cB ? 1 << 16 : 0);
+    c = __reduce_add_sync(kFull, c);
+    const int nD = c & 0xffff, nB = c >> 16;
+    if (!doneD && nD >= m) {
+      bD = cD;
+      doneD = nD == m;
+    }
+    if (!doneB && nB >= m) {
+      bB = cB;
+      doneB = nB == m;
+    }
+  }
+  constexpr int kHalf = kSurvivors / 2;
+  const uint32_t below = (1u << lane) - 1u;
+  int cntD = 0, cntB = 0;
+  for (int x0 = 0; x0 < n; x0 += 32) {
+    const int x = x0 + lane;
+    const bool in = x < n;
+    const uint32_t v = in ? kk[x] : 0u;
+    const bool inD = in && ((Dw[x0 >> 5] >> lane) & 1u);
+    const bool kd = inD && v >= bD, kb = in && !inD && v >= bB;
+    const uint32_t BD = __ballot_sync(kFull, kd), BB = __ballot_sync(kFull, kb);
+    if (kd) {
+      const int pos = cntD + __popc(BD & below);
+      if (pos < kHalf) {
+        sk[pos] = v;
+        si[pos] = (uint16_t)x;
+      }
+    }
+    if (kb) {
+      const int pos = cntB + __popc(BB & below);
+      if (pos < kHalf) {
+        sk[kHalf + pos] = v;
+        si[kHalf + pos] = (uint16_t)x;
+      }
+    }
+    cntD += __popc(BD);
+    cntB += __popc(BB);
+  }
+  __syncwarp();
+  if (cntD > kHalf)
+    select_exact(kk, nullptr, n, m, Dw, true, selD);
+  else
+    select_exact(sk, si, cntD, m, nullptr, true, selD);
+  if (cntB > kHalf)
+    select_exact(kk, nullptr, n, m, Dw, false, selB);
+  else
+    select_exact(sk + kHalf, si + kHalf, cntB, m, nullptr, true, selB);
+  __syncwarp();
+}
+
 __device__ __forceinline__ float warp_sum(float v) {
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(kFull, v, o);
   return v;
 }
 
-// Bits of word w that are valid key blocks (< nb).
 // g~ of row ri (this lane's channels 2 lane, 2 lane + 1), its three bf16 terms (the A
 // operands of the tensor-core gains) and c_i = y~_i . g~_i.
 __device__ __forceinline__ void store_gtil(const SelPtrs& p, int64_t ri, int lane, float2 y,
@@ -477,6 +559,7 @@ __device__ __forceinline__ void store_gtil(const SelPtrs& p, int64_t ri, int lan
   if (lane == 0) p.cdot[ri] = c;
 }
 
+// Bits of word w that are valid key blocks (< nb).
 __device__ __forceinline__ uint32_t valid_bits(int w, int n) {
   const int rem = n - w * 32;
   return rem >= 32 ? kFull : (rem <= 0 ? 0u : ((1u << rem) - 1u));
@@ -842,6 +925,7 @@ __global__ void __launch_bounds__(32 * kRowWarps, 8) k_round_rows(SelPtrs p, Bud
   for (int w = lane; w < p.words; w += 32) Dw[w] = p.dmask[ri * p.words + w];
   const float K = p.K[ri], G = p.G[ri];
   __syncwarp();
+  LaneTop2 top;  // this lane's two largest keys in D and outside it
   // one pass over the candidates: a block k in D is a restore candidate (u = +P_k,
   // dG = -2 P_k t_k + P_k^2 q_k, Eq. 13-14), a kept candidate a drop candidate (u = -P_k,
   // dG = +2 P_k t_k + P_k^2 q_k, Eq. 15); the key is the exact decrease of J (Eq. 16)
@@ -858,10 +942,15 @@ __global__ void __launch_bounds__(32 * kRowWarps, 8) k_round_rows(SelPtrs p, Bud
       const float s2 = pv[u] * pv[u] * qv[u];
       const float dG = inD ? fmaf(-2.0f * pv[u], tv[u], s2) : fmaf(2.0f * pv[u], tv[u], s2);
       k4[u] = order_key(delta_J(G, K, dG, inD ? pv[u] : -pv[u]));
+      if (j + u < p.ncand) top.add(k4[u], inD);
     }
   });
-  warp_topm(kk, p.ncand, m, Rw, p.words, sk, si, Dw, true);
-  warp_topm(kk, p.ncand, m, Xw, p.words, sk, si, Dw, false);
+  if (m <= 64) {
+    warp_topm_pair(kk, p.ncand, m, Dw, top, Rw, Xw, p.words, sk, si);
+  } else {
+    warp_topm(kk, p.ncand, m, Rw, p.words, sk, si, Dw, true);
+    warp_topm(kk, p.ncand, m, Xw, p.words, sk, si, Dw, false);
+  }
   for (int w = lane; w < p.words; w += 32) Dw[w] = (Dw[w] & ~Rw[w]) | Xw[w];
   __syncwarp();
   // state of the new set (Eq. 10-12): the swapped blocks update g~ and K
