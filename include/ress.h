@@ -36,7 +36,7 @@
 extern "C" {
 #endif
 
-#define RESS_ABI_VERSION 2
+#define RESS_ABI_VERSION 3
 #define RESS_HEAD_DIM 64
 #define RESS_BLOCK 64
 #define RESS_MAX_HEADS 32
@@ -78,8 +78,12 @@ typedef struct {
   int64_t K, G, J, Jbest, J0; /* [H, nb] remaining mass, G, J of Eq. 12                  */
   int64_t dmask, bmask; /* uint32 [H, nb, words] current and best drop sets (bit j)      */
   int64_t plen;        /* int32 [H, ceil(nb/2)] union lengths of query-block pairs          */
-  int64_t gsplit, zsplit; /* bf16 [3, H, nb, 64]: g~ and z~ as sums of three bf16 terms     */
-  int64_t cdot;        /* float [H, nb] y~_i . g~_i                                         */
+  int64_t asplit;      /* bf16 [3, H, nb, 64]: row operand as three bf16 terms (hi, mid, lo):
+                          q_bar, then y~, then g~ (tensor-core products)                   */
+  int64_t ksplit, zsplit; /* bf16 [3, H, nb, 64]: k_bar and z~ as three bf16 terms          */
+  int64_t cdot, ny, nz;   /* float [H, nb]: y~_i . g~_i, ||y~_i||^2, ||z~_j||^2              */
+  int64_t lstat;       /* float2 [H, nb, ceil(nb/128)]: per 128-block slice of a row of
+                          pooled logits, its max and sum of exp(logit - max)               */
   int64_t ld;          /* row stride of P, q, t                                          */
   int64_t words;       /* uint32 words per drop-set bitmask = ceil(nb / 32)              */
   int64_t total;       /* bytes                                                          */

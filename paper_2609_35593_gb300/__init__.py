@@ -46,8 +46,8 @@ class WsLayout(ctypes.Structure):
     """ress_ws_layout: byte offsets of the workspace arrays."""
     _fields_ = [(n, ctypes.c_int64) for n in
                 ("status", "counter", "qbar", "kbar", "vbar", "ztil", "ytil", "gtil", "P", "q", "t",
-                 "K", "G", "J", "Jbest", "J0", "dmask", "bmask", "plen", "gsplit", "zsplit", "cdot",
-                 "ld", "words", "total")]
+                 "K", "G", "J", "Jbest", "J0", "dmask", "bmask", "plen", "asplit", "ksplit", "zsplit",
+                 "cdot", "ny", "nz", "lstat", "ld", "words", "total")]
 
 
 _c = ctypes

@@ -1,5 +1,8 @@
 // ReSS block selection on sm_103a: pooling, pooled attention map, drift scoring, initial
-// top-c selection and the restoration rounds (Sec. 4.1-4.3 of the paper).
+// top-c selection and the restoration rounds (Sec. 4.1-4.3 of the paper).  This file holds
+// pooling, the F-space projection, the per-row selection kernels and the kept-block lists;
+// the row-by-block products (pooled logits, q, round gains) run on the tensor cores in
+// k_dot.cu and the pooled map with y~ in k_yagg.cu.
 //
 // Arithmetic is float32 with fixed-order reductions (deterministic, Appendix B.4).  The
 // per-head Gram matrix M_h = W_O^h^T W_O^h (Eq. 8) enters through its Cholesky factor F_h
@@ -20,9 +23,6 @@
 namespace ress {
 
 constexpr int kThreads = 256;
-constexpr int RT = 32;    // query rows per CTA (score and round kernels)
-constexpr int BN = 128;   // key blocks per staged chunk
-constexpr int LDA = 68;   // padded float stride of a staged 64-vector (17 x 16 B)
 constexpr unsigned kFull = 0xffffffffu;
 
 // ------------------------------------------------------------------------------------
@@ -101,11 +101,15 @@ __global__ void __launch_bounds__(kThreads) k_pool(const uint16_t* __restrict__ 
                                                     const uint16_t* __restrict__ V, int N,
                                                     int H, int nb, float* __restrict__ qbar,
                                                     float* __restrict__ kbar,
-                                                    float* __restrict__ vbar) {
+                                                    float* __restrict__ vbar,
+                                                    uint16_t* __restrict__ qsplit,
+                                                    uint16_t* __restrict__ ksplit) {
   __shared__ float part[kThreads * 8];
   const int j = blockIdx.x, which = blockIdx.y;
   const uint16_t* X = which == 0 ? Q : (which == 1 ? K : V);
   float* out = which == 0 ? qbar : (which == 1 ? kbar : vbar);
+  uint16_t* terms = which == 0 ? qsplit : (which == 1 ? ksplit : nullptr);  // tensor-core operands
+  const int64_t term_stride = (int64_t)H * nb * kHeadDim;
   const int C = 8 * H;
   const int tpp = kThreads / C;
   const int tok0 = j * kBlock;
@@ -133,7 +137,15 @@ __global__ void __launch_bounds__(kThreads) k_pool(const uint16_t* __restrict__ 
     float s = 0.f;
     for (int sl = 0; sl < tpp; ++sl) s += part[sl * C * 8 + f];
     const int h = f >> 6, d = f & 63;
-    out[((int64_t)h * nb + j) * kHeadDim + d] = s * inv;
+    const int64_t at = ((int64_t)h * nb + j) * kHeadDim + d;
+    out[at] = s * inv;
+    if (terms) {
+      uint16_t hi, mid, lo;
+      split3_bf16(s * inv, hi, mid, lo);
+      terms[at] = hi;
+      terms[at + term_stride] = mid;
+      terms[at + 2 * term_stride] = lo;
+    }
   }
 }
 
@@ -144,7 +156,8 @@ __global__ void __launch_bounds__(kThreads) k_zproj(const float* __restrict__ F,
                                                      const float* __restrict__ vbar, int nb,
                                                      float* __restrict__ ztil,
                                                      uint2* __restrict__ zsplit,
-                                                     int64_t term_stride) {
+                                                     int64_t term_stride,
+                                                     float* __restrict__ nz) {
   __shared__ __align__(16) float Ft[64][64];  // Ft[b][a] = F[a][b]
   __shared__ float Vs[16][65];
   const int h = blockIdx.y, j0 = blockIdx.x * 16, t = threadIdx.x;
@@ -175,24 +188,20 @@ __global__ void __launch_bounds__(kThreads) k_zproj(const float* __restrict__ F,
   zsplit[at / 4] = hi;
   zsplit[at / 4 + term_stride] = mid;
   zsplit[at / 4 + 2 * term_stride] = lo;
+  // ||z~_j||^2 over the 16 threads of block jj (one half-warp), fixed order
+  const unsigned group = 0xFFFFu << (threadIdx.x & 16);
+  float n2 = fmaf(acc.w, acc.w, fmaf(acc.z, acc.z, fmaf(acc.y, acc.y, acc.x * acc.x)));
+#pragma unroll
+  for (int o = 8; o > 0; o >>= 1) n2 += __shfl_xor_sync(group, n2, o);
+  if ((t & 15) == 0) nz[(int64_t)h * nb + j0 + jj] = n2;
 }
-
-// ------------------------------------------------------------------------------------
-// Shared pieces of the score and round kernels.
-// ------------------------------------------------------------------------------------
-struct SelSmem {
-  float A[RT][LDA];      // per-row 64-vectors: q_bar, then y~
-  float B[BN][LDA];      // staged chunk of per-block 64-vectors (k_bar or z~)
-  float Pc[RT][BN + 4];  // staged chunk of P (score kernel)
-  float rowm[RT], rowiz[RT];
-};
 
 struct SelPtrs {
   int nb, ncand, words, ld;
   const float *qbar, *kbar, *ztil;
   float *ytil, *gtil, *P, *q, *t, *K, *G, *J, *Jbest, *J0;
   uint32_t *dmask, *bmask;
-  uint32_t* gsplit;      // bf16x2 [3][H][nb][32]: g~ as three bf16 terms (tensor-core gains)
+  uint32_t* asplit;      // bf16x2 [3][H][nb][32]: g~ as three bf16 terms (tensor-core gains)
   float* cdot;           // [H, nb] y~_i . g~_i
   int64_t split_stride;  // H nb 32: uint32 words per term
 };
@@ -218,99 +227,10 @@ __host__ __device__ inline SelPtrs sel_ptrs(const Shape& s, char* ws, const ress
   p.J0 = (float*)(ws + L.J0);
   p.dmask = (uint32_t*)(ws + L.dmask);
   p.bmask = (uint32_t*)(ws + L.bmask);
-  p.gsplit = (uint32_t*)(ws + L.gsplit);
+  p.asplit = (uint32_t*)(ws + L.asplit);
   p.cdot = (float*)(ws + L.cdot);
   p.split_stride = (int64_t)s.H * s.nb * 32;
   return p;
-}
-
-// Stage rows [j0, j0+BN) of a [nb, 64] float matrix into B (zeros past nb).
-__device__ __forceinline__ void stage_blocks(float (*B)[LDA], const float* __restrict__ src,
-                                             int j0, int nb) {
-  for (int f = threadIdx.x; f < BN * 16; f += kThreads) {
-    const int jj = f >> 4, d4 = (f & 15) << 2;
-    float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
-    if (j0 + jj < nb) v = *reinterpret_cast<const float4*>(src + (int64_t)(j0 + jj) * 64 + d4);
-    *reinterpret_cast<float4*>(&B[jj][d4]) = v;
-  }
-}
-
-// Stage RT per-row 64-vectors (rows past `nrows` are zero).
-__device__ __forceinline__ void stage_rows(float (*A)[LDA], const float* __restrict__ src,
-                                           int nrows) {
-  for (int f = threadIdx.x; f < RT * 16; f += kThreads) {
-    const int r = f >> 4, d4 = (f & 15) << 2;
-    float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
-    if (r < nrows) v = *reinterpret_cast<const float4*>(src + (int64_t)r * 64 + d4);
-    *reinterpret_cast<float4*>(&A[r][d4]) = v;
-  }
-}
-
-enum { kOpDot = 0, kOpDist = 1 };
-
-// Packed pairs of floats (two fp32 lanes of one 64-bit register) for the f32x2 FMA path.
-__device__ __forceinline__ uint64_t ffma2(uint64_t a, uint64_t b, uint64_t c) {
-  uint64_t d;
-  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
-  return d;
-}
-__device__ __forceinline__ uint64_t fsub2(uint64_t a, uint64_t b) {
-  uint64_t d;
-  asm("sub.rn.f32x2 %0, %1, %2;" : "=l"(d) : "l"(a), "l"(b));
-  return d;
-}
-__device__ __forceinline__ uint64_t pack2(float lo, float hi) {
-  uint64_t d;
-  asm("mov.b64 %0, {%1, %2};" : "=l"(d) : "f"(lo), "f"(hi));
-  return d;
-}
-__device__ __forceinline__ float2 unpack2(uint64_t v) {
-  float2 r;
-  asm("mov.b64 {%0, %1}, %2;" : "=f"(r.x), "=f"(r.y) : "l"(v));
-  return r;
-}
-__device__ __forceinline__ float hsum2(uint64_t v) {
-  float lo, hi;
-  asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(v));
-  return lo + hi;
-}
-
-// Warp tile of 8 rows (8*rg ..) x 2 staged blocks (jb, jb + 32), reduced over the 64
-// channels; each accumulator is a pair (even channels, odd channels) updated by packed
-// f32x2 instructions straight from the float4 operands, the halves added at the end:
-//   kOpDot  : sum_d A[r][d] B[j][d]
-//   kOpDist : sum_d (A[r][d] - B[j][d])^2
-template <int OP>
-__device__ __forceinline__ void tile8x2(const SelSmem& S, int rg, int jb, float out[8][2]) {
-  uint64_t acc[8][2];
-#pragma unroll
-  for (int x = 0; x < 8; ++x) acc[x][0] = acc[x][1] = 0ull;
-#pragma unroll 2
-  for (int d = 0; d < 64; d += 4) {
-    const ulonglong2 b0 = *reinterpret_cast<const ulonglong2*>(&S.B[jb][d]);
-    const ulonglong2 b1 = *reinterpret_cast<const ulonglong2*>(&S.B[jb + 32][d]);
-#pragma unroll
-    for (int x = 0; x < 8; ++x) {
-      const ulonglong2 a = *reinterpret_cast<const ulonglong2*>(&S.A[rg * 8 + x][d]);
-      if (OP == kOpDot) {
-        acc[x][0] = ffma2(a.x, b0.x, acc[x][0]);
-        acc[x][0] = ffma2(a.y, b0.y, acc[x][0]);
-        acc[x][1] = ffma2(a.x, b1.x, acc[x][1]);
-        acc[x][1] = ffma2(a.y, b1.y, acc[x][1]);
-      } else {
-        uint64_t e;
-        e = fsub2(a.x, b0.x); acc[x][0] = ffma2(e, e, acc[x][0]);
-        e = fsub2(a.y, b0.y); acc[x][0] = ffma2(e, e, acc[x][0]);
-        e = fsub2(a.x, b1.x); acc[x][1] = ffma2(e, e, acc[x][1]);
-        e = fsub2(a.y, b1.y); acc[x][1] = ffma2(e, e, acc[x][1]);
-      }
-    }
-  }
-#pragma unroll
-  for (int x = 0; x < 8; ++x) {
-    out[x][0] = hsum2(acc[x][0]);
-    out[x][1] = hsum2(acc[x][1]);
-  }
 }
 
 // Order-preserving map of a float to uint32; every non-NaN value maps above 0, so 0 can
@@ -551,7 +471,7 @@ __device__ __forceinline__ void store_gtil(const SelPtrs& p, int64_t ri, int lan
   *reinterpret_cast<float2*>(p.gtil + ri * 64 + 2 * lane) = make_float2(g0, g1);
   uint32_t hi, mid, lo;
   split3_bf16x2(g0, g1, hi, mid, lo);
-  uint32_t* gs = p.gsplit + ri * 32 + lane;
+  uint32_t* gs = p.asplit + ri * 32 + lane;
   gs[0] = hi;
   gs[p.split_stride] = mid;
   gs[2 * p.split_stride] = lo;
@@ -647,171 +567,14 @@ __device__ __forceinline__ void swap_drift(const uint32_t* R, const uint32_t* X,
   __syncwarp();
 }
 
-// Per-warp scratch of the per-row phase: keys [ld] u32, survivor keys [kSurvivors] u32,
-// survivor indices [kSurvivors] u16, bitmask words.  It reuses the GEMM staging area (B,
-// Pc), which the per-row phase no longer needs, when that area is large enough.
+// Per-warp scratch of the per-row kernels: keys [ld] u32, survivor keys [kSurvivors] u32,
+// survivor indices [kSurvivors] u16, bitmask words.
 __host__ __device__ constexpr size_t warp_scratch_words(int ld, int words_per_warp) {
   return (size_t)ld + kSurvivors + kSurvivors / 2 + words_per_warp;
 }
 
-struct WarpScratch {
-  uint32_t* kk;
-  uint32_t* sk;
-  uint16_t* si;
-  uint32_t* words;
-};
-
-// Offset of the per-warp scratch from the start of SelSmem.
-__host__ __device__ inline size_t scratch_offset(int ld, int wpw) {
-  const size_t need = (size_t)8 * warp_scratch_words(ld, wpw) * 4;
-  const size_t staged = sizeof(SelSmem) - offsetof(SelSmem, B);
-  return need <= staged ? offsetof(SelSmem, B) : sizeof(SelSmem);
-}
-
-__device__ __forceinline__ WarpScratch warp_scratch(unsigned char* smem, int warp, int ld, int wpw) {
-  uint32_t* w0 = reinterpret_cast<uint32_t*>(smem + scratch_offset(ld, wpw)) +
-                 (size_t)warp * warp_scratch_words(ld, wpw);
-  WarpScratch ws;
-  ws.kk = w0;
-  ws.sk = w0 + ld;
-  ws.si = reinterpret_cast<uint16_t*>(ws.sk + kSurvivors);
-  ws.words = ws.sk + kSurvivors + kSurvivors / 2;
-  return ws;
-}
 
 
-// ------------------------------------------------------------------------------------
-// Score kernel: Sec. 4.1-4.2 and the initial state of Sec. 4.3 for RT query rows of one
-// head.  grid (ceil(ncand / RT), H).
-// ------------------------------------------------------------------------------------
-__global__ void __launch_bounds__(kThreads, 3) k_score(SelPtrs p, Budgets bud) {
-  extern __shared__ __align__(16) unsigned char smem_raw[];
-  SelSmem& S = *reinterpret_cast<SelSmem*>(smem_raw);
-  const int h = blockIdx.y, i0 = blockIdx.x * RT;
-  const int nrows = min(RT, p.ncand - i0);
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int rg = warp & 3, jb = (warp >> 2) * 64 + lane;
-  const int64_t hrow = (int64_t)h * p.nb;
-  float* Pbase = p.P + (hrow + i0) * p.ld;
-  float* qbase = p.q + (hrow + i0) * p.ld;
-  const float* kb_h = p.kbar + hrow * 64;
-  const float* zt_h = p.ztil + hrow * 64;
-
-  // ---- pass 1: pooled logits q_bar_i . k_bar_j / sqrt(64) into P (as logits) --------
-  stage_rows(S.A, p.qbar + (hrow + i0) * 64, nrows);
-  for (int j0 = 0; j0 < p.nb; j0 += BN) {
-    stage_blocks(S.B, kb_h, j0, p.nb);
-    __syncthreads();
-    float acc[8][2];
-    tile8x2<kOpDot>(S, rg, jb, acc);
-#pragma unroll
-    for (int x = 0; x < 8; ++x) {
-      const int r = rg * 8 + x;
-      if (r < nrows) {
-        if (j0 + jb < p.nb) Pbase[(int64_t)r * p.ld + j0 + jb] = acc[x][0] * 0.125f;
-        if (j0 + jb + 32 < p.nb) Pbase[(int64_t)r * p.ld + j0 + jb + 32] = acc[x][1] * 0.125f;
-      }
-    }
-    __syncthreads();
-  }
-
-  // ---- softmax statistics per row (max and normaliser, fixed order) ------------------
-  for (int r = warp; r < nrows; r += 8) {
-    const float* row = Pbase + (int64_t)r * p.ld;
-    float m = -INFINITY, z = 0.f;
-#pragma unroll 4
-    for (int j = lane; j < p.nb; j += 32) {
-      const float x = row[j];
-      if (x > m) {
-        z = z * expf(m - x) + 1.f;
-        m = x;
-      } else {
-        z += expf(x - m);
-      }
-    }
-    float mall = m;
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) mall = fmaxf(mall, __shfl_xor_sync(kFull, mall, o));
-    z = (m == -INFINITY) ? 0.f : z * expf(m - mall);
-    z = warp_sum(z);
-    if (lane == 0) {
-      S.rowm[r] = mall;
-      S.rowiz[r] = 1.0f / z;
-    }
-  }
-  __syncthreads();
-
-  // ---- pass 2: P_ij = softmax, y~_i = sum_j P_ij z~_j (Eq. 1 in F space) -----------
-  uint64_t ya[4];  // (channel 2 lane, channel 2 lane + 1) of 4 rows, packed f32x2
-#pragma unroll
-  for (int x = 0; x < 4; ++x) ya[x] = 0ull;
-  for (int j0 = 0; j0 < p.nb; j0 += BN) {
-    stage_blocks(S.B, zt_h, j0, p.nb);
-    for (int f = threadIdx.x; f < RT * (BN / 4); f += kThreads) {
-      const int r = f / (BN / 4), c4 = (f % (BN / 4)) * 4;
-      float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
-      if (r < nrows) {
-        float* src = Pbase + (int64_t)r * p.ld + j0 + c4;
-        const float m = S.rowm[r], iz = S.rowiz[r];
-        float e[4];
-#pragma unroll
-        for (int u = 0; u < 4; ++u) {
-          e[u] = 0.f;
-          if (j0 + c4 + u < p.nb) {
-            e[u] = expf(src[u] - m) * iz;
-            src[u] = e[u];
-          }
-        }
-        v = make_float4(e[0], e[1], e[2], e[3]);
-      }
-      *reinterpret_cast<float4*>(&S.Pc[r][c4]) = v;
-    }
-    __syncthreads();
-#pragma unroll 2
-    for (int jj = 0; jj < BN; jj += 4) {
-      float4 pv[4];
-#pragma unroll
-      for (int x = 0; x < 4; ++x) pv[x] = *reinterpret_cast<const float4*>(&S.Pc[warp * 4 + x][jj]);
-#pragma unroll
-      for (int u = 0; u < 4; ++u) {
-        const uint64_t z = *reinterpret_cast<const uint64_t*>(&S.B[jj + u][2 * lane]);
-#pragma unroll
-        for (int x = 0; x < 4; ++x) {
-          const float pu = u == 0 ? pv[x].x : (u == 1 ? pv[x].y : (u == 2 ? pv[x].z : pv[x].w));
-          ya[x] = ffma2(pack2(pu, pu), z, ya[x]);  // each half an fma.rn, as fmaf
-        }
-      }
-    }
-    __syncthreads();
-  }
-#pragma unroll
-  for (int x = 0; x < 4; ++x) {
-    const int r = warp * 4 + x;
-    const float2 y = unpack2(ya[x]);
-    S.A[r][2 * lane] = y.x;
-    S.A[r][2 * lane + 1] = y.y;
-    if (r < nrows) *reinterpret_cast<float2*>(p.ytil + (hrow + i0 + r) * 64 + 2 * lane) = y;
-  }
-  __syncthreads();
-
-  // ---- pass 3: q_ij = ||y~_i - z~_j||^2 (Eq. 9) --------------------------------------
-  for (int j0 = 0; j0 < p.nb; j0 += BN) {
-    stage_blocks(S.B, zt_h, j0, p.nb);
-    __syncthreads();
-    float acc[8][2];
-    tile8x2<kOpDist>(S, rg, jb, acc);
-#pragma unroll
-    for (int x = 0; x < 8; ++x) {
-      const int r = rg * 8 + x;
-      if (r < nrows) {
-        if (j0 + jb < p.nb) qbase[(int64_t)r * p.ld + j0 + jb] = acc[x][0];
-        if (j0 + jb + 32 < p.nb) qbase[(int64_t)r * p.ld + j0 + jb + 32] = acc[x][1];
-      }
-    }
-    __syncthreads();
-  }
-
-}
 
 // Exact decrease of J (Eq. 16) when G changes by dG and K by u, with the denominators
 // clamped at eps as in Eq. 7.  When no clamp applies the two fractions are combined over
@@ -1035,14 +798,18 @@ cudaError_t launch_score(const SelectArgs& a, cudaStream_t st) {
   float* kbar = (float*)(a.ws + a.L.kbar);
   float* vbar = (float*)(a.ws + a.L.vbar);
   float* ztil = (float*)(a.ws + a.L.ztil);
-  k_pool<<<dim3(s.nb, 3), kThreads, 0, st>>>(a.Q, a.K, a.V, s.N, s.H, s.nb, qbar, kbar, vbar);
+  k_pool<<<dim3(s.nb, 3), kThreads, 0, st>>>(a.Q, a.K, a.V, s.N, s.H, s.nb, qbar, kbar, vbar,
+                                              (uint16_t*)(a.ws + a.L.asplit),
+                                              (uint16_t*)(a.ws + a.L.ksplit));
   k_zproj<<<dim3((s.nb + 15) / 16, s.H), kThreads, 0, st>>>(
-      a.F, vbar, s.nb, ztil, (uint2*)(a.ws + a.L.zsplit), p.split_stride / 2);
-  if (s.ncand <= 0) return cudaGetLastError();
-  const size_t smem = sizeof(SelSmem);
-  cudaError_t e = cudaFuncSetAttribute(k_score, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-  if (e != cudaSuccess) return e;
-  k_score<<<dim3((s.ncand + RT - 1) / RT, s.H), kThreads, smem, st>>>(p, budgets_of(a));
+      a.F, vbar, s.nb, ztil, (uint2*)(a.ws + a.L.zsplit), p.split_stride / 2,
+      (float*)(a.ws + a.L.nz));
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess || s.ncand <= 0) return e;
+  // pooled logits, then P and y~, then q (Sec. 4.1, Eq. 1, Eq. 9), on the tensor cores
+  if ((e = launch_logits(a, st)) != cudaSuccess) return e;
+  if ((e = launch_yagg(a, st)) != cudaSuccess) return e;
+  if ((e = launch_drift_norms(a, st)) != cudaSuccess) return e;
   const size_t rsmem = (size_t)kRowWarps * warp_scratch_words(s.ld, s.words) * 4;
   e = cudaFuncSetAttribute(k_score_rows, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)rsmem);
   if (e != cudaSuccess) return e;

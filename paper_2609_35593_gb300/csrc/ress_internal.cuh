@@ -69,9 +69,13 @@ inline ress_ws_layout make_layout(const Shape& s) {
   L.dmask = take(msk);
   L.bmask = take(msk);
   L.plen = take((int64_t)s.H * ((s.nb + 1) / 2) * 4);
-  L.gsplit = take(3 * (int64_t)s.H * s.nb * kHeadDim * 2);
+  L.asplit = take(3 * (int64_t)s.H * s.nb * kHeadDim * 2);
+  L.ksplit = take(3 * (int64_t)s.H * s.nb * kHeadDim * 2);
   L.zsplit = take(3 * (int64_t)s.H * s.nb * kHeadDim * 2);
   L.cdot = take(row);
+  L.ny = take(row);
+  L.nz = take(row);
+  L.lstat = take((int64_t)s.H * s.nb * ((s.nb + 127) / 128) * 8);
   L.ld = s.ld;
   L.words = s.words;
   L.total = off;
@@ -105,6 +109,18 @@ __device__ __forceinline__ uint32_t cvt_bf16x2(float lo_elem, float hi_elem) {
   asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(hi_elem), "f"(lo_elem));
   return r;
 }
+__device__ __forceinline__ uint16_t cvt_bf16(float x) {
+  uint16_t r;
+  asm("cvt.rn.bf16.f32 %0, %1;" : "=h"(r) : "f"(x));
+  return r;
+}
+// One float as three bf16 terms (same rule as split3_bf16x2).
+__device__ __forceinline__ void split3_bf16(float x, uint16_t& hi, uint16_t& mid, uint16_t& lo) {
+  hi = cvt_bf16(x);
+  const float r = x - __uint_as_float((uint32_t)hi << 16);
+  mid = cvt_bf16(r);
+  lo = cvt_bf16(r - __uint_as_float((uint32_t)mid << 16));
+}
 __device__ __forceinline__ void split3_bf16x2(float x0, float x1, uint32_t& hi, uint32_t& mid,
                                               uint32_t& lo) {
   hi = cvt_bf16x2(x0, x1);
@@ -137,6 +153,9 @@ cudaError_t launch_prepare_wo(const Shape& s, const uint16_t* W_o, float* F, cud
 cudaError_t launch_score(const SelectArgs& a, cudaStream_t st);
 cudaError_t launch_round(const SelectArgs& a, int round, float rho, cudaStream_t st);
 cudaError_t launch_gain(const SelectArgs& a, int round, float rho, cudaStream_t st);
+cudaError_t launch_logits(const SelectArgs& a, cudaStream_t st);
+cudaError_t launch_drift_norms(const SelectArgs& a, cudaStream_t st);
+cudaError_t launch_yagg(const SelectArgs& a, cudaStream_t st);
 cudaError_t launch_csr(const SelectArgs& a, const int64_t* head_base, int32_t* row_ptr,
                        int32_t* col_idx, int64_t col_capacity, float* J_best,
                        uint32_t* drop_mask, cudaStream_t st);

@@ -314,7 +314,7 @@ def test_gain_products(fixture_name):
     z = layer.ws("ztil", shape=(H, nb, 64)).astype(np.float64)
     g = layer.ws("gtil", shape=(H, nb, 64)).astype(np.float64)
     cdot = layer.ws("cdot", shape=(H, nb)).astype(np.float64)
-    for name, x, rows in (("gsplit", g, nc), ("zsplit", z, nb)):
+    for name, x, rows in (("asplit", g, nc), ("zsplit", z, nb)):
         terms = synth.bf16_to_f32(layer.ws(name, torch.int16, (3, H, nb, 64)).view(np.uint16))
         hi, mid, lo = (terms[k].astype(np.float64)[:, :rows] for k in range(3))
         xs = x[:, :rows]
@@ -337,3 +337,39 @@ def test_gain_products(fixture_name):
         assert np.all(err <= bound), (h, float((err / bound).max()))
         checked += 1
     assert checked > 0
+
+
+@pytest.mark.parametrize("fixture_name", ["tiny_v2", "vggt_v8"])
+def test_tensor_core_scoring(fixture_name):
+    """Pooled map P, y~ and q (Sec. 4.1, Eq. 1, Eq. 9), computed on the tensor cores from
+    three-term bf16 splits, against float64 arithmetic on the same float32 pooled vectors
+    q_bar, k_bar and z~ that the GPU produced."""
+    layer, wl = layer_for(fixture_name)
+    r, b = layer.ress, layer.buf
+    r.prepare_wo(layer.d, layer.W, b.F)
+    r.score(layer.d, layer.Q, layer.K, layer.V, b.F, layer.c_h, b.ws)
+    r.status(b.ws)
+    torch.cuda.synchronize()
+    H, nb, nc, L = layer.H, layer.nb, layer.ncand, b.layout
+    qb = layer.ws("qbar", shape=(H, nb, 64)).astype(np.float64)
+    kb = layer.ws("kbar", shape=(H, nb, 64)).astype(np.float64)
+    z = layer.ws("ztil", shape=(H, nb, 64)).astype(np.float64)
+    y = layer.ws("ytil", shape=(H, nb, 64)).astype(np.float64)
+    P = layer.ws("P", shape=(H, nb, L.ld))
+    q = layer.ws("q", shape=(H, nb, L.ld))
+    nz = layer.ws("nz", shape=(H, nb)).astype(np.float64)
+    np.testing.assert_allclose(nz, (z * z).sum(2), rtol=1e-5)
+    for h in range(H):
+        logit = qb[h, :nc] @ kb[h].T / 8.0
+        Pr = np.exp(logit - logit.max(1, keepdims=True))
+        Pr /= Pr.sum(1, keepdims=True)
+        np.testing.assert_allclose(P[h, :nc, :nb], Pr, rtol=2e-5, atol=1e-7 * Pr.max())
+        assert np.all(P[h, :nc, nb:L.ld] == 0)
+        yr = Pr @ z[h]
+        yn = np.linalg.norm(yr, axis=1, keepdims=True)
+        assert np.all(np.abs(y[h, :nc] - yr) <= 1e-5 * (yn + np.abs(yr)) + 1e-30)
+        # q from the GPU's own y~ (its rounding is not q's error)
+        qr = ((y[h, :nc, None, :] - z[h, None, :, :]) ** 2).sum(2)
+        scale = (y[h, :nc] ** 2).sum(1)[:, None] + nz[h][None, :]
+        assert np.all(np.abs(q[h, :nc, :nb] - qr) <= 2e-6 * scale + 1e-30), h
+        assert np.all(q[h, :nc, :nb] >= 0)
