@@ -1,11 +1,12 @@
 // The row-by-block inner products of the selection on the tensor cores.  For one head and
 // every candidate row i and block j, with x_i a per-row 64-vector and w_j a per-block one:
-//   logits (Sec. 4.1):        L_ij = q_bar_i . k_bar_j / sqrt(64)            (j < nb)
+//   logits (Sec. 4.1):        L_ij = q_bar_i . k_bar_j / sqrt(64) * log2(e)  (j < nb)
 //   drift norms (Eq. 9):      q_ij = ||y~_i||^2 + ||z~_j||^2 - 2 y~_i . z~_j   (j < nb)
 //   round gains (Eq. 14/15):  t_ij = c_i - g~_i . z~_j,  c_i = y~_i . g~_i     (j < |P|)
-// The rows P (as logits), q or t of the workspace receive the results.  For the logits each
-// 128-block slice of a row also yields its max and its sum of exp(L - max), from which the
-// softmax of the row (the pooled map P) is assembled by k_yagg.
+// The rows P (as logits), q or t of the workspace receive the results.  The logits are kept
+// in base-2 units, so that P_ij = 2^(L_ij - m_i) / Z_i; each 128-block slice of a row also
+// yields its max and its sum of 2^(L - max), from which k_yagg assembles the softmax of the
+// row (the pooled map P).
 //
 // Both operands are fp32; each is held as the sum of three bf16 terms (hi + mid + lo,
 // written by the kernels that produce the vectors), and the product is accumulated in fp32
@@ -44,6 +45,7 @@ constexpr uint64_t kDotWaitNs = 2000000000ull;    // 2 s per wait
 constexpr uint64_t kDotDrainNs = 200000000ull;    // 0.2 s to drain after an abort
 
 enum DotMode { kDotGain = 0, kDotLogit = 1, kDotDist = 2 };
+constexpr float kLogitScale = 0.125f * 1.4426950408889634f;  // 1/sqrt(64) * log2(e)
 
 struct __align__(1024) DotSmem {
   uint8_t A[3][kTermBytes];  // row-vector terms (hi, mid, lo) of rows i0 .. i0 + 127
@@ -58,7 +60,7 @@ struct DotParams {
   float rho;
   const float* a;     // per row: c_i (gains) or ||y~_i||^2 (drift norms), [H, nb]
   const float* b;     // per block: ||z~_j||^2 (drift norms), [H, nb]
-  float2* lstat;      // logits: per row and 128-block slice (max, sum exp(L - max))
+  float2* lstat;      // logits: per row and 128-block slice (max, sum 2^(L - max))
   int nslices;        // ceil(nb / 128)
   int ld;             // row stride of the output
   uint32_t* status;
@@ -180,16 +182,16 @@ __global__ void __launch_bounds__(kDotThreads)
         float cm = -INFINITY;
 #pragma unroll
         for (int k = 0; k < 32; ++k) {
-          o[k] = __uint_as_float(v[k]) * 0.125f;
+          o[k] = __uint_as_float(v[k]) * kLogitScale;
           if (jq + k < p.nb) cm = fmaxf(cm, o[k]);
         }
         if (cm > pm) {
-          ps = (pm == -INFINITY) ? 0.f : ps * expf(pm - cm);
+          ps = (pm == -INFINITY) ? 0.f : ps * exp2f(pm - cm);
           pm = cm;
         }
 #pragma unroll
         for (int k = 0; k < 32; ++k)
-          if (jq + k < p.nb) ps += expf(o[k] - pm);
+          if (jq + k < p.nb) ps += exp2f(o[k] - pm);
       } else {
         const int jq = j0 + 32 * q;
 #pragma unroll

@@ -1,22 +1,23 @@
 // Pooled attention map and pooled output in F space (Sec. 4.1, Eq. 1) on the tensor cores:
-//   P_ij = exp(L_ij - m_i) / Z_i  over all key blocks j < nb   (L = pooled logits, k_dot)
+//   P_ij = 2^(L_ij - m_i) / Z_i   over all key blocks j < nb   (L = pooled logits in base-2
+//                                                                 units, from k_dot)
 //   y~_i = sum_j P_ij z~_j                                     (z~_j = F_h V_j)
 // for the candidate rows of one head.  m_i and Z_i come from the per-slice maxima and sums
 // k_dot left in lstat.  P overwrites L in place; y~ is written in fp32, as three bf16
 // terms (the row operand of the drift-norm products) and as ||y~_i||^2.
 //
-// One CTA per 128 candidate rows of a head, 288 threads, 64 key blocks per chunk, two
+// One CTA per 128 candidate rows of a head, 544 threads, 64 key blocks per chunk, two
 // pipeline stages:
-//   warp 8     lane 0 loads chunk c + 1 by TMA (L: two 32-column fp32 boxes; z~: its three
+//   warp 16    lane 0 loads chunk c + 1 by TMA (L: two 32-column fp32 boxes; z~: its three
 //              bf16 term tiles, 64 blocks x 64 channels) while the chunk c is converted;
 //              then the converged warp, one elected lane, issues the chunk's MMAs
 //                y~ += P_c^(a) z~_c^(b)   for the six term pairs (a, b) of k_dot,
 //              M128 N64 K16 x 4 each, P terms K-major, z~ terms MN-major, both from shared
 //              memory, and commits them to the stage's "empty" barrier;
-//   warps 0-7  one row and 32 of the chunk's blocks per thread: P from L, P back to global
+//   warps 0-15 one row and 16 of the chunk's blocks per thread: P from L, P back to global
 //              memory, P as three bf16 terms into the stage's A tiles (128-byte swizzle),
 //              then an arrive on the stage's "converted" barrier; after the last chunk the
-//              epilogue (warp w: TMEM lanes 32 (w mod 4).., columns 32 (w / 4)..).
+//              epilogue (warp w: TMEM lanes 32 (w mod 4).., columns 16 (w / 4)..).
 // Every mbarrier wait is bounded; a wait that gives up records RESS_ETIMEOUT, lets copies
 // and MMAs already issued finish (again bounded), frees TMEM and returns.
 
@@ -33,7 +34,9 @@ bool make_row_map(CUtensorMap* m, void* base, int nb, int H, int ld);
 
 namespace {
 
-constexpr int kYThreads = 288;
+constexpr int kConvWarps = 16;
+constexpr int kYThreads = 32 * kConvWarps + 32;
+constexpr int kMmaWarp = kConvWarps;
 constexpr int kYRows = 128;      // candidate rows per CTA
 constexpr int kYChunk = 64;      // key blocks per pipeline step
 constexpr int kYStages = 2;
@@ -45,7 +48,7 @@ struct __align__(1024) YSmem {
   uint8_t L[kYStages][2][16384];  // logits: 2 boxes of 128 rows x 32 fp32 (swizzled)
   uint8_t A[kYStages][3][16384];  // P terms: 128 rows x 64 blocks bf16 (K-major, swizzled)
   uint8_t Z[kYStages][3][8192];   // z~ terms: 64 blocks x 64 channels bf16 (MN-major)
-  float ny_half[2][kYRows];
+  float ny_part[4][kYRows];
   uint64_t full[kYStages], conv[kYStages], empty[kYStages];
   uint64_t done;
   uint32_t tmem_base;
@@ -94,7 +97,7 @@ __global__ void __launch_bounds__(kYThreads, 1)
   if (threadIdx.x == 0) {
     for (int s = 0; s < kYStages; ++s) {
       mbar_init(&S.full[s], 1);
-      mbar_init(&S.conv[s], 8);
+      mbar_init(&S.conv[s], kConvWarps);
       mbar_init(&S.empty[s], 1);
     }
     mbar_init(&S.done, 1);
@@ -103,13 +106,13 @@ __global__ void __launch_bounds__(kYThreads, 1)
     prefetch_tensormap(&tmL);
     prefetch_tensormap(&tmZ);
   }
-  if (warp == 8) tmem_alloc(&S.tmem_base, kYCols);
+  if (warp == kMmaWarp) tmem_alloc(&S.tmem_base, kYCols);
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = S.tmem_base;
 
-  if (warp == 8) {
+  if (warp == kMmaWarp) {
     // ============================ loads and MMAs ====================================
     const bool leader = elect_one();
     bool failed = false;
@@ -179,7 +182,7 @@ __global__ void __launch_bounds__(kYThreads, 1)
     }
   } else {
     // ============================ conversion ========================================
-    const int r = 32 * (warp & 3) + lane, hf = warp >> 2;  // row of the tile, column half
+    const int r = 32 * (warp & 3) + lane, qq = warp >> 2;  // row of the tile, column quarter
     const int i = i0 + r;
     const bool row_ok = i < p.ncand;
     const int64_t ri = (int64_t)h * p.nb + i;
@@ -190,7 +193,7 @@ __global__ void __launch_bounds__(kYThreads, 1)
       float z = 0.f;
       for (int t = 0; t < p.nslices; ++t) {
         const float2 st = p.lstat[ri * p.nslices + t];
-        if (st.x != -INFINITY) z += st.y * expf(st.x - m);
+        if (st.x != -INFINITY) z += st.y * exp2f(st.x - m);
       }
       iz = 1.0f / z;
     }
@@ -202,31 +205,32 @@ __global__ void __launch_bounds__(kYThreads, 1)
         failed = true;
         break;
       }
-      const int jb = c * kYChunk + 32 * hf;  // first block of this thread's 32
-      const uint8_t* lrow = S.L[s][hf] + r * 128;
-      float pv[32];
+      const int jb = c * kYChunk + 16 * qq;  // first block of this thread's 16
+      // L: box qq / 2, 16-byte chunks 4 (qq mod 2) .. + 3 of row r
+      const uint8_t* lrow = S.L[s][qq >> 1] + r * 128;
+      float pv[16];
 #pragma unroll
-      for (int k = 0; k < 8; ++k) {
-        const float4 v = *reinterpret_cast<const float4*>(lrow + ((k ^ (r & 7)) << 4));
+      for (int k = 0; k < 4; ++k) {
+        const float4 v = *reinterpret_cast<const float4*>(lrow + (((4 * (qq & 1) + k) ^ (r & 7)) << 4));
         const float lv[4] = {v.x, v.y, v.z, v.w};
 #pragma unroll
         for (int e = 0; e < 4; ++e)
-          pv[4 * k + e] = (row_ok && jb + 4 * k + e < p.nb) ? expf(lv[e] - m) * iz : 0.f;
+          pv[4 * k + e] = (row_ok && jb + 4 * k + e < p.nb) ? exp2f(lv[e] - m) * iz : 0.f;
       }
-      if (row_ok && jb < p.ld) {
+      if (row_ok && jb < p.ld) {  // ld is a multiple of 16
 #pragma unroll
-        for (int k = 0; k < 8; ++k)
+        for (int k = 0; k < 4; ++k)
           *reinterpret_cast<float4*>(Prow + jb + 4 * k) =
               make_float4(pv[4 * k], pv[4 * k + 1], pv[4 * k + 2], pv[4 * k + 3]);
       }
-      // P terms: this thread's 32 blocks are 16-byte chunks 4 hf .. 4 hf + 3 of row r
+      // P terms: this thread's 16 blocks are 16-byte chunks 2 qq, 2 qq + 1 of row r
 #pragma unroll
-      for (int k = 0; k < 4; ++k) {
+      for (int k = 0; k < 2; ++k) {
         uint32_t hi[4], mid[4], lo[4];
 #pragma unroll
         for (int e = 0; e < 4; ++e)
           split3_bf16x2(pv[8 * k + 2 * e], pv[8 * k + 2 * e + 1], hi[e], mid[e], lo[e]);
-        const int off = r * 128 + (((4 * hf + k) ^ (r & 7)) << 4);
+        const int off = r * 128 + (((2 * qq + k) ^ (r & 7)) << 4);
         *reinterpret_cast<uint4*>(S.A[s][0] + off) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
         *reinterpret_cast<uint4*>(S.A[s][1] + off) = make_uint4(mid[0], mid[1], mid[2], mid[3]);
         *reinterpret_cast<uint4*>(S.A[s][2] + off) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
@@ -236,22 +240,22 @@ __global__ void __launch_bounds__(kYThreads, 1)
       if (lane == 0) mbar_arrive(&S.conv[s]);
     }
     if (failed && lane == 0) y_give_up(S, p.status);
-    // ---- epilogue: y~ row r, channels 32 hf .. 32 hf + 31 ------------------------------
+    // ---- epilogue: y~ row r, channels 16 qq .. 16 qq + 15 ------------------------------
     float nyp = 0.f;
     if (!failed && y_wait(&S.done, 0, abort)) {
       tc_fence_after();
-      uint32_t v[32];
-      RESS_TMEM_LD32(tmem + ((uint32_t)(32 * (warp & 3)) << 16) + 32 * hf, v);
+      uint32_t v[16];
+      RESS_TMEM_LD16(tmem + ((uint32_t)(32 * (warp & 3)) << 16) + 16 * qq, v);
       if (row_ok) {
-        float* yrow = p.ytil + ri * 64 + 32 * hf;
+        float* yrow = p.ytil + ri * 64 + 16 * qq;
 #pragma unroll
-        for (int k = 0; k < 8; ++k)
+        for (int k = 0; k < 4; ++k)
           *reinterpret_cast<float4*>(yrow + 4 * k) =
               make_float4(__uint_as_float(v[4 * k]), __uint_as_float(v[4 * k + 1]),
                           __uint_as_float(v[4 * k + 2]), __uint_as_float(v[4 * k + 3]));
-        uint32_t* as = p.asplit + ri * 32 + 16 * hf;
+        uint32_t* as = p.asplit + ri * 32 + 8 * qq;
 #pragma unroll
-        for (int k = 0; k < 4; ++k) {
+        for (int k = 0; k < 2; ++k) {
           uint32_t hi[4], mid[4], lo[4];
 #pragma unroll
           for (int e = 0; e < 4; ++e)
@@ -264,21 +268,22 @@ __global__ void __launch_bounds__(kYThreads, 1)
               make_uint4(lo[0], lo[1], lo[2], lo[3]);
         }
 #pragma unroll
-        for (int k = 0; k < 32; ++k) nyp = fmaf(__uint_as_float(v[k]), __uint_as_float(v[k]), nyp);
+        for (int k = 0; k < 16; ++k) nyp = fmaf(__uint_as_float(v[k]), __uint_as_float(v[k]), nyp);
       }
     } else if (lane == 0) {
       y_give_up(S, p.status);
     }
-    S.ny_half[hf][r] = nyp;
+    S.ny_part[qq][r] = nyp;
   }
   tc_fence_before();
   __syncthreads();
   if (threadIdx.x < kYRows) {
     const int i = i0 + threadIdx.x;
     if (i < p.ncand && !*abort)
-      p.ny[(int64_t)h * p.nb + i] = S.ny_half[0][threadIdx.x] + S.ny_half[1][threadIdx.x];
+      p.ny[(int64_t)h * p.nb + i] = (S.ny_part[0][threadIdx.x] + S.ny_part[1][threadIdx.x]) +
+                                    (S.ny_part[2][threadIdx.x] + S.ny_part[3][threadIdx.x]);
   }
-  if (warp == 8) {
+  if (warp == kMmaWarp) {
     tc_fence_after();
     tmem_dealloc(tmem, kYCols);
   }
