@@ -92,6 +92,12 @@ __global__ void __launch_bounds__(kThreads) k_prepare_wo(const uint16_t* __restr
   }
 }
 
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(kFull, v, o);
+  return v;
+}
+
 // ------------------------------------------------------------------------------------
 // Sec. 3 step (1): block means of Q, K and V over the valid tokens of each block.
 // grid (nb, 3); one token is H*64 bf16 = 8H 16-byte chunks (H <= 32).
@@ -150,50 +156,69 @@ __global__ void __launch_bounds__(kThreads) k_pool(const uint16_t* __restrict__ 
 }
 
 // ------------------------------------------------------------------------------------
-// z~_j = F_h V_j.  grid (ceil(nb/16), H); thread (block jj, channels 4a..4a+3).
+// z~_j = F_h V_j.  grid (ceil(nb/16), H); thread (channel a, blocks 4q..4q+3 of the 16).
+// F_h and the 16 pooled values sit in shared memory with rows padded to 68 floats, so that
+// the float4 reads of a warp (32 channels, one column group) hit every bank once per pass.
 // ------------------------------------------------------------------------------------
 __global__ void __launch_bounds__(kThreads) k_zproj(const float* __restrict__ F,
                                                      const float* __restrict__ vbar, int nb,
                                                      float* __restrict__ ztil,
-                                                     uint2* __restrict__ zsplit,
+                                                     uint16_t* __restrict__ zsplit,
                                                      int64_t term_stride,
                                                      float* __restrict__ nz) {
-  __shared__ __align__(16) float Ft[64][64];  // Ft[b][a] = F[a][b]
-  __shared__ float Vs[16][65];
+  constexpr int kPad = 68;
+  __shared__ __align__(16) float Fs[64][kPad];  // Fs[a][b] = F[a][b]
+  __shared__ __align__(16) float Vs[16][kPad];
+  __shared__ float npart[8][4];
   const int h = blockIdx.y, j0 = blockIdx.x * 16, t = threadIdx.x;
-  for (int f = t; f < 4096; f += kThreads) Ft[f & 63][f >> 6] = F[(int64_t)h * 4096 + f];
-  for (int f = t; f < 16 * 64; f += kThreads) {
-    const int r = f >> 6, c = f & 63;
-    Vs[r][c] = (j0 + r < nb) ? vbar[((int64_t)h * nb + j0 + r) * 64 + c] : 0.f;
+  const int warp = t >> 5, lane = t & 31;
+  for (int f = t; f < 1024; f += kThreads) {  // float4 units
+    const int r = f >> 4, c4 = (f & 15) * 4;
+    *reinterpret_cast<float4*>(&Fs[r][c4]) =
+        *reinterpret_cast<const float4*>(F + (int64_t)h * 4096 + r * 64 + c4);
+  }
+  for (int f = t; f < 256; f += kThreads) {
+    const int r = f >> 4, c4 = (f & 15) * 4;
+    float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (j0 + r < nb) v = *reinterpret_cast<const float4*>(vbar + ((int64_t)h * nb + j0 + r) * 64 + c4);
+    *reinterpret_cast<float4*>(&Vs[r][c4]) = v;
   }
   __syncthreads();
-  const int jj = t >> 4, a4 = (t & 15) * 4;
-  if (j0 + jj >= nb) return;
-  float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-#pragma unroll 8
-  for (int b = 0; b < 64; ++b) {
-    const float v = Vs[jj][b];
-    const float4 f = *reinterpret_cast<const float4*>(&Ft[b][a4]);
-    acc.x = fmaf(f.x, v, acc.x);
-    acc.y = fmaf(f.y, v, acc.y);
-    acc.z = fmaf(f.z, v, acc.z);
-    acc.w = fmaf(f.w, v, acc.w);
-  }
-  const int64_t at = ((int64_t)h * nb + j0 + jj) * 64 + a4;
-  *reinterpret_cast<float4*>(ztil + at) = acc;
-  // the same vectors as three bf16 terms, the B operands of the tensor-core gains
-  uint2 hi, mid, lo;
-  split3_bf16x2(acc.x, acc.y, hi.x, mid.x, lo.x);
-  split3_bf16x2(acc.z, acc.w, hi.y, mid.y, lo.y);
-  zsplit[at / 4] = hi;
-  zsplit[at / 4 + term_stride] = mid;
-  zsplit[at / 4 + 2 * term_stride] = lo;
-  // ||z~_j||^2 over the 16 threads of block jj (one half-warp), fixed order
-  const unsigned group = 0xFFFFu << (threadIdx.x & 16);
-  float n2 = fmaf(acc.w, acc.w, fmaf(acc.z, acc.z, fmaf(acc.y, acc.y, acc.x * acc.x)));
+  const int a = t & 63, q = t >> 6;  // q is uniform across a warp
+  float acc[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll 4
+  for (int b4 = 0; b4 < 64; b4 += 4) {
+    const float4 f = *reinterpret_cast<const float4*>(&Fs[a][b4]);
 #pragma unroll
-  for (int o = 8; o > 0; o >>= 1) n2 += __shfl_xor_sync(group, n2, o);
-  if ((t & 15) == 0) nz[(int64_t)h * nb + j0 + jj] = n2;
+    for (int u = 0; u < 4; ++u) {
+      const float4 v = *reinterpret_cast<const float4*>(&Vs[4 * q + u][b4]);
+      acc[u] = fmaf(f.x, v.x, acc[u]);
+      acc[u] = fmaf(f.y, v.y, acc[u]);
+      acc[u] = fmaf(f.z, v.z, acc[u]);
+      acc[u] = fmaf(f.w, v.w, acc[u]);
+    }
+  }
+#pragma unroll
+  for (int u = 0; u < 4; ++u) {
+    const int j = j0 + 4 * q + u;
+    if (j < nb) {
+      const int64_t at = ((int64_t)h * nb + j) * 64 + a;
+      ztil[at] = acc[u];
+      // the same vector as three bf16 terms: an operand of the tensor-core products
+      uint16_t hi, mid, lo;
+      split3_bf16(acc[u], hi, mid, lo);
+      zsplit[at] = hi;
+      zsplit[at + term_stride] = mid;
+      zsplit[at + 2 * term_stride] = lo;
+    }
+    const float n2 = warp_sum(acc[u] * acc[u]);  // this warp's 32 channels
+    if (lane == 0) npart[warp][u] = n2;
+  }
+  __syncthreads();
+  if (t < 16) {  // ||z~_j||^2: the two warps of block group q, fixed order
+    const int qq = t >> 2, u = t & 3, j = j0 + t;
+    if (j < nb) nz[(int64_t)h * nb + j] = npart[2 * qq][u] + npart[2 * qq + 1][u];
+  }
 }
 
 struct SelPtrs {
@@ -456,12 +481,6 @@ __device__ void warp_topm_pair(const uint32_t* kk, int n, int m, const uint32_t*
   else
     select_exact(sk + kHalf, si + kHalf, cntB, m, nullptr, true, selB);
   __syncwarp();
-}
-
-__device__ __forceinline__ float warp_sum(float v) {
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(kFull, v, o);
-  return v;
 }
 
 // g~ of row ri (this lane's channels 2 lane, 2 lane + 1), its three bf16 terms (the A
@@ -740,7 +759,7 @@ __global__ void __launch_bounds__(32 * kRowWarps, 8) k_round_rows(SelPtrs p, Bud
 
 // ------------------------------------------------------------------------------------
 // Kept-block lists (CSR) from the best drop sets; special query rows keep everything.
-// grid (nb, H), one warp per row.
+// grid (ceil(nb / 8), H) x 256 threads, one warp per row.
 // ------------------------------------------------------------------------------------
 struct CsrBases {
   int64_t base[RESS_MAX_HEADS + 1];
@@ -749,7 +768,8 @@ struct CsrBases {
 __global__ void k_csr(SelPtrs p, Budgets bud, CsrBases cb, int H, int32_t* __restrict__ row_ptr,
                       int32_t* __restrict__ col_idx, int64_t cap, float* __restrict__ J_best,
                       uint32_t* __restrict__ drop_mask, uint32_t* status) {
-  const int i = blockIdx.x, h = blockIdx.y, lane = threadIdx.x;
+  const int i = blockIdx.x * 8 + (threadIdx.x >> 5), h = blockIdx.y, lane = threadIdx.x & 31;
+  if (i >= p.nb) return;
   const int64_t ri = (int64_t)h * p.nb + i;
   const int c = bud.c[h];
   const int ns = p.nb - p.ncand;
@@ -758,15 +778,20 @@ __global__ void k_csr(SelPtrs p, Budgets bud, CsrBases cb, int H, int32_t* __res
                                           : (int64_t)i * (c + ns));
   const int expect = dense ? p.nb : c + ns;
   int pos = 0;
-  for (int w = 0; w < p.words; ++w) {
-    const uint32_t dm = dense ? 0u : p.bmask[ri * p.words + w];
-    const uint32_t keep = ~dm & valid_bits(w, p.nb);
-    if (drop_mask && lane == 0) drop_mask[ri * p.words + w] = dm;
-    const int j = w * 32 + lane;
-    const bool k = (keep >> lane) & 1u;
-    const int at = pos + __popc(keep & ((1u << lane) - 1u));
-    if (k && at < expect && off + at < cap) col_idx[off + at] = j;
-    pos += __popc(keep);
+  for (int w0 = 0; w0 < p.words; w0 += 32) {
+    // 32 words per coalesced load, handed out by shuffle
+    const uint32_t mine =
+        (!dense && w0 + lane < p.words) ? p.bmask[ri * p.words + w0 + lane] : 0u;
+    if (drop_mask && w0 + lane < p.words) drop_mask[ri * p.words + w0 + lane] = mine;
+    const int nw = min(32, p.words - w0);
+    for (int k = 0; k < nw; ++k) {
+      const int w = w0 + k;
+      const uint32_t dm = __shfl_sync(kFull, mine, k);
+      const uint32_t keep = ~dm & valid_bits(w, p.nb);
+      const int at = pos + __popc(keep & ((1u << lane) - 1u));
+      if (((keep >> lane) & 1u) && at < expect && off + at < cap) col_idx[off + at] = w * 32 + lane;
+      pos += __popc(keep);
+    }
   }
   if (lane == 0) {
     if (pos != expect) flag_status(status, kStatusBadRow);
@@ -802,7 +827,7 @@ cudaError_t launch_score(const SelectArgs& a, cudaStream_t st) {
                                               (uint16_t*)(a.ws + a.L.asplit),
                                               (uint16_t*)(a.ws + a.L.ksplit));
   k_zproj<<<dim3((s.nb + 15) / 16, s.H), kThreads, 0, st>>>(
-      a.F, vbar, s.nb, ztil, (uint2*)(a.ws + a.L.zsplit), p.split_stride / 2,
+      a.F, vbar, s.nb, ztil, (uint16_t*)(a.ws + a.L.zsplit), (int64_t)s.H * s.nb * kHeadDim,
       (float*)(a.ws + a.L.nz));
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess || s.ncand <= 0) return e;
@@ -839,7 +864,7 @@ cudaError_t launch_csr(const SelectArgs& a, const int64_t* head_base, int32_t* r
   SelPtrs p = sel_ptrs(s, a.ws, a.L);
   CsrBases cb;
   for (int h = 0; h <= s.H; ++h) cb.base[h] = head_base[h];
-  k_csr<<<dim3(s.nb, s.H), 32, 0, st>>>(p, budgets_of(a), cb, s.H, row_ptr, col_idx, col_capacity,
+  k_csr<<<dim3((s.nb + 7) / 8, s.H), 256, 0, st>>>(p, budgets_of(a), cb, s.H, row_ptr, col_idx, col_capacity,
                                         J_best, drop_mask, (uint32_t*)(a.ws + a.L.status));
   return cudaGetLastError();
 }
