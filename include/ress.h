@@ -93,6 +93,12 @@ typedef struct {
 const char* ress_last_error(void);
 int32_t ress_abi_version(void);
 
+/* Number of kernels this library has enqueued since it was loaded, over all calls, streams
+ * and threads of the process (host-side count, incremented at each launch).  For telemetry
+ * and benchmarks: the difference around a sequence of calls is the number of kernels they
+ * put on the GPU.  No paper counterpart. */
+uint64_t ress_kernel_launches(void);
+
 /* Number of key blocks nb = ceil(N / 64) and candidate blocks |P|; -1 on bad dims. */
 int32_t ress_num_blocks(const ress_dims* dims);
 int32_t ress_num_candidates(const ress_dims* dims);

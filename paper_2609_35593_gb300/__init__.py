@@ -55,6 +55,7 @@ _P = _c.c_void_p
 _SIGS = {
     "ress_last_error": (_c.c_char_p, []),
     "ress_abi_version": (_c.c_int32, []),
+    "ress_kernel_launches": (_c.c_uint64, []),
     "ress_num_blocks": (_c.c_int32, [_c.POINTER(Dims)]),
     "ress_num_candidates": (_c.c_int32, [_c.POINTER(Dims)]),
     "ress_workspace_bytes": (_c.c_size_t, [_c.POINTER(Dims)]),
@@ -96,6 +97,11 @@ def _check(rc: int):
 
 def dims(n_tokens: int, n_heads: int, n_special: int, d_model: int) -> Dims:
     return Dims(n_tokens, n_heads, HEAD_DIM, BLOCK, n_special, d_model)
+
+
+def kernel_launches() -> int:
+    """ress_kernel_launches: kernels this library has enqueued so far in the process."""
+    return int(_lib.ress_kernel_launches())
 
 
 def num_blocks(d: Dims) -> int:

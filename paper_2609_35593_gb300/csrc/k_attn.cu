@@ -608,6 +608,7 @@ cudaError_t launch_sparse_attn(const AttnArgs& x, cudaStream_t st) {
   const int pairs = s.H * npairs;
   k_pairs<<<(pairs + 7) / 8, 256, 0, st>>>(x.row_ptr, x.col_idx, x.col_capacity, x.scratch_cap,
                                            s.nb, npairs, s.H, x.plist, x.plen, x.status);
+  note_launch();
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
   e = cudaMemsetAsync(x.counter, 0, sizeof(uint32_t), st);
@@ -631,6 +632,7 @@ cudaError_t launch_sparse_attn(const AttnArgs& x, cudaStream_t st) {
   if (e != cudaSuccess) return e;
   const int grid = min(pairs, 2 * sm_count());
   kern<<<grid, kAttnThreads, smem, st>>>(tq, tk, tv, p);
+  note_launch();
   return cudaGetLastError();
 }
 

@@ -305,6 +305,7 @@ cudaError_t launch_dot(const SelectArgs& a, int64_t a_terms, int64_t b_terms, in
   if (e != cudaSuccess) return e;
   const dim3 grid((ncols + kDotTile - 1) / kDotTile, (s.ncand + kDotTile - 1) / kDotTile, s.H);
   k_dot<MODE><<<grid, kDotThreads, smem, st>>>(ta, tb, to, p);
+  note_launch();
   return cudaGetLastError();
 }
 

@@ -807,6 +807,7 @@ __global__ void k_csr(SelPtrs p, Budgets bud, CsrBases cb, int H, int32_t* __res
 
 cudaError_t launch_prepare_wo(const Shape& s, const uint16_t* W_o, float* F, cudaStream_t st) {
   k_prepare_wo<<<s.H, kThreads, 0, st>>>(W_o, s.d_model, s.H, F);
+  note_launch();
   return cudaGetLastError();
 }
 
@@ -826,9 +827,11 @@ cudaError_t launch_score(const SelectArgs& a, cudaStream_t st) {
   k_pool<<<dim3(s.nb, 3), kThreads, 0, st>>>(a.Q, a.K, a.V, s.N, s.H, s.nb, qbar, kbar, vbar,
                                               (uint16_t*)(a.ws + a.L.asplit),
                                               (uint16_t*)(a.ws + a.L.ksplit));
+  note_launch();
   k_zproj<<<dim3((s.nb + 15) / 16, s.H), kThreads, 0, st>>>(
       a.F, vbar, s.nb, ztil, (uint16_t*)(a.ws + a.L.zsplit), (int64_t)s.H * s.nb * kHeadDim,
       (float*)(a.ws + a.L.nz));
+  note_launch();
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess || s.ncand <= 0) return e;
   // pooled logits, then P and y~, then q (Sec. 4.1, Eq. 1, Eq. 9), on the tensor cores
@@ -840,6 +843,7 @@ cudaError_t launch_score(const SelectArgs& a, cudaStream_t st) {
   if (e != cudaSuccess) return e;
   k_score_rows<<<dim3((s.ncand + kRowWarps - 1) / kRowWarps, s.H), 32 * kRowWarps, rsmem, st>>>(
       p, budgets_of(a));
+  note_launch();
   return cudaGetLastError();
 }
 
@@ -854,6 +858,7 @@ cudaError_t launch_round(const SelectArgs& a, int round, float rho, cudaStream_t
   if (e != cudaSuccess) return e;
   k_round_rows<<<dim3((s.ncand + kRowWarps - 1) / kRowWarps, s.H), 32 * kRowWarps, rsmem, st>>>(
       p, budgets_of(a), round, rho);
+  note_launch();
   return cudaGetLastError();
 }
 
@@ -866,6 +871,7 @@ cudaError_t launch_csr(const SelectArgs& a, const int64_t* head_base, int32_t* r
   for (int h = 0; h <= s.H; ++h) cb.base[h] = head_base[h];
   k_csr<<<dim3((s.nb + 7) / 8, s.H), 256, 0, st>>>(p, budgets_of(a), cb, s.H, row_ptr, col_idx, col_capacity,
                                         J_best, drop_mask, (uint32_t*)(a.ws + a.L.status));
+  note_launch();
   return cudaGetLastError();
 }
 

@@ -315,6 +315,7 @@ cudaError_t launch_yagg(const SelectArgs& a, cudaStream_t st) {
   cudaError_t e = cudaFuncSetAttribute(k_yagg, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   k_yagg<<<dim3((s.ncand + kYRows - 1) / kYRows, s.H), kYThreads, smem, st>>>(tl, tz, p);
+  note_launch();
   return cudaGetLastError();
 }
 

@@ -5,9 +5,13 @@
 #include <stdio.h>
 #include <string.h>
 
+#include <atomic>
+
 #include "ress_internal.cuh"
 
 namespace {
+
+std::atomic<uint64_t> g_kernel_launches{0};
 
 thread_local char g_err[512] = "";
 
@@ -99,11 +103,17 @@ ress::SelectArgs select_args(const ress::Shape& s, const uint16_t* Q, const uint
 
 }  // namespace
 
+namespace ress {
+void note_launch() { g_kernel_launches.fetch_add(1, std::memory_order_relaxed); }
+}  // namespace ress
+
 extern "C" {
 
 const char* ress_last_error(void) { return g_err; }
 
 int32_t ress_abi_version(void) { return RESS_ABI_VERSION; }
+
+uint64_t ress_kernel_launches(void) { return g_kernel_launches.load(std::memory_order_relaxed); }
 
 int32_t ress_num_blocks(const ress_dims* d) {
   if (check_dims(d)) return -1;

@@ -139,6 +139,9 @@ __device__ __forceinline__ uint4 ld_stream(const uint4* p) {
   return r;
 }
 
+// Counts one kernel launch of this library (host side, process-wide; ress_kernel_launches).
+void note_launch();
+
 // Kernel launchers (defined in k_select.cu / k_attn.cu); each returns a cudaError_t.
 struct SelectArgs {
   Shape s;

@@ -120,3 +120,8 @@ def test_binding_refuses_host_tensors():
     with pytest.raises(ValueError):
         ress.sparse_attn(d, x, x, x, torch.zeros(3, dtype=torch.int32), torch.zeros(3, dtype=torch.int32),
                          x, torch.zeros(8, dtype=torch.uint8))
+
+
+def test_launch_counter_is_exported_and_monotone():
+    a = ress.kernel_launches()
+    assert a >= 0 and ress.kernel_launches() >= a

@@ -373,3 +373,17 @@ def test_tensor_core_scoring(fixture_name):
         scale = (y[h, :nc] ** 2).sum(1)[:, None] + nz[h][None, :]
         assert np.all(np.abs(q[h, :nc, :nb] - qr) <= 2e-6 * scale + 1e-30), h
         assert np.all(q[h, :nc, :nb] >= 0)
+
+
+def test_kernel_launch_counter():
+    """ress_kernel_launches counts every kernel of a forward: six for scoring (pooling,
+    z-projection, logits, P with y~, q, score rows), two per restoration round, the CSR
+    kernel, and the pair unions with the attention kernel."""
+    layer, wl = layer_for("tiny_v2")
+    r, b = layer.ress, layer.buf
+    r.prepare_wo(layer.d, layer.W, b.F)
+    n0 = r.kernel_launches()
+    r.forward(layer.d, layer.Q, layer.K, layer.V, b.F, layer.c_h, layer.rounds, layer.rho, b.ws,
+              b.row_ptr, b.col_idx, b.O, b.J_best)
+    torch.cuda.synchronize()
+    assert r.kernel_launches() - n0 == 6 + 2 * layer.rounds + 1 + 2
