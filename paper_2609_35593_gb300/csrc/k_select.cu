@@ -681,7 +681,7 @@ __global__ void __launch_bounds__(32 * kRowWarps, 8) k_score_rows(SelPtrs p, Bud
 
 // ------------------------------------------------------------------------------------
 // Restoration round r (Sec. 4.3, Eq. 13-17).  The gain inner products t_ij of the round
-// come from k_gain (tensor cores, k_gain.cu); the rest of the round runs per row here.
+// come from k_dot (tensor cores, k_dot.cu); the rest of the round runs per row here.
 // ------------------------------------------------------------------------------------
 // Restoration round r, per row: exact top-m restores and drops from the round-start state,
 // update, track-best.  grid (ceil(|P| / 4), H).
