@@ -187,6 +187,26 @@ int ress_forward_host(const ress_dims* dims, const uint16_t* Q_host, const uint1
                       int32_t rounds, float rho, void* ws, size_t ws_bytes, int32_t* row_ptr,
                       int32_t* col_idx, int64_t col_capacity, float* J_best, void* stream);
 
+/* Sec. 3: the attention sublayer's residual update, y = x + O W_o^T (pre-LN structure
+ * x_{l+1} = x_l + f_l(x_l); O W_o^T is what the sublayer adds to the residual stream).
+ * O: device bf16 [N, H*64] (the attention output, [N, H, 64]); W_o: device bf16 [d_model,
+ * H*64] (Linear weight, out x in); x, y: device bf16 [N, d_model] (x may equal y for an in-
+ * place update; x NULL gives y = O W_o^T).  fp32 accumulation on the tensor cores (tcgen05),
+ * one rounding to bf16.  d_model must be a multiple of 64.  Uses the workspace's status word
+ * only. */
+int ress_out_proj(const ress_dims* dims, const uint16_t* O, const uint16_t* W_o,
+                  const uint16_t* x, uint16_t* y, void* ws, size_t ws_bytes, void* stream);
+
+/* Sec. 3's token-level reference for the drift: for every query block b,
+ *   drift[b] = sum over the query tokens t of block b of || W_o (O_a[t] - O_b[t]) ||^2,
+ * the squared change one attention output leaves in the residual stream relative to another
+ * (O_a sparse, O_b dense in the paper's use).  O_a, O_b: device bf16 [N, H*64]; W_o as in
+ * ress_out_proj; drift: device float [ceil(N/64)].  Both products are accumulated in fp32
+ * TMEM and subtracted there; each block's sum is formed in a fixed order (deterministic).
+ * d_model must be a multiple of 64.  Uses the workspace's status word only. */
+int ress_token_drift(const ress_dims* dims, const uint16_t* O_a, const uint16_t* O_b,
+                     const uint16_t* W_o, float* drift, void* ws, size_t ws_bytes, void* stream);
+
 /* Allocation-free variant of ress_sparse_attn (the paper has no counterpart: this is an
  * interface for callers, not part of the method).  It is for callers that cannot allocate
  * device memory when they call in: a host framework that owns all device memory through

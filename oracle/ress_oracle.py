@@ -330,3 +330,25 @@ def csr_from_selection(sel: dict, H: int, nb: int):
             cols.append(k)
             row_ptr[h * nb + i + 1] = row_ptr[h * nb + i] + k.size
     return row_ptr.astype(np.int32), np.concatenate(cols).astype(np.int32)
+
+
+# ----------------------------------------------------------------------------------------
+# Sec. 3: what the attention sublayer adds to the residual stream
+# ----------------------------------------------------------------------------------------
+def residual_update(x, O, W_o):
+    """x + O W_o^T: the pre-LN residual update x_{l+1} = x_l + f_l(x_l) of the attention
+    sublayer (Sec. 3), with O [N, H d_h] the concatenated head outputs and W_o [d, H d_h] the
+    output projection as a Linear weight (out x in).  x may be None (the update alone)."""
+    y = np.asarray(O, dtype=np.float64) @ np.asarray(W_o, dtype=np.float64).T
+    return y if x is None else np.asarray(x, dtype=np.float64) + y
+
+
+def token_drift(O_a, O_b, W_o, block: int = BLOCK) -> np.ndarray:
+    """Per query block: the squared Euclidean norm, over the block's query tokens and the
+    residual dimension, of W_o (O_a - O_b), the change one attention output leaves in the
+    residual stream relative to another (Sec. 3's token-level reference, with O_a the sparse
+    and O_b the dense output).  Returns float64 [nb]."""
+    delta = residual_update(None, np.asarray(O_a, np.float64) - np.asarray(O_b, np.float64), W_o)
+    N = delta.shape[0]
+    return np.array([float((delta[i * block: min(N, (i + 1) * block)] ** 2).sum())
+                     for i in range(n_blocks(N, block))])

@@ -75,6 +75,8 @@ _SIGS = {
                                      _c.c_int32, _c.c_float, _P, _c.c_size_t, _P, _P, _c.c_int64,
                                      _P, _P]),
     "ress_status": (_c.c_int, [_P, _P]),
+    "ress_out_proj": (_c.c_int, [_c.POINTER(Dims), _P, _P, _P, _P, _P, _c.c_size_t, _P]),
+    "ress_token_drift": (_c.c_int, [_c.POINTER(Dims), _P, _P, _P, _P, _P, _c.c_size_t, _P]),
     "ress_sparse_attn_noalloc": (_c.c_int, [_c.POINTER(Dims), _P, _P, _P, _P, _P, _c.c_int64, _P,
                                             _c.c_int32, _P]),
 }
@@ -217,6 +219,22 @@ def sparse_attn(d: Dims, Q, K, V, row_ptr, col_idx, O, ws, stream=None):
                                  _dev(col_idx, (torch.int32,), "col_idx"), col_idx.numel(),
                                  _dev(O, _bf16(), "O"), _dev(ws, None, "ws"),
                                  ws.numel() * ws.element_size(), _stream(stream)))
+
+
+def out_proj(d: Dims, O, W_o, x, y, ws, stream=None):
+    """ress_out_proj: y = x + O W_o^T (x None: y = O W_o^T); bf16 tensors."""
+    _check(_lib.ress_out_proj(_c.byref(d), _dev(O, _bf16(), "O"), _dev(W_o, _bf16(), "W_o"),
+                              _dev(x, _bf16(), "x"), _dev(y, _bf16(), "y"), _dev(ws, None, "ws"),
+                              ws.numel() * ws.element_size(), _stream(stream)))
+
+
+def token_drift(d: Dims, O_a, O_b, W_o, drift, ws, stream=None):
+    """ress_token_drift: drift[b] = sum over block b's tokens of ||W_o (O_a - O_b)||^2."""
+    torch = _torch()
+    _check(_lib.ress_token_drift(_c.byref(d), _dev(O_a, _bf16(), "O_a"), _dev(O_b, _bf16(), "O_b"),
+                                 _dev(W_o, _bf16(), "W_o"), _dev(drift, (torch.float32,), "drift"),
+                                 _dev(ws, None, "ws"), ws.numel() * ws.element_size(),
+                                 _stream(stream)))
 
 
 def sparse_attn_f32(d: Dims, Q, K, V, row_ptr, col_idx, O, ws, stream=None):

@@ -19,7 +19,7 @@ CSRC = os.path.join(HERE, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 OBJDIR = os.path.join(HERE, "_build")
 LIB = os.path.join(HERE, "libress.so")
-SOURCES = ["ress_abi.cu", "k_select.cu", "k_attn.cu", "k_dot.cu", "k_yagg.cu"]
+SOURCES = ["ress_abi.cu", "k_select.cu", "k_attn.cu", "k_dot.cu", "k_yagg.cu", "k_oproj.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-Xcompiler", "-fPIC", "-Xcompiler", "-Wall",
          "--expt-relaxed-constexpr", "-I", INCLUDE, "-I", CSRC]

@@ -334,6 +334,66 @@ int ress_status(void* ws, void* stream) {
   return fail(RESS_EDEVICE, "device-side argument check failed (code %u)", word);
 }
 
+static int oproj_checks(const ress_dims* d, const void* W_o, void* ws, size_t ws_bytes,
+                        ress::Shape* s, ress_ws_layout* L) {
+  int e = check_dims(d);
+  if (e) return e;
+  if ((e = check_ptr(W_o, 16, "W_o"))) return e;
+  if (d->d_model % 64 != 0)
+    return fail(RESS_EUNSUPPORTED, "d_model %d must be a multiple of 64", d->d_model);
+  *s = ress::make_shape(*d);
+  return check_ws(*s, ws, ws_bytes, L);
+}
+
+int ress_out_proj(const ress_dims* d, const uint16_t* O, const uint16_t* W_o, const uint16_t* x,
+                  uint16_t* y, void* ws, size_t ws_bytes, void* stream) {
+  ress::Shape s{};
+  ress_ws_layout L{};
+  int e = oproj_checks(d, W_o, ws, ws_bytes, &s, &L);
+  if (e) return e;
+  if ((e = check_ptr(O, 16, "O")) || (e = check_ptr(y, 16, "y"))) return e;
+  if (x && (e = check_ptr(x, 16, "x"))) return e;
+  ress::OProjArgs a;
+  a.N = s.N;
+  a.H = s.H;
+  a.Dm = d->d_model;
+  a.O = O;
+  a.O2 = nullptr;
+  a.W_o = W_o;
+  a.x = x;
+  a.y = y;
+  a.drift = nullptr;
+  a.status = reinterpret_cast<uint32_t*>(static_cast<char*>(ws) + L.status);
+  cudaError_t ce = ress::launch_out_proj(a, static_cast<cudaStream_t>(stream));
+  if (ce != cudaSuccess) return cuda_fail(ce, "ress_out_proj");
+  return ok();
+}
+
+int ress_token_drift(const ress_dims* d, const uint16_t* O_a, const uint16_t* O_b,
+                     const uint16_t* W_o, float* drift, void* ws, size_t ws_bytes, void* stream) {
+  ress::Shape s{};
+  ress_ws_layout L{};
+  int e = oproj_checks(d, W_o, ws, ws_bytes, &s, &L);
+  if (e) return e;
+  if ((e = check_ptr(O_a, 16, "O_a")) || (e = check_ptr(O_b, 16, "O_b")) ||
+      (e = check_ptr(drift, 4, "drift")))
+    return e;
+  ress::OProjArgs a;
+  a.N = s.N;
+  a.H = s.H;
+  a.Dm = d->d_model;
+  a.O = O_a;
+  a.O2 = O_b;
+  a.W_o = W_o;
+  a.x = nullptr;
+  a.y = nullptr;
+  a.drift = drift;
+  a.status = reinterpret_cast<uint32_t*>(static_cast<char*>(ws) + L.status);
+  cudaError_t ce = ress::launch_token_drift(a, static_cast<cudaStream_t>(stream));
+  if (ce != cudaSuccess) return cuda_fail(ce, "ress_token_drift");
+  return ok();
+}
+
 }  // extern "C"
 
 // ---------------------------------------------------------------------------------------

@@ -178,4 +178,14 @@ struct AttnArgs {
 };
 cudaError_t launch_sparse_attn(const AttnArgs& a, cudaStream_t st);
 
+struct OProjArgs {
+  int N, H, Dm;                      // tokens, heads (K = 64 H), d_model
+  const uint16_t *O, *O2, *W_o, *x;  // O2: the second output (token drift)
+  uint16_t* y;
+  float* drift;
+  uint32_t* status;
+};
+cudaError_t launch_out_proj(const OProjArgs& a, cudaStream_t st);
+cudaError_t launch_token_drift(const OProjArgs& a, cudaStream_t st);
+
 }  // namespace ress

@@ -387,3 +387,60 @@ def test_kernel_launch_counter():
               b.row_ptr, b.col_idx, b.O, b.J_best)
     torch.cuda.synchronize()
     assert r.kernel_launches() - n0 == 6 + 2 * layer.rounds + 1 + 2
+
+
+def _bf16_tensor(a):
+    """float array -> (device bf16 tensor, the float64 values it holds)."""
+    t = torch.from_numpy(np.ascontiguousarray(a, dtype=np.float32)).to(torch.bfloat16)
+    return t.cuda(), t.float().numpy().astype(np.float64)
+
+
+@pytest.mark.parametrize("fixture", ["tiny", "v8"])
+def test_out_proj_residual_update(fixture, request):
+    """y = x + O W_o^T (Sec. 3) on the tensor cores against float64 on the same bf16 inputs:
+    the attention output of the layer, a random residual x; also x = NULL and in place."""
+    layer = request.getfixturevalue(fixture)
+    N, Dm = layer.N, layer.d_model
+    rng = np.random.default_rng(11)
+    x, xf = _bf16_tensor(rng.normal(size=(N, Dm)))
+    Of = layer.buf.O.float().cpu().numpy().reshape(N, -1).astype(np.float64)
+    Wf = layer.W_o()
+    ref = O.residual_update(xf, Of, Wf)
+    scale = np.abs(Of) @ np.abs(Wf).T + np.abs(xf)  # bound of the accumulated magnitudes
+    y = torch.empty(N, Dm, dtype=torch.bfloat16, device="cuda")
+    layer.ress.out_proj(layer.d, layer.buf.O, layer.W, x, y, layer.buf.ws)
+    layer.ress.status(layer.buf.ws)
+    got = y.float().cpu().numpy()
+    assert np.all(np.abs(got - ref) <= 2.0 ** -8 * np.abs(ref) + 1e-5 * scale + 1e-6)
+    y0 = torch.empty_like(y)
+    layer.ress.out_proj(layer.d, layer.buf.O, layer.W, None, y0, layer.buf.ws)
+    ref0 = O.residual_update(None, Of, Wf)
+    assert np.all(np.abs(y0.float().cpu().numpy() - ref0) <= 2.0 ** -8 * np.abs(ref0) + 1e-5 * scale + 1e-6)
+    xi = x.clone()
+    layer.ress.out_proj(layer.d, layer.buf.O, layer.W, xi, xi, layer.buf.ws)  # in place
+    torch.cuda.synchronize()
+    assert torch.equal(xi.view(torch.int16), y.view(torch.int16))
+
+
+@pytest.mark.parametrize("fixture", ["tiny", "v8"])
+def test_token_drift_sparse_vs_dense(fixture, request):
+    """Sec. 3's token-level drift per query block, ||W_o (O_sparse - O_dense)||^2 over the
+    block's tokens, on the tensor cores against float64 on the same bf16 outputs."""
+    layer = request.getfixturevalue(fixture)
+    H, nb, N = layer.H, layer.nb, layer.N
+    rp = torch.arange(0, H * nb * nb + 1, nb, dtype=torch.int32, device="cuda")
+    ci = torch.arange(nb, dtype=torch.int32, device="cuda").repeat(H * nb)
+    O_dense = torch.empty_like(layer.buf.O)
+    layer.ress.sparse_attn(layer.d, layer.Q, layer.K, layer.V, rp, ci, O_dense, layer.buf.ws)
+    drift = torch.empty(nb, dtype=torch.float32, device="cuda")
+    layer.ress.token_drift(layer.d, layer.buf.O, O_dense, layer.W, drift, layer.buf.ws)
+    layer.ress.status(layer.buf.ws)
+    got = drift.cpu().numpy().astype(np.float64)
+    Oa = layer.buf.O.float().cpu().numpy().reshape(N, -1)
+    Ob = O_dense.float().cpu().numpy().reshape(N, -1)
+    ref = O.token_drift(Oa, Ob, layer.W_o())
+    ya, yb = (O.residual_update(None, o, layer.W_o()) for o in (Oa, Ob))
+    mag = np.array([float((ya[64 * b: 64 * (b + 1)] ** 2).sum() + (yb[64 * b: 64 * (b + 1)] ** 2).sum())
+                    for b in range(nb)])
+    assert np.all(np.abs(got - ref) <= 1e-4 * ref + 1e-6 * mag + 1e-12), np.max(np.abs(got - ref) / (ref + 1e-30))
+    assert np.all(got[layer.ncand:] <= 1e-6 * mag[layer.ncand:] + 1e-12)  # special rows are dense

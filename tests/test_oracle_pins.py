@@ -354,3 +354,50 @@ def test_csr_layout(layer):
     lens = np.diff(rp).reshape(2, pooled.nb)
     assert (lens[0, :pooled.n_cand] == 3 + ns).all() and (lens[1, :pooled.n_cand] == 8 + ns).all()
     assert (lens[:, pooled.n_cand:] == pooled.nb).all()
+
+
+# ---------------------------------------------------------------------------------------
+# Sec. 3: residual update and token-level drift
+# ---------------------------------------------------------------------------------------
+def test_residual_update_elementwise_by_loops():
+    """y[t, o] = x[t, o] + sum_k O[t, k] W_o[o, k], written out with loops on a small case
+    whose W_o is not symmetric (a transposed operand fails it)."""
+    rng = np.random.default_rng(7)
+    N, d = 5, 6
+    x, Ob, W = rng.normal(size=(N, d)), rng.normal(size=(N, d)), rng.normal(size=(d, d))
+    y = O.residual_update(x, Ob, W)
+    for t in range(N):
+        for o in range(d):
+            acc = x[t, o]
+            for k in range(d):
+                acc += Ob[t, k] * W[o, k]
+            assert y[t, o] == pytest.approx(acc, rel=1e-13, abs=1e-13)
+    assert np.allclose(O.residual_update(None, Ob, W), y - x, rtol=0, atol=1e-13)
+
+
+def test_residual_update_is_the_output_projection_linear():
+    """The update equals F.linear with W_o as the Linear weight (out x in), and with an
+    identity W_o it is x + O."""
+    rng = np.random.default_rng(8)
+    x, Ob = rng.normal(size=(9, 16)), rng.normal(size=(9, 16))
+    W = rng.normal(size=(16, 16))
+    ref = torch.from_numpy(x) + F.linear(torch.from_numpy(Ob), torch.from_numpy(W))
+    assert np.allclose(O.residual_update(x, Ob, W), ref.numpy(), rtol=1e-12, atol=1e-12)
+    assert np.allclose(O.residual_update(x, Ob, np.eye(16)), x + Ob, rtol=0, atol=1e-14)
+
+
+def test_token_drift_definition_and_invariants(layer):
+    """Token drift per block: zero for identical outputs, the squared norm of the difference
+    of the two residual updates, scaling by alpha^2 with W_o, blocks summing to the whole."""
+    rng = np.random.default_rng(9)
+    N, d = 200, 32
+    Oa, Ob, W = rng.normal(size=(N, d)), rng.normal(size=(N, d)), rng.normal(size=(d, d))
+    dr = O.token_drift(Oa, Ob, W, block=64)
+    assert dr.shape == (4,)
+    assert np.all(O.token_drift(Oa, Oa, W, block=64) == 0)
+    ya, yb = O.residual_update(None, Oa, W), O.residual_update(None, Ob, W)
+    for b in range(4):
+        sl = slice(64 * b, min(N, 64 * (b + 1)))
+        assert dr[b] == pytest.approx(float(np.linalg.norm(ya[sl] - yb[sl]) ** 2), rel=1e-12)
+    assert np.allclose(O.token_drift(Oa, Ob, 3.0 * W, block=64), 9.0 * dr, rtol=1e-12)
+    assert dr.sum() == pytest.approx(float(((ya - yb) ** 2).sum()), rel=1e-12)
