@@ -423,8 +423,44 @@ def run_ours(a, wl):
         dfl = kept_flops(rpd.cpu().numpy(), cid.cpu().numpy(), N, H, nb)
         dense = {"attn_ms": dms, "tflops": dfl / dms / 1e9, "frac_of_bf16_peak": dfl / dms / 1e9 / bf16,
                  "speedup_of_sparse_layer": dms / ms}
+        # token-level drift of the sparse output against the dense one (Sec. 3's reference)
+        drift = torch.empty(nb, dtype=torch.float32, device="cuda")
+        ress.token_drift(d, buf.O, Od, W, drift, buf.ws)
+        e0.record(stream)
+        for _ in range(nd):
+            ress.token_drift(d, buf.O, Od, W, drift, buf.ws)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        tms = e0.elapsed_time(e1) / nd
+        tdr = drift.cpu().numpy().astype(np.float64)
+        ncb = ress.num_candidates(d)
+        dense["token_drift"] = {"sum_candidate_blocks": float(tdr[:ncb].sum()),
+                                "sum_all_blocks": float(tdr.sum()), "ms": tms,
+                                "tflops": 2 * 2.0 * N * d.d_model * H * 64 / tms / 1e9}
         ress.status(buf.ws)
         del Od, rpd, cid
+
+    # ---- the sublayer's residual update y = x + O W_o^T (tensor-core GEMM) ----------
+    xres = torch.randn(N, d.d_model, dtype=torch.bfloat16, device="cuda",
+                       generator=torch.Generator(device="cuda").manual_seed(0))
+    yres = torch.empty_like(xres)
+    for _ in range(3):
+        ress.out_proj(d, buf.O, W, xres, yres, buf.ws)
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    no = 20
+    e0.record(stream)
+    for _ in range(no):
+        ress.out_proj(d, buf.O, W, xres, yres, buf.ws)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    oms = e0.elapsed_time(e1) / no
+    ofl = 2.0 * N * d.d_model * H * 64
+    obytes = 2.0 * (N * H * 64 + d.d_model * H * 64 + 2 * N * d.d_model)
+    out_proj = {"ms": oms, "tflops": ofl / oms / 1e9, "frac_of_bf16_peak": ofl / oms / 1e9 / bf16,
+                "gbs": obytes / oms / 1e6, "flop": ofl, "bytes": obytes}
+    ress.status(buf.ws)
+    del xres, yres
 
     # ---- end to end through the public API with host buffers -------------------------
     # ress_forward_host per step: the copies of the step's Q, K, V in, the forward, the copy
@@ -501,6 +537,7 @@ def run_ours(a, wl):
         "kept_tflop": flops / 1e12, "realized_pair_sparsity": 1.0 - kept_pairs / (H * nb * nb),
         "drift": {"sum_J_best": float(Jb[cand_rows].sum()), "sum_J0": float(J0[cand_rows].sum())},
         "dense": dense,
+        "out_proj": out_proj,
         "roofline": {"bound": "tensor", "kernel": "k_attn (ress_sparse_attn)",
                      "achieved": flops / attn_ms / 1e9, "peak": bf16, "unit": "TFLOP/s",
                      "frac": flops / attn_ms / 1e9 / bf16,
