@@ -190,12 +190,60 @@ class RowSelection:
         return np.nonzero(~self.D_best)[0].astype(np.int32)
 
 
+@dataclass(frozen=True)
+class Variant:
+    """Selection variants of the paper's ablations (Sec. 6: Fig. 8's sign flip, Table 3's
+    probability selection; the random baseline of Fig. 8).
+
+    key:      "drift" (Eq. 7, ReSS), "probability" (the pooled P_ij alone: top-k by attention
+              mass, the rule of the probability-based methods) or "random" (SplitMix64 of a
+              counter, see random_keys).
+    maximize: "none" (ReSS minimises the drift), "swap" (restoration maximises J, the initial
+              selection is unchanged) or "full" (the initial selection keeps the c_h smallest
+              keys and restoration maximises J).
+    """
+    key: str = "drift"
+    maximize: str = "none"
+    seed: int = 0
+
+
+RESS = Variant()
+_MASK64 = (1 << 64) - 1
+
+
+def splitmix64(x: int) -> int:
+    """SplitMix64 (Steele, Lea and Flood, OOPSLA 2014): the state advanced by the golden-ratio
+    increment, then the variant-13 mix of that paper.  Returns the output for state x."""
+    z = (x + 0x9E3779B97F4A7C15) & _MASK64
+    z = ((z ^ (z >> 30)) * 0xBF58476D1CE4E5B9) & _MASK64
+    z = ((z ^ (z >> 27)) * 0x94D049BB133111EB) & _MASK64
+    return z ^ (z >> 31)
+
+
+def random_keys(seed: int, h: int, i: int, nb: int) -> np.ndarray:
+    """Random selection keys of row (h, i): the top 24 bits of SplitMix64 at the counter
+    seed + ((h * 4096 + i) * 4096 + j) for block j (exact integers, so the GPU's order,
+    ties to the lower index, is the same)."""
+    base = (seed + (h * 4096 + i) * 4096) & _MASK64
+    return np.array([float(splitmix64((base + j) & _MASK64) >> 40) for j in range(nb)])
+
+
 def select_row(P_i, vbar_i, Vb_h, WOh, n_cand: int, c: int, rounds: int, rho: float,
-               h: int = 0, i: int = 0) -> RowSelection:
+               h: int = 0, i: int = 0, variant: Variant = RESS) -> RowSelection:
     """Initial selection (Eq. 7) and R restoration rounds (Eq. 13-17) for one row."""
     nb = P_i.size
     _, _, r = residual_contributions(P_i, vbar_i, Vb_h, WOh)
-    key = cut_keys(drift_scores(r), P_i)
+    if variant.key == "drift":
+        key = cut_keys(drift_scores(r), P_i)
+    elif variant.key == "probability":
+        key = np.array(P_i, dtype=np.float64)
+    elif variant.key == "random":
+        key = random_keys(variant.seed, h, i, nb)
+    else:
+        raise ValueError(variant.key)
+    if variant.maximize == "full":  # keep the smallest keys: drop the largest drifts
+        key = -key
+    sign = -1.0 if variant.maximize in ("swap", "full") else 1.0  # restoration direction
 
     # initial selection: keep the c_h candidates with the largest key, drop the rest
     keep = top_m(key[:n_cand], c)
@@ -213,6 +261,7 @@ def select_row(P_i, vbar_i, Vb_h, WOh, n_cand: int, c: int, rounds: int, rho: fl
             res.J_trace.append(J)
             continue
         floor = 1e-30 * J
+        gain_res, gain_drop = sign * gain_res, sign * gain_drop
         res.margin = min(res.margin, _gap(ranked(gain_res), m, floor),
                          _gap(ranked(gain_drop), m, floor))
         restore = inD[top_m(gain_res, m)]
@@ -224,7 +273,7 @@ def select_row(P_i, vbar_i, Vb_h, WOh, n_cand: int, c: int, rounds: int, rho: fl
         res.J_trace.append(J)
         if res.J_best > 0:
             res.margin = min(res.margin, abs(J - res.J_best) / res.J_best)
-        if J < res.J_best:
+        if (J < res.J_best) if sign > 0 else (J > res.J_best):
             res.J_best = J
             res.D_best = D.copy()
     return res
@@ -268,8 +317,10 @@ def row_quantities(pooled: Pooled, h: int, i: int):
     return P_i, dense_pooled_output(P_i, pooled.Vb[h])
 
 
-def ress_select(pooled: Pooled, W_o, c_h, rounds: int, rho: float = 0.5, rows=None):
-    """ReSS selection for every (h, i) row, or for the given list of rows.
+def ress_select(pooled: Pooled, W_o, c_h, rounds: int, rho: float = 0.5, rows=None,
+                variant: Variant = RESS):
+    """ReSS selection (or one of its ablation variants) for every (h, i) row, or for the
+    given list of rows.
 
     Returns {(h, i): RowSelection}.
     """
@@ -284,7 +335,7 @@ def ress_select(pooled: Pooled, W_o, c_h, rounds: int, rho: float = 0.5, rows=No
             continue
         P_i, vbar_i = row_quantities(pooled, h, i)
         out[(h, i)] = select_row(P_i, vbar_i, pooled.Vb[h], head_projection(W_o, h, d_h),
-                                 n_cand, int(c_h[h]), rounds, rho, h, i)
+                                 n_cand, int(c_h[h]), rounds, rho, h, i, variant)
     return out
 
 

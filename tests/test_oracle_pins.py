@@ -401,3 +401,72 @@ def test_token_drift_definition_and_invariants(layer):
         assert dr[b] == pytest.approx(float(np.linalg.norm(ya[sl] - yb[sl]) ** 2), rel=1e-12)
     assert np.allclose(O.token_drift(Oa, Ob, 3.0 * W, block=64), 9.0 * dr, rtol=1e-12)
     assert dr.sum() == pytest.approx(float(((ya - yb) ** 2).sum()), rel=1e-12)
+
+
+# ---------------------------------------------------------------------------------------
+# Ablation variants (Sec. 6): probability keys, random keys, maximised drift
+# ---------------------------------------------------------------------------------------
+def test_splitmix64_reference_outputs():
+    """The counter-based generator behind the random variant reproduces SplitMix64's
+    published outputs for seed 0 (tests/golden/splitmix64_seed0.txt)."""
+    import pathlib
+    path = pathlib.Path(__file__).with_name("golden") / "splitmix64_seed0.txt"
+    want = [int(l, 16) for l in path.read_text().splitlines() if l.startswith("0x")]
+    state, got = 0, []
+    for _ in want:
+        got.append(O.splitmix64(state))
+        state = (state + 0x9E3779B97F4A7C15) & ((1 << 64) - 1)
+    assert got == want
+
+
+def _variant_rows(layer, variant, rounds=3):
+    X, pooled = layer
+    H, nb = pooled.heads, pooled.nb
+    c = [max(2, pooled.n_cand // 4)] * H
+    rows = [(h, i) for h in range(H) for i in range(0, pooled.n_cand, 3)]
+    return pooled, c, O.ress_select(pooled, X["W_o"], c, rounds, 0.5, rows=rows, variant=variant)
+
+
+def test_probability_variant_is_top_k_by_pooled_mass(layer):
+    """key = P_ij with no rounds keeps exactly the c_h candidates of largest pooled
+    probability (ties to the lower index), found here by a stable argsort."""
+    pooled, c, sel = _variant_rows(layer, O.Variant(key="probability"), rounds=0)
+    for (h, i), s in sel.items():
+        P_i, _ = O.row_quantities(pooled, h, i)
+        order = np.argsort(-P_i[:pooled.n_cand], kind="stable")[:c[h]]
+        assert set(np.nonzero(~s.D_best[:pooled.n_cand])[0]) == set(order)
+
+
+def test_random_variant_keys(layer):
+    """Random keys: the same seed gives the same sets, another seed other sets, and every
+    row keeps exactly c_h candidates."""
+    pooled, c, a = _variant_rows(layer, O.Variant(key="random", seed=5), rounds=0)
+    _, _, b = _variant_rows(layer, O.Variant(key="random", seed=5), rounds=0)
+    _, _, o = _variant_rows(layer, O.Variant(key="random", seed=6), rounds=0)
+    assert all(np.array_equal(a[k].D_best, b[k].D_best) for k in a)
+    assert any(not np.array_equal(a[k].D_best, o[k].D_best) for k in a)
+    for (h, i), s in a.items():
+        assert (~s.D_best).sum() == c[h] + (pooled.nb - pooled.n_cand)
+
+
+def test_maximised_drift_variants(layer):
+    """Flipping the sign (Fig. 8): "swap" keeps ReSS's initial set and its rounds never
+    lower the best J below J0; "full" keeps the smallest Eq. 7 keys; the best J is the
+    largest J seen, and it does not decrease with more rounds."""
+    pooled, c, ress = _variant_rows(layer, O.RESS)
+    _, _, swap = _variant_rows(layer, O.Variant(maximize="swap"))
+    _, _, full = _variant_rows(layer, O.Variant(maximize="full"))
+    _, _, full2 = _variant_rows(layer, O.Variant(maximize="full"), rounds=2)
+    for k in ress:
+        assert np.array_equal(swap[k].D0, ress[k].D0)
+        for v in (swap[k], full[k]):
+            assert v.J_best >= v.J0
+            assert v.J_best == max([v.J0] + v.J_trace)
+        assert full[k].J_best >= full2[k].J_best
+        h, i = k
+        P_i, vbar_i = O.row_quantities(pooled, h, i)
+        _, _, r = O.residual_contributions(P_i, vbar_i, pooled.Vb[h],
+                                           O.head_projection(layer[0]["W_o"], h, 64))
+        key = O.cut_keys(O.drift_scores(r), P_i)[:pooled.n_cand]
+        smallest = set(np.argsort(key, kind="stable")[:c[h]])
+        assert set(np.nonzero(~full[k].D0[:pooled.n_cand])[0]) == smallest
