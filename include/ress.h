@@ -131,6 +131,28 @@ int ress_score(const ress_dims* dims, const uint16_t* Q, const uint16_t* K, cons
                const float* F, const int32_t* c_h_host, void* ws, size_t ws_bytes,
                void* stream);
 
+/* Selection variants of the paper's ablations (Sec. 6: the sign flip of Fig. 8 and the
+ * probability selection of Table 3; the random baseline of Fig. 8).  `key` picks what the
+ * initial selection ranks: the Eq. 7 drift key (ReSS), the pooled probability P_ij alone
+ * (top-k by attention mass) or random keys (the top 24 bits of SplitMix64 at the counter
+ * seed + (h * 4096 + i) * 4096 + j for row (h, i) and block j; ties to the lower index).
+ * `direction` flips the objective: RESS_MAXIMIZE_SWAP makes the restoration rounds maximise
+ * J (track-best keeps the largest J), RESS_MAXIMIZE_FULL also makes the initial selection
+ * keep the c_h smallest keys.  A NULL variant is ReSS: {RESS_KEY_DRIFT, RESS_MINIMIZE, 0}. */
+typedef enum { RESS_KEY_DRIFT = 0, RESS_KEY_PROBABILITY = 1, RESS_KEY_RANDOM = 2 } ress_key_kind;
+typedef enum { RESS_MINIMIZE = 0, RESS_MAXIMIZE_SWAP = 1, RESS_MAXIMIZE_FULL = 2 } ress_direction;
+typedef struct {
+  int32_t key;       /* ress_key_kind  */
+  int32_t direction; /* ress_direction */
+  uint64_t seed;     /* RESS_KEY_RANDOM */
+} ress_variant;
+
+/* ress_score with a selection variant (NULL: ReSS).  RESS_EINVAL on an unknown key or
+ * direction. */
+int ress_score_variant(const ress_dims* dims, const uint16_t* Q, const uint16_t* K,
+                       const uint16_t* V, const float* F, const int32_t* c_h_host,
+                       const ress_variant* variant, void* ws, size_t ws_bytes, void* stream);
+
 /* Sec. 4.3: `rounds` budget-neutral swap rounds on the drop sets left by ress_score.
  * Round r exchanges m_r = floor(rho c_h / 2^(r+1)) blocks (Eq. 17), capped by the sizes of
  * the two sides: the m_r restores and the m_r drops with the largest exact decrease of
@@ -144,6 +166,13 @@ int ress_score(const ress_dims* dims, const uint16_t* Q, const uint16_t* K, cons
 int ress_restore(const ress_dims* dims, const int32_t* c_h_host, int32_t rounds, float rho,
                  void* ws, size_t ws_bytes, int32_t* row_ptr, int32_t* col_idx,
                  int64_t col_capacity, float* J_best, uint32_t* drop_mask, void* stream);
+
+/* ress_restore with a selection variant (NULL: ReSS); pass the same variant as to
+ * ress_score_variant.  RESS_EINVAL on an unknown key or direction. */
+int ress_restore_variant(const ress_dims* dims, const int32_t* c_h_host, int32_t rounds,
+                         float rho, const ress_variant* variant, void* ws, size_t ws_bytes,
+                         int32_t* row_ptr, int32_t* col_idx, int64_t col_capacity,
+                         float* J_best, uint32_t* drop_mask, void* stream);
 
 /* Sec. 3 step (3): for every head h, query block i and query token of that block,
  * O = softmax(q K^T / 8) V over the tokens of the key blocks listed in row h*nb + i of the

@@ -42,6 +42,22 @@ class Dims(ctypes.Structure):
                 ("n_special", ctypes.c_int32), ("d_model", ctypes.c_int32)]
 
 
+class Variant(ctypes.Structure):
+    """ress_variant: selection variant of the ablations (key: 0 drift, 1 probability,
+    2 random; direction: 0 minimise, 1 restoration maximises, 2 everything maximises)."""
+    _fields_ = [("key", ctypes.c_int32), ("direction", ctypes.c_int32), ("seed", ctypes.c_uint64)]
+
+
+_KEYS = {"drift": 0, "probability": 1, "random": 2}
+_DIRECTIONS = {"none": 0, "swap": 1, "full": 2}
+
+
+def variant(key: str = "drift", maximize: str = "none", seed: int = 0) -> Variant:
+    """A ress_variant from names: key in {drift, probability, random}, maximize in
+    {none, swap, full}."""
+    return Variant(_KEYS[key], _DIRECTIONS[maximize], seed)
+
+
 class WsLayout(ctypes.Structure):
     """ress_ws_layout: byte offsets of the workspace arrays."""
     _fields_ = [(n, ctypes.c_int64) for n in
@@ -75,6 +91,11 @@ _SIGS = {
                                      _c.c_int32, _c.c_float, _P, _c.c_size_t, _P, _P, _c.c_int64,
                                      _P, _P]),
     "ress_status": (_c.c_int, [_P, _P]),
+    "ress_score_variant": (_c.c_int, [_c.POINTER(Dims), _P, _P, _P, _P, _P, _c.POINTER(Variant), _P,
+                                      _c.c_size_t, _P]),
+    "ress_restore_variant": (_c.c_int, [_c.POINTER(Dims), _P, _c.c_int32, _c.c_float,
+                                        _c.POINTER(Variant), _P, _c.c_size_t, _P, _P, _c.c_int64,
+                                        _P, _P, _P]),
     "ress_out_proj": (_c.c_int, [_c.POINTER(Dims), _P, _P, _P, _P, _P, _c.c_size_t, _P]),
     "ress_token_drift": (_c.c_int, [_c.POINTER(Dims), _P, _P, _P, _P, _P, _c.c_size_t, _P]),
     "ress_sparse_attn_noalloc": (_c.c_int, [_c.POINTER(Dims), _P, _P, _P, _P, _P, _c.c_int64, _P,
@@ -192,24 +213,31 @@ def prepare_wo(d: Dims, W_o, F, stream=None):
                                 _stream(stream)))
 
 
-def score(d: Dims, Q, K, V, F, c_h, ws, stream=None):
+def score(d: Dims, Q, K, V, F, c_h, ws, stream=None, variant: Variant = None):
+    """ress_score, or ress_score_variant when a Variant is given."""
     torch = _torch()
-    _check(_lib.ress_score(_c.byref(d), _dev(Q, _bf16(), "Q"), _dev(K, _bf16(), "K"),
-                           _dev(V, _bf16(), "V"), _dev(F, (torch.float32,), "F"),
-                           _c.cast(_budget_array(c_h), _P), _dev(ws, None, "ws"),
-                           ws.numel() * ws.element_size(), _stream(stream)))
+    args = (_dev(Q, _bf16(), "Q"), _dev(K, _bf16(), "K"), _dev(V, _bf16(), "V"),
+            _dev(F, (torch.float32,), "F"), _c.cast(_budget_array(c_h), _P))
+    tail = (_dev(ws, None, "ws"), ws.numel() * ws.element_size(), _stream(stream))
+    if variant is None:
+        _check(_lib.ress_score(_c.byref(d), *args, *tail))
+    else:
+        _check(_lib.ress_score_variant(_c.byref(d), *args, _c.byref(variant), *tail))
 
 
 def restore(d: Dims, c_h, rounds: int, rho: float, ws, row_ptr, col_idx, J_best=None,
-            drop_mask=None, stream=None):
+            drop_mask=None, stream=None, variant: Variant = None):
+    """ress_restore, or ress_restore_variant when a Variant is given."""
     torch = _torch()
-    _check(_lib.ress_restore(_c.byref(d), _c.cast(_budget_array(c_h), _P), int(rounds), float(rho),
-                             _dev(ws, None, "ws"), ws.numel() * ws.element_size(),
-                             _dev(row_ptr, (torch.int32,), "row_ptr"),
-                             _dev(col_idx, (torch.int32,), "col_idx"), col_idx.numel(),
-                             _dev(J_best, (torch.float32,), "J_best"),
-                             _dev(drop_mask, (torch.int32, torch.uint32), "drop_mask"),
-                             _stream(stream)))
+    head = (_c.cast(_budget_array(c_h), _P), int(rounds), float(rho))
+    tail = (_dev(ws, None, "ws"), ws.numel() * ws.element_size(),
+            _dev(row_ptr, (torch.int32,), "row_ptr"), _dev(col_idx, (torch.int32,), "col_idx"),
+            col_idx.numel(), _dev(J_best, (torch.float32,), "J_best"),
+            _dev(drop_mask, (torch.int32, torch.uint32), "drop_mask"), _stream(stream))
+    if variant is None:
+        _check(_lib.ress_restore(_c.byref(d), *head, *tail))
+    else:
+        _check(_lib.ress_restore_variant(_c.byref(d), *head, _c.byref(variant), *tail))
 
 
 def sparse_attn(d: Dims, Q, K, V, row_ptr, col_idx, O, ws, stream=None):

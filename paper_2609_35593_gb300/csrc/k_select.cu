@@ -631,8 +631,21 @@ __device__ __forceinline__ void row_keys(int n, uint32_t* kk, KeyFn key_of) {
   __syncwarp();
 }
 
+// SplitMix64 (Steele, Lea and Flood, OOPSLA 2014) at state x: advance by the golden-ratio
+// increment, then that paper's mix.  The random selection keys of the ablation variant.
+__device__ __forceinline__ unsigned long long splitmix64(unsigned long long x) {
+  unsigned long long z = x + 0x9E3779B97F4A7C15ull;
+  z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+  z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+  return z ^ (z >> 31);
+}
+
 // Initial selection (Eq. 7) and the state of Eq. 10-12.  grid (ceil(|P| / 4), H).
-__global__ void __launch_bounds__(32 * kRowWarps, 8) k_score_rows(SelPtrs p, Budgets bud) {
+// The variant picks the key: the Eq. 7 drift key (ReSS), the pooled probability, or the top
+// 24 bits of SplitMix64 at seed + (h 4096 + i) 4096 + j; the full sign flip keeps the
+// smallest keys (complemented keys, ties still to the lower index).
+__global__ void __launch_bounds__(32 * kRowWarps, 8) k_score_rows(SelPtrs p, Budgets bud,
+                                                                  Variant v) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int h = blockIdx.y, i = blockIdx.x * kRowWarps + warp;
@@ -651,8 +664,17 @@ __global__ void __launch_bounds__(32 * kRowWarps, 8) k_score_rows(SelPtrs p, Bud
     const float4 q4 = *reinterpret_cast<const float4*>(qrow + j);
     const float pv[4] = {P4.x, P4.y, P4.z, P4.w}, qv[4] = {q4.x, q4.y, q4.z, q4.w};
 #pragma unroll
-    for (int u = 0; u < 4; ++u)  // s_ij / max(1 - P_ij, eps), s_ij = P_ij sqrt(q_ij)
-      k4[u] = order_key(pv[u] * sqrtf(qv[u]) / fmaxf(1.0f - pv[u], kEps));
+    for (int u = 0; u < 4; ++u) {
+      uint32_t key;
+      if (v.key == 0)  // s_ij / max(1 - P_ij, eps), s_ij = P_ij sqrt(q_ij)
+        key = order_key(pv[u] * sqrtf(qv[u]) / fmaxf(1.0f - pv[u], kEps));
+      else if (v.key == 1)
+        key = order_key(pv[u]);
+      else
+        key = (uint32_t)(splitmix64(v.seed + ((unsigned long long)h * 4096ull + (unsigned long long)i) *
+                                                 4096ull + (unsigned long long)(j + u)) >> 40) + 1u;
+      k4[u] = (v.direction == 2) ? ~key : key;
+    }
   });
   warp_topm(kk, p.ncand, bud.c[h], sel, p.words, sk, si);  // sel = kept candidates
   // drop set D0 = candidates not kept
@@ -684,9 +706,11 @@ __global__ void __launch_bounds__(32 * kRowWarps, 8) k_score_rows(SelPtrs p, Bud
 // come from k_dot (tensor cores, k_dot.cu); the rest of the round runs per row here.
 // ------------------------------------------------------------------------------------
 // Restoration round r, per row: exact top-m restores and drops from the round-start state,
-// update, track-best.  grid (ceil(|P| / 4), H).
+// update, track-best.  grid (ceil(|P| / 4), H).  With a maximising variant the keys are the
+// increases of J and track-best keeps the largest J.
 __global__ void __launch_bounds__(32 * kRowWarps, 8) k_round_rows(SelPtrs p, Budgets bud,
-                                                                  int round, float rho) {
+                                                                  int round, float rho,
+                                                                  int maximize) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int h = blockIdx.y, i = blockIdx.x * kRowWarps + warp;
@@ -723,7 +747,8 @@ __global__ void __launch_bounds__(32 * kRowWarps, 8) k_round_rows(SelPtrs p, Bud
       const bool inD = (dword >> u) & 1u;
       const float s2 = pv[u] * pv[u] * qv[u];
       const float dG = inD ? fmaf(-2.0f * pv[u], tv[u], s2) : fmaf(2.0f * pv[u], tv[u], s2);
-      k4[u] = order_key(delta_J(G, K, dG, inD ? pv[u] : -pv[u]));
+      const float dJ = delta_J(G, K, dG, inD ? pv[u] : -pv[u]);
+      k4[u] = order_key(maximize ? -dJ : dJ);
       if (j + u < p.ncand) top.add(k4[u], inD);
     }
   });
@@ -743,7 +768,7 @@ __global__ void __launch_bounds__(32 * kRowWarps, 8) k_round_rows(SelPtrs p, Bud
   const float Gn = warp_sum(g0 * g0 + g1 * g1);
   const float Kc = fmaxf(Kn, kEps);
   const float Jn = Gn / (Kc * Kc);
-  const bool better = Jn < p.Jbest[ri];
+  const bool better = maximize ? (Jn > p.Jbest[ri]) : (Jn < p.Jbest[ri]);
   for (int w = lane; w < p.words; w += 32) {
     p.dmask[ri * p.words + w] = Dw[w];
     if (better) p.bmask[ri * p.words + w] = Dw[w];
@@ -842,7 +867,7 @@ cudaError_t launch_score(const SelectArgs& a, cudaStream_t st) {
   e = cudaFuncSetAttribute(k_score_rows, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)rsmem);
   if (e != cudaSuccess) return e;
   k_score_rows<<<dim3((s.ncand + kRowWarps - 1) / kRowWarps, s.H), 32 * kRowWarps, rsmem, st>>>(
-      p, budgets_of(a));
+      p, budgets_of(a), a.v);
   note_launch();
   return cudaGetLastError();
 }
@@ -857,7 +882,7 @@ cudaError_t launch_round(const SelectArgs& a, int round, float rho, cudaStream_t
   e = cudaFuncSetAttribute(k_round_rows, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)rsmem);
   if (e != cudaSuccess) return e;
   k_round_rows<<<dim3((s.ncand + kRowWarps - 1) / kRowWarps, s.H), 32 * kRowWarps, rsmem, st>>>(
-      p, budgets_of(a), round, rho);
+      p, budgets_of(a), round, rho, a.v.direction != 0 ? 1 : 0);
   note_launch();
   return cudaGetLastError();
 }

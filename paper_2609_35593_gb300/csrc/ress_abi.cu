@@ -98,7 +98,20 @@ ress::SelectArgs select_args(const ress::Shape& s, const uint16_t* Q, const uint
   a.ws = static_cast<char*>(ws);
   a.L = L;
   for (int h = 0; h < RESS_MAX_HEADS; ++h) a.c[h] = (c && h < s.H) ? c[h] : 0;
+  a.v = ress::Variant{0, 0, 0ull};
   return a;
+}
+
+// NULL -> ReSS; otherwise the variant after a range check.
+int check_variant(const ress_variant* v, ress::Variant* out) {
+  *out = ress::Variant{0, 0, 0ull};
+  if (!v) return RESS_OK;
+  if (v->key < RESS_KEY_DRIFT || v->key > RESS_KEY_RANDOM)
+    return fail(RESS_EINVAL, "variant key %d unknown", v->key);
+  if (v->direction < RESS_MINIMIZE || v->direction > RESS_MAXIMIZE_FULL)
+    return fail(RESS_EINVAL, "variant direction %d unknown", v->direction);
+  *out = ress::Variant{v->key, v->direction, (unsigned long long)v->seed};
+  return RESS_OK;
 }
 
 }  // namespace
@@ -157,8 +170,9 @@ int ress_prepare_wo(const ress_dims* d, const uint16_t* W_o, float* F, void* str
   return ok();
 }
 
-int ress_score(const ress_dims* d, const uint16_t* Q, const uint16_t* K, const uint16_t* V,
-               const float* F, const int32_t* c_h, void* ws, size_t ws_bytes, void* stream) {
+int ress_score_variant(const ress_dims* d, const uint16_t* Q, const uint16_t* K,
+                       const uint16_t* V, const float* F, const int32_t* c_h,
+                       const ress_variant* variant, void* ws, size_t ws_bytes, void* stream) {
   int e = check_dims(d);
   if (e) return e;
   if ((e = check_ptr(Q, 16, "Q")) || (e = check_ptr(K, 16, "K")) || (e = check_ptr(V, 16, "V")) ||
@@ -168,15 +182,22 @@ int ress_score(const ress_dims* d, const uint16_t* Q, const uint16_t* K, const u
   if ((e = check_budgets(s, c_h))) return e;
   ress_ws_layout L;
   if ((e = check_ws(s, ws, ws_bytes, &L))) return e;
-  const ress::SelectArgs a = select_args(s, Q, K, V, F, c_h, ws, L);
+  ress::SelectArgs a = select_args(s, Q, K, V, F, c_h, ws, L);
+  if ((e = check_variant(variant, &a.v))) return e;
   cudaError_t ce = ress::launch_score(a, static_cast<cudaStream_t>(stream));
   if (ce != cudaSuccess) return cuda_fail(ce, "ress_score");
   return ok();
 }
 
-int ress_restore(const ress_dims* d, const int32_t* c_h, int32_t rounds, float rho, void* ws,
-                 size_t ws_bytes, int32_t* row_ptr, int32_t* col_idx, int64_t col_capacity,
-                 float* J_best, uint32_t* drop_mask, void* stream) {
+int ress_score(const ress_dims* d, const uint16_t* Q, const uint16_t* K, const uint16_t* V,
+               const float* F, const int32_t* c_h, void* ws, size_t ws_bytes, void* stream) {
+  return ress_score_variant(d, Q, K, V, F, c_h, nullptr, ws, ws_bytes, stream);
+}
+
+int ress_restore_variant(const ress_dims* d, const int32_t* c_h, int32_t rounds, float rho,
+                         const ress_variant* variant, void* ws, size_t ws_bytes, int32_t* row_ptr,
+                         int32_t* col_idx, int64_t col_capacity, float* J_best,
+                         uint32_t* drop_mask, void* stream) {
   int e = check_dims(d);
   if (e) return e;
   const ress::Shape s = ress::make_shape(*d);
@@ -194,7 +215,8 @@ int ress_restore(const ress_dims* d, const int32_t* c_h, int32_t rounds, float r
     return fail(RESS_EWORKSPACE, "col_capacity %lld < %lld", (long long)col_capacity, (long long)base[s.H]);
   if (base[s.H] > INT32_MAX) return fail(RESS_EUNSUPPORTED, "CSR larger than 2^31 entries");
   cudaStream_t st = static_cast<cudaStream_t>(stream);
-  const ress::SelectArgs a = select_args(s, nullptr, nullptr, nullptr, nullptr, c_h, ws, L);
+  ress::SelectArgs a = select_args(s, nullptr, nullptr, nullptr, nullptr, c_h, ws, L);
+  if ((e = check_variant(variant, &a.v))) return e;
   for (int r = 0; r < rounds; ++r) {
     cudaError_t ce = ress::launch_round(a, r, rho, st);
     if (ce != cudaSuccess) return cuda_fail(ce, "ress_restore round");
@@ -202,6 +224,13 @@ int ress_restore(const ress_dims* d, const int32_t* c_h, int32_t rounds, float r
   cudaError_t ce = ress::launch_csr(a, base, row_ptr, col_idx, col_capacity, J_best, drop_mask, st);
   if (ce != cudaSuccess) return cuda_fail(ce, "ress_restore csr");
   return ok();
+}
+
+int ress_restore(const ress_dims* d, const int32_t* c_h, int32_t rounds, float rho, void* ws,
+                 size_t ws_bytes, int32_t* row_ptr, int32_t* col_idx, int64_t col_capacity,
+                 float* J_best, uint32_t* drop_mask, void* stream) {
+  return ress_restore_variant(d, c_h, rounds, rho, nullptr, ws, ws_bytes, row_ptr, col_idx,
+                              col_capacity, J_best, drop_mask, stream);
 }
 
 static int sparse_attn_impl(const ress_dims* d, const uint16_t* Q, const uint16_t* K,

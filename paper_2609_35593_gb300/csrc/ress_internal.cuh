@@ -143,6 +143,13 @@ __device__ __forceinline__ uint4 ld_stream(const uint4* p) {
 void note_launch();
 
 // Kernel launchers (defined in k_select.cu / k_attn.cu); each returns a cudaError_t.
+// Selection variant (ress_variant) as the kernels take it.
+struct Variant {
+  int key;        // 0 drift (Eq. 7), 1 pooled probability, 2 random
+  int direction;  // 0 minimise J, 1 restoration maximises J, 2 initial selection too
+  unsigned long long seed;
+};
+
 struct SelectArgs {
   Shape s;
   const uint16_t *Q, *K, *V;
@@ -150,6 +157,7 @@ struct SelectArgs {
   char* ws;
   ress_ws_layout L;
   int c[RESS_MAX_HEADS];
+  Variant v;
 };
 
 cudaError_t launch_prepare_wo(const Shape& s, const uint16_t* W_o, float* F, cudaStream_t st);

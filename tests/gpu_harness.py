@@ -33,7 +33,8 @@ def widen(bits: np.ndarray) -> np.ndarray:
 class Layer:
     """Inputs of one layer, their device copies and the GPU results."""
 
-    def __init__(self, inputs: dict, n_special: int, c_h, rounds: int, rho: float = 0.5):
+    def __init__(self, inputs: dict, n_special: int, c_h, rounds: int, rho: float = 0.5,
+                 variant=None):
         import paper_2609_35593_gb300 as ress
         self.ress = ress
         self.bits = inputs
@@ -43,6 +44,7 @@ class Layer:
         self.c_h = [int(c) for c in c_h]
         self.rounds = rounds
         self.rho = rho
+        self.variant = variant  # oracle.Variant or None (ReSS)
         self.d = ress.dims(self.N, self.H, n_special, self.d_model)
         self.Q = bits_to_device(inputs["Q"])
         self.K = bits_to_device(inputs["K"])
@@ -57,8 +59,11 @@ class Layer:
     def run(self, attention: bool = True):
         r, b = self.ress, self.buf
         r.prepare_wo(self.d, self.W, b.F)
-        r.score(self.d, self.Q, self.K, self.V, b.F, self.c_h, b.ws)
-        r.restore(self.d, self.c_h, self.rounds, self.rho, b.ws, b.row_ptr, b.col_idx, b.J_best)
+        v = None if self.variant is None else r.variant(self.variant.key, self.variant.maximize,
+                                                          self.variant.seed)
+        r.score(self.d, self.Q, self.K, self.V, b.F, self.c_h, b.ws, variant=v)
+        r.restore(self.d, self.c_h, self.rounds, self.rho, b.ws, b.row_ptr, b.col_idx, b.J_best,
+                  variant=v)
         if attention:
             r.sparse_attn(self.d, self.Q, self.K, self.V, b.row_ptr, b.col_idx, b.O, b.ws)
             r.sparse_attn_f32(self.d, self.Q, self.K, self.V, b.row_ptr, b.col_idx, self.O32, b.ws)
@@ -112,7 +117,8 @@ class Layer:
         return widen(self.bits["W_o"]).astype(np.float64)
 
     def oracle_select(self, rows=None):
-        return O.ress_select(self.pooled(), self.W_o(), self.c_h, self.rounds, self.rho, rows=rows)
+        return O.ress_select(self.pooled(), self.W_o(), self.c_h, self.rounds, self.rho, rows=rows,
+                             variant=self.variant or O.RESS)
 
     def oracle_attention(self, rows, kept=None):
         kept = kept if kept is not None else self.kept()

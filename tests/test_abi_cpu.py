@@ -125,3 +125,9 @@ def test_binding_refuses_host_tensors():
 def test_launch_counter_is_exported_and_monotone():
     a = ress.kernel_launches()
     assert a >= 0 and ress.kernel_launches() >= a
+
+
+def test_variant_names_map_to_the_header_values():
+    v = ress.variant("random", "full", seed=9)
+    assert (v.key, v.direction, v.seed) == (2, 2, 9)
+    assert (ress.variant().key, ress.variant().direction) == (0, 0)

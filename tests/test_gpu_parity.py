@@ -444,3 +444,32 @@ def test_token_drift_sparse_vs_dense(fixture, request):
                     for b in range(nb)])
     assert np.all(np.abs(got - ref) <= 1e-4 * ref + 1e-6 * mag + 1e-12), np.max(np.abs(got - ref) / (ref + 1e-30))
     assert np.all(got[layer.ncand:] <= 1e-6 * mag[layer.ncand:] + 1e-12)  # special rows are dense
+
+
+@pytest.mark.parametrize("name", ["tiny_v2", "vggt_v8"])
+@pytest.mark.parametrize("variant,rounds", [
+    (O.Variant(key="probability"), 0),     # top-k by pooled mass (Table 3's probability rule)
+    (O.Variant(key="probability"), 3),     # the same set refined by restoration
+    (O.Variant(key="random", seed=5), 0),  # random selection (Fig. 8)
+    (O.Variant(key="random", seed=5), 2),
+    (O.Variant(maximize="swap"), 3),       # sign flip in the rounds only (Fig. 8, swap only)
+    (O.Variant(maximize="full"), 3),       # sign flip from the initial selection (Fig. 8, full)
+])
+def test_selection_variants(name, variant, rounds):
+    """The ablation variants of the selection against the oracle's: identical drop sets on
+    every row outside the decision margin, drift within 1e-3."""
+    wl = synth.WORKLOADS[name]
+    layer = G.Layer(synth.make_inputs(wl), wl.n_special, wl.budgets(), rounds, wl.rho,
+                    variant=variant).run(attention=False)
+    r = G.compare_selection(layer, layer.oracle_select())
+    assert r["mismatched"] == 0, r
+    assert r["exact"] >= 0.95 * (r["exact"] + r["near"]), r
+    assert r["worst_row_rel"] <= G.DRIFT_REL and r["sum_rel_gpu_vs_oracle"] <= G.DRIFT_REL, r
+
+
+def test_invalid_variant_is_rejected(tiny):
+    import paper_2609_35593_gb300 as ress
+    bad = ress.Variant(7, 0, 0)
+    with pytest.raises(ress.RessError) as e:
+        ress.score(tiny.d, tiny.Q, tiny.K, tiny.V, tiny.buf.F, tiny.c_h, tiny.buf.ws, variant=bad)
+    assert e.value.code == -1
