@@ -6,7 +6,7 @@ and the initial selection, R restoration rounds, the kept-block lists, and the
 block-sparse attention.  Prints one JSON line (rank 0).
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
-                  [--workload vggt_v32] [--sweep]
+                  [--workload vggt_v32] [--sweep] [--variants]
 
 N > 1 runs as independent replicas (one per GPU, launched by torchrun): the method has no
 exchange step, so there is no collective on the data path.  --impl reference times the
@@ -41,6 +41,8 @@ def parse(argv=None):
     ap.add_argument("--cpu-budget", type=float, default=15.0, help="seconds of oracle work")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--sweep", action="store_true", help="64-view sparsity x rounds sweep lines")
+    ap.add_argument("--variants", action="store_true",
+                    help="drift of the ablation variants (probability, random, maximised) lines")
     return ap.parse_args(argv)
 
 
@@ -563,6 +565,8 @@ def run_ours(a, wl):
 
     if a.sweep and rank == 0:
         sweep(a)
+    if a.variants and rank == 0:
+        variants(a, wl)
     if dist:
         dist.destroy_process_group()
 
@@ -603,6 +607,43 @@ def sweep(a):
                           "sum_J_best": float(Jb.astype(np.float64).sum()),
                           "select_ms": float(m[0] + m[1]), "attn_ms": float(m[2])}), flush=True)
         del buf
+
+
+def variants(a, wl):
+    """The drift side of Fig. 8 on the synthetic layer: for ReSS and each ablation variant,
+    the pooled objective sum_J(D_best) over candidate rows and the token-level drift of its
+    sparse output against the dense output (ress_token_drift), at the workload's budget."""
+    import torch
+    import synth
+    import paper_2609_35593_gb300 as ress
+    bits = synth.make_inputs(wl)
+    dev = lambda b: torch.from_numpy(b.view(np.int16)).view(torch.bfloat16).cuda()
+    Q, K, V, W = (dev(bits[k]) for k in ("Q", "K", "V", "W_o"))
+    c_h = wl.budgets()
+    d = ress.dims(wl.n_tokens, wl.heads, wl.n_special, wl.d_model)
+    buf = ress.Buffers(d, c_h)
+    ress.prepare_wo(d, W, buf.F)
+    H, nb, nc = wl.heads, buf.nb, wl.n_candidates
+    rpd = torch.arange(0, H * nb * nb + 1, nb, dtype=torch.int32, device="cuda")
+    cid = torch.arange(nb, dtype=torch.int32, device="cuda").repeat(H * nb)
+    Od = torch.empty_like(buf.O)
+    ress.sparse_attn(d, Q, K, V, rpd, cid, Od, buf.ws)
+    drift = torch.empty(nb, dtype=torch.float32, device="cuda")
+    cases = [("ress", "drift", "none", wl.rounds), ("probability", "probability", "none", 0),
+             ("random", "random", "none", 0), ("maximize_swap", "drift", "swap", wl.rounds),
+             ("maximize_full", "drift", "full", wl.rounds)]
+    for name, key, mx, R in cases:
+        v = ress.variant(key, mx, seed=1)
+        ress.score(d, Q, K, V, buf.F, c_h, buf.ws, variant=v)
+        ress.restore(d, c_h, R, wl.rho, buf.ws, buf.row_ptr, buf.col_idx, buf.J_best, variant=v)
+        ress.sparse_attn(d, Q, K, V, buf.row_ptr, buf.col_idx, buf.O, buf.ws)
+        ress.token_drift(d, buf.O, Od, W, drift, buf.ws)
+        ress.status(buf.ws)
+        Jb = buf.J_best.cpu().numpy().reshape(H, nb)[:, :nc].astype(np.float64)
+        print(json.dumps({"variants": wl.name, "variant": name, "key": key, "maximize": mx,
+                          "rounds": R, "c_h": int(c_h[0]), "sum_J_best": float(Jb.sum()),
+                          "token_drift": float(drift.cpu().numpy().astype(np.float64).sum())}),
+              flush=True)
 
 
 def main():
