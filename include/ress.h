@@ -36,7 +36,7 @@
 extern "C" {
 #endif
 
-#define RESS_ABI_VERSION 3
+#define RESS_ABI_VERSION 4
 #define RESS_HEAD_DIM 64
 #define RESS_BLOCK 64
 #define RESS_MAX_HEADS 32
@@ -64,6 +64,11 @@ typedef struct {
   int32_t block;     /* block size, must be 64                                    */
   int32_t n_special; /* trailing special tokens, 0..N-1                           */
   int32_t d_model;   /* d: rows of the output projection W_o ([d, H*64])          */
+  int32_t q_block;   /* query block size: 64 (0 means 64) or 128, the paper's own grid
+                        of 128-token query blocks over 64-token key blocks (Appendix F).
+                        Selection rows, CSR rows, J_best and drop masks are per (head,
+                        query block): H * nq rows, nq = ceil(N / q_block); query blocks
+                        that contain special tokens attend densely.                  */
 } ress_dims;
 
 /* Byte offsets of the arrays inside the workspace (for inspection and tests).  All
@@ -102,6 +107,10 @@ uint64_t ress_kernel_launches(void);
 /* Number of key blocks nb = ceil(N / 64) and candidate blocks |P|; -1 on bad dims. */
 int32_t ress_num_blocks(const ress_dims* dims);
 int32_t ress_num_candidates(const ress_dims* dims);
+/* Query blocks nq = ceil(N / q_block) (the rows of the selection and of the CSR), and the
+ * candidate query blocks, floor((N - n_special) / q_block), that are sparsified. */
+int32_t ress_num_query_blocks(const ress_dims* dims);
+int32_t ress_num_query_candidates(const ress_dims* dims);
 
 /* Workspace needed by ress_score / ress_restore / ress_sparse_attn / ress_forward
  * (0 on invalid dims).  The same workspace serves every call on that layer shape; it

@@ -287,12 +287,14 @@ def dense_row(h: int, i: int, nb: int) -> RowSelection:
 
 @dataclass
 class Pooled:
-    """Block-pooled inputs of one layer."""
+    """Block-pooled inputs of one layer: queries over query blocks of q_block tokens (64, or
+    128 on the paper's own grid, Appendix F), keys and values over 64-token key blocks."""
     Qb: np.ndarray
     Kb: np.ndarray
     Vb: np.ndarray
     n_tokens: int
     n_special: int
+    q_block: int = BLOCK
 
     @property
     def heads(self):
@@ -300,15 +302,28 @@ class Pooled:
 
     @property
     def nb(self):
+        """Key blocks."""
+        return self.Kb.shape[1]
+
+    @property
+    def nq(self):
+        """Query blocks (the rows of the selection)."""
         return self.Qb.shape[1]
 
     @property
     def n_cand(self):
+        """Candidate key blocks |cal_P|."""
         return n_candidates(self.n_tokens, self.n_special)
 
+    @property
+    def n_qcand(self):
+        """Query blocks made of patch tokens only: the sparsified rows."""
+        return n_candidates(self.n_tokens, self.n_special, self.q_block)
 
-def pool(Q, K, V, n_special: int) -> Pooled:
-    return Pooled(pool_blocks(Q), pool_blocks(K), pool_blocks(V), Q.shape[0], n_special)
+
+def pool(Q, K, V, n_special: int, q_block: int = BLOCK) -> Pooled:
+    return Pooled(pool_blocks(Q, q_block), pool_blocks(K), pool_blocks(V), Q.shape[0], n_special,
+                  q_block)
 
 
 def row_quantities(pooled: Pooled, h: int, i: int):
@@ -324,13 +339,13 @@ def ress_select(pooled: Pooled, W_o, c_h, rounds: int, rho: float = 0.5, rows=No
 
     Returns {(h, i): RowSelection}.
     """
-    H, nb, d_h = pooled.Qb.shape
-    n_cand = pooled.n_cand
+    H, nq, d_h = pooled.Qb.shape
+    nb, n_cand = pooled.nb, pooled.n_cand
     if rows is None:
-        rows = [(h, i) for h in range(H) for i in range(nb)]
+        rows = [(h, i) for h in range(H) for i in range(nq)]
     out = {}
     for h, i in rows:
-        if i >= n_cand:
+        if i >= pooled.n_qcand:
             out[(h, i)] = dense_row(h, i, nb)
             continue
         P_i, vbar_i = row_quantities(pooled, h, i)
@@ -350,16 +365,18 @@ def drift_of(pooled: Pooled, W_o, h: int, i: int, D: np.ndarray) -> float:
 # ----------------------------------------------------------------------------------------
 # Sec. 3 step (3): exact attention over the kept blocks
 # ----------------------------------------------------------------------------------------
-def block_sparse_attention(Q, K, V, kept, rows, block: int = BLOCK) -> dict:
-    """For every query token of block i and head h: softmax(q k^T / sqrt(d_h)) over the
-    tokens of the kept key blocks of (h, i), renormalised among them, times V.
+def block_sparse_attention(Q, K, V, kept, rows, block: int = BLOCK, q_block: int = None) -> dict:
+    """For every query token of query block i and head h: softmax(q k^T / sqrt(d_h)) over
+    the tokens of the kept key blocks of (h, i), renormalised among them, times V.  Query
+    blocks are q_block tokens (default: the key block size).
 
     kept: {(h, i): ascending key-block indices}.  Returns {(h, i): [rows_i, d_h] float64}.
     """
     N, H, d = Q.shape
+    qb = block if q_block is None else q_block
     out = {}
     for h, i in rows:
-        q = np.asarray(Q[i * block: min(N, (i + 1) * block), h], dtype=np.float64)
+        q = np.asarray(Q[i * qb: min(N, (i + 1) * qb), h], dtype=np.float64)
         idx = np.concatenate([np.arange(j * block, min(N, (j + 1) * block))
                               for j in kept[(h, i)]])
         k = np.asarray(K[idx, h], dtype=np.float64)

@@ -39,7 +39,8 @@ class Dims(ctypes.Structure):
     """ress_dims: one global-attention layer."""
     _fields_ = [("n_tokens", ctypes.c_int32), ("n_heads", ctypes.c_int32),
                 ("head_dim", ctypes.c_int32), ("block", ctypes.c_int32),
-                ("n_special", ctypes.c_int32), ("d_model", ctypes.c_int32)]
+                ("n_special", ctypes.c_int32), ("d_model", ctypes.c_int32),
+                ("q_block", ctypes.c_int32)]
 
 
 class Variant(ctypes.Structure):
@@ -74,6 +75,8 @@ _SIGS = {
     "ress_kernel_launches": (_c.c_uint64, []),
     "ress_num_blocks": (_c.c_int32, [_c.POINTER(Dims)]),
     "ress_num_candidates": (_c.c_int32, [_c.POINTER(Dims)]),
+    "ress_num_query_blocks": (_c.c_int32, [_c.POINTER(Dims)]),
+    "ress_num_query_candidates": (_c.c_int32, [_c.POINTER(Dims)]),
     "ress_workspace_bytes": (_c.c_size_t, [_c.POINTER(Dims)]),
     "ress_workspace_layout": (_c.c_int, [_c.POINTER(Dims), _c.POINTER(WsLayout)]),
     "ress_csr_capacity": (_c.c_int64, [_c.POINTER(Dims), _P]),
@@ -118,8 +121,9 @@ def _check(rc: int):
         raise RessError(rc, _lib.ress_last_error().decode())
 
 
-def dims(n_tokens: int, n_heads: int, n_special: int, d_model: int) -> Dims:
-    return Dims(n_tokens, n_heads, HEAD_DIM, BLOCK, n_special, d_model)
+def dims(n_tokens: int, n_heads: int, n_special: int, d_model: int, q_block: int = 64) -> Dims:
+    """ress_dims; q_block 128 selects the paper's grid of 128-token query blocks."""
+    return Dims(n_tokens, n_heads, HEAD_DIM, BLOCK, n_special, d_model, q_block)
 
 
 def kernel_launches() -> int:
@@ -133,6 +137,14 @@ def num_blocks(d: Dims) -> int:
 
 def num_candidates(d: Dims) -> int:
     return _lib.ress_num_candidates(_c.byref(d))
+
+
+def num_query_blocks(d: Dims) -> int:
+    return _lib.ress_num_query_blocks(_c.byref(d))
+
+
+def num_query_candidates(d: Dims) -> int:
+    return _lib.ress_num_query_candidates(_c.byref(d))
 
 
 def workspace_bytes(d: Dims) -> int:
@@ -329,13 +341,14 @@ class Buffers:
         self.d = d
         self.c_h = [int(c) for c in c_h]
         self.nb = num_blocks(d)
+        self.nq = num_query_blocks(d)
         H = d.n_heads
         self.ws = torch.zeros(workspace_bytes(d), dtype=torch.uint8, device=device)
         self.F = torch.zeros(H, 64, 64, dtype=torch.float32, device=device)
-        self.row_ptr = torch.zeros(H * self.nb + 1, dtype=torch.int32, device=device)
+        self.row_ptr = torch.zeros(H * self.nq + 1, dtype=torch.int32, device=device)
         self.col_idx = torch.zeros(csr_capacity(d, c_h), dtype=torch.int32, device=device)
         self.O = torch.zeros(d.n_tokens, H, 64, dtype=torch.bfloat16, device=device)
-        self.J_best = torch.zeros(H * self.nb, dtype=torch.float32, device=device)
+        self.J_best = torch.zeros(H * self.nq, dtype=torch.float32, device=device)
         self.layout = workspace_layout(d)
 
     def ws_view(self, name: str, dtype=None, shape=None):

@@ -76,6 +76,7 @@ struct __align__(1024) AttnSmem {
 
 struct AttnParams {
   int N, H, nb, npairs, nitems;
+  int rows_per_head, row_step;  // CSR row of item (h, p): h * rows_per_head + row_step * p
   int nsparse;           // pairs 0..nsparse-1 of a head hold only candidate query blocks
   const int32_t* row_ptr;
   const int32_t* plist;  // union lists: entry = j | mask << 16, at row_ptr[h*nb + 2p]
@@ -121,13 +122,15 @@ __device__ __forceinline__ void give_up(AttnSmem& S, uint32_t* status) {
 }
 
 // ------------------------------------------------------------------------------------
-// Union of the two kept lists of every query-block pair, via per-warp bitmaps.
-// One warp per pair; grid ceil(H * npairs / 8) x 256 threads.
+// Union of the two kept lists of every query-block pair, via per-warp bitmaps.  With
+// 128-token query blocks (one block per 128-row item) the list is the block's own, every
+// entry kept by both halves.  One warp per item; grid ceil(H * npairs / 8) x 256 threads.
 // ------------------------------------------------------------------------------------
 __global__ void __launch_bounds__(256) k_pairs(const int32_t* __restrict__ row_ptr,
                                                const int32_t* __restrict__ col_idx,
                                                int64_t cap, int64_t scratch_cap, int nb,
-                                               int npairs, int H, int32_t* __restrict__ plist,
+                                               int npairs, int H, bool qb128,
+                                               int32_t* __restrict__ plist,
                                                int32_t* __restrict__ plen, uint32_t* status) {
   __shared__ uint32_t bits[8][2][RESS_MAX_BLOCKS / 32];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -138,8 +141,8 @@ __global__ void __launch_bounds__(256) k_pairs(const int32_t* __restrict__ row_p
   uint32_t* bA = bits[warp][0];
   uint32_t* bB = bits[warp][1];
   for (int w = lane; w < words; w += 32) bA[w] = bB[w] = 0u;
-  const int64_t ra = (int64_t)h * nb + 2 * p;
-  const bool has_b = 2 * p + 1 < nb;
+  const int64_t ra = qb128 ? (int64_t)h * npairs + p : (int64_t)h * nb + 2 * p;
+  const bool has_b = !qb128 && 2 * p + 1 < nb;
   const int64_t sa = row_ptr[ra], ea = row_ptr[ra + 1];
   const int64_t eb = has_b ? row_ptr[ra + 2] : ea;
   const bool ok = sa >= 0 && sa <= ea && ea <= eb && eb <= cap && eb <= scratch_cap &&
@@ -165,7 +168,7 @@ __global__ void __launch_bounds__(256) k_pairs(const int32_t* __restrict__ row_p
   // union in ascending block order, 32 blocks per step: lane l looks at block 32 w + l
   int pos = 0;
   for (int w = 0; w < words; ++w) {
-    const uint32_t a = bA[w], b = bB[w], u = a | b;
+    const uint32_t a = bA[w], b = qb128 ? a : bB[w], u = a | b;
     if ((u >> lane) & 1u) {
       const int m = (int)((a >> lane) & 1u) | (int)(((b >> lane) & 1u) << 1);
       plist[sa + pos + __popc(u & ((1u << lane) - 1u))] = (w * 32 + lane) | (m << 16);
@@ -233,7 +236,7 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
       item_pair(a, item, h, p);
       const int n = a.plen[h * a.npairs + p];
       if (n <= 0) continue;
-      const int32_t* lst = a.plist + a.row_ptr[(int64_t)h * a.nb + 2 * p];
+      const int32_t* lst = a.plist + a.row_ptr[(int64_t)h * a.rows_per_head + a.row_step * p];
       if (it > 0 && !warp_wait(&S.q_empty, (it - 1) & 1, abort)) {
         failed = true;
         break;
@@ -606,8 +609,9 @@ cudaError_t launch_sparse_attn(const AttnArgs& x, cudaStream_t st) {
     return cudaErrorInvalidValue;
   const int npairs = (s.nb + 1) / 2;
   const int pairs = s.H * npairs;
+  const bool qb128 = s.qb == 128;
   k_pairs<<<(pairs + 7) / 8, 256, 0, st>>>(x.row_ptr, x.col_idx, x.col_capacity, x.scratch_cap,
-                                           s.nb, npairs, s.H, x.plist, x.plen, x.status);
+                                           s.nb, npairs, s.H, qb128, x.plist, x.plen, x.status);
   note_launch();
   cudaError_t e = cudaGetLastError();
   if (e != cudaSuccess) return e;
@@ -618,7 +622,10 @@ cudaError_t launch_sparse_attn(const AttnArgs& x, cudaStream_t st) {
   p.H = s.H;
   p.nb = s.nb;
   p.npairs = npairs;
-  p.nsparse = s.ncand / 2;
+  // items whose rows are all candidate query rows come first in each head's order
+  p.nsparse = qb128 ? s.nqc : s.ncand / 2;
+  p.rows_per_head = qb128 ? s.nq : s.nb;
+  p.row_step = qb128 ? 1 : 2;
   p.nitems = pairs;
   p.row_ptr = x.row_ptr;
   p.plist = x.plist;

@@ -56,7 +56,8 @@ struct __align__(1024) DotSmem {
 };
 
 struct DotParams {
-  int nb, ncand, round;
+  int nb, ncand, round;  // key blocks (columns), candidate key blocks
+  int nq, nqc;           // query blocks (rows), candidate query blocks
   float rho;
   const float* a;     // per row: c_i (gains) or ||y~_i||^2 (drift norms), [H, nb]
   const float* b;     // per block: ||z~_j||^2 (drift norms), [H, nb]
@@ -164,9 +165,9 @@ __global__ void __launch_bounds__(kDotThreads)
     tc_fence_after();
     const int r = 32 * warp + lane;  // row of the tile = TMEM lane
     const int i = i0 + r;
-    const int64_t ri = (int64_t)h * p.nb + i;
+    const int64_t ri = (int64_t)h * p.nq + i;
     float a = 0.f;
-    if (MODE != kDotLogit && i < p.nb) a = p.a[ri];
+    if (MODE != kDotLogit && i < p.nq) a = p.a[ri];
     float pm = -INFINITY, ps = 0.f;  // logits: running max and sum over the slice
     uint8_t* stage = &S.A[0][0];     // 4 boxes of 128 rows x 32 fp32, 16 KB each
 #pragma unroll 1
@@ -206,7 +207,7 @@ __global__ void __launch_bounds__(kDotThreads)
         *reinterpret_cast<float4*>(row + ((k ^ (r & 7)) << 4)) =
             make_float4(o[4 * k], o[4 * k + 1], o[4 * k + 2], o[4 * k + 3]);
     }
-    if (MODE == kDotLogit && i < p.ncand)
+    if (MODE == kDotLogit && i < p.nqc)
       p.lstat[ri * p.nslices + blockIdx.x] = make_float2(pm, ps);
     fence_proxy_async_smem();
   }
@@ -281,15 +282,17 @@ cudaError_t launch_dot(const SelectArgs& a, int64_t a_terms, int64_t b_terms, in
                        const float* rowv, const float* colv, int ncols, int round, float rho,
                        cudaStream_t st) {
   const Shape& s = a.s;
-  if (s.ncand <= 0) return cudaSuccess;
+  if (s.ncand <= 0 || s.nqc <= 0) return cudaSuccess;
   CUtensorMap ta, tb, to;
-  if (!make_term_map(&ta, a.ws + a_terms, s.nb, s.H, kDotTile) ||
+  if (!make_term_map(&ta, a.ws + a_terms, s.nq, s.H, kDotTile) ||
       !make_term_map(&tb, a.ws + b_terms, s.nb, s.H, kDotTile) ||
-      !make_row_map(&to, a.ws + out, s.nb, s.H, s.ld))
+      !make_row_map(&to, a.ws + out, s.nq, s.H, s.ld))
     return cudaErrorInvalidValue;
   DotParams p;
   p.nb = s.nb;
   p.ncand = s.ncand;
+  p.nq = s.nq;
+  p.nqc = s.nqc;
   p.round = round;
   p.rho = rho;
   p.a = rowv;
@@ -303,7 +306,7 @@ cudaError_t launch_dot(const SelectArgs& a, int64_t a_terms, int64_t b_terms, in
   cudaError_t e =
       cudaFuncSetAttribute(k_dot<MODE>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
-  const dim3 grid((ncols + kDotTile - 1) / kDotTile, (s.ncand + kDotTile - 1) / kDotTile, s.H);
+  const dim3 grid((ncols + kDotTile - 1) / kDotTile, (s.nqc + kDotTile - 1) / kDotTile, s.H);
   k_dot<MODE><<<grid, kDotThreads, smem, st>>>(ta, tb, to, p);
   note_launch();
   return cudaGetLastError();

@@ -99,27 +99,32 @@ __device__ __forceinline__ float warp_sum(float v) {
 }
 
 // ------------------------------------------------------------------------------------
-// Sec. 3 step (1): block means of Q, K and V over the valid tokens of each block.
-// grid (nb, 3); one token is H*64 bf16 = 8H 16-byte chunks (H <= 32).
+// Sec. 3 step (1): block means of Q (over query blocks of qb tokens), K and V (over 64-token
+// key blocks), each over the valid tokens of its block.  grid (nb, 3); one token is H*64
+// bf16 = 8H 16-byte chunks (H <= 32).
 // ------------------------------------------------------------------------------------
 __global__ void __launch_bounds__(kThreads) k_pool(const uint16_t* __restrict__ Q,
                                                     const uint16_t* __restrict__ K,
                                                     const uint16_t* __restrict__ V, int N,
-                                                    int H, int nb, float* __restrict__ qbar,
+                                                    int H, int nb, int qb, int nq,
+                                                    float* __restrict__ qbar,
                                                     float* __restrict__ kbar,
                                                     float* __restrict__ vbar,
                                                     uint16_t* __restrict__ qsplit,
                                                     uint16_t* __restrict__ ksplit) {
   __shared__ float part[kThreads * 8];
   const int j = blockIdx.x, which = blockIdx.y;
+  const int bs = which == 0 ? qb : kBlock;        // tokens per block
+  const int nblocks = which == 0 ? nq : nb;
+  if (j >= nblocks) return;
   const uint16_t* X = which == 0 ? Q : (which == 1 ? K : V);
   float* out = which == 0 ? qbar : (which == 1 ? kbar : vbar);
   uint16_t* terms = which == 0 ? qsplit : (which == 1 ? ksplit : nullptr);  // tensor-core operands
-  const int64_t term_stride = (int64_t)H * nb * kHeadDim;
+  const int64_t term_stride = (int64_t)H * nblocks * kHeadDim;
   const int C = 8 * H;
   const int tpp = kThreads / C;
-  const int tok0 = j * kBlock;
-  const int valid = min(kBlock, N - tok0);
+  const int tok0 = j * bs;
+  const int valid = min(bs, N - tok0);
   const int c = threadIdx.x % C, slot = threadIdx.x / C;
   float acc[8];
 #pragma unroll
@@ -143,7 +148,7 @@ __global__ void __launch_bounds__(kThreads) k_pool(const uint16_t* __restrict__ 
     float s = 0.f;
     for (int sl = 0; sl < tpp; ++sl) s += part[sl * C * 8 + f];
     const int h = f >> 6, d = f & 63;
-    const int64_t at = ((int64_t)h * nb + j) * kHeadDim + d;
+    const int64_t at = ((int64_t)h * nblocks + j) * kHeadDim + d;
     out[at] = s * inv;
     if (terms) {
       uint16_t hi, mid, lo;
@@ -222,7 +227,8 @@ __global__ void __launch_bounds__(kThreads) k_zproj(const float* __restrict__ F,
 }
 
 struct SelPtrs {
-  int nb, ncand, words, ld;
+  int nb, ncand, words, ld;  // key blocks (columns), candidate key blocks, mask words, row stride
+  int nq, nqc;               // query blocks (rows), candidate query blocks
   const float *qbar, *kbar, *ztil;
   float *ytil, *gtil, *P, *q, *t, *K, *G, *J, *Jbest, *J0;
   uint32_t *dmask, *bmask;
@@ -235,6 +241,8 @@ __host__ __device__ inline SelPtrs sel_ptrs(const Shape& s, char* ws, const ress
   SelPtrs p;
   p.nb = s.nb;
   p.ncand = s.ncand;
+  p.nq = s.nq;
+  p.nqc = s.nqc;
   p.words = s.words;
   p.ld = s.ld;
   p.qbar = (const float*)(ws + L.qbar);
@@ -254,7 +262,7 @@ __host__ __device__ inline SelPtrs sel_ptrs(const Shape& s, char* ws, const ress
   p.bmask = (uint32_t*)(ws + L.bmask);
   p.asplit = (uint32_t*)(ws + L.asplit);
   p.cdot = (float*)(ws + L.cdot);
-  p.split_stride = (int64_t)s.H * s.nb * 32;
+  p.split_stride = (int64_t)s.H * s.nq * 32;
   return p;
 }
 
@@ -649,8 +657,8 @@ __global__ void __launch_bounds__(32 * kRowWarps, 8) k_score_rows(SelPtrs p, Bud
   extern __shared__ __align__(16) unsigned char smem_raw[];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int h = blockIdx.y, i = blockIdx.x * kRowWarps + warp;
-  if (i >= p.ncand) return;
-  const int64_t ri = (int64_t)h * p.nb + i;
+  if (i >= p.nqc) return;
+  const int64_t ri = (int64_t)h * p.nq + i;
   const float* Prow = p.P + ri * p.ld;
   const float* qrow = p.q + ri * p.ld;
   const float* zt_h = p.ztil + (int64_t)h * p.nb * 64;
@@ -715,8 +723,8 @@ __global__ void __launch_bounds__(32 * kRowWarps, 8) k_round_rows(SelPtrs p, Bud
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int h = blockIdx.y, i = blockIdx.x * kRowWarps + warp;
   const int m = swap_count(bud.c[h], p.ncand, round, rho);
-  if (m <= 0 || i >= p.ncand) return;
-  const int64_t ri = (int64_t)h * p.nb + i;
+  if (m <= 0 || i >= p.nqc) return;
+  const int64_t ri = (int64_t)h * p.nq + i;
   const float* Prow = p.P + ri * p.ld;
   const float* qrow = p.q + ri * p.ld;
   const float* trow = p.t + ri * p.ld;
@@ -784,7 +792,7 @@ __global__ void __launch_bounds__(32 * kRowWarps, 8) k_round_rows(SelPtrs p, Bud
 
 // ------------------------------------------------------------------------------------
 // Kept-block lists (CSR) from the best drop sets; special query rows keep everything.
-// grid (ceil(nb / 8), H) x 256 threads, one warp per row.
+// grid (ceil(nq / 8), H) x 256 threads, one warp per (head, query block) row.
 // ------------------------------------------------------------------------------------
 struct CsrBases {
   int64_t base[RESS_MAX_HEADS + 1];
@@ -794,12 +802,12 @@ __global__ void k_csr(SelPtrs p, Budgets bud, CsrBases cb, int H, int32_t* __res
                       int32_t* __restrict__ col_idx, int64_t cap, float* __restrict__ J_best,
                       uint32_t* __restrict__ drop_mask, uint32_t* status) {
   const int i = blockIdx.x * 8 + (threadIdx.x >> 5), h = blockIdx.y, lane = threadIdx.x & 31;
-  if (i >= p.nb) return;
-  const int64_t ri = (int64_t)h * p.nb + i;
+  if (i >= p.nq) return;
+  const int64_t ri = (int64_t)h * p.nq + i;
   const int c = bud.c[h];
-  const int ns = p.nb - p.ncand;
-  const bool dense = i >= p.ncand;
-  const int64_t off = cb.base[h] + (dense ? (int64_t)p.ncand * (c + ns) + (int64_t)(i - p.ncand) * p.nb
+  const int ns = p.nb - p.ncand;  // always-kept key blocks
+  const bool dense = i >= p.nqc;
+  const int64_t off = cb.base[h] + (dense ? (int64_t)p.nqc * (c + ns) + (int64_t)(i - p.nqc) * p.nb
                                           : (int64_t)i * (c + ns));
   const int expect = dense ? p.nb : c + ns;
   int pos = 0;
@@ -821,7 +829,7 @@ __global__ void k_csr(SelPtrs p, Budgets bud, CsrBases cb, int H, int32_t* __res
   if (lane == 0) {
     if (pos != expect) flag_status(status, kStatusBadRow);
     row_ptr[ri] = (int32_t)off;
-    if (h == H - 1 && i == p.nb - 1) row_ptr[(int64_t)H * p.nb] = (int32_t)cb.base[H];
+    if (h == H - 1 && i == p.nq - 1) row_ptr[(int64_t)H * p.nq] = (int32_t)cb.base[H];
     if (J_best) J_best[ri] = dense ? 0.f : p.Jbest[ri];
   }
 }
@@ -849,7 +857,8 @@ cudaError_t launch_score(const SelectArgs& a, cudaStream_t st) {
   float* kbar = (float*)(a.ws + a.L.kbar);
   float* vbar = (float*)(a.ws + a.L.vbar);
   float* ztil = (float*)(a.ws + a.L.ztil);
-  k_pool<<<dim3(s.nb, 3), kThreads, 0, st>>>(a.Q, a.K, a.V, s.N, s.H, s.nb, qbar, kbar, vbar,
+  k_pool<<<dim3(s.nb, 3), kThreads, 0, st>>>(a.Q, a.K, a.V, s.N, s.H, s.nb, s.qb, s.nq, qbar,
+                                              kbar, vbar,
                                               (uint16_t*)(a.ws + a.L.asplit),
                                               (uint16_t*)(a.ws + a.L.ksplit));
   note_launch();
@@ -858,7 +867,7 @@ cudaError_t launch_score(const SelectArgs& a, cudaStream_t st) {
       (float*)(a.ws + a.L.nz));
   note_launch();
   cudaError_t e = cudaGetLastError();
-  if (e != cudaSuccess || s.ncand <= 0) return e;
+  if (e != cudaSuccess || s.ncand <= 0 || s.nqc <= 0) return e;
   // pooled logits, then P and y~, then q (Sec. 4.1, Eq. 1, Eq. 9), on the tensor cores
   if ((e = launch_logits(a, st)) != cudaSuccess) return e;
   if ((e = launch_yagg(a, st)) != cudaSuccess) return e;
@@ -866,7 +875,7 @@ cudaError_t launch_score(const SelectArgs& a, cudaStream_t st) {
   const size_t rsmem = (size_t)kRowWarps * warp_scratch_words(s.ld, s.words) * 4;
   e = cudaFuncSetAttribute(k_score_rows, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)rsmem);
   if (e != cudaSuccess) return e;
-  k_score_rows<<<dim3((s.ncand + kRowWarps - 1) / kRowWarps, s.H), 32 * kRowWarps, rsmem, st>>>(
+  k_score_rows<<<dim3((s.nqc + kRowWarps - 1) / kRowWarps, s.H), 32 * kRowWarps, rsmem, st>>>(
       p, budgets_of(a), a.v);
   note_launch();
   return cudaGetLastError();
@@ -874,14 +883,14 @@ cudaError_t launch_score(const SelectArgs& a, cudaStream_t st) {
 
 cudaError_t launch_round(const SelectArgs& a, int round, float rho, cudaStream_t st) {
   const Shape& s = a.s;
-  if (s.ncand <= 0) return cudaSuccess;
+  if (s.ncand <= 0 || s.nqc <= 0) return cudaSuccess;
   SelPtrs p = sel_ptrs(s, a.ws, a.L);
   cudaError_t e = launch_gain(a, round, rho, st);  // t_ij on the tensor cores
   if (e != cudaSuccess) return e;
   const size_t rsmem = (size_t)kRowWarps * warp_scratch_words(s.ld, 3 * s.words) * 4;
   e = cudaFuncSetAttribute(k_round_rows, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)rsmem);
   if (e != cudaSuccess) return e;
-  k_round_rows<<<dim3((s.ncand + kRowWarps - 1) / kRowWarps, s.H), 32 * kRowWarps, rsmem, st>>>(
+  k_round_rows<<<dim3((s.nqc + kRowWarps - 1) / kRowWarps, s.H), 32 * kRowWarps, rsmem, st>>>(
       p, budgets_of(a), round, rho, a.v.direction != 0 ? 1 : 0);
   note_launch();
   return cudaGetLastError();
@@ -894,7 +903,7 @@ cudaError_t launch_csr(const SelectArgs& a, const int64_t* head_base, int32_t* r
   SelPtrs p = sel_ptrs(s, a.ws, a.L);
   CsrBases cb;
   for (int h = 0; h <= s.H; ++h) cb.base[h] = head_base[h];
-  k_csr<<<dim3((s.nb + 7) / 8, s.H), 256, 0, st>>>(p, budgets_of(a), cb, s.H, row_ptr, col_idx, col_capacity,
+  k_csr<<<dim3((s.nq + 7) / 8, s.H), 256, 0, st>>>(p, budgets_of(a), cb, s.H, row_ptr, col_idx, col_capacity,
                                         J_best, drop_mask, (uint32_t*)(a.ws + a.L.status));
   note_launch();
   return cudaGetLastError();

@@ -56,7 +56,7 @@ struct __align__(1024) YSmem {
 };
 
 struct YParams {
-  int nb, ncand, ld, nslices, nchunks;
+  int nb, nq, nqc, ld, nslices, nchunks;  // key blocks, query blocks, candidate query blocks
   const float2* lstat;
   float* P;         // [H, nb, ld]: logits in, probabilities out
   float* ytil;      // [H, nb, 64]
@@ -184,8 +184,8 @@ __global__ void __launch_bounds__(kYThreads, 1)
     // ============================ conversion ========================================
     const int r = 32 * (warp & 3) + lane, qq = warp >> 2;  // row of the tile, column quarter
     const int i = i0 + r;
-    const bool row_ok = i < p.ncand;
-    const int64_t ri = (int64_t)h * p.nb + i;
+    const bool row_ok = i < p.nqc;
+    const int64_t ri = (int64_t)h * p.nq + i;
     float m = 0.f, iz = 0.f;
     if (row_ok) {  // the row's softmax from its per-slice maxima and sums
       m = -INFINITY;
@@ -279,8 +279,8 @@ __global__ void __launch_bounds__(kYThreads, 1)
   __syncthreads();
   if (threadIdx.x < kYRows) {
     const int i = i0 + threadIdx.x;
-    if (i < p.ncand && !*abort)
-      p.ny[(int64_t)h * p.nb + i] = (S.ny_part[0][threadIdx.x] + S.ny_part[1][threadIdx.x]) +
+    if (i < p.nqc && !*abort)
+      p.ny[(int64_t)h * p.nq + i] = (S.ny_part[0][threadIdx.x] + S.ny_part[1][threadIdx.x]) +
                                     (S.ny_part[2][threadIdx.x] + S.ny_part[3][threadIdx.x]);
   }
   if (warp == kMmaWarp) {
@@ -293,14 +293,15 @@ __global__ void __launch_bounds__(kYThreads, 1)
 
 cudaError_t launch_yagg(const SelectArgs& a, cudaStream_t st) {
   const Shape& s = a.s;
-  if (s.ncand <= 0) return cudaSuccess;
+  if (s.ncand <= 0 || s.nqc <= 0) return cudaSuccess;
   CUtensorMap tl, tz;
-  if (!make_row_map(&tl, a.ws + a.L.P, s.nb, s.H, s.ld) ||
+  if (!make_row_map(&tl, a.ws + a.L.P, s.nq, s.H, s.ld) ||
       !make_term_map(&tz, a.ws + a.L.zsplit, s.nb, s.H, kYChunk))
     return cudaErrorInvalidValue;
   YParams p;
   p.nb = s.nb;
-  p.ncand = s.ncand;
+  p.nq = s.nq;
+  p.nqc = s.nqc;
   p.ld = s.ld;
   p.nslices = (s.nb + 127) / 128;
   p.nchunks = (s.nb + kYChunk - 1) / kYChunk;
@@ -309,12 +310,12 @@ cudaError_t launch_yagg(const SelectArgs& a, cudaStream_t st) {
   p.ytil = (float*)(a.ws + a.L.ytil);
   p.asplit = (uint32_t*)(a.ws + a.L.asplit);
   p.ny = (float*)(a.ws + a.L.ny);
-  p.term_words = (int64_t)s.H * s.nb * 32;
+  p.term_words = (int64_t)s.H * s.nq * 32;
   p.status = (uint32_t*)(a.ws + a.L.status);
   const size_t smem = sizeof(YSmem) + 1024;
   cudaError_t e = cudaFuncSetAttribute(k_yagg, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
-  k_yagg<<<dim3((s.ncand + kYRows - 1) / kYRows, s.H), kYThreads, smem, st>>>(tl, tz, p);
+  k_yagg<<<dim3((s.nqc + kYRows - 1) / kYRows, s.H), kYThreads, smem, st>>>(tl, tz, p);
   note_launch();
   return cudaGetLastError();
 }

@@ -39,6 +39,8 @@ int check_dims(const ress_dims* d) {
   if (d->n_special < 0 || d->n_special >= d->n_tokens)
     return fail(RESS_EINVAL, "n_special %d outside 0..n_tokens-1", d->n_special);
   if (d->d_model < 1) return fail(RESS_EINVAL, "d_model %d < 1", d->d_model);
+  if (d->q_block != 0 && d->q_block != 64 && d->q_block != 128)
+    return fail(RESS_EUNSUPPORTED, "q_block %d unsupported (0, 64 or 128)", d->q_block);
   const int64_t nb = ((int64_t)d->n_tokens + RESS_BLOCK - 1) / RESS_BLOCK;
   if (nb > RESS_MAX_BLOCKS)
     return fail(RESS_EUNSUPPORTED, "%lld blocks exceed the limit of %d", (long long)nb, RESS_MAX_BLOCKS);
@@ -76,9 +78,11 @@ int cuda_fail(cudaError_t e, const char* where) {
   return fail(RESS_ECUDA, "%s: %s", where, cudaGetErrorString(e));
 }
 
+// col_idx entries of one head: every candidate query block keeps c_h candidates plus the
+// always-kept key blocks, every other query block keeps all key blocks.
 int64_t head_rows(const ress::Shape& s, int c) {
-  const int ns = s.nb - s.ncand;
-  return (int64_t)s.ncand * (c + ns) + (int64_t)ns * s.nb;
+  const int nsk = s.nb - s.ncand;
+  return (int64_t)s.nqc * (c + nsk) + (int64_t)(s.nq - s.nqc) * s.nb;
 }
 
 void head_bases(const ress::Shape& s, const int32_t* c, int64_t* base) {
@@ -136,6 +140,14 @@ int32_t ress_num_blocks(const ress_dims* d) {
 int32_t ress_num_candidates(const ress_dims* d) {
   if (check_dims(d)) return -1;
   return ress::make_shape(*d).ncand;
+}
+int32_t ress_num_query_blocks(const ress_dims* d) {
+  if (check_dims(d)) return -1;
+  return ress::make_shape(*d).nq;
+}
+int32_t ress_num_query_candidates(const ress_dims* d) {
+  if (check_dims(d)) return -1;
+  return ress::make_shape(*d).nqc;
 }
 
 size_t ress_workspace_bytes(const ress_dims* d) {
@@ -262,7 +274,7 @@ static int sparse_attn_impl(const ress_dims* d, const uint16_t* Q, const uint16_
   a.counter = reinterpret_cast<uint32_t*>(w + L.counter);
   a.plist = reinterpret_cast<int32_t*>(w + L.t);  // the gains buffer is free during attention
   a.plen = reinterpret_cast<int32_t*>(w + L.plen);
-  a.scratch_cap = (int64_t)s.H * s.nb * s.ld;
+  a.scratch_cap = (int64_t)s.H * s.nq * s.ld;  // entries of the t array
   cudaError_t ce = ress::launch_sparse_attn(a, static_cast<cudaStream_t>(stream));
   if (ce != cudaSuccess) return cuda_fail(ce, "ress_sparse_attn");
   return ok();

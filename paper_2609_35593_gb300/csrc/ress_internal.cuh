@@ -19,8 +19,11 @@ constexpr uint32_t kStatusBadIndex = 2;
 constexpr uint32_t kStatusBadRow = 3;
 
 // Derived sizes of one layer.
+// Key blocks are 64 tokens (columns of the selection); query blocks qb = 64 or 128 tokens
+// (rows of the selection, the CSR and the attention items).
 struct Shape {
   int N, H, nb, ncand, nspecial_blocks, words, ld, d_model;
+  int qb, nq, nqc;  // query block size, query blocks, candidate (sparsified) query blocks
 };
 
 inline Shape make_shape(const ress_dims& d) {
@@ -33,6 +36,9 @@ inline Shape make_shape(const ress_dims& d) {
   s.words = (s.nb + 31) / 32;
   s.ld = (s.nb + 31) / 32 * 32;
   s.d_model = d.d_model;
+  s.qb = d.q_block == 128 ? 128 : kBlock;
+  s.nq = (d.n_tokens + s.qb - 1) / s.qb;
+  s.nqc = (d.n_tokens - d.n_special) / s.qb;
   return s;
 }
 
@@ -46,18 +52,19 @@ inline ress_ws_layout make_layout(const Shape& s) {
     off = align256(off + bytes);
     return o;
   };
-  const int64_t vec = (int64_t)s.H * s.nb * kHeadDim * 4;
-  const int64_t mat = (int64_t)s.H * s.nb * s.ld * 4;
-  const int64_t row = (int64_t)s.H * s.nb * 4;
-  const int64_t msk = (int64_t)s.H * s.nb * s.words * 4;
+  const int64_t vec = (int64_t)s.H * s.nb * kHeadDim * 4;   // per key block
+  const int64_t qvec = (int64_t)s.H * s.nq * kHeadDim * 4;  // per query block
+  const int64_t mat = (int64_t)s.H * s.nq * s.ld * 4;
+  const int64_t row = (int64_t)s.H * s.nq * 4;
+  const int64_t msk = (int64_t)s.H * s.nq * s.words * 4;
   L.status = take(64);
   L.counter = take(64);
-  L.qbar = take(vec);
+  L.qbar = take(qvec);
   L.kbar = take(vec);
   L.vbar = take(vec);
   L.ztil = take(vec);
-  L.ytil = take(vec);
-  L.gtil = take(vec);
+  L.ytil = take(qvec);
+  L.gtil = take(qvec);
   L.P = take(mat);
   L.q = take(mat);
   L.t = take(mat);
@@ -69,13 +76,13 @@ inline ress_ws_layout make_layout(const Shape& s) {
   L.dmask = take(msk);
   L.bmask = take(msk);
   L.plen = take((int64_t)s.H * ((s.nb + 1) / 2) * 4);
-  L.asplit = take(3 * (int64_t)s.H * s.nb * kHeadDim * 2);
+  L.asplit = take(3 * (int64_t)s.H * s.nq * kHeadDim * 2);
   L.ksplit = take(3 * (int64_t)s.H * s.nb * kHeadDim * 2);
   L.zsplit = take(3 * (int64_t)s.H * s.nb * kHeadDim * 2);
   L.cdot = take(row);
   L.ny = take(row);
-  L.nz = take(row);
-  L.lstat = take((int64_t)s.H * s.nb * ((s.nb + 127) / 128) * 8);
+  L.nz = take((int64_t)s.H * s.nb * 4);
+  L.lstat = take((int64_t)s.H * s.nq * ((s.nb + 127) / 128) * 8);
   L.ld = s.ld;
   L.words = s.words;
   L.total = off;

@@ -34,7 +34,7 @@ class Layer:
     """Inputs of one layer, their device copies and the GPU results."""
 
     def __init__(self, inputs: dict, n_special: int, c_h, rounds: int, rho: float = 0.5,
-                 variant=None):
+                 variant=None, q_block: int = 64):
         import paper_2609_35593_gb300 as ress
         self.ress = ress
         self.bits = inputs
@@ -45,15 +45,18 @@ class Layer:
         self.rounds = rounds
         self.rho = rho
         self.variant = variant  # oracle.Variant or None (ReSS)
-        self.d = ress.dims(self.N, self.H, n_special, self.d_model)
+        self.q_block = q_block
+        self.d = ress.dims(self.N, self.H, n_special, self.d_model, q_block)
         self.Q = bits_to_device(inputs["Q"])
         self.K = bits_to_device(inputs["K"])
         self.V = bits_to_device(inputs["V"])
         self.W = bits_to_device(inputs["W_o"])
         self.buf = ress.Buffers(self.d, self.c_h)
         self.O32 = torch.zeros(self.N, self.H, 64, dtype=torch.float32, device="cuda")
-        self.nb = self.buf.nb
-        self.ncand = ress.num_candidates(self.d)
+        self.nb = self.buf.nb                          # key blocks
+        self.nq = self.buf.nq                          # query blocks (selection and CSR rows)
+        self.ncand = ress.num_candidates(self.d)       # candidate key blocks
+        self.nqc = ress.num_query_candidates(self.d)   # sparsified query blocks
 
     # ---- GPU -----------------------------------------------------------------------
     def run(self, attention: bool = True):
@@ -85,10 +88,10 @@ class Layer:
         return self.buf.ws_view(name, dtype, shape).cpu().numpy()
 
     def drop_sets(self, which="bmask") -> np.ndarray:
-        """[H, nb, nb] bool: the GPU drop sets (best by default)."""
+        """[H, nq, nb] bool: the GPU drop sets (best by default)."""
         L = self.buf.layout
-        w = self.ws(which, torch.int32, (self.H, self.nb, L.words)).view(np.uint32)
-        bits = np.unpackbits(w.view(np.uint8), bitorder="little").reshape(self.H, self.nb, -1)
+        w = self.ws(which, torch.int32, (self.H, self.nq, L.words)).view(np.uint32)
+        bits = np.unpackbits(w.view(np.uint8), bitorder="little").reshape(self.H, self.nq, -1)
         return bits[:, :, :self.nb].astype(bool)
 
     def csr(self):
@@ -96,8 +99,8 @@ class Layer:
 
     def kept(self) -> dict:
         rp, ci = self.csr()
-        return {(h, i): ci[rp[h * self.nb + i]:rp[h * self.nb + i + 1]]
-                for h in range(self.H) for i in range(self.nb)}
+        return {(h, i): ci[rp[h * self.nq + i]:rp[h * self.nq + i + 1]]
+                for h in range(self.H) for i in range(self.nq)}
 
     def output(self) -> np.ndarray:
         """The kernel's float32 attention output."""
@@ -110,7 +113,7 @@ class Layer:
     def pooled(self):
         if not hasattr(self, "_pooled"):
             self._pooled = O.pool(widen(self.bits["Q"]), widen(self.bits["K"]), widen(self.bits["V"]),
-                                  self.n_special)
+                                  self.n_special, self.q_block)
         return self._pooled
 
     def W_o(self):
@@ -123,13 +126,13 @@ class Layer:
     def oracle_attention(self, rows, kept=None):
         kept = kept if kept is not None else self.kept()
         X = [widen(self.bits[k]) for k in ("Q", "K", "V")]
-        return O.block_sparse_attention(*X, kept, rows)
+        return O.block_sparse_attention(*X, kept, rows, q_block=self.q_block)
 
 
 def compare_selection(layer: Layer, sel: dict) -> dict:
     """Drop-set and drift parity on the rows in `sel`."""
     D = layer.drop_sets()
-    Jg = layer.buf.J_best.cpu().numpy().reshape(layer.H, layer.nb)
+    Jg = layer.buf.J_best.cpu().numpy().reshape(layer.H, layer.nq)
     exact = near = mismatched = 0
     bad_rows = []
     J_gpu_sum = J_ref_gpu_D = J_oracle = 0.0
@@ -166,7 +169,7 @@ def compare_attention(layer: Layer, rows) -> dict:
     num = den = 0.0
     mx = 0.0
     for (h, i), o in ref.items():
-        g = out[i * 64:i * 64 + o.shape[0], h, :]
+        g = out[i * layer.q_block:i * layer.q_block + o.shape[0], h, :]
         diff = np.abs(g - o)
         mx = max(mx, float(diff.max()))
         num += float(diff.sum())

@@ -23,7 +23,7 @@ def test_every_declared_function_is_exported():
         assert hasattr(ress._lib, n), n
     for n in ("ress_score", "ress_restore", "ress_sparse_attn", "ress_forward"):
         assert n in names
-    assert ress._lib.ress_abi_version() == 3
+    assert ress._lib.ress_abi_version() == 4
 
 
 @pytest.mark.parametrize("name", list(synth.WORKLOADS))
@@ -131,3 +131,26 @@ def test_variant_names_map_to_the_header_values():
     v = ress.variant("random", "full", seed=9)
     assert (v.key, v.direction, v.seed) == (2, 2, 9)
     assert (ress.variant().key, ress.variant().direction) == (0, 0)
+
+
+@pytest.mark.parametrize("name", ["tiny_v2", "vggt_v8", "vggt_v32"])
+def test_query_block_128_shapes(name):
+    """On the paper's grid the selection and CSR rows are 128-token query blocks: their
+    count, the sparsified ones, and the CSR capacity match the oracle's row structure."""
+    wl = synth.WORKLOADS[name]
+    d = ress.dims(wl.n_tokens, wl.heads, wl.n_special, wl.d_model, 128)
+    nq = -(-wl.n_tokens // 128)
+    nqc = (wl.n_tokens - wl.n_special) // 128
+    assert ress.num_query_blocks(d) == nq and ress.num_query_candidates(d) == nqc
+    nb, nc = ress.num_blocks(d), ress.num_candidates(d)
+    c = wl.budgets()
+    assert ress.csr_capacity(d, c) == sum(nqc * (ch + nb - nc) + (nq - nqc) * nb for ch in c)
+    L = ress.workspace_layout(d)
+    assert L.total == ress.workspace_bytes(d)
+    d64 = ress.dims(wl.n_tokens, wl.heads, wl.n_special, wl.d_model)
+    assert ress.workspace_bytes(d) < ress.workspace_bytes(d64)  # half the selection rows
+
+
+def test_query_block_must_be_64_or_128():
+    d = ress.dims(1000, 2, 0, 128, 96)
+    assert ress.num_query_blocks(d) == -1

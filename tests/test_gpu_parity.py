@@ -473,3 +473,51 @@ def test_invalid_variant_is_rejected(tiny):
     with pytest.raises(ress.RessError) as e:
         ress.score(tiny.d, tiny.Q, tiny.K, tiny.V, tiny.buf.F, tiny.c_h, tiny.buf.ws, variant=bad)
     assert e.value.code == -1
+
+
+@pytest.mark.parametrize("name", ["tiny_v2", "vggt_v8"])
+def test_paper_grid_query_block_128(name):
+    """The paper's own grid (Appendix F): 128-token query blocks over 64-token key blocks.
+    Selection against the oracle on that grid, the CSR's row structure, and attention of
+    every (sampled) query block against the oracle over the GPU's kept lists."""
+    wl = synth.WORKLOADS[name]
+    layer = G.Layer(synth.make_inputs(wl), wl.n_special, wl.budgets(), wl.rounds, wl.rho,
+                    q_block=128).run()
+    assert layer.nq == -(-layer.N // 128)
+    r = G.compare_selection(layer, layer.oracle_select())
+    assert r["mismatched"] == 0, r
+    assert r["exact"] >= 0.95 * (r["exact"] + r["near"]), r
+    assert r["worst_row_rel"] <= G.DRIFT_REL and r["sum_rel_gpu_vs_oracle"] <= G.DRIFT_REL, r
+    rp, ci = layer.csr()
+    D = layer.drop_sets()
+    assert rp.size == layer.H * layer.nq + 1 and rp[-1] == ci.size
+    for h in range(layer.H):
+        for i in range(layer.nq):
+            k = ci[rp[h * layer.nq + i]:rp[h * layer.nq + i + 1]]
+            if i >= layer.nqc:
+                assert k.tolist() == list(range(layer.nb))
+            else:
+                assert k.size == layer.c_h[h] + layer.nb - layer.ncand
+                assert np.array_equal(k, np.nonzero(~D[h, i])[0])
+    rows = [(h, i) for h in range(layer.H) for i in range(layer.nq)]
+    if len(rows) > 60:
+        idx = np.random.default_rng(1).choice(len(rows), 48, replace=False)
+        rows = [rows[k] for k in sorted(idx)] + [(0, layer.nq - 1), (layer.H - 1, layer.nqc - 1)]
+    a = G.compare_attention(layer, rows)
+    assert a["max_abs"] <= G.ATT_MAX_ABS and a["mean_rel"] <= G.ATT_MEAN_REL, a
+
+
+@pytest.mark.parametrize("N,H,ns,c,R", [
+    (100, 1, 0, 1, 1),          # one ragged query block, two key blocks
+    (64 * 9 + 30, 2, 40, 3, 2),  # special tokens straddling the last query blocks
+    (1300, 2, 7, 20, 3),         # nothing dropped
+])
+def test_paper_grid_edge_shapes(N, H, ns, c, R):
+    inp = synth.make_random_layer(N, H, 64 * H, seed=N + 7 * H)
+    nc = O.n_candidates(N, ns)
+    c = min(c, nc)
+    layer = G.Layer(inp, ns, [c] * H, R, q_block=128).run()
+    r = G.compare_selection(layer, layer.oracle_select())
+    assert r["mismatched"] == 0, r
+    a = G.compare_attention(layer, [(h, i) for h in range(H) for i in range(layer.nq)])
+    assert a["max_abs"] <= G.ATT_MAX_ABS and a["mean_rel"] <= G.ATT_MEAN_REL, a

@@ -470,3 +470,36 @@ def test_maximised_drift_variants(layer):
         key = O.cut_keys(O.drift_scores(r), P_i)[:pooled.n_cand]
         smallest = set(np.argsort(key, kind="stable")[:c[h]])
         assert set(np.nonzero(~full[k].D0[:pooled.n_cand])[0]) == smallest
+
+
+# ---------------------------------------------------------------------------------------
+# The paper's grid (Appendix F): 128-token query blocks over 64-token key blocks
+# ---------------------------------------------------------------------------------------
+def test_query_block_128_pooling_is_the_weighted_pair_mean(layer):
+    """A 128-token query block's mean is the token-count-weighted mean of its two 64-token
+    halves (the ragged tail included)."""
+    X, _ = layer
+    Q = X["Q"]
+    N = Q.shape[0]
+    q64 = O.pool_blocks(Q, 64)
+    q128 = O.pool_blocks(Q, 128)
+    for i in range(q128.shape[1]):
+        n0 = min(64, N - 128 * i)
+        n1 = max(0, min(64, N - 128 * i - 64))
+        want = (n0 * q64[:, 2 * i] + (n1 * q64[:, 2 * i + 1] if n1 else 0.0)) / (n0 + n1)
+        assert np.allclose(q128[:, i], want, rtol=1e-12, atol=1e-12)
+
+
+def test_query_block_128_attention_is_two_64_blocks_with_the_same_list(layer):
+    """Attention of a 128-token query block over a kept list equals that of its two 64-token
+    halves over the same list (each query token attends the same keys)."""
+    X, _ = layer
+    nb = O.n_blocks(X["Q"].shape[0])
+    rng = np.random.default_rng(3)
+    kept = {(0, i): np.sort(rng.choice(nb, 5, replace=False)) for i in range(3)}
+    a128 = O.block_sparse_attention(X["Q"], X["K"], X["V"], kept, list(kept), q_block=128)
+    kept64 = {(0, 2 * i + s): kept[(0, i)] for i in range(3) for s in range(2)}
+    a64 = O.block_sparse_attention(X["Q"], X["K"], X["V"], kept64, list(kept64))
+    for i in range(3):
+        assert np.allclose(a128[(0, i)], np.vstack([a64[(0, 2 * i)], a64[(0, 2 * i + 1)]]),
+                           rtol=1e-12, atol=1e-12)
