@@ -716,7 +716,7 @@ __global__ void __launch_bounds__(32 * kRowWarps, 8) k_score_rows(SelPtrs p, Bud
 // Restoration round r, per row: exact top-m restores and drops from the round-start state,
 // update, track-best.  grid (ceil(|P| / 4), H).  With a maximising variant the keys are the
 // increases of J and track-best keeps the largest J.
-__global__ void __launch_bounds__(32 * kRowWarps, 8) k_round_rows(SelPtrs p, Budgets bud,
+__global__ void __launch_bounds__(32 * kRowWarps, 10) k_round_rows(SelPtrs p, Budgets bud,
                                                                   int round, float rho,
                                                                   int maximize) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
