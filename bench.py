@@ -41,6 +41,8 @@ def parse(argv=None):
     ap.add_argument("--cpu-budget", type=float, default=15.0, help="seconds of oracle work")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--sweep", action="store_true", help="64-view sparsity x rounds sweep lines")
+    ap.add_argument("--q-block", type=int, default=64, choices=[64, 128],
+                    help="query block size: 64 (the configs' grid) or 128 (the paper's grid)")
     ap.add_argument("--variants", action="store_true",
                     help="drift of the ablation variants (probability, random, maximised) lines")
     return ap.parse_args(argv)
@@ -76,14 +78,16 @@ def kept_flops(row_ptr, col_idx, N, H, nb, q_block=64):
     return 4.0 * 64.0 * float((q * keys).sum())
 
 
-def selection_bytes(N, H, nb, ld, rounds, csr_entries):
+def selection_bytes(N, H, nb, ld, rounds, csr_entries, nq=None):
     """Algorithmic bytes of scoring + restoration, a fixed formula whatever the kernels move:
     read Q, K, V once and write P and q (score); per round read P and q and read/write the
-    drop masks (one bit per pair); write the CSR (col_idx and row_ptr)."""
-    mat = H * nb * nb * 4
+    drop masks (one bit per pair); write the CSR (col_idx and row_ptr).  Rows are the nq
+    query blocks (nb by default), columns the nb key blocks."""
+    nq = nb if nq is None else nq
+    mat = H * nq * nb * 4
     score = 3 * N * H * 64 * 2 + 2 * mat
-    per_round = 2 * mat + 2 * H * nb * nb // 8
-    return score + rounds * per_round + 4 * csr_entries + 4 * (H * nb + 1)
+    per_round = 2 * mat + 2 * H * nq * nb // 8
+    return score + rounds * per_round + 4 * csr_entries + 4 * (H * nq + 1)
 
 
 # ----------------------------------------------------------------------------------------
@@ -337,7 +341,8 @@ def run_ours(a, wl):
     local = int(os.environ.get("LOCAL_RANK", "0"))
     pool = None
     workers = os.cpu_count() or 1
-    if rank == 0 and world == 1 and not a.no_cpu_baseline:
+    # the oracle's row sampling follows the 64-token grid; no CPU baseline on the 128 grid
+    if rank == 0 and world == 1 and not a.no_cpu_baseline and a.q_block == 64:
         pool = make_pool(workers, wl.name)  # spawned processes, started before the first CUDA call
     import torch
     import synth
@@ -353,9 +358,9 @@ def run_ours(a, wl):
     Q, K, V, W = (dev(bits[k]) for k in ("Q", "K", "V", "W_o"))
     c_h = wl.budgets()
     N, H = wl.n_tokens, wl.heads
-    d = ress.dims(N, H, wl.n_special, wl.d_model)
+    d = ress.dims(N, H, wl.n_special, wl.d_model, a.q_block)
     buf = ress.Buffers(d, c_h)
-    nb = buf.nb
+    nb, nq, nqc = buf.nb, buf.nq, ress.num_query_candidates(d)
     ress.prepare_wo(d, W, buf.F)  # model-load time (Eq. 8), outside the step
     stream = torch.cuda.current_stream()
 
@@ -405,12 +410,12 @@ def run_ours(a, wl):
 
     rp = buf.row_ptr.cpu().numpy()
     ci = buf.col_idx.cpu().numpy()
-    flops = kept_flops(rp, ci, N, H, nb)
+    flops = kept_flops(rp, ci, N, H, nb, a.q_block)
     hbm, bf16, bf16_sus, peak_kind = peaks()
 
     # ---- dense run of the same attention kernel (no block dropped) -------------------
     dense = None
-    if wl.name == "vggt_v32":
+    if wl.name == "vggt_v32" and a.q_block == 64:
         rpd = torch.arange(0, H * nb * nb + 1, nb, dtype=torch.int32, device="cuda")
         cid = torch.arange(nb, dtype=torch.int32, device="cuda").repeat(H * nb)
         Od = torch.empty_like(buf.O)
@@ -447,7 +452,7 @@ def run_ours(a, wl):
 
     # ---- the paper's own grid: 128-token query blocks over 64-token key blocks ------
     paper_grid = None
-    if wl.name == "vggt_v32":
+    if wl.name == "vggt_v32" and a.q_block == 64:
         d2 = ress.dims(N, H, wl.n_special, wl.d_model, 128)
         buf2 = ress.Buffers(d2, c_h)
         ress.prepare_wo(d2, W, buf2.F)
@@ -562,11 +567,11 @@ def run_ours(a, wl):
 
     # ---- realised drift and sparsity ---------------------------------------------------
     Jb = buf.J_best.cpu().numpy().astype(np.float64)
-    J0 = buf.ws_view("J0", torch.float32).cpu().numpy()[:H * nb].astype(np.float64)
-    cand_rows = np.tile(np.arange(nb) < wl.n_candidates, H)
+    J0 = buf.ws_view("J0", torch.float32).cpu().numpy()[:H * nq].astype(np.float64)
+    cand_rows = np.tile(np.arange(nq) < nqc, H)
     kept_pairs = int(np.diff(rp.astype(np.int64)).sum())
 
-    sel_bytes = selection_bytes(N, H, nb, buf.layout.ld, wl.rounds, ci.size)
+    sel_bytes = selection_bytes(N, H, nb, buf.layout.ld, wl.rounds, ci.size, nq)
     sel_ms = score_ms + restore_ms
     dev = "cuda" if dist and dist.get_backend() == "nccl" else "cpu"
     ms_job, flops_job = job_totals(dist, ms, flops, dev)      # device-timed step
@@ -577,7 +582,8 @@ def run_ours(a, wl):
         "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
         "data": "synthetic (seeded VGGT-shaped Q/K/V and W_o; inputs 3x larger than L2, no flush)",
         "config": {"workload": wl.name, "views": wl.views, "heads": H, "tokens": N, "head_dim": 64,
-                   "block": 64, "sparsity": wl.sparsity, "rounds": wl.rounds, "rho": wl.rho,
+                   "block": 64, "q_block": a.q_block, "sparsity": wl.sparsity,
+                   "rounds": wl.rounds, "rho": wl.rho,
                    "c_h": int(c_h[0]), "parallelism": f"replicas{world}",
                    "l2": "inputs larger than L2 (270 MB Q/K/V at 32 views)"},
         "layer_ms": ms_job, "stage_ms": {"score": score_ms, "restore": restore_ms, "attn": attn_ms},
@@ -585,7 +591,7 @@ def run_ours(a, wl):
         "attn_tflops": flops / attn_ms / 1e9,
         "selection": {"algorithmic_bytes": sel_bytes, "gbs": sel_bytes / sel_ms / 1e6,
                       "frac_of_hbm": sel_bytes / sel_ms / 1e6 / hbm, "hbm_peak_gbs": hbm},
-        "kept_tflop": flops / 1e12, "realized_pair_sparsity": 1.0 - kept_pairs / (H * nb * nb),
+        "kept_tflop": flops / 1e12, "realized_pair_sparsity": 1.0 - kept_pairs / (H * nq * nb),
         "drift": {"sum_J_best": float(Jb[cand_rows].sum()), "sum_J0": float(J0[cand_rows].sum())},
         "dense": dense,
         "paper_grid": paper_grid,
@@ -593,7 +599,7 @@ def run_ours(a, wl):
         "roofline": {"bound": "tensor", "kernel": "k_attn (ress_sparse_attn)",
                      "achieved": flops / attn_ms / 1e9, "peak": bf16, "unit": "TFLOP/s",
                      "frac": flops / attn_ms / 1e9 / bf16,
-                     "traffic": attn_traffic() if wl.name == "vggt_v32" else None,
+                     "traffic": attn_traffic() if wl.name == "vggt_v32" and a.q_block == 64 else None,
                      "peak_kind": f"{peak_kind} bf16 burst"},
         # kernels the library enqueued inside the timed region (its own launch counter)
         "gpu_launches": launches,
