@@ -76,18 +76,19 @@ typedef struct {
 typedef struct {
   int64_t status;      /* uint32 status word (first device-side error, sticky)          */
   int64_t counter;     /* uint32 tile-scheduler counters of the attention kernel        */
-  int64_t qbar, kbar, vbar, ztil; /* [H, nb, 64] block means; z~_j = F_h V_j              */
-  int64_t ytil, gtil;  /* [H, nb, 64] y~_i = F_h v_bar_i (Eq. 1); g~ = F_h g (Eq. 10)    */
-  int64_t P, q, t;     /* [H, nb, ld] pooled P_ij, q_ij = ||F_h e_ij||^2 (Eq. 9), gains;
+  /* Rows i are the nq query blocks, columns j the nb key blocks (nq = nb on the 64 grid). */
+  int64_t qbar, kbar, vbar, ztil; /* [H, nq, 64] q_bar; [H, nb, 64] k_bar, V_bar, z~_j = F_h V_j */
+  int64_t ytil, gtil;  /* [H, nq, 64] y~_i = F_h v_bar_i (Eq. 1); g~ = F_h g (Eq. 10)    */
+  int64_t P, q, t;     /* [H, nq, ld] pooled P_ij, q_ij = ||F_h e_ij||^2 (Eq. 9), gains;
                           t doubles as the attention kernel's pair-list scratch            */
-  int64_t K, G, J, Jbest, J0; /* [H, nb] remaining mass, G, J of Eq. 12                  */
-  int64_t dmask, bmask; /* uint32 [H, nb, words] current and best drop sets (bit j)      */
-  int64_t plen;        /* int32 [H, ceil(nb/2)] union lengths of query-block pairs          */
-  int64_t asplit;      /* bf16 [3, H, nb, 64]: row operand as three bf16 terms (hi, mid, lo):
+  int64_t K, G, J, Jbest, J0; /* [H, nq] remaining mass, G, J of Eq. 12                  */
+  int64_t dmask, bmask; /* uint32 [H, nq, words] current and best drop sets (bit j)      */
+  int64_t plen;        /* int32 [H, ceil(nb/2)] lengths of the attention items' lists       */
+  int64_t asplit;      /* bf16 [3, H, nq, 64]: row operand as three bf16 terms (hi, mid, lo):
                           q_bar, then y~, then g~ (tensor-core products)                   */
   int64_t ksplit, zsplit; /* bf16 [3, H, nb, 64]: k_bar and z~ as three bf16 terms          */
-  int64_t cdot, ny, nz;   /* float [H, nb]: y~_i . g~_i, ||y~_i||^2, ||z~_j||^2              */
-  int64_t lstat;       /* float2 [H, nb, ceil(nb/128)]: per 128-block slice of a row of
+  int64_t cdot, ny, nz;   /* float [H, nq]: y~_i . g~_i, ||y~_i||^2; [H, nb]: ||z~_j||^2    */
+  int64_t lstat;       /* float2 [H, nq, ceil(nb/128)]: per 128-block slice of a row of
                           pooled logits, its max and sum of exp(logit - max)               */
   int64_t ld;          /* row stride of P, q, t                                          */
   int64_t words;       /* uint32 words per drop-set bitmask = ceil(nb / 32)              */
@@ -119,8 +120,8 @@ size_t ress_workspace_bytes(const ress_dims* dims);
 int ress_workspace_layout(const ress_dims* dims, ress_ws_layout* out);
 
 /* Entries of col_idx that ress_restore writes for the budgets c_h (host array [H]):
- * every candidate query row keeps c_h + (nb - |P|) blocks, every special query row keeps
- * all nb blocks.  -1 on invalid arguments. */
+ * every candidate query block keeps c_h + (nb - |P|) key blocks, every other query block
+ * keeps all nb.  -1 on invalid arguments. */
 int64_t ress_csr_capacity(const ress_dims* dims, const int32_t* c_h_host);
 
 /* Eq. 8 at model-load time.  W_o: device bf16 [d_model, H*64] (Linear.weight layout,
@@ -166,11 +167,12 @@ int ress_score_variant(const ress_dims* dims, const uint16_t* Q, const uint16_t*
  * Round r exchanges m_r = floor(rho c_h / 2^(r+1)) blocks (Eq. 17), capped by the sizes of
  * the two sides: the m_r restores and the m_r drops with the largest exact decrease of
  * J (Eq. 13-16), both taken from the round-start state.  The set with the smallest J seen
- * (track-best, strict <) is returned as kept-block lists in CSR form over the H*nb query
- * rows (h-major): row_ptr device int32 [H*nb + 1], col_idx device int32 [col_capacity] with
+ * (track-best, strict <) is returned as kept-block lists in CSR form over the H*nq query
+ * rows (h-major; nq query blocks, see ress_dims.q_block): row_ptr device int32 [H*nq + 1],
+ * col_idx device int32 [col_capacity] with
  * ascending block indices; col_capacity >= ress_csr_capacity().  Optional device outputs
- * (NULL to skip): J_best float [H*nb] (0 for special query rows), drop_mask uint32
- * [H*nb, ceil(nb/32)] (bit j of row (h, i) set when block j is dropped).
+ * (NULL to skip): J_best float [H*nq] (0 for special query rows), drop_mask uint32
+ * [H*nq, ceil(nb/32)] (bit j of row (h, i) set when key block j is dropped).
  * rounds in [0, 32]; rho in [0, 1]. */
 int ress_restore(const ress_dims* dims, const int32_t* c_h_host, int32_t rounds, float rho,
                  void* ws, size_t ws_bytes, int32_t* row_ptr, int32_t* col_idx,
@@ -184,7 +186,7 @@ int ress_restore_variant(const ress_dims* dims, const int32_t* c_h_host, int32_t
                          float* J_best, uint32_t* drop_mask, void* stream);
 
 /* Sec. 3 step (3): for every head h, query block i and query token of that block,
- * O = softmax(q K^T / 8) V over the tokens of the key blocks listed in row h*nb + i of the
+ * O = softmax(q K^T / 8) V over the tokens of the key blocks listed in row h*nq + i of the
  * CSR (renormalised among them); keys past N are excluded.  Q, K, V: device bf16 [N, H, 64];
  * O: device bf16 [N, H, 64].  Lists must hold ascending, distinct block indices < nb and be
  * non-empty; entries past col_capacity or >= nb are skipped and flagged as RESS_EDEVICE in
