@@ -521,3 +521,21 @@ def test_paper_grid_edge_shapes(N, H, ns, c, R):
     assert r["mismatched"] == 0, r
     a = G.compare_attention(layer, [(h, i) for h in range(H) for i in range(layer.nq)])
     assert a["max_abs"] <= G.ATT_MAX_ABS and a["mean_rel"] <= G.ATT_MEAN_REL, a
+
+
+def test_paper_grid_headline_shape_sampled():
+    """The 32-view headline layer on the paper's grid (128-token query blocks): sampled rows
+    of the selection and of the attention against the oracle, and J_best <= J0 on every
+    sparsified row."""
+    wl = synth.WORKLOADS["vggt_v32"]
+    layer = G.Layer(synth.make_inputs(wl), wl.n_special, wl.budgets(), wl.rounds, wl.rho,
+                    q_block=128).run()
+    rng = np.random.default_rng(2)
+    rows = [(int(h), int(i)) for h, i in zip(rng.integers(0, wl.heads, 20), rng.integers(0, layer.nqc, 20))]
+    r = G.compare_selection(layer, layer.oracle_select(rows))
+    assert r["mismatched"] == 0, r
+    J0 = layer.ws("J0", shape=(layer.H, layer.nq))
+    Jb = layer.buf.J_best.cpu().numpy().reshape(layer.H, layer.nq)
+    assert np.all(Jb[:, :layer.nqc] <= J0[:, :layer.nqc])
+    a = G.compare_attention(layer, rows[:8] + [(0, layer.nq - 1), (7, layer.nqc - 1)])
+    assert a["max_abs"] <= G.ATT_MAX_ABS and a["mean_rel"] <= G.ATT_MEAN_REL, a
