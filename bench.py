@@ -45,6 +45,8 @@ def parse(argv=None):
                     help="query block size: 64 (the configs' grid) or 128 (the paper's grid)")
     ap.add_argument("--variants", action="store_true",
                     help="drift of the ablation variants (probability, random, maximised) lines")
+    ap.add_argument("--cdf", type=float, default=0.9,
+                    help="threshold tau of the CDF-threshold variant in --variants")
     return ap.parse_args(argv)
 
 
@@ -677,7 +679,7 @@ def variants(a, wl):
     Q, K, V, W = (dev(bits[k]) for k in ("Q", "K", "V", "W_o"))
     c_h = wl.budgets()
     d = ress.dims(wl.n_tokens, wl.heads, wl.n_special, wl.d_model)
-    buf = ress.Buffers(d, c_h)
+    buf = ress.Buffers(d, c_h, variant=ress.variant(cdf=1.0))  # room for whole rows
     ress.prepare_wo(d, W, buf.F)
     H, nb, nc = wl.heads, buf.nb, wl.n_candidates
     rpd = torch.arange(0, H * nb * nb + 1, nb, dtype=torch.int32, device="cuda")
@@ -685,19 +687,24 @@ def variants(a, wl):
     Od = torch.empty_like(buf.O)
     ress.sparse_attn(d, Q, K, V, rpd, cid, Od, buf.ws)
     drift = torch.empty(nb, dtype=torch.float32, device="cuda")
-    cases = [("ress", "drift", "none", wl.rounds), ("probability", "probability", "none", 0),
-             ("random", "random", "none", 0), ("maximize_swap", "drift", "swap", wl.rounds),
-             ("maximize_full", "drift", "full", wl.rounds)]
-    for name, key, mx, R in cases:
-        v = ress.variant(key, mx, seed=1)
+    cases = [("ress", "drift", "none", wl.rounds, 0.0),
+             ("probability", "probability", "none", 0, 0.0),
+             ("probability_cdf", "probability", "none", 0, a.cdf),  # top-k plus the CDF rule
+             ("random", "random", "none", 0, 0.0), ("maximize_swap", "drift", "swap", wl.rounds, 0.0),
+             ("maximize_full", "drift", "full", wl.rounds, 0.0)]
+    for name, key, mx, R, cdf in cases:
+        v = ress.variant(key, mx, seed=1, cdf=cdf)
         ress.score(d, Q, K, V, buf.F, c_h, buf.ws, variant=v)
         ress.restore(d, c_h, R, wl.rho, buf.ws, buf.row_ptr, buf.col_idx, buf.J_best, variant=v)
         ress.sparse_attn(d, Q, K, V, buf.row_ptr, buf.col_idx, buf.O, buf.ws)
         ress.token_drift(d, buf.O, Od, W, drift, buf.ws)
         ress.status(buf.ws)
         Jb = buf.J_best.cpu().numpy().reshape(H, nb)[:, :nc].astype(np.float64)
+        kept = int(buf.row_ptr[-1].item())  # CSR entries: every query row's kept key blocks
         print(json.dumps({"variants": wl.name, "variant": name, "key": key, "maximize": mx,
-                          "rounds": R, "c_h": int(c_h[0]), "sum_J_best": float(Jb.sum()),
+                          "rounds": R, "cdf": cdf, "c_h": int(c_h[0]),
+                          "kept_block_fraction": kept / float(H * nb * nb),
+                          "sum_J_best": float(Jb.sum()),
                           "token_drift": float(drift.cpu().numpy().astype(np.float64).sum())}),
               flush=True)
 

@@ -36,7 +36,7 @@
 extern "C" {
 #endif
 
-#define RESS_ABI_VERSION 4
+#define RESS_ABI_VERSION 5
 #define RESS_HEAD_DIM 64
 #define RESS_BLOCK 64
 #define RESS_MAX_HEADS 32
@@ -90,6 +90,7 @@ typedef struct {
   int64_t cdot, ny, nz;   /* float [H, nq]: y~_i . g~_i, ||y~_i||^2; [H, nb]: ||z~_j||^2    */
   int64_t lstat;       /* float2 [H, nq, ceil(nb/128)]: per 128-block slice of a row of
                           pooled logits, its max and sum of exp(logit - max)               */
+  int64_t kcount;      /* int32 [H, nq]: key blocks kept by each candidate query row       */
   int64_t ld;          /* row stride of P, q, t                                          */
   int64_t words;       /* uint32 words per drop-set bitmask = ceil(nb / 32)              */
   int64_t total;       /* bytes                                                          */
@@ -155,10 +156,25 @@ typedef struct {
   int32_t key;       /* ress_key_kind  */
   int32_t direction; /* ress_direction */
   uint64_t seed;     /* RESS_KEY_RANDOM */
+  float cdf;         /* 0: off.  tau in (0, 1]: the CDF threshold of Table 3 (the top-p rule
+                        of probability-based selection on the pooled map).  After its c_h
+                        largest keys a candidate row keeps further candidates in key order
+                        (ties to the lower index) until the pooled mass P of its kept blocks,
+                        the always-kept ones included, reaches tau.  Row lengths then depend
+                        on the data; needs rounds = 0 and direction RESS_MINIMIZE.        */
+  int32_t reserved;  /* must be 0 */
 } ress_variant;
 
+/* col_idx entries that ress_restore_variant may write for this variant: ress_csr_capacity
+ * for a fixed budget; with a CDF threshold every query row may keep all nb key blocks, so
+ * H * nq * nb.  The entries actually written are row_ptr[H * nq] after the call.  -1 on
+ * invalid arguments. */
+int64_t ress_csr_capacity_variant(const ress_dims* dims, const int32_t* c_h_host,
+                                  const ress_variant* variant);
+
 /* ress_score with a selection variant (NULL: ReSS).  RESS_EINVAL on an unknown key or
- * direction. */
+ * direction, a CDF threshold outside [0, 1] or combined with a maximising direction, or a
+ * nonzero reserved field. */
 int ress_score_variant(const ress_dims* dims, const uint16_t* Q, const uint16_t* K,
                        const uint16_t* V, const float* F, const int32_t* c_h_host,
                        const ress_variant* variant, void* ws, size_t ws_bytes, void* stream);
@@ -179,7 +195,9 @@ int ress_restore(const ress_dims* dims, const int32_t* c_h_host, int32_t rounds,
                  int64_t col_capacity, float* J_best, uint32_t* drop_mask, void* stream);
 
 /* ress_restore with a selection variant (NULL: ReSS); pass the same variant as to
- * ress_score_variant.  RESS_EINVAL on an unknown key or direction. */
+ * ress_score_variant.  RESS_EINVAL as ress_score_variant, or rounds > 0 with a CDF
+ * threshold.  With a CDF threshold the row lengths come from the device (row_ptr is a
+ * scan of the per-row kept counts) and col_capacity >= ress_csr_capacity_variant(). */
 int ress_restore_variant(const ress_dims* dims, const int32_t* c_h_host, int32_t rounds,
                          float rho, const ress_variant* variant, void* ws, size_t ws_bytes,
                          int32_t* row_ptr, int32_t* col_idx, int64_t col_capacity,

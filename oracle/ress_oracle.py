@@ -201,10 +201,16 @@ class Variant:
     maximize: "none" (ReSS minimises the drift), "swap" (restoration maximises J, the initial
               selection is unchanged) or "full" (the initial selection keeps the c_h smallest
               keys and restoration maximises J).
+    cdf:      0 (off) or a threshold tau in (0, 1]: the CDF threshold of Table 3 (the top-p
+              rule of probability-based selection on the pooled map).  Beyond its c_h
+              top-key candidates a row keeps further candidates, in key order (value desc,
+              index asc), until the pooled mass of its kept blocks, the always-kept ones
+              included, reaches tau.  Defined without restoration rounds.
     """
     key: str = "drift"
     maximize: str = "none"
     seed: int = 0
+    cdf: float = 0.0
 
 
 RESS = Variant()
@@ -251,7 +257,26 @@ def select_row(P_i, vbar_i, Vb_h, WOh, n_cand: int, c: int, rounds: int, rho: fl
     D[:n_cand] = True
     D[keep] = False
     margin = _gap(ranked(key[:n_cand]), c, 0.0)
-
+    if variant.cdf > 0:
+        if rounds:
+            raise ValueError("the CDF threshold is defined without restoration rounds")
+        tau = variant.cdf
+        mass = float(P_i[~D].sum())  # kept candidates and the always-kept blocks
+        rest = np.nonzero(D[:n_cand])[0]
+        order = rest[top_m(key[rest], rest.size)] if rest.size else rest
+        masses = [mass]
+        n_add = 0
+        while n_add < order.size and mass < tau:
+            mass += float(P_i[order[n_add]])
+            masses.append(mass)
+            n_add += 1
+        D[order[:n_add]] = False
+        # decision margins: every running mass against tau, and the key gaps on both sides
+        # of the last added block (a swap there changes which blocks cross the threshold)
+        margin = min([margin] + [abs(x - tau) / tau for x in masses])
+        if rest.size:
+            keys_sorted = ranked(key[rest])
+            margin = min(margin, _gap(keys_sorted, n_add, 0.0), _gap(keys_sorted, n_add - 1, 0.0))
     J, a, K = objective(D, P_i, r)
     res = RowSelection(h, i, False, D.copy(), D.copy(), J, J, [], margin)
     for m_r in swap_schedule(c, rounds, rho):

@@ -45,18 +45,21 @@ class Dims(ctypes.Structure):
 
 class Variant(ctypes.Structure):
     """ress_variant: selection variant of the ablations (key: 0 drift, 1 probability,
-    2 random; direction: 0 minimise, 1 restoration maximises, 2 everything maximises)."""
-    _fields_ = [("key", ctypes.c_int32), ("direction", ctypes.c_int32), ("seed", ctypes.c_uint64)]
+    2 random; direction: 0 minimise, 1 restoration maximises, 2 everything maximises;
+    cdf: 0, or the threshold tau of the CDF rule, which keeps further candidates until the
+    kept pooled mass reaches tau)."""
+    _fields_ = [("key", ctypes.c_int32), ("direction", ctypes.c_int32), ("seed", ctypes.c_uint64),
+                ("cdf", ctypes.c_float), ("reserved", ctypes.c_int32)]
 
 
 _KEYS = {"drift": 0, "probability": 1, "random": 2}
 _DIRECTIONS = {"none": 0, "swap": 1, "full": 2}
 
 
-def variant(key: str = "drift", maximize: str = "none", seed: int = 0) -> Variant:
+def variant(key: str = "drift", maximize: str = "none", seed: int = 0, cdf: float = 0.0) -> Variant:
     """A ress_variant from names: key in {drift, probability, random}, maximize in
-    {none, swap, full}."""
-    return Variant(_KEYS[key], _DIRECTIONS[maximize], seed)
+    {none, swap, full}; cdf the CDF threshold tau (0: off)."""
+    return Variant(_KEYS[key], _DIRECTIONS[maximize], seed, cdf, 0)
 
 
 class WsLayout(ctypes.Structure):
@@ -64,7 +67,7 @@ class WsLayout(ctypes.Structure):
     _fields_ = [(n, ctypes.c_int64) for n in
                 ("status", "counter", "qbar", "kbar", "vbar", "ztil", "ytil", "gtil", "P", "q", "t",
                  "K", "G", "J", "Jbest", "J0", "dmask", "bmask", "plen", "asplit", "ksplit", "zsplit",
-                 "cdot", "ny", "nz", "lstat", "ld", "words", "total")]
+                 "cdot", "ny", "nz", "lstat", "kcount", "ld", "words", "total")]
 
 
 _c = ctypes
@@ -80,6 +83,7 @@ _SIGS = {
     "ress_workspace_bytes": (_c.c_size_t, [_c.POINTER(Dims)]),
     "ress_workspace_layout": (_c.c_int, [_c.POINTER(Dims), _c.POINTER(WsLayout)]),
     "ress_csr_capacity": (_c.c_int64, [_c.POINTER(Dims), _P]),
+    "ress_csr_capacity_variant": (_c.c_int64, [_c.POINTER(Dims), _P, _c.POINTER(Variant)]),
     "ress_prepare_wo": (_c.c_int, [_c.POINTER(Dims), _P, _P, _P]),
     "ress_score": (_c.c_int, [_c.POINTER(Dims), _P, _P, _P, _P, _P, _P, _c.c_size_t, _P]),
     "ress_restore": (_c.c_int, [_c.POINTER(Dims), _P, _c.c_int32, _c.c_float, _P, _c.c_size_t,
@@ -165,8 +169,13 @@ def _budget_array(c_h):
     return arr
 
 
-def csr_capacity(d: Dims, c_h) -> int:
-    n = _lib.ress_csr_capacity(_c.byref(d), _c.cast(_budget_array(c_h), _P))
+def csr_capacity(d: Dims, c_h, variant: Variant = None) -> int:
+    """col_idx entries the restore may write (every row kept whole under a CDF threshold)."""
+    if variant is None:
+        n = _lib.ress_csr_capacity(_c.byref(d), _c.cast(_budget_array(c_h), _P))
+    else:
+        n = _lib.ress_csr_capacity_variant(_c.byref(d), _c.cast(_budget_array(c_h), _P),
+                                           _c.byref(variant))
     if n < 0:
         raise RessError(-1, _lib.ress_last_error().decode())
     return n
@@ -336,7 +345,7 @@ def status(ws, stream=None):
 class Buffers:
     """Device buffers of one layer shape (workspace, F, CSR, output), allocated by torch."""
 
-    def __init__(self, d: Dims, c_h, device="cuda"):
+    def __init__(self, d: Dims, c_h, device="cuda", variant: Variant = None):
         torch = _torch()
         self.d = d
         self.c_h = [int(c) for c in c_h]
@@ -346,7 +355,7 @@ class Buffers:
         self.ws = torch.zeros(workspace_bytes(d), dtype=torch.uint8, device=device)
         self.F = torch.zeros(H, 64, 64, dtype=torch.float32, device=device)
         self.row_ptr = torch.zeros(H * self.nq + 1, dtype=torch.int32, device=device)
-        self.col_idx = torch.zeros(csr_capacity(d, c_h), dtype=torch.int32, device=device)
+        self.col_idx = torch.zeros(csr_capacity(d, c_h, variant), dtype=torch.int32, device=device)
         self.O = torch.zeros(d.n_tokens, H, 64, dtype=torch.bfloat16, device=device)
         self.J_best = torch.zeros(H * self.nq, dtype=torch.float32, device=device)
         self.layout = workspace_layout(d)

@@ -235,6 +235,7 @@ struct SelPtrs {
   uint32_t* asplit;      // bf16x2 [3][H][nb][32]: g~ as three bf16 terms (tensor-core gains)
   float* cdot;           // [H, nb] y~_i . g~_i
   int64_t split_stride;  // H nb 32: uint32 words per term
+  int32_t* kcount;       // [H, nq] key blocks kept by each candidate row
 };
 
 __host__ __device__ inline SelPtrs sel_ptrs(const Shape& s, char* ws, const ress_ws_layout& L) {
@@ -263,6 +264,7 @@ __host__ __device__ inline SelPtrs sel_ptrs(const Shape& s, char* ws, const ress
   p.asplit = (uint32_t*)(ws + L.asplit);
   p.cdot = (float*)(ws + L.cdot);
   p.split_stride = (int64_t)s.H * s.nq * 32;
+  p.kcount = (int32_t*)(ws + L.kcount);
   return p;
 }
 
@@ -648,6 +650,63 @@ __device__ __forceinline__ unsigned long long splitmix64(unsigned long long x) {
   return z ^ (z >> 31);
 }
 
+// CDF threshold (Table 3, the top-p rule of probability-based selection): after the c_h
+// largest keys a row keeps further candidates in key order (ties to the lower index) until
+// the pooled mass of its kept blocks, the always-kept ones included, reaches tau.  kk holds
+// the candidates' keys and D the drop set (the candidates not yet kept).  The blocks that
+// join are the shortest prefix of D in key order whose mass reaches tau - (kept mass); it
+// is found without sorting: bit by bit, the largest key T such that the mass of the blocks
+// of D with key >= T still reaches that need, then, among the blocks whose key is exactly T,
+// the shortest prefix by index.  Each pass sums per lane in ascending j and then across the
+// warp in a fixed order, so a pass's sum never decreases when its set grows.
+__device__ void cdf_extend(const uint32_t* kk, const float* __restrict__ Prow, uint32_t* D,
+                           int ncand, int nb, int words, float tau) {
+  const int lane = threadIdx.x & 31;
+  auto in_D = [&](int j) { return ((D[j >> 5] >> (j & 31)) & 1u) != 0u; };
+  float kept = 0.f;
+  for (int j = lane; j < nb; j += 32)
+    if (!in_D(j)) kept += Prow[j];
+  const float need = tau - warp_sum(kept);
+  if (!(need > 0.f)) return;
+  auto mass_from = [&](uint32_t T) {  // mass of the blocks of D with key >= T
+    float s = 0.f;
+    for (int j = lane; j < ncand; j += 32)
+      if (in_D(j) && kk[j] >= T) s += Prow[j];
+    return warp_sum(s);
+  };
+  uint32_t T = 0u;  // mass_from(T) >= need holds throughout, unless even all of D falls short
+  int L = ncand;    // the blocks with key T and index <= L join
+  if (mass_from(0u) >= need) {
+    for (int bit = 31; bit >= 0; --bit) {
+      const uint32_t cand = T | (1u << bit);
+      if (mass_from(cand) >= need) T = cand;
+    }
+    // every block with key > T is needed (their mass alone falls short); the ties at T join
+    // in ascending index until the rest of the need is met
+    const float need_t = need - (T == 0xffffffffu ? 0.f : mass_from(T + 1u));
+    auto tie_mass_below = [&](int x) {
+      float s = 0.f;
+      for (int j = lane; j < min(x, ncand); j += 32)
+        if (in_D(j) && kk[j] == T) s += Prow[j];
+      return warp_sum(s);
+    };
+    L = 0;  // the largest L with the ties below index L still short of need_t
+    for (int bit = 12; bit >= 0; --bit) {
+      const int cand = L | (1 << bit);
+      if (cand <= ncand && tie_mass_below(cand) < need_t) L = cand;
+    }
+  }
+  for (int w = 0; w < words; ++w) {
+    const int j = w * 32 + lane;
+    const bool joins =
+        j < ncand && in_D(j) && (kk[j] > T || (kk[j] == T && j <= L));
+    const uint32_t m = __ballot_sync(kFull, joins);
+    __syncwarp();
+    if (lane == 0) D[w] &= ~m;
+    __syncwarp();
+  }
+}
+
 // Initial selection (Eq. 7) and the state of Eq. 10-12.  grid (ceil(|P| / 4), H).
 // The variant picks the key: the Eq. 7 drift key (ReSS), the pooled probability, or the top
 // 24 bits of SplitMix64 at seed + (h 4096 + i) 4096 + j; the full sign flip keeps the
@@ -686,12 +745,18 @@ __global__ void __launch_bounds__(32 * kRowWarps, 8) k_score_rows(SelPtrs p, Bud
   });
   warp_topm(kk, p.ncand, bud.c[h], sel, p.words, sk, si);  // sel = kept candidates
   // drop set D0 = candidates not kept
+  for (int w = lane; w < p.words; w += 32) sel[w] = valid_bits(w, p.ncand) & ~sel[w];
+  __syncwarp();
+  if (v.cdf > 0.f) cdf_extend(kk, Prow, sel, p.ncand, p.nb, p.words, v.cdf);
+  int ndrop = 0;
   for (int w = lane; w < p.words; w += 32) {
-    const uint32_t d = valid_bits(w, p.ncand) & ~sel[w];
-    sel[w] = d;
+    const uint32_t d = sel[w];
     p.dmask[ri * p.words + w] = d;
     p.bmask[ri * p.words + w] = d;
+    ndrop += __popc(d);
   }
+  ndrop = __reduce_add_sync(kFull, ndrop);
+  if (lane == 0) p.kcount[ri] = p.nb - ndrop;
   __syncwarp();
   const float2 y = *reinterpret_cast<const float2*>(p.ytil + ri * 64 + 2 * lane);
   float g0, g1, K;
@@ -798,18 +863,61 @@ struct CsrBases {
   int64_t base[RESS_MAX_HEADS + 1];
 };
 
+// Row offsets of variable-length kept lists (CDF threshold): row_ptr = exclusive scan of the
+// kept counts over the H * nq rows (candidate rows: kcount; special query rows: nb).  One
+// CTA of 1024 threads, each owning a contiguous run of rows.
+__global__ void __launch_bounds__(1024) k_rowptr(const int32_t* __restrict__ kcount, int H,
+                                                 int nq, int nqc, int nb,
+                                                 int32_t* __restrict__ row_ptr) {
+  __shared__ long long wsum[32];
+  const long long R = (long long)H * nq;
+  const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
+  const long long per = (R + 1023) / 1024;
+  const long long r0 = min(R, (long long)t * per), r1 = min(R, r0 + per);
+  auto count = [&](long long r) -> long long { return (r % nq) >= nqc ? nb : kcount[r]; };
+  long long local = 0;
+  for (long long r = r0; r < r1; ++r) local += count(r);
+  long long inc = local;  // inclusive scan over the warp, then over the warps
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const long long y = __shfl_up_sync(kFull, inc, o);
+    if (lane >= o) inc += y;
+  }
+  if (lane == 31) wsum[warp] = inc;
+  __syncthreads();
+  if (warp == 0) {
+    long long w = wsum[lane];
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const long long y = __shfl_up_sync(kFull, w, o);
+      if (lane >= o) w += y;
+    }
+    wsum[lane] = w;
+  }
+  __syncthreads();
+  long long off = inc - local + (warp ? wsum[warp - 1] : 0);
+  for (long long r = r0; r < r1; ++r) {
+    row_ptr[r] = (int32_t)off;
+    off += count(r);
+  }
+  if (t == 1023) row_ptr[R] = (int32_t)off;
+}
+
 __global__ void k_csr(SelPtrs p, Budgets bud, CsrBases cb, int H, int32_t* __restrict__ row_ptr,
                       int32_t* __restrict__ col_idx, int64_t cap, float* __restrict__ J_best,
-                      uint32_t* __restrict__ drop_mask, uint32_t* status) {
+                      uint32_t* __restrict__ drop_mask, uint32_t* status, bool variable) {
   const int i = blockIdx.x * 8 + (threadIdx.x >> 5), h = blockIdx.y, lane = threadIdx.x & 31;
   if (i >= p.nq) return;
   const int64_t ri = (int64_t)h * p.nq + i;
   const int c = bud.c[h];
   const int ns = p.nb - p.ncand;  // always-kept key blocks
   const bool dense = i >= p.nqc;
-  const int64_t off = cb.base[h] + (dense ? (int64_t)p.nqc * (c + ns) + (int64_t)(i - p.nqc) * p.nb
-                                          : (int64_t)i * (c + ns));
-  const int expect = dense ? p.nb : c + ns;
+  // fixed budgets: offsets by formula; variable lengths: the offsets k_rowptr wrote
+  const int64_t off = variable ? (int64_t)row_ptr[ri]
+                               : cb.base[h] + (dense ? (int64_t)p.nqc * (c + ns) +
+                                                           (int64_t)(i - p.nqc) * p.nb
+                                                     : (int64_t)i * (c + ns));
+  const int expect = variable ? (int)(row_ptr[ri + 1] - off) : (dense ? p.nb : c + ns);
   int pos = 0;
   for (int w0 = 0; w0 < p.words; w0 += 32) {
     // 32 words per coalesced load, handed out by shuffle
@@ -828,8 +936,10 @@ __global__ void k_csr(SelPtrs p, Budgets bud, CsrBases cb, int H, int32_t* __res
   }
   if (lane == 0) {
     if (pos != expect) flag_status(status, kStatusBadRow);
-    row_ptr[ri] = (int32_t)off;
-    if (h == H - 1 && i == p.nq - 1) row_ptr[(int64_t)H * p.nq] = (int32_t)cb.base[H];
+    if (!variable) {
+      row_ptr[ri] = (int32_t)off;
+      if (h == H - 1 && i == p.nq - 1) row_ptr[(int64_t)H * p.nq] = (int32_t)cb.base[H];
+    }
     if (J_best) J_best[ri] = dense ? 0.f : p.Jbest[ri];
   }
 }
@@ -903,8 +1013,13 @@ cudaError_t launch_csr(const SelectArgs& a, const int64_t* head_base, int32_t* r
   SelPtrs p = sel_ptrs(s, a.ws, a.L);
   CsrBases cb;
   for (int h = 0; h <= s.H; ++h) cb.base[h] = head_base[h];
+  const bool variable = a.v.cdf > 0.f;
+  if (variable) {
+    k_rowptr<<<1, 1024, 0, st>>>(p.kcount, s.H, s.nq, s.nqc, s.nb, row_ptr);
+    note_launch();
+  }
   k_csr<<<dim3((s.nq + 7) / 8, s.H), 256, 0, st>>>(p, budgets_of(a), cb, s.H, row_ptr, col_idx, col_capacity,
-                                        J_best, drop_mask, (uint32_t*)(a.ws + a.L.status));
+                                        J_best, drop_mask, (uint32_t*)(a.ws + a.L.status), variable);
   note_launch();
   return cudaGetLastError();
 }

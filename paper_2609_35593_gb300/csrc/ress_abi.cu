@@ -102,19 +102,24 @@ ress::SelectArgs select_args(const ress::Shape& s, const uint16_t* Q, const uint
   a.ws = static_cast<char*>(ws);
   a.L = L;
   for (int h = 0; h < RESS_MAX_HEADS; ++h) a.c[h] = (c && h < s.H) ? c[h] : 0;
-  a.v = ress::Variant{0, 0, 0ull};
+  a.v = ress::Variant{0, 0, 0ull, 0.0f};
   return a;
 }
 
 // NULL -> ReSS; otherwise the variant after a range check.
 int check_variant(const ress_variant* v, ress::Variant* out) {
-  *out = ress::Variant{0, 0, 0ull};
+  *out = ress::Variant{0, 0, 0ull, 0.0f};
   if (!v) return RESS_OK;
   if (v->key < RESS_KEY_DRIFT || v->key > RESS_KEY_RANDOM)
     return fail(RESS_EINVAL, "variant key %d unknown", v->key);
   if (v->direction < RESS_MINIMIZE || v->direction > RESS_MAXIMIZE_FULL)
     return fail(RESS_EINVAL, "variant direction %d unknown", v->direction);
-  *out = ress::Variant{v->key, v->direction, (unsigned long long)v->seed};
+  if (!(v->cdf >= 0.0f && v->cdf <= 1.0f))
+    return fail(RESS_EINVAL, "variant cdf %g outside [0, 1]", (double)v->cdf);
+  if (v->cdf > 0.0f && v->direction != RESS_MINIMIZE)
+    return fail(RESS_EINVAL, "a CDF threshold needs direction RESS_MINIMIZE");
+  if (v->reserved != 0) return fail(RESS_EINVAL, "variant reserved field is %d, not 0", v->reserved);
+  *out = ress::Variant{v->key, v->direction, (unsigned long long)v->seed, v->cdf};
   return RESS_OK;
 }
 
@@ -172,6 +177,18 @@ int64_t ress_csr_capacity(const ress_dims* d, const int32_t* c) {
   return base[s.H];
 }
 
+int64_t ress_csr_capacity_variant(const ress_dims* d, const int32_t* c, const ress_variant* v) {
+  if (check_dims(d)) return -1;
+  const ress::Shape s = ress::make_shape(*d);
+  if (check_budgets(s, c)) return -1;
+  ress::Variant var;
+  if (check_variant(v, &var)) return -1;
+  if (var.cdf > 0.0f) return (int64_t)s.H * s.nq * s.nb;
+  int64_t base[RESS_MAX_HEADS + 1];
+  head_bases(s, c, base);
+  return base[s.H];
+}
+
 int ress_prepare_wo(const ress_dims* d, const uint16_t* W_o, float* F, void* stream) {
   int e = check_dims(d);
   if (e) return e;
@@ -221,14 +238,19 @@ int ress_restore_variant(const ress_dims* d, const int32_t* c_h, int32_t rounds,
   if ((e = check_ptr(row_ptr, 4, "row_ptr")) || (e = check_ptr(col_idx, 4, "col_idx"))) return e;
   if (J_best && (e = check_ptr(J_best, 4, "J_best"))) return e;
   if (drop_mask && (e = check_ptr(drop_mask, 4, "drop_mask"))) return e;
-  int64_t base[RESS_MAX_HEADS + 1];
-  head_bases(s, c_h, base);
-  if (col_capacity < base[s.H])
-    return fail(RESS_EWORKSPACE, "col_capacity %lld < %lld", (long long)col_capacity, (long long)base[s.H]);
-  if (base[s.H] > INT32_MAX) return fail(RESS_EUNSUPPORTED, "CSR larger than 2^31 entries");
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   ress::SelectArgs a = select_args(s, nullptr, nullptr, nullptr, nullptr, c_h, ws, L);
   if ((e = check_variant(variant, &a.v))) return e;
+  if (a.v.cdf > 0.0f && rounds != 0)
+    return fail(RESS_EINVAL, "a CDF threshold is defined without restoration rounds (rounds %d)", rounds);
+  int64_t base[RESS_MAX_HEADS + 1];
+  head_bases(s, c_h, base);
+  // a CDF threshold may keep every key block of every row; the lists are written then at
+  // the offsets of a device-side scan of the kept counts
+  const int64_t need = a.v.cdf > 0.0f ? (int64_t)s.H * s.nq * s.nb : base[s.H];
+  if (col_capacity < need)
+    return fail(RESS_EWORKSPACE, "col_capacity %lld < %lld", (long long)col_capacity, (long long)need);
+  if (need > INT32_MAX) return fail(RESS_EUNSUPPORTED, "CSR larger than 2^31 entries");
   for (int r = 0; r < rounds; ++r) {
     cudaError_t ce = ress::launch_round(a, r, rho, st);
     if (ce != cudaSuccess) return cuda_fail(ce, "ress_restore round");

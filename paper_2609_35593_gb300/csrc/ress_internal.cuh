@@ -83,6 +83,7 @@ inline ress_ws_layout make_layout(const Shape& s) {
   L.ny = take(row);
   L.nz = take((int64_t)s.H * s.nb * 4);
   L.lstat = take((int64_t)s.H * s.nq * ((s.nb + 127) / 128) * 8);
+  L.kcount = take(row);
   L.ld = s.ld;
   L.words = s.words;
   L.total = off;
@@ -155,6 +156,7 @@ struct Variant {
   int key;        // 0 drift (Eq. 7), 1 pooled probability, 2 random
   int direction;  // 0 minimise J, 1 restoration maximises J, 2 initial selection too
   unsigned long long seed;
+  float cdf;      // 0 off; tau: keep further candidates until the kept mass reaches tau
 };
 
 struct SelectArgs {

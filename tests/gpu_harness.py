@@ -51,7 +51,7 @@ class Layer:
         self.K = bits_to_device(inputs["K"])
         self.V = bits_to_device(inputs["V"])
         self.W = bits_to_device(inputs["W_o"])
-        self.buf = ress.Buffers(self.d, self.c_h)
+        self.buf = ress.Buffers(self.d, self.c_h, variant=self.device_variant())
         self.O32 = torch.zeros(self.N, self.H, 64, dtype=torch.float32, device="cuda")
         self.nb = self.buf.nb                          # key blocks
         self.nq = self.buf.nq                          # query blocks (selection and CSR rows)
@@ -59,11 +59,15 @@ class Layer:
         self.nqc = ress.num_query_candidates(self.d)   # sparsified query blocks
 
     # ---- GPU -----------------------------------------------------------------------
+    def device_variant(self):
+        """The library's ress_variant for the oracle's Variant (None: ReSS)."""
+        v = self.variant
+        return None if v is None else self.ress.variant(v.key, v.maximize, v.seed, v.cdf)
+
     def run(self, attention: bool = True):
         r, b = self.ress, self.buf
         r.prepare_wo(self.d, self.W, b.F)
-        v = None if self.variant is None else r.variant(self.variant.key, self.variant.maximize,
-                                                          self.variant.seed)
+        v = self.device_variant()
         r.score(self.d, self.Q, self.K, self.V, b.F, self.c_h, b.ws, variant=v)
         r.restore(self.d, self.c_h, self.rounds, self.rho, b.ws, b.row_ptr, b.col_idx, b.J_best,
                   variant=v)

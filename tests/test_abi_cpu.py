@@ -23,7 +23,7 @@ def test_every_declared_function_is_exported():
         assert hasattr(ress._lib, n), n
     for n in ("ress_score", "ress_restore", "ress_sparse_attn", "ress_forward"):
         assert n in names
-    assert ress._lib.ress_abi_version() == 4
+    assert ress._lib.ress_abi_version() == 5
 
 
 @pytest.mark.parametrize("name", list(synth.WORKLOADS))
@@ -130,7 +130,42 @@ def test_launch_counter_is_exported_and_monotone():
 def test_variant_names_map_to_the_header_values():
     v = ress.variant("random", "full", seed=9)
     assert (v.key, v.direction, v.seed) == (2, 2, 9)
+    assert ress.variant(cdf=0.75).cdf == 0.75 and ctypes.sizeof(ress.Variant) == 24
     assert (ress.variant().key, ress.variant().direction) == (0, 0)
+
+
+def test_cdf_variant_capacity_and_validation():
+    """A CDF threshold may keep every block: the capacity is H * nq * nb.  Out-of-range
+    thresholds, a maximising direction, a nonzero reserved field and restoration rounds
+    are rejected on the host (fake device pointers: nothing is launched)."""
+    wl = synth.WORKLOADS["vggt_v8"]
+    c = wl.budgets()
+    for qb in (64, 128):
+        d = ress.dims(wl.n_tokens, wl.heads, wl.n_special, wl.d_model, qb)
+        nq, nb = ress.num_query_blocks(d), ress.num_blocks(d)
+        assert ress.csr_capacity(d, c, ress.variant(cdf=0.9)) == wl.heads * nq * nb
+        assert ress.csr_capacity(d, c, ress.variant(key="probability")) == ress.csr_capacity(d, c)
+    d = ress.dims(wl.n_tokens, wl.heads, wl.n_special, wl.d_model)
+    bad = [ress.variant(cdf=1.5), ress.variant(cdf=-0.1), ress.variant(maximize="swap", cdf=0.5),
+           ress.variant(cdf=float("nan"))]
+    r = ress.variant(cdf=0.5)
+    r.reserved = 1
+    bad.append(r)
+    for v in bad:
+        with pytest.raises(ress.RessError):
+            ress.csr_capacity(d, c, v)
+    L = ress.workspace_layout(d)
+    cap = ress.csr_capacity(d, c, ress.variant(cdf=0.9))
+    ptr = ctypes.c_void_p(1 << 20)
+    budgets = (ctypes.c_int32 * len(c))(*[int(x) for x in c])
+    def restore(v, rounds, capacity):
+        return ress._lib.ress_restore_variant(ctypes.byref(d), ctypes.cast(budgets, ctypes.c_void_p),
+                                              rounds, 0.5, ctypes.byref(v), ptr, L.total, ptr,
+                                              ptr, capacity, None, None, None)
+    assert restore(ress.variant(cdf=0.9), 1, cap) == EINVAL
+    assert restore(ress.variant(cdf=0.9), 0, cap - 1) == EWORKSPACE
+    assert restore(ress.variant(cdf=2.0), 0, cap) == EINVAL
+    assert L.kcount > 0
 
 
 @pytest.mark.parametrize("name", ["tiny_v2", "vggt_v8", "vggt_v32"])

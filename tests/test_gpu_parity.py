@@ -467,6 +467,55 @@ def test_selection_variants(name, variant, rounds):
     assert r["worst_row_rel"] <= G.DRIFT_REL and r["sum_rel_gpu_vs_oracle"] <= G.DRIFT_REL, r
 
 
+@pytest.mark.parametrize("name,q_block", [("tiny_v2", 64), ("vggt_v8", 64), ("vggt_v8", 128)])
+@pytest.mark.parametrize("variant", [
+    O.Variant(key="probability", cdf=0.9),  # SparseVGGT's rule: top-k plus the CDF threshold
+    O.Variant(key="probability", cdf=0.5),
+    O.Variant(cdf=0.8),                     # the drift key with the threshold on top
+    O.Variant(key="random", seed=3, cdf=0.7),
+])
+def test_cdf_threshold_variant(name, q_block, variant):
+    """CDF threshold (Table 3): drop sets against the oracle row by row, variable-length
+    CSR rows (a device-side scan of the kept counts) that list exactly the kept blocks, the
+    kept mass of every row at least tau unless the row keeps everything, and attention over
+    those lists against the oracle on sampled rows."""
+    wl = synth.WORKLOADS[name]
+    layer = G.Layer(synth.make_inputs(wl), wl.n_special, wl.budgets(), 0, wl.rho,
+                    variant=variant, q_block=q_block).run()
+    sel = layer.oracle_select()
+    r = G.compare_selection(layer, sel)
+    assert r["mismatched"] == 0, r
+    assert r["exact"] >= 0.95 * (r["exact"] + r["near"]), r
+    assert r["worst_row_rel"] <= G.DRIFT_REL and r["sum_rel_gpu_vs_oracle"] <= G.DRIFT_REL, r
+    rp, ci = layer.csr()
+    D = layer.drop_sets()
+    P = layer.ws("P", shape=(layer.H, layer.nq, layer.buf.layout.ld))
+    lengths = np.diff(rp)
+    assert rp[0] == 0 and np.all(lengths >= 1) and rp[-1] <= ci.size
+    for h in range(layer.H):
+        for i in range(layer.nq):
+            k = ci[rp[h * layer.nq + i]:rp[h * layer.nq + i + 1]]
+            if i >= layer.nqc:
+                assert k.tolist() == list(range(layer.nb))
+                continue
+            assert np.array_equal(k, np.nonzero(~D[h, i])[0])
+            assert k.size >= layer.c_h[h] + layer.nb - layer.ncand
+            mass = float(P[h, i, k].astype(np.float64).sum())
+            assert mass >= variant.cdf - 1e-4 or k.size == layer.nb, (h, i, mass)
+    # the rule lengthens rows on the GPU exactly when it does in the oracle
+    fixed = np.array([layer.c_h[h] + layer.nb - layer.ncand for h in range(layer.H)])
+    gpu_ext = [lengths[h * layer.nq:h * layer.nq + layer.nqc].max() > fixed[h] for h in range(layer.H)]
+    ora_ext = [any((~sel[(h, i)].D_best).sum() > fixed[h] for i in range(layer.nqc))
+               for h in range(layer.H)]
+    assert gpu_ext == ora_ext
+    rows = [(h, i) for h in range(layer.H) for i in range(layer.nq)]
+    if len(rows) > 60:
+        idx = np.random.default_rng(2).choice(len(rows), 40, replace=False)
+        rows = [rows[k] for k in sorted(idx)] + [(layer.H - 1, layer.nq - 1)]
+    a = G.compare_attention(layer, rows)
+    assert a["max_abs"] <= G.ATT_MAX_ABS and a["mean_rel"] <= G.ATT_MEAN_REL, a
+
+
 def test_invalid_variant_is_rejected(tiny):
     import paper_2609_35593_gb300 as ress
     bad = ress.Variant(7, 0, 0)

@@ -472,6 +472,55 @@ def test_maximised_drift_variants(layer):
         assert set(np.nonzero(~full[k].D0[:pooled.n_cand])[0]) == smallest
 
 
+def test_cdf_threshold_probability_key_is_top_p(layer):
+    """CDF threshold on the probability key (Table 3's "+ CDF threshold" row): the kept
+    candidates are the first n of a stable descending argsort of P, n the larger of c_h and
+    the shortest prefix whose mass, with the always-kept blocks, reaches tau (np.cumsum)."""
+    for tau in (0.3, 0.6, 0.9, 0.99):
+        pooled, c, sel = _variant_rows(layer, O.Variant(key="probability", cdf=tau), rounds=0)
+        nc = pooled.n_cand
+        for (h, i), s in sel.items():
+            P_i, _ = O.row_quantities(pooled, h, i)
+            order = np.argsort(-P_i[:nc], kind="stable")
+            reach = P_i[nc:].sum() + np.cumsum(P_i[order])
+            n_tau = int(np.searchsorted(reach >= tau, True)) + 1 if reach[-1] >= tau else nc
+            n = max(c[h], n_tau)
+            assert set(np.nonzero(~s.D_best[:nc])[0]) == set(order[:n]), (tau, h, i)
+
+
+def test_cdf_threshold_invariants(layer):
+    """With the drift key: a threshold at or below the mass of the top-c_h set changes
+    nothing; otherwise the kept set contains ReSS's initial set, its mass reaches tau, and
+    taking back its lowest-key added block falls below tau (the prefix is the shortest)."""
+    pooled, c, base = _variant_rows(layer, O.RESS, rounds=0)
+    _, _, low = _variant_rows(layer, O.Variant(cdf=1e-9), rounds=0)
+    assert all(np.array_equal(low[k].D_best, base[k].D_best) for k in base)
+    X = layer[0]
+    for tau in (0.5, 0.8, 0.95):
+        _, _, sel = _variant_rows(layer, O.Variant(cdf=tau), rounds=0)
+        for (h, i), s in sel.items():
+            P_i, vbar_i = O.row_quantities(pooled, h, i)
+            kept = ~s.D_best
+            assert (~base[(h, i)].D_best <= kept).all()
+            added = np.nonzero(kept & base[(h, i)].D_best)[0]
+            mass = P_i[kept].sum()
+            if added.size == 0:
+                assert P_i[~base[(h, i)].D_best].sum() >= tau or kept.all()
+                continue
+            _, _, r = O.residual_contributions(P_i, vbar_i, pooled.Vb[h],
+                                               O.head_projection(X["W_o"], h, 64))
+            key = O.cut_keys(O.drift_scores(r), P_i)
+            last = added[np.lexsort((-added, key[added]))[0]]  # lowest key, highest index
+            assert mass >= tau - 1e-12 or kept[:pooled.n_cand].all()
+            assert mass - P_i[last] < tau
+            # every added block outranks every candidate still dropped
+            still = np.nonzero(s.D_best[:pooled.n_cand])[0]
+            if still.size:
+                assert key[added].min() >= key[still].max()
+    with pytest.raises(ValueError):
+        _variant_rows(layer, O.Variant(cdf=0.9), rounds=1)
+
+
 # ---------------------------------------------------------------------------------------
 # The paper's grid (Appendix F): 128-token query blocks over 64-token key blocks
 # ---------------------------------------------------------------------------------------
