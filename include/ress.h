@@ -231,8 +231,13 @@ int ress_forward(const ress_dims* dims, const uint16_t* Q, const uint16_t* K, co
 /* ress_forward from host memory to host memory, for callers that keep a layer's Q, K, V
  * and O on the host (the paper has no counterpart: an interface, not part of the method).
  * Enqueued on `stream`, in order: host -> device copies of Q, K, V into the caller's device
- * buffers Q_dev, K_dev, V_dev, then ress_forward on them, then the device -> host copy of
- * O_dev into O_host; nothing waits for completion.  Host buffers should be page-locked (for
+ * buffers Q_dev, K_dev, V_dev, then ress_forward on them, with the output brought back while
+ * the attention still runs: the attention is split into up to 8 chunks of 128-token query
+ * rows, and as each chunk completes its rows of O_dev are copied into O_host on a copy
+ * stream the library owns (one per device, with a second compute stream for alternate
+ * chunks; both are joined back into `stream` before the call's work ends, so `stream`
+ * passing the call means O_host is complete).  Nothing waits for completion on the host.
+ * Host buffers should be page-locked (for
  * example cudaHostAlloc) for the copies to overlap other work; every buffer belongs to the
  * caller and must stay untouched until the stream has passed the call.  Two calls on two
  * streams with separate device buffers, workspaces and CSR arrays overlap one layer's copies

@@ -76,6 +76,7 @@ struct __align__(1024) AttnSmem {
 
 struct AttnParams {
   int N, H, nb, npairs, nitems;
+  int p0, p1;                   // pairs [p0, p1) of every head are this launch's items
   int rows_per_head, row_step;  // CSR row of item (h, p): h * rows_per_head + row_step * p
   int nsparse;           // pairs 0..nsparse-1 of a head hold only candidate query blocks
   const int32_t* row_ptr;
@@ -86,18 +87,20 @@ struct AttnParams {
   uint32_t* counter;
 };
 
-// Work order: the pairs that hold special (dense) query blocks of every head first (they
-// are the longest), then the remaining pairs head by head, so that the CTAs running at the
-// same time share one head's K and V in L2.
+// Work order within the launch's pairs [p0, p1): those that hold special (dense) query
+// blocks, of every head, first (they are the longest), then the others head by head, so
+// that the CTAs running at the same time share one head's K and V in L2.
 __device__ __forceinline__ void item_pair(const AttnParams& a, int item, int& h, int& p) {
-  const int ndense = a.npairs - a.nsparse;
+  const int dlo = max(a.p0, a.nsparse);  // first pair of the range with a dense block
+  const int ndense = max(0, a.p1 - dlo);
+  const int nsp = max(0, min(a.p1, a.nsparse) - a.p0);
   const int first = a.H * ndense;
   if (item < first) {
     h = item / ndense;
-    p = a.nsparse + item % ndense;
+    p = dlo + item % ndense;
   } else {
-    h = (item - first) / a.nsparse;
-    p = (item - first) % a.nsparse;
+    h = (item - first) / nsp;
+    p = a.p0 + (item - first) % nsp;
   }
 }
 
@@ -601,46 +604,63 @@ static int sm_count() {
   return n > 0 ? n : 1;
 }
 
-cudaError_t launch_sparse_attn(const AttnArgs& x, cudaStream_t st) {
+int attn_num_pairs(const Shape& s) { return (s.nb + 1) / 2; }
+
+cudaError_t launch_attn_pairs(const AttnArgs& x, cudaStream_t st) {
   const Shape& s = x.s;
+  const int npairs = attn_num_pairs(s);
+  const int pairs = s.H * npairs;
+  k_pairs<<<(pairs + 7) / 8, 256, 0, st>>>(x.row_ptr, x.col_idx, x.col_capacity, x.scratch_cap,
+                                           s.nb, npairs, s.H, s.qb == 128, x.plist, x.plen,
+                                           x.status);
+  note_launch();
+  return cudaGetLastError();
+}
+
+cudaError_t launch_attn_range(const AttnArgs& x, int p0, int p1, int slot, cudaStream_t st) {
+  const Shape& s = x.s;
+  const int npairs = attn_num_pairs(s);
+  if (p0 < 0 || p1 > npairs || p0 >= p1 || slot < 0 || slot >= kAttnCounterSlots)
+    return cudaErrorInvalidValue;
   CUtensorMap tq, tk, tv;
   if (!make_map(&tq, x.Q, s.N, s.H, kRows) || !make_map(&tk, x.K, s.N, s.H, 64) ||
       !make_map(&tv, x.V, s.N, s.H, 64))
     return cudaErrorInvalidValue;
-  const int npairs = (s.nb + 1) / 2;
-  const int pairs = s.H * npairs;
+  const int items = s.H * (p1 - p0);
   const bool qb128 = s.qb == 128;
-  k_pairs<<<(pairs + 7) / 8, 256, 0, st>>>(x.row_ptr, x.col_idx, x.col_capacity, x.scratch_cap,
-                                           s.nb, npairs, s.H, qb128, x.plist, x.plen, x.status);
-  note_launch();
-  cudaError_t e = cudaGetLastError();
-  if (e != cudaSuccess) return e;
-  e = cudaMemsetAsync(x.counter, 0, sizeof(uint32_t), st);
-  if (e != cudaSuccess) return e;
   AttnParams p;
   p.N = s.N;
   p.H = s.H;
   p.nb = s.nb;
   p.npairs = npairs;
+  p.p0 = p0;
+  p.p1 = p1;
   // items whose rows are all candidate query rows come first in each head's order
   p.nsparse = qb128 ? s.nqc : s.ncand / 2;
   p.rows_per_head = qb128 ? s.nq : s.nb;
   p.row_step = qb128 ? 1 : 2;
-  p.nitems = pairs;
+  p.nitems = items;
   p.row_ptr = x.row_ptr;
   p.plist = x.plist;
   p.plen = x.plen;
   p.O = x.O;
   p.status = x.status;
-  p.counter = x.counter;
+  p.counter = x.counter + slot;
   const size_t smem = sizeof(AttnSmem) + 1024;
   auto kern = x.out_f32 ? k_attn<true> : k_attn<false>;
-  e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
-  const int grid = min(pairs, 2 * sm_count());
+  const int grid = min(items, 2 * sm_count());
   kern<<<grid, kAttnThreads, smem, st>>>(tq, tk, tv, p);
   note_launch();
   return cudaGetLastError();
+}
+
+cudaError_t launch_sparse_attn(const AttnArgs& x, cudaStream_t st) {
+  cudaError_t e = launch_attn_pairs(x, st);
+  if (e != cudaSuccess) return e;
+  if ((e = cudaMemsetAsync(x.counter, 0, sizeof(uint32_t), st)) != cudaSuccess) return e;
+  return launch_attn_range(x, 0, attn_num_pairs(x.s), 0, st);
 }
 
 }  // namespace ress

@@ -6,6 +6,7 @@
 #include <string.h>
 
 #include <atomic>
+#include <mutex>
 
 #include "ress_internal.cuh"
 
@@ -76,6 +77,42 @@ int check_ws(const ress::Shape& s, void* ws, size_t ws_bytes, ress_ws_layout* L)
 
 int cuda_fail(cudaError_t e, const char* where) {
   return fail(RESS_ECUDA, "%s: %s", where, cudaGetErrorString(e));
+}
+
+// Streams and events the host-buffer forward owns: a second compute stream (the attention
+// runs as chunks of query rows that alternate between it and the caller's stream, so that a
+// chunk's CTAs take the SMs the previous chunk frees at its tail) and a copy stream that
+// brings each chunk's output rows to the host while later chunks compute.  Created once per
+// device on first use (never device memory); every call enqueues under one mutex because
+// it re-records the same events.
+constexpr int kOutChunks = 8;
+constexpr int kMaxDevices = 64;
+struct OverlapStreams {
+  cudaStream_t aux = nullptr, copy = nullptr;
+  cudaEvent_t ready = nullptr, copied = nullptr, done[kOutChunks] = {};
+};
+std::mutex g_overlap_mu;
+OverlapStreams g_overlap[kMaxDevices];
+
+cudaError_t overlap_streams(OverlapStreams** out) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
+  OverlapStreams& o = g_overlap[dev];
+  if (!o.copied) {
+    OverlapStreams n;
+    if ((e = cudaStreamCreateWithFlags(&n.aux, cudaStreamNonBlocking)) != cudaSuccess ||
+        (e = cudaStreamCreateWithFlags(&n.copy, cudaStreamNonBlocking)) != cudaSuccess ||
+        (e = cudaEventCreateWithFlags(&n.ready, cudaEventDisableTiming)) != cudaSuccess)
+      return e;
+    for (int c = 0; c < kOutChunks; ++c)
+      if ((e = cudaEventCreateWithFlags(&n.done[c], cudaEventDisableTiming)) != cudaSuccess) return e;
+    if ((e = cudaEventCreateWithFlags(&n.copied, cudaEventDisableTiming)) != cudaSuccess) return e;
+    o = n;
+  }
+  *out = &o;
+  return cudaSuccess;
 }
 
 // col_idx entries of one head: every candidate query block keeps c_h candidates plus the
@@ -267,20 +304,10 @@ int ress_restore(const ress_dims* d, const int32_t* c_h, int32_t rounds, float r
                               col_capacity, J_best, drop_mask, stream);
 }
 
-static int sparse_attn_impl(const ress_dims* d, const uint16_t* Q, const uint16_t* K,
-                            const uint16_t* V, const int32_t* row_ptr, const int32_t* col_idx,
-                            int64_t col_capacity, void* O, bool out_f32, void* ws, size_t ws_bytes,
-                            void* stream) {
-  int e = check_dims(d);
-  if (e) return e;
-  if ((e = check_ptr(Q, 16, "Q")) || (e = check_ptr(K, 16, "K")) || (e = check_ptr(V, 16, "V")) ||
-      (e = check_ptr(O, 16, "O")) || (e = check_ptr(row_ptr, 4, "row_ptr")) ||
-      (e = check_ptr(col_idx, 4, "col_idx")))
-    return e;
-  if (col_capacity < 0) return fail(RESS_EINVAL, "col_capacity %lld < 0", (long long)col_capacity);
-  const ress::Shape s = ress::make_shape(*d);
-  ress_ws_layout L;
-  if ((e = check_ws(s, ws, ws_bytes, &L))) return e;
+static ress::AttnArgs attn_args(const ress::Shape& s, const ress_ws_layout& L,
+                                const uint16_t* Q, const uint16_t* K, const uint16_t* V,
+                                const int32_t* row_ptr, const int32_t* col_idx,
+                                int64_t col_capacity, void* O, bool out_f32, void* ws) {
   char* w = static_cast<char*>(ws);
   ress::AttnArgs a;
   a.s = s;
@@ -297,6 +324,24 @@ static int sparse_attn_impl(const ress_dims* d, const uint16_t* Q, const uint16_
   a.plist = reinterpret_cast<int32_t*>(w + L.t);  // the gains buffer is free during attention
   a.plen = reinterpret_cast<int32_t*>(w + L.plen);
   a.scratch_cap = (int64_t)s.H * s.nq * s.ld;  // entries of the t array
+  return a;
+}
+
+static int sparse_attn_impl(const ress_dims* d, const uint16_t* Q, const uint16_t* K,
+                            const uint16_t* V, const int32_t* row_ptr, const int32_t* col_idx,
+                            int64_t col_capacity, void* O, bool out_f32, void* ws, size_t ws_bytes,
+                            void* stream) {
+  int e = check_dims(d);
+  if (e) return e;
+  if ((e = check_ptr(Q, 16, "Q")) || (e = check_ptr(K, 16, "K")) || (e = check_ptr(V, 16, "V")) ||
+      (e = check_ptr(O, 16, "O")) || (e = check_ptr(row_ptr, 4, "row_ptr")) ||
+      (e = check_ptr(col_idx, 4, "col_idx")))
+    return e;
+  if (col_capacity < 0) return fail(RESS_EINVAL, "col_capacity %lld < 0", (long long)col_capacity);
+  const ress::Shape s = ress::make_shape(*d);
+  ress_ws_layout L;
+  if ((e = check_ws(s, ws, ws_bytes, &L))) return e;
+  const ress::AttnArgs a = attn_args(s, L, Q, K, V, row_ptr, col_idx, col_capacity, O, out_f32, ws);
   cudaError_t ce = ress::launch_sparse_attn(a, static_cast<cudaStream_t>(stream));
   if (ce != cudaSuccess) return cuda_fail(ce, "ress_sparse_attn");
   return ok();
@@ -373,11 +418,46 @@ int ress_forward_host(const ress_dims* d, const uint16_t* Q_host, const uint16_t
     cudaError_t ce = cudaMemcpyAsync(dst[k], src[k], bytes, cudaMemcpyHostToDevice, st);
     if (ce != cudaSuccess) return cuda_fail(ce, "ress_forward_host input copy");
   }
-  if ((e = ress_forward(d, Q_dev, K_dev, V_dev, F, c_h, rounds, rho, ws, ws_bytes, row_ptr, col_idx,
-                        col_capacity, O_dev, J_best, stream)))
+  if ((e = ress_score(d, Q_dev, K_dev, V_dev, F, c_h, ws, ws_bytes, stream))) return e;
+  if ((e = ress_restore(d, c_h, rounds, rho, ws, ws_bytes, row_ptr, col_idx, col_capacity, J_best,
+                        nullptr, stream)))
     return e;
-  cudaError_t ce = cudaMemcpyAsync(O_host, O_dev, bytes, cudaMemcpyDeviceToHost, st);
-  if (ce != cudaSuccess) return cuda_fail(ce, "ress_forward_host output copy");
+  // attention in chunks of 128-token query rows; each chunk's output rows go to the host on
+  // the copy stream as soon as the chunk is done, while the next chunks compute
+  const ress::Shape s = ress::make_shape(*d);
+  ress_ws_layout L;
+  if ((e = check_ws(s, ws, ws_bytes, &L))) return e;
+  const ress::AttnArgs a =
+      attn_args(s, L, Q_dev, K_dev, V_dev, row_ptr, col_idx, col_capacity, O_dev, false, ws);
+  std::lock_guard<std::mutex> lock(g_overlap_mu);
+  OverlapStreams* o = nullptr;
+  cudaError_t ce = overlap_streams(&o);
+  if (ce != cudaSuccess) return cuda_fail(ce, "ress_forward_host streams");
+  if ((ce = ress::launch_attn_pairs(a, st)) != cudaSuccess ||
+      (ce = cudaMemsetAsync(a.counter, 0, kOutChunks * sizeof(uint32_t), st)) != cudaSuccess ||
+      (ce = cudaEventRecord(o->ready, st)) != cudaSuccess ||
+      (ce = cudaStreamWaitEvent(o->aux, o->ready, 0)) != cudaSuccess)
+    return cuda_fail(ce, "ress_forward_host attention");
+  const int np = ress::attn_num_pairs(s);
+  const int chunks = np < kOutChunks ? np : kOutChunks;
+  const size_t row_bytes = bytes / (size_t)d->n_tokens;  // one token: H * 64 bf16
+  for (int c = 0; c < chunks && ce == cudaSuccess; ++c) {
+    const int p0 = (int)((int64_t)np * c / chunks), p1 = (int)((int64_t)np * (c + 1) / chunks);
+    cudaStream_t cs = (c & 1) ? o->aux : st;
+    const int64_t t0 = 128 * (int64_t)p0;
+    const int64_t t1 = 128 * (int64_t)p1 < d->n_tokens ? 128 * (int64_t)p1 : d->n_tokens;
+    if ((ce = ress::launch_attn_range(a, p0, p1, c, cs)) == cudaSuccess &&
+        (ce = cudaEventRecord(o->done[c], cs)) == cudaSuccess &&
+        (ce = cudaStreamWaitEvent(o->copy, o->done[c], 0)) == cudaSuccess)
+      ce = cudaMemcpyAsync(reinterpret_cast<char*>(O_host) + t0 * row_bytes,
+                           reinterpret_cast<const char*>(O_dev) + t0 * row_bytes,
+                           (size_t)(t1 - t0) * row_bytes, cudaMemcpyDeviceToHost, o->copy);
+  }
+  // the caller's stream resumes after every chunk and copy (also after a failed enqueue)
+  cudaError_t je = cudaEventRecord(o->copied, o->copy);
+  if (je == cudaSuccess) je = cudaStreamWaitEvent(st, o->copied, 0);
+  if (ce != cudaSuccess) return cuda_fail(ce, "ress_forward_host attention chunk");
+  if (je != cudaSuccess) return cuda_fail(je, "ress_forward_host join");
   return ok();
 }
 

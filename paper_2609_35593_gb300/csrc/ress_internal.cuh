@@ -194,6 +194,15 @@ struct AttnArgs {
   int64_t scratch_cap;
 };
 cudaError_t launch_sparse_attn(const AttnArgs& a, cudaStream_t st);
+// The two halves of launch_sparse_attn, for callers that split the attention: the union
+// lists of the query-block pairs, then the attention over pairs [p0, p1) of every head
+// (query tokens [128 p0, 128 p1)) with tile-scheduler counter `slot`, which the caller
+// zeroes before the launch.  Pairs are 128 query rows: two 64-token query blocks, or one
+// 128-token block on the paper's grid.
+constexpr int kAttnCounterSlots = 16;  // uint32 counters in the workspace's 64-byte slot
+int attn_num_pairs(const Shape& s);
+cudaError_t launch_attn_pairs(const AttnArgs& a, cudaStream_t st);
+cudaError_t launch_attn_range(const AttnArgs& a, int p0, int p1, int slot, cudaStream_t st);
 
 struct OProjArgs {
   int N, H, Dm;                      // tokens, heads (K = 64 H), d_model

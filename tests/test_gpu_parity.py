@@ -282,21 +282,33 @@ def test_large_shapes_sampled(name, kw):
     assert a["max_abs"] <= G.ATT_MAX_ABS and a["mean_rel"] <= G.ATT_MEAN_REL, a
 
 
-def test_forward_host_equals_forward(tiny):
-    """ress_forward_host (copies in, forward, copy out, one stream) gives the bits of the
-    staged device calls."""
-    layer, _ = layer_for("tiny_v2")
+@pytest.mark.parametrize("name,q_block", [("tiny_v2", 64), ("tiny_v2", 128), ("vggt_v8", 64)])
+def test_forward_host_equals_forward(name, q_block):
+    """ress_forward_host (copies in, selection, then the attention in chunks of query rows
+    whose output rows are copied out as each chunk completes, on library streams joined back
+    into the caller's) gives the bits of the staged device calls, and the caller's stream
+    alone orders the result: every output row is on the host once that stream is done."""
+    wl = synth.WORKLOADS[name]
+    ref = G.Layer(synth.make_inputs(wl), wl.n_special, wl.budgets(), wl.rounds, wl.rho,
+                  q_block=q_block).run()
+    layer = G.Layer(synth.make_inputs(wl), wl.n_special, wl.budgets(), wl.rounds, wl.rho,
+                    q_block=q_block)
     r, b = layer.ress, layer.buf
     r.prepare_wo(layer.d, layer.W, b.F)
+    torch.cuda.synchronize()
     Qh, Kh, Vh = (t.cpu().pin_memory() for t in (layer.Q, layer.K, layer.V))
     Oh = torch.empty(b.O.shape, dtype=torch.bfloat16).pin_memory()
+    Oh.view(torch.int16).fill_(-1)  # NaN bits: a row the copies miss stays visible
     Qd, Kd, Vd, Od = (torch.empty_like(t) for t in (layer.Q, layer.K, layer.V, b.O))
-    r.forward_host(layer.d, Qh, Kh, Vh, Oh, Qd, Kd, Vd, Od, b.F, layer.c_h, layer.rounds,
-                   layer.rho, b.ws, b.row_ptr, b.col_idx, b.J_best)
-    r.status(b.ws)
-    torch.cuda.synchronize()
-    assert torch.equal(Oh.view(torch.int16), tiny.buf.O.cpu().view(torch.int16))
-    assert np.array_equal(layer.csr()[1], tiny.csr()[1])
+    s = torch.cuda.Stream()
+    for _ in range(2):  # the second call reuses the library's streams and events
+        r.forward_host(layer.d, Qh, Kh, Vh, Oh, Qd, Kd, Vd, Od, b.F, layer.c_h, layer.rounds,
+                       layer.rho, b.ws, b.row_ptr, b.col_idx, b.J_best, stream=s)
+        s.synchronize()
+        assert torch.equal(Oh.view(torch.int16), ref.buf.O.cpu().view(torch.int16))
+        Oh.view(torch.int16).fill_(-1)
+    r.status(b.ws, stream=s)
+    assert np.array_equal(layer.csr()[1], ref.csr()[1])
 
 
 @pytest.mark.parametrize("fixture_name", ["tiny_v2", "vggt_v8"])
