@@ -857,10 +857,29 @@ __global__ void __launch_bounds__(32 * kRowWarps, 10) k_round_rows(SelPtrs p, Bu
 
 // ------------------------------------------------------------------------------------
 // Kept-block lists (CSR) from the best drop sets; special query rows keep everything.
-// grid (ceil(nq / 8), H) x 256 threads, one warp per (head, query block) row.
+// One warp per attention item: query rows 2u and 2u + 1 on the 64-token grid, row u on the
+// 128-token grid.  With plist set the warp also writes the item's list for the attention
+// kernel (what k_pairs builds from a caller's CSR): the union of its rows' lists in
+// ascending order, entry j | mask << 16 (bit 0: the item's first 64 query rows keep j, bit 1:
+// the second 64), at the offset of the item's first row, and the union's length in plen.
+// grid (ceil(items / 8), H) x 256 threads.
 // ------------------------------------------------------------------------------------
 struct CsrBases {
   int64_t base[RESS_MAX_HEADS + 1];
+};
+
+struct CsrOut {
+  int32_t* row_ptr;
+  int32_t* col_idx;
+  int64_t cap;           // col_idx entries
+  float* J_best;         // optional
+  uint32_t* drop_mask;   // optional
+  int32_t* plist;        // optional: attention item lists
+  int32_t* plen;         // [H * items] with plist
+  int64_t plist_cap;
+  uint32_t* status;
+  int rows_per_item;     // 2 on the 64-token grid, 1 on the 128-token grid
+  bool variable;         // row offsets from row_ptr (k_rowptr) instead of the fixed budgets
 };
 
 // Row offsets of variable-length kept lists (CDF threshold): row_ptr = exclusive scan of the
@@ -903,44 +922,75 @@ __global__ void __launch_bounds__(1024) k_rowptr(const int32_t* __restrict__ kco
   if (t == 1023) row_ptr[R] = (int32_t)off;
 }
 
-__global__ void k_csr(SelPtrs p, Budgets bud, CsrBases cb, int H, int32_t* __restrict__ row_ptr,
-                      int32_t* __restrict__ col_idx, int64_t cap, float* __restrict__ J_best,
-                      uint32_t* __restrict__ drop_mask, uint32_t* status, bool variable) {
-  const int i = blockIdx.x * 8 + (threadIdx.x >> 5), h = blockIdx.y, lane = threadIdx.x & 31;
-  if (i >= p.nq) return;
-  const int64_t ri = (int64_t)h * p.nq + i;
+__global__ void k_csr(SelPtrs p, Budgets bud, CsrBases cb, int H, CsrOut o) {
+  const int h = blockIdx.y, lane = threadIdx.x & 31;
+  const int rpi = o.rows_per_item;
+  const int items = (p.nq + rpi - 1) / rpi;
+  const int u = blockIdx.x * 8 + (threadIdx.x >> 5);
+  if (u >= items) return;
+  const int i0 = u * rpi;
+  const int nr = min(rpi, p.nq - i0);  // rows of this item: 1 or 2
+  const int ns = p.nb - p.ncand;        // always-kept key blocks
   const int c = bud.c[h];
-  const int ns = p.nb - p.ncand;  // always-kept key blocks
-  const bool dense = i >= p.nqc;
-  // fixed budgets: offsets by formula; variable lengths: the offsets k_rowptr wrote
-  const int64_t off = variable ? (int64_t)row_ptr[ri]
-                               : cb.base[h] + (dense ? (int64_t)p.nqc * (c + ns) +
-                                                           (int64_t)(i - p.nqc) * p.nb
-                                                     : (int64_t)i * (c + ns));
-  const int expect = variable ? (int)(row_ptr[ri + 1] - off) : (dense ? p.nb : c + ns);
-  int pos = 0;
+  int64_t ri[2], off[2];
+  int expect[2], pos[2] = {0, 0};
+  bool dense[2];
+#pragma unroll
+  for (int r = 0; r < 2; ++r) {
+    const int i = min(i0 + r, p.nq - 1);
+    ri[r] = (int64_t)h * p.nq + i;
+    dense[r] = i >= p.nqc;
+    // fixed budgets: offsets by formula; variable lengths: the offsets k_rowptr wrote
+    off[r] = o.variable ? (int64_t)o.row_ptr[ri[r]]
+                        : cb.base[h] + (dense[r] ? (int64_t)p.nqc * (c + ns) +
+                                                       (int64_t)(i - p.nqc) * p.nb
+                                                 : (int64_t)i * (c + ns));
+    expect[r] = o.variable ? (int)(o.row_ptr[ri[r] + 1] - off[r]) : (dense[r] ? p.nb : c + ns);
+  }
+  const uint32_t below = (1u << lane) - 1u;
+  int posU = 0;
   for (int w0 = 0; w0 < p.words; w0 += 32) {
-    // 32 words per coalesced load, handed out by shuffle
-    const uint32_t mine =
-        (!dense && w0 + lane < p.words) ? p.bmask[ri * p.words + w0 + lane] : 0u;
-    if (drop_mask && w0 + lane < p.words) drop_mask[ri * p.words + w0 + lane] = mine;
+    // 32 words of each row per coalesced load, handed out by shuffle
+    uint32_t mine[2];
+#pragma unroll
+    for (int r = 0; r < 2; ++r) {
+      mine[r] = (r < nr && !dense[r] && w0 + lane < p.words) ? p.bmask[ri[r] * p.words + w0 + lane] : 0u;
+      if (r < nr && o.drop_mask && w0 + lane < p.words) o.drop_mask[ri[r] * p.words + w0 + lane] = mine[r];
+    }
     const int nw = min(32, p.words - w0);
     for (int k = 0; k < nw; ++k) {
       const int w = w0 + k;
-      const uint32_t dm = __shfl_sync(kFull, mine, k);
-      const uint32_t keep = ~dm & valid_bits(w, p.nb);
-      const int at = pos + __popc(keep & ((1u << lane) - 1u));
-      if (((keep >> lane) & 1u) && at < expect && off + at < cap) col_idx[off + at] = w * 32 + lane;
-      pos += __popc(keep);
+      const uint32_t valid = valid_bits(w, p.nb);
+      uint32_t keep[2];
+#pragma unroll
+      for (int r = 0; r < 2; ++r) {
+        keep[r] = r < nr ? ~__shfl_sync(kFull, mine[r], k) & valid : 0u;
+        const int at = pos[r] + __popc(keep[r] & below);
+        if (((keep[r] >> lane) & 1u) && at < expect[r] && off[r] + at < o.cap)
+          o.col_idx[off[r] + at] = w * 32 + lane;
+        pos[r] += __popc(keep[r]);
+      }
+      if (o.plist) {
+        // a 128-token query block keeps its list for both 64-row halves of the tile
+        const uint32_t kb = rpi == 1 ? keep[0] : keep[1];
+        const uint32_t un = keep[0] | kb;
+        const int at = posU + __popc(un & below);
+        if (((un >> lane) & 1u) && off[0] + at < o.plist_cap) {
+          const int m = (int)((keep[0] >> lane) & 1u) | (int)(((kb >> lane) & 1u) << 1);
+          o.plist[off[0] + at] = (w * 32 + lane) | (m << 16);
+        }
+        posU += __popc(un);
+      }
     }
   }
   if (lane == 0) {
-    if (pos != expect) flag_status(status, kStatusBadRow);
-    if (!variable) {
-      row_ptr[ri] = (int32_t)off;
-      if (h == H - 1 && i == p.nq - 1) row_ptr[(int64_t)H * p.nq] = (int32_t)cb.base[H];
+    for (int r = 0; r < nr; ++r) {
+      if (pos[r] != expect[r]) flag_status(o.status, kStatusBadRow);
+      if (!o.variable) o.row_ptr[ri[r]] = (int32_t)off[r];
+      if (o.J_best) o.J_best[ri[r]] = dense[r] ? 0.f : p.Jbest[ri[r]];
     }
-    if (J_best) J_best[ri] = dense ? 0.f : p.Jbest[ri];
+    if (!o.variable && h == H - 1 && u == items - 1) o.row_ptr[(int64_t)H * p.nq] = (int32_t)cb.base[H];
+    if (o.plist) o.plen[(int64_t)h * items + u] = posU;
   }
 }
 
@@ -1008,18 +1058,30 @@ cudaError_t launch_round(const SelectArgs& a, int round, float rho, cudaStream_t
 
 cudaError_t launch_csr(const SelectArgs& a, const int64_t* head_base, int32_t* row_ptr,
                        int32_t* col_idx, int64_t col_capacity, float* J_best,
-                       uint32_t* drop_mask, cudaStream_t st) {
+                       uint32_t* drop_mask, int32_t* plist, int32_t* plen, int64_t plist_cap,
+                       cudaStream_t st) {
   const Shape& s = a.s;
   SelPtrs p = sel_ptrs(s, a.ws, a.L);
   CsrBases cb;
   for (int h = 0; h <= s.H; ++h) cb.base[h] = head_base[h];
-  const bool variable = a.v.cdf > 0.f;
-  if (variable) {
+  CsrOut o;
+  o.row_ptr = row_ptr;
+  o.col_idx = col_idx;
+  o.cap = col_capacity;
+  o.J_best = J_best;
+  o.drop_mask = drop_mask;
+  o.plist = plist;
+  o.plen = plen;
+  o.plist_cap = plist_cap;
+  o.status = (uint32_t*)(a.ws + a.L.status);
+  o.rows_per_item = s.qb == 128 ? 1 : 2;
+  o.variable = a.v.cdf > 0.f;
+  if (o.variable) {
     k_rowptr<<<1, 1024, 0, st>>>(p.kcount, s.H, s.nq, s.nqc, s.nb, row_ptr);
     note_launch();
   }
-  k_csr<<<dim3((s.nq + 7) / 8, s.H), 256, 0, st>>>(p, budgets_of(a), cb, s.H, row_ptr, col_idx, col_capacity,
-                                        J_best, drop_mask, (uint32_t*)(a.ws + a.L.status), variable);
+  const int items = (s.nq + o.rows_per_item - 1) / o.rows_per_item;
+  k_csr<<<dim3((items + 7) / 8, s.H), 256, 0, st>>>(p, budgets_of(a), cb, s.H, o);
   note_launch();
   return cudaGetLastError();
 }

@@ -260,10 +260,14 @@ int ress_score(const ress_dims* d, const uint16_t* Q, const uint16_t* K, const u
   return ress_score_variant(d, Q, K, V, F, c_h, nullptr, ws, ws_bytes, stream);
 }
 
-int ress_restore_variant(const ress_dims* d, const int32_t* c_h, int32_t rounds, float rho,
-                         const ress_variant* variant, void* ws, size_t ws_bytes, int32_t* row_ptr,
-                         int32_t* col_idx, int64_t col_capacity, float* J_best,
-                         uint32_t* drop_mask, void* stream) {
+}  // extern "C"
+
+// The restoration rounds and the CSR; with items set, the CSR kernel also writes the
+// attention items' union lists into the workspace (a forward then skips k_pairs).
+static int restore_impl(const ress_dims* d, const int32_t* c_h, int32_t rounds, float rho,
+                        const ress_variant* variant, void* ws, size_t ws_bytes, int32_t* row_ptr,
+                        int32_t* col_idx, int64_t col_capacity, float* J_best,
+                        uint32_t* drop_mask, bool items, void* stream) {
   int e = check_dims(d);
   if (e) return e;
   const ress::Shape s = ress::make_shape(*d);
@@ -292,9 +296,23 @@ int ress_restore_variant(const ress_dims* d, const int32_t* c_h, int32_t rounds,
     cudaError_t ce = ress::launch_round(a, r, rho, st);
     if (ce != cudaSuccess) return cuda_fail(ce, "ress_restore round");
   }
-  cudaError_t ce = ress::launch_csr(a, base, row_ptr, col_idx, col_capacity, J_best, drop_mask, st);
+  char* w = static_cast<char*>(ws);
+  int32_t* plist = items ? reinterpret_cast<int32_t*>(w + L.t) : nullptr;  // t is free by now
+  int32_t* plen = items ? reinterpret_cast<int32_t*>(w + L.plen) : nullptr;
+  cudaError_t ce = ress::launch_csr(a, base, row_ptr, col_idx, col_capacity, J_best, drop_mask,
+                                    plist, plen, (int64_t)s.H * s.nq * s.ld, st);
   if (ce != cudaSuccess) return cuda_fail(ce, "ress_restore csr");
   return ok();
+}
+
+extern "C" {
+
+int ress_restore_variant(const ress_dims* d, const int32_t* c_h, int32_t rounds, float rho,
+                         const ress_variant* variant, void* ws, size_t ws_bytes, int32_t* row_ptr,
+                         int32_t* col_idx, int64_t col_capacity, float* J_best,
+                         uint32_t* drop_mask, void* stream) {
+  return restore_impl(d, c_h, rounds, rho, variant, ws, ws_bytes, row_ptr, col_idx, col_capacity,
+                      J_best, drop_mask, false, stream);
 }
 
 int ress_restore(const ress_dims* d, const int32_t* c_h, int32_t rounds, float rho, void* ws,
@@ -377,11 +395,19 @@ int ress_forward(const ress_dims* d, const uint16_t* Q, const uint16_t* K, const
   head_bases(s, c_h, base);
   if (col_capacity < base[s.H])
     return fail(RESS_EWORKSPACE, "col_capacity %lld < %lld", (long long)col_capacity, (long long)base[s.H]);
+  ress_ws_layout L;
+  if ((e = check_ws(s, ws, ws_bytes, &L))) return e;
   if ((e = ress_score(d, Q, K, V, F, c_h, ws, ws_bytes, stream))) return e;
-  if ((e = ress_restore(d, c_h, rounds, rho, ws, ws_bytes, row_ptr, col_idx, col_capacity, J_best,
-                        nullptr, stream)))
+  // the CSR kernel also writes the attention items' lists, so the attention starts directly
+  if ((e = restore_impl(d, c_h, rounds, rho, nullptr, ws, ws_bytes, row_ptr, col_idx, col_capacity,
+                        J_best, nullptr, true, stream)))
     return e;
-  return ress_sparse_attn(d, Q, K, V, row_ptr, col_idx, col_capacity, O, ws, ws_bytes, stream);
+  const ress::AttnArgs a = attn_args(s, L, Q, K, V, row_ptr, col_idx, col_capacity, O, false, ws);
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  cudaError_t ce = cudaMemsetAsync(a.counter, 0, sizeof(uint32_t), st);
+  if (ce == cudaSuccess) ce = ress::launch_attn_range(a, 0, ress::attn_num_pairs(s), 0, st);
+  if (ce != cudaSuccess) return cuda_fail(ce, "ress_forward attention");
+  return ok();
 }
 
 int ress_forward_host(const ress_dims* d, const uint16_t* Q_host, const uint16_t* K_host,
@@ -419,8 +445,8 @@ int ress_forward_host(const ress_dims* d, const uint16_t* Q_host, const uint16_t
     if (ce != cudaSuccess) return cuda_fail(ce, "ress_forward_host input copy");
   }
   if ((e = ress_score(d, Q_dev, K_dev, V_dev, F, c_h, ws, ws_bytes, stream))) return e;
-  if ((e = ress_restore(d, c_h, rounds, rho, ws, ws_bytes, row_ptr, col_idx, col_capacity, J_best,
-                        nullptr, stream)))
+  if ((e = restore_impl(d, c_h, rounds, rho, nullptr, ws, ws_bytes, row_ptr, col_idx, col_capacity,
+                        J_best, nullptr, true, stream)))
     return e;
   // attention in chunks of 128-token query rows; each chunk's output rows go to the host on
   // the copy stream as soon as the chunk is done, while the next chunks compute
@@ -433,8 +459,7 @@ int ress_forward_host(const ress_dims* d, const uint16_t* Q_host, const uint16_t
   OverlapStreams* o = nullptr;
   cudaError_t ce = overlap_streams(&o);
   if (ce != cudaSuccess) return cuda_fail(ce, "ress_forward_host streams");
-  if ((ce = ress::launch_attn_pairs(a, st)) != cudaSuccess ||
-      (ce = cudaMemsetAsync(a.counter, 0, kOutChunks * sizeof(uint32_t), st)) != cudaSuccess ||
+  if ((ce = cudaMemsetAsync(a.counter, 0, kOutChunks * sizeof(uint32_t), st)) != cudaSuccess ||
       (ce = cudaEventRecord(o->ready, st)) != cudaSuccess ||
       (ce = cudaStreamWaitEvent(o->aux, o->ready, 0)) != cudaSuccess)
     return cuda_fail(ce, "ress_forward_host attention");

@@ -176,9 +176,13 @@ cudaError_t launch_gain(const SelectArgs& a, int round, float rho, cudaStream_t 
 cudaError_t launch_logits(const SelectArgs& a, cudaStream_t st);
 cudaError_t launch_drift_norms(const SelectArgs& a, cudaStream_t st);
 cudaError_t launch_yagg(const SelectArgs& a, cudaStream_t st);
+// Kept-block lists in CSR form; with plist set, also the attention items' union lists and
+// their lengths (what launch_attn_pairs builds from a caller's CSR), so that a forward can
+// go straight to launch_attn_range.
 cudaError_t launch_csr(const SelectArgs& a, const int64_t* head_base, int32_t* row_ptr,
                        int32_t* col_idx, int64_t col_capacity, float* J_best,
-                       uint32_t* drop_mask, cudaStream_t st);
+                       uint32_t* drop_mask, int32_t* plist, int32_t* plen, int64_t plist_cap,
+                       cudaStream_t st);
 
 struct AttnArgs {
   Shape s;

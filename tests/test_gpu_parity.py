@@ -138,6 +138,39 @@ def test_forward_equals_staged_calls(tiny):
     assert np.array_equal(layer.buf.J_best.cpu().numpy(), tiny.buf.J_best.cpu().numpy())
 
 
+@pytest.mark.parametrize("name,q_block", [("tiny_v2", 64), ("tiny_v2", 128), ("vggt_v8", 64),
+                                          ("vggt_v8", 128)])
+def test_forward_item_lists_match_pair_unions(name, q_block):
+    """ress_forward's CSR kernel also writes the attention items' lists (entry j | mask << 16
+    at each item's first row offset, lengths in plen).  They equal what ress_sparse_attn's
+    own union kernel builds from the same CSR, and both attention runs give the same bits."""
+    wl = synth.WORKLOADS[name]
+    layer = G.Layer(synth.make_inputs(wl), wl.n_special, wl.budgets(), wl.rounds, wl.rho,
+                    q_block=q_block)
+    r, b = layer.ress, layer.buf
+    r.prepare_wo(layer.d, layer.W, b.F)
+    r.forward(layer.d, layer.Q, layer.K, layer.V, b.F, layer.c_h, layer.rounds, layer.rho, b.ws,
+              b.row_ptr, b.col_idx, b.O, b.J_best)
+    r.status(b.ws)
+    rpi = 1 if q_block == 128 else 2
+    items = -(-layer.nq // rpi)
+    plen_f = layer.ws("plen", torch.int32)[:layer.H * items].copy()
+    plist_f = layer.ws("t", torch.int32).copy()
+    O_f = b.O.clone()
+    r.sparse_attn(layer.d, layer.Q, layer.K, layer.V, b.row_ptr, b.col_idx, b.O, b.ws)
+    r.status(b.ws)
+    plen_p = layer.ws("plen", torch.int32)[:layer.H * items]
+    plist_p = layer.ws("t", torch.int32)
+    assert np.array_equal(plen_f, plen_p)
+    rp = layer.csr()[0]
+    for h in range(layer.H):
+        for u in range(items):
+            s0, n = rp[h * layer.nq + u * rpi], plen_f[h * items + u]
+            assert n >= rp[h * layer.nq + u * rpi + 1] - s0
+            assert np.array_equal(plist_f[s0:s0 + n], plist_p[s0:s0 + n]), (h, u)
+    assert torch.equal(O_f.view(torch.int16), b.O.view(torch.int16))
+
+
 def test_deterministic_bits():
     a, _ = layer_for("tiny_v2")
     b, _ = layer_for("tiny_v2")
@@ -390,7 +423,7 @@ def test_tensor_core_scoring(fixture_name):
 def test_kernel_launch_counter():
     """ress_kernel_launches counts every kernel of a forward: six for scoring (pooling,
     z-projection, logits, P with y~, q, score rows), two per restoration round, the CSR
-    kernel, and the pair unions with the attention kernel."""
+    kernel (which also writes the attention items' lists) and the attention kernel."""
     layer, wl = layer_for("tiny_v2")
     r, b = layer.ress, layer.buf
     r.prepare_wo(layer.d, layer.W, b.F)
@@ -398,7 +431,7 @@ def test_kernel_launch_counter():
     r.forward(layer.d, layer.Q, layer.K, layer.V, b.F, layer.c_h, layer.rounds, layer.rho, b.ws,
               b.row_ptr, b.col_idx, b.O, b.J_best)
     torch.cuda.synchronize()
-    assert r.kernel_launches() - n0 == 6 + 2 * layer.rounds + 1 + 2
+    assert r.kernel_launches() - n0 == 6 + 2 * layer.rounds + 1 + 1
 
 
 def _bf16_tensor(a):
