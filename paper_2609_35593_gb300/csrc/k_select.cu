@@ -356,10 +356,85 @@ __device__ void select_exact(const uint32_t* keys, const uint16_t* idx, int n, i
   }
 }
 
-// Requires m <= number of participating blocks.  sk/si: survivor scratch (kSurvivors).
+// Exact selection over a survivor list (keys[0..n) with block indices idx[], in ascending
+// index order): the m largest keys, ties to the lower index, by a most-significant-first
+// radix select with 8-bit digits whose 256 counters live in `hist` (per-warp shared
+// scratch, 16-byte aligned).  Each pass fixes one byte of the m-th largest key and stops
+// early once the keys that share the fixed bytes are exactly the ones still needed; a final
+// pass in index order takes the keys above that prefix and the first `need` equal to it.
+__device__ void select_radix(const uint32_t* keys, const uint16_t* idx, int n, int m,
+                             uint32_t* hist, uint32_t* sel) {
+  const int lane = threadIdx.x & 31;
+  uint32_t prefix = 0u, pmask = 0u;
+  int need = m;  // keys still to choose among those matching the prefix
+  uint4* h4 = reinterpret_cast<uint4*>(hist);
+  for (int shift = 24; shift >= 0; shift -= 8) {
+    h4[2 * lane] = make_uint4(0u, 0u, 0u, 0u);
+    h4[2 * lane + 1] = make_uint4(0u, 0u, 0u, 0u);
+    __syncwarp();
+    for (int x = lane; x < n; x += 32) {
+      const uint32_t k = keys[x];
+      if ((k & pmask) == prefix) atomicAdd(&hist[(k >> shift) & 255u], 1u);
+    }
+    __syncwarp();
+    // lane l owns digits base + 7 .. base, base = 8 (31 - l): lane 0 the highest
+    const int base = 8 * (31 - lane);
+    const uint4 lo4 = h4[2 * (31 - lane)], hi4 = h4[2 * (31 - lane) + 1];
+    const uint32_t c[8] = {hi4.w, hi4.z, hi4.y, hi4.x, lo4.w, lo4.z, lo4.y, lo4.x};
+    int sum = 0;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) sum += (int)c[i];
+    int inc = sum;  // inclusive count over lanes 0..l (digits above and at this lane's)
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int y = __shfl_up_sync(kFull, inc, o);
+      if (lane >= o) inc += y;
+    }
+    const int exc = inc - sum;
+    const uint32_t who = __ballot_sync(kFull, exc < need && need <= inc);
+    const int src = __ffs(who) - 1;
+    int digit = 0, before = 0, cnt = 0;
+    if (lane == src) {
+      int run = exc;
+#pragma unroll
+      for (int i = 0; i < 8; ++i) {
+        if (cnt == 0 && run + (int)c[i] >= need) {
+          digit = base + 7 - i;
+          before = run;
+          cnt = (int)c[i];
+        }
+        run += (int)c[i];
+      }
+    }
+    digit = __shfl_sync(kFull, digit, src);
+    before = __shfl_sync(kFull, before, src);
+    cnt = __shfl_sync(kFull, cnt, src);
+    need -= before;
+    prefix |= (uint32_t)digit << shift;
+    pmask |= 255u << shift;
+    if (cnt == need) break;  // every key with this prefix is chosen
+  }
+  int taken = 0;
+  for (int x0 = 0; x0 < n; x0 += 32) {
+    const int x = x0 + lane;
+    const bool in = x < n;
+    const uint32_t v = in ? (keys[x] & pmask) : 0u;
+    const bool is_eq = in && v == prefix;
+    const uint32_t eqb = __ballot_sync(kFull, is_eq);
+    const int rank = taken + __popc(eqb & ((1u << lane) - 1u));
+    if ((in && v > prefix) || (is_eq && rank < need)) {
+      const int j = (int)idx[x];
+      atomicOr(&sel[j >> 5], 1u << (j & 31));
+    }
+    taken += __popc(eqb);
+  }
+}
+
+// Requires m <= number of participating blocks.  sk/si: survivor scratch (kSurvivors);
+// hist: 256 words for select_radix on the survivors (NULL: bit-by-bit select_exact).
 __device__ void warp_topm(const uint32_t* kk, int n, int m, uint32_t* sel, int words,
                           uint32_t* sk, uint16_t* si, const uint32_t* member = nullptr,
-                          bool want = true) {
+                          bool want = true, uint32_t* hist = nullptr) {
   const int lane = threadIdx.x & 31;
   for (int w = lane; w < words; w += 32) sel[w] = 0u;
   __syncwarp();
@@ -405,6 +480,8 @@ __device__ void warp_topm(const uint32_t* kk, int n, int m, uint32_t* sel, int w
   // 3. exact selection on the survivors (or on every participating key if they overflowed)
   if (cnt > kSurvivors)
     select_exact(kk, nullptr, n, m, member, want, sel);
+  else if (hist)
+    select_radix(sk, si, cnt, m, hist, sel);
   else
     select_exact(sk, si, cnt, m, nullptr, true, sel);
   __syncwarp();
@@ -482,6 +559,13 @@ __device__ void warp_topm_pair(const uint32_t* kk, int n, int m, const uint32_t*
     cntB += __popc(BB);
   }
   __syncwarp();
+  if (cntD <= kHalf && cntB <= kHalf) {
+    // the keys are no longer needed: their first 256 words hold the radix counters
+    select_radix(sk, si, cntD, m, const_cast<uint32_t*>(kk), selD);
+    select_radix(sk + kHalf, si + kHalf, cntB, m, const_cast<uint32_t*>(kk), selB);
+    __syncwarp();
+    return;
+  }
   if (cntD > kHalf)
     select_exact(kk, nullptr, n, m, Dw, true, selD);
   else
@@ -596,11 +680,17 @@ __device__ __forceinline__ void swap_drift(const uint32_t* R, const uint32_t* X,
   __syncwarp();
 }
 
-// Per-warp scratch of the per-row kernels: keys [ld] u32, survivor keys [kSurvivors] u32,
-// survivor indices [kSurvivors] u16, bitmask words.
+// Per-warp scratch of the per-row kernels: keys [key_words(ld)] u32, survivor keys
+// [kSurvivors] u32, survivor indices [kSurvivors] u16, bitmask words (and, in the score
+// kernel, 256 radix counters after them).
+// The key area holds at least 256 words, so that it can serve as radix counters once the
+// keys are spent; the total is a multiple of 4 words (16-byte aligned per-warp areas).
+__host__ __device__ constexpr int key_words(int ld) { return ld > 256 ? ld : 256; }
 __host__ __device__ constexpr size_t warp_scratch_words(int ld, int words_per_warp) {
-  return (size_t)ld + kSurvivors + kSurvivors / 2 + words_per_warp;
+  return ((size_t)key_words(ld) + kSurvivors + kSurvivors / 2 + words_per_warp + 3) / 4 * 4;
 }
+// the score kernel's words after the survivors: its drop-set mask, then 256 radix counters
+__host__ __device__ constexpr int score_mask_words(int words) { return (words + 3) / 4 * 4 + 256; }
 
 
 
@@ -615,7 +705,7 @@ __device__ __forceinline__ float delta_J(float G, float K, float dG, float u) {
     return __fdividef(num, (K * K) * (K2 * K2));
   }
   const float Kc = fmaxf(K, kEps), K2c = fmaxf(K2, kEps);
-  return G / (Kc * Kc) - (G + dG) / (K2c * K2c);
+  return __fdividef(G, Kc * Kc) - __fdividef(G + dG, K2c * K2c);
 }
 
 
@@ -721,11 +811,13 @@ __global__ void __launch_bounds__(32 * kRowWarps, 8) k_score_rows(SelPtrs p, Bud
   const float* Prow = p.P + ri * p.ld;
   const float* qrow = p.q + ri * p.ld;
   const float* zt_h = p.ztil + (int64_t)h * p.nb * 64;
-  uint32_t* base = reinterpret_cast<uint32_t*>(smem_raw) + (size_t)warp * warp_scratch_words(p.ld, p.words);
+  uint32_t* base =
+      reinterpret_cast<uint32_t*>(smem_raw) + (size_t)warp * warp_scratch_words(p.ld, score_mask_words(p.words));
   uint32_t* kk = base;
-  uint32_t* sk = base + p.ld;
+  uint32_t* sk = base + key_words(p.ld);
   uint16_t* si = reinterpret_cast<uint16_t*>(sk + kSurvivors);
   uint32_t* sel = sk + kSurvivors + kSurvivors / 2;
+  uint32_t* hist = sel + (p.words + 3) / 4 * 4;  // radix counters (the keys stay for the CDF rule)
   row_keys(p.ncand, kk, [&](int j, uint32_t (&k4)[4]) {
     const float4 P4 = *reinterpret_cast<const float4*>(Prow + j);
     const float4 q4 = *reinterpret_cast<const float4*>(qrow + j);
@@ -734,7 +826,7 @@ __global__ void __launch_bounds__(32 * kRowWarps, 8) k_score_rows(SelPtrs p, Bud
     for (int u = 0; u < 4; ++u) {
       uint32_t key;
       if (v.key == 0)  // s_ij / max(1 - P_ij, eps), s_ij = P_ij sqrt(q_ij)
-        key = order_key(pv[u] * sqrtf(qv[u]) / fmaxf(1.0f - pv[u], kEps));
+        key = order_key(__fdividef(pv[u] * sqrtf(qv[u]), fmaxf(1.0f - pv[u], kEps)));
       else if (v.key == 1)
         key = order_key(pv[u]);
       else
@@ -743,7 +835,7 @@ __global__ void __launch_bounds__(32 * kRowWarps, 8) k_score_rows(SelPtrs p, Bud
       k4[u] = (v.direction == 2) ? ~key : key;
     }
   });
-  warp_topm(kk, p.ncand, bud.c[h], sel, p.words, sk, si);  // sel = kept candidates
+  warp_topm(kk, p.ncand, bud.c[h], sel, p.words, sk, si, nullptr, true, hist);  // sel = kept
   // drop set D0 = candidates not kept
   for (int w = lane; w < p.words; w += 32) sel[w] = valid_bits(w, p.ncand) & ~sel[w];
   __syncwarp();
@@ -796,7 +888,7 @@ __global__ void __launch_bounds__(32 * kRowWarps, 10) k_round_rows(SelPtrs p, Bu
   const float* zt_h = p.ztil + (int64_t)h * p.nb * 64;
   uint32_t* base = reinterpret_cast<uint32_t*>(smem_raw) + (size_t)warp * warp_scratch_words(p.ld, 3 * p.words);
   uint32_t* kk = base;
-  uint32_t* sk = base + p.ld;
+  uint32_t* sk = base + key_words(p.ld);
   uint16_t* si = reinterpret_cast<uint16_t*>(sk + kSurvivors);
   uint32_t* Dw = sk + kSurvivors + kSurvivors / 2;  // current drop set
   uint32_t* Rw = Dw + p.words;                       // chosen restores
@@ -1032,7 +1124,7 @@ cudaError_t launch_score(const SelectArgs& a, cudaStream_t st) {
   if ((e = launch_logits(a, st)) != cudaSuccess) return e;
   if ((e = launch_yagg(a, st)) != cudaSuccess) return e;
   if ((e = launch_drift_norms(a, st)) != cudaSuccess) return e;
-  const size_t rsmem = (size_t)kRowWarps * warp_scratch_words(s.ld, s.words) * 4;
+  const size_t rsmem = (size_t)kRowWarps * warp_scratch_words(s.ld, score_mask_words(s.words)) * 4;
   e = cudaFuncSetAttribute(k_score_rows, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)rsmem);
   if (e != cudaSuccess) return e;
   k_score_rows<<<dim3((s.nqc + kRowWarps - 1) / kRowWarps, s.H), 32 * kRowWarps, rsmem, st>>>(
