@@ -365,10 +365,47 @@ __device__ void select_exact(const uint32_t* keys, const uint16_t* idx, int n, i
 __device__ void select_radix(const uint32_t* keys, const uint16_t* idx, int n, int m,
                              uint32_t* hist, uint32_t* sel) {
   const int lane = threadIdx.x & 31;
+  if (n <= m) {  // every survivor is chosen
+    for (int x = lane; x < n; x += 32) {
+      const int j = (int)idx[x];
+      atomicOr(&sel[j >> 5], 1u << (j & 31));
+    }
+    return;
+  }
+  if (n <= 32) {
+    // one survivor per lane: a bitonic sort of (key, lower index first) composites,
+    // descending; lanes 0..m-1 then hold the chosen blocks
+    unsigned long long c = 0ull;  // below every survivor (keys are >= 1)
+    if (lane < n) c = ((unsigned long long)keys[lane] << 32) | (0xffffu - (uint32_t)idx[lane]);
+#pragma unroll
+    for (int k = 2; k <= 32; k <<= 1) {
+#pragma unroll
+      for (int j = k >> 1; j >= 1; j >>= 1) {
+        const unsigned long long o = __shfl_xor_sync(kFull, c, j);
+        const bool keep_max = ((lane & k) == 0) == ((lane & j) == 0);
+        c = keep_max ? (c > o ? c : o) : (c < o ? c : o);
+      }
+    }
+    if (lane < m) {
+      const int j = 0xffff - (int)(c & 0xffffu);
+      atomicOr(&sel[j >> 5], 1u << (j & 31));
+    }
+    return;
+  }
   uint32_t prefix = 0u, pmask = 0u;
   int need = m;  // keys still to choose among those matching the prefix
   uint4* h4 = reinterpret_cast<uint4*>(hist);
-  for (int shift = 24; shift >= 0; shift -= 8) {
+  // bytes above the highest bit in which the survivors differ are common to all: start
+  // below them
+  uint32_t diff = 0u;
+  for (int x = lane; x < n; x += 32) diff |= keys[x] ^ keys[0];
+  diff = __reduce_or_sync(kFull, diff);
+  const int top_shift = diff ? (31 - __clz(diff)) / 8 * 8 : 0;
+  if (top_shift < 24) {
+    pmask = 0xffffffffu << (top_shift + 8);
+    prefix = keys[0] & pmask;
+  }
+  for (int shift = top_shift; shift >= 0; shift -= 8) {
     h4[2 * lane] = make_uint4(0u, 0u, 0u, 0u);
     h4[2 * lane + 1] = make_uint4(0u, 0u, 0u, 0u);
     __syncwarp();
@@ -498,14 +535,43 @@ struct LaneTop2 {
   }
 };
 
+// The m-th largest (1 <= m <= 64) of the 64 values held two per lane (element 2 lane + s
+// holds v[s]): a bitonic sort of the 64 values across the warp, descending.
+__device__ __forceinline__ uint32_t mth_of_64(uint32_t a, uint32_t b, int m) {
+  const int lane = threadIdx.x & 31;
+  uint32_t v[2] = {a, b};
+#pragma unroll
+  for (int k = 2; k <= 64; k <<= 1) {
+#pragma unroll
+    for (int j = k >> 1; j >= 1; j >>= 1) {
+      if (j == 1) {  // the partner is the lane's other element
+        const bool desc = ((2 * lane) & k) == 0;
+        const uint32_t hi = max(v[0], v[1]), lo = min(v[0], v[1]);
+        v[0] = desc ? hi : lo;
+        v[1] = desc ? lo : hi;
+      } else {
+#pragma unroll
+        for (int s = 0; s < 2; ++s) {
+          const int e = 2 * lane + s;
+          const uint32_t o = __shfl_xor_sync(kFull, v[s], j >> 1);
+          // in a descending run the lower element of a pair keeps the larger value
+          v[s] = (((e & k) == 0) == ((e & j) == 0)) ? max(v[s], o) : min(v[s], o);
+        }
+      }
+    }
+  }
+  const uint32_t mine = ((m - 1) & 1) ? v[1] : v[0];
+  return __shfl_sync(kFull, mine, (m - 1) >> 1);
+}
+
 // Both selections of a restoration round at once, for m <= 64: the m largest keys among
 // the blocks in D (bit set in Dw) into selD and the m largest among the other candidates
 // into selB, ties to the lower block index.  `top` holds this lane's two largest keys on
 // each side (0 where it has none), taken while the keys were written, so the lane-local
-// pass of warp_topm is not needed: the m-th largest of the 64 lane values of a side bounds
-// that side's m-th key from below.  Both bounds come from one bit search (counts packed in
-// one reduction) and both survivor lists from one ballot pass; each side then selects
-// exactly.
+// pass of warp_topm is not needed: the m-th largest of the 64 lane values of a side (a
+// bitonic sort across the warp) bounds that side's m-th key from below.  Both survivor
+// lists come from one pass (four blocks per lane and step, one warp scan for the store
+// positions); each side then selects exactly (radix select on its survivors).
 __device__ void warp_topm_pair(const uint32_t* kk, int n, int m, const uint32_t* Dw,
                                const LaneTop2& top, uint32_t* selD, uint32_t* selB,
                                int words, uint32_t* sk, uint16_t* si) {
@@ -513,50 +579,60 @@ __device__ void warp_topm_pair(const uint32_t* kk, int n, int m, const uint32_t*
   for (int w = lane; w < words; w += 32) selD[w] = selB[w] = 0u;
   __syncwarp();
   if (m <= 0) return;
-  uint32_t bD = 0, bB = 0;
-  bool doneD = false, doneB = false;
-  for (int bit = 31; bit >= 0 && !(doneD && doneB); --bit) {
-    const uint32_t cD = bD | (1u << bit), cB = bB | (1u << bit);
-    int c = 0;
-    if (!doneD) c += (top.d1 >= cD ? 1 : 0) + (top.d2 >= cD ? 1 : 0);
-    if (!doneB) c += (top.b1 >= cB ? 1 << 16 : 0) + (top.b2 >= cB ? 1 << 16 : 0);
-    c = __reduce_add_sync(kFull, c);
-    const int nD = c & 0xffff, nB = c >> 16;
-    if (!doneD && nD >= m) {
-      bD = cD;
-      doneD = nD == m;
-    }
-    if (!doneB && nB >= m) {
-      bB = cB;
-      doneB = nB == m;
-    }
-  }
+  // the m-th largest of the 64 lane values of a side bounds that side's m-th key from below
+  const uint32_t bD = mth_of_64(top.d1, top.d2, m), bB = mth_of_64(top.b1, top.b2, m);
   constexpr int kHalf = kSurvivors / 2;
-  const uint32_t below = (1u << lane) - 1u;
   int cntD = 0, cntB = 0;
-  for (int x0 = 0; x0 < n; x0 += 32) {
-    const int x = x0 + lane;
-    const bool in = x < n;
-    const uint32_t v = in ? kk[x] : 0u;
-    const bool inD = in && ((Dw[x0 >> 5] >> lane) & 1u);
-    const bool kd = inD && v >= bD, kb = in && !inD && v >= bB;
-    const uint32_t BD = __ballot_sync(kFull, kd), BB = __ballot_sync(kFull, kb);
-    if (kd) {
-      const int pos = cntD + __popc(BD & below);
-      if (pos < kHalf) {
-        sk[pos] = v;
-        si[pos] = (uint16_t)x;
+  // survivors in ascending block order, four consecutive blocks per lane and step: each
+  // lane's counts on both sides (packed) go through one warp scan for the store positions
+  for (int x0 = 0; x0 < n; x0 += 128) {
+    const int x = x0 + 4 * lane;
+    uint32_t fD = 0u, fB = 0u;
+    uint4 v = make_uint4(0u, 0u, 0u, 0u);
+    if (x < n) {
+      v = *reinterpret_cast<const uint4*>(kk + x);  // 16-byte aligned, inside the key area
+      const uint32_t dbits = Dw[x >> 5] >> (x & 31);
+      const uint32_t k4[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        if (x + u < n) {
+          const bool inD = (dbits >> u) & 1u;
+          if (inD && k4[u] >= bD) fD |= 1u << u;
+          if (!inD && k4[u] >= bB) fB |= 1u << u;
+        }
       }
     }
-    if (kb) {
-      const int pos = cntB + __popc(BB & below);
-      if (pos < kHalf) {
-        sk[kHalf + pos] = v;
-        si[kHalf + pos] = (uint16_t)x;
+    const int c = __popc(fD) | (__popc(fB) << 16);
+    int inc = c;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int y = __shfl_up_sync(kFull, inc, o);
+      if (lane >= o) inc += y;
+    }
+    const int total = __shfl_sync(kFull, inc, 31);
+    if (fD | fB) {
+      int pD = cntD + ((inc - c) & 0xffff), pB = cntB + ((inc - c) >> 16);
+      const uint32_t k4[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        if ((fD >> u) & 1u) {
+          if (pD < kHalf) {
+            sk[pD] = k4[u];
+            si[pD] = (uint16_t)(x + u);
+          }
+          ++pD;
+        }
+        if ((fB >> u) & 1u) {
+          if (pB < kHalf) {
+            sk[kHalf + pB] = k4[u];
+            si[kHalf + pB] = (uint16_t)(x + u);
+          }
+          ++pB;
+        }
       }
     }
-    cntD += __popc(BD);
-    cntB += __popc(BB);
+    cntD += total & 0xffff;
+    cntB += total >> 16;
   }
   __syncwarp();
   if (cntD <= kHalf && cntB <= kHalf) {
@@ -696,16 +772,15 @@ __host__ __device__ constexpr int score_mask_words(int words) { return (words + 
 
 
 // Exact decrease of J (Eq. 16) when G changes by dG and K by u, with the denominators
-// clamped at eps as in Eq. 7.  When no clamp applies the two fractions are combined over
-// one denominator so that the result carries no cancellation of J-sized terms.
+// clamped at eps as in Eq. 7.  The two fractions are combined over one denominator so that
+// the result carries no cancellation of J-sized terms, and no branch is taken per block.
 __device__ __forceinline__ float delta_J(float G, float K, float dG, float u) {
-  const float K2 = K + u;
-  if (K >= kEps && K2 >= kEps) {
-    const float num = fmaf(G * u, 2.0f * K + u, -dG * (K * K));
-    return __fdividef(num, (K * K) * (K2 * K2));
-  }
-  const float Kc = fmaxf(K, kEps), K2c = fmaxf(K2, kEps);
-  return __fdividef(G, Kc * Kc) - __fdividef(G + dG, K2c * K2c);
+  // G / Kc^2 - (G + dG) / K2c^2 = (G (K2c - Kc)(K2c + Kc) - dG Kc^2) / (Kc^2 K2c^2), with
+  // Kc = max(K, eps) and K2c = max(K + u, eps); K2c - Kc is u when no clamp applies
+  const float Kc = fmaxf(K, kEps), K2c = fmaxf(K + u, kEps);
+  const float KK = Kc * Kc;
+  const float num = fmaf(G * (K2c - Kc), K2c + Kc, -dG * KK);
+  return __fdividef(num, KK * (K2c * K2c));
 }
 
 
