@@ -356,20 +356,29 @@ __device__ void select_exact(const uint32_t* keys, const uint16_t* idx, int n, i
   }
 }
 
+// A chosen block: bit j of the bitmask sel, or entry `pos` of the list lst as j | flag.
+__device__ __forceinline__ void choose_block(uint32_t* sel, uint16_t* lst, uint16_t flag, int j,
+                                             int pos) {
+  if (lst)
+    lst[pos] = (uint16_t)(j | flag);
+  else
+    atomicOr(&sel[j >> 5], 1u << (j & 31));
+}
+
 // Exact selection over a survivor list (keys[0..n) with block indices idx[], in ascending
 // index order): the m largest keys, ties to the lower index, by a most-significant-first
 // radix select with 8-bit digits whose 256 counters live in `hist` (per-warp shared
 // scratch, 16-byte aligned).  Each pass fixes one byte of the m-th largest key and stops
 // early once the keys that share the fixed bytes are exactly the ones still needed; a final
 // pass in index order takes the keys above that prefix and the first `need` equal to it.
+// The chosen blocks go to the bitmask sel, or, with lst set, to lst[0..m) as j | flag (in an
+// order fixed by the data, so that sums over the list are reproducible).
 __device__ void select_radix(const uint32_t* keys, const uint16_t* idx, int n, int m,
-                             uint32_t* hist, uint32_t* sel) {
+                             uint32_t* hist, uint32_t* sel, uint16_t* lst = nullptr,
+                             uint16_t flag = 0) {
   const int lane = threadIdx.x & 31;
   if (n <= m) {  // every survivor is chosen
-    for (int x = lane; x < n; x += 32) {
-      const int j = (int)idx[x];
-      atomicOr(&sel[j >> 5], 1u << (j & 31));
-    }
+    for (int x = lane; x < n; x += 32) choose_block(sel, lst, flag, (int)idx[x], x);
     return;
   }
   if (n <= 32) {
@@ -386,10 +395,7 @@ __device__ void select_radix(const uint32_t* keys, const uint16_t* idx, int n, i
         c = keep_max ? (c > o ? c : o) : (c < o ? c : o);
       }
     }
-    if (lane < m) {
-      const int j = 0xffff - (int)(c & 0xffffu);
-      atomicOr(&sel[j >> 5], 1u << (j & 31));
-    }
+    if (lane < m) choose_block(sel, lst, flag, 0xffff - (int)(c & 0xffffu), lane);
     return;
   }
   uint32_t prefix = 0u, pmask = 0u;
@@ -451,19 +457,20 @@ __device__ void select_radix(const uint32_t* keys, const uint16_t* idx, int n, i
     pmask |= 255u << shift;
     if (cnt == need) break;  // every key with this prefix is chosen
   }
-  int taken = 0;
+  int taken = 0, out = 0;
+  const uint32_t below = (1u << lane) - 1u;
   for (int x0 = 0; x0 < n; x0 += 32) {
     const int x = x0 + lane;
     const bool in = x < n;
     const uint32_t v = in ? (keys[x] & pmask) : 0u;
     const bool is_eq = in && v == prefix;
     const uint32_t eqb = __ballot_sync(kFull, is_eq);
-    const int rank = taken + __popc(eqb & ((1u << lane) - 1u));
-    if ((in && v > prefix) || (is_eq && rank < need)) {
-      const int j = (int)idx[x];
-      atomicOr(&sel[j >> 5], 1u << (j & 31));
-    }
+    const int rank = taken + __popc(eqb & below);
+    const bool chosen = (in && v > prefix) || (is_eq && rank < need);
+    const uint32_t cb = __ballot_sync(kFull, chosen);
+    if (chosen) choose_block(sel, lst, flag, (int)idx[x], out + __popc(cb & below));
     taken += __popc(eqb);
+    out += __popc(cb);
   }
 }
 
@@ -572,13 +579,16 @@ __device__ __forceinline__ uint32_t mth_of_64(uint32_t a, uint32_t b, int m) {
 // bitonic sort across the warp) bounds that side's m-th key from below.  Both survivor
 // lists come from one pass (four blocks per lane and step, one warp scan for the store
 // positions); each side then selects exactly (radix select on its survivors).
-__device__ void warp_topm_pair(const uint32_t* kk, int n, int m, const uint32_t* Dw,
+// Returns true when the chosen blocks went to lst (restores at lst[0..m), drops at
+// lst[m..2m) with bit 15 set) instead of the bitmasks; lst lies in the key area after its
+// first 256 words (the radix counters).
+__device__ bool warp_topm_pair(const uint32_t* kk, int n, int m, const uint32_t* Dw,
                                const LaneTop2& top, uint32_t* selD, uint32_t* selB,
-                               int words, uint32_t* sk, uint16_t* si) {
+                               int words, uint32_t* sk, uint16_t* si, uint16_t* lst) {
   const int lane = threadIdx.x & 31;
   for (int w = lane; w < words; w += 32) selD[w] = selB[w] = 0u;
   __syncwarp();
-  if (m <= 0) return;
+  if (m <= 0) return false;
   // the m-th largest of the 64 lane values of a side bounds that side's m-th key from below
   const uint32_t bD = mth_of_64(top.d1, top.d2, m), bB = mth_of_64(top.b1, top.b2, m);
   constexpr int kHalf = kSurvivors / 2;
@@ -637,10 +647,10 @@ __device__ void warp_topm_pair(const uint32_t* kk, int n, int m, const uint32_t*
   __syncwarp();
   if (cntD <= kHalf && cntB <= kHalf) {
     // the keys are no longer needed: their first 256 words hold the radix counters
-    select_radix(sk, si, cntD, m, const_cast<uint32_t*>(kk), selD);
-    select_radix(sk + kHalf, si + kHalf, cntB, m, const_cast<uint32_t*>(kk), selB);
+    select_radix(sk, si, cntD, m, const_cast<uint32_t*>(kk), selD, lst, 0);
+    select_radix(sk + kHalf, si + kHalf, cntB, m, const_cast<uint32_t*>(kk), selB, lst + m, 0x8000);
     __syncwarp();
-    return;
+    return true;
   }
   if (cntD > kHalf)
     select_exact(kk, nullptr, n, m, Dw, true, selD);
@@ -651,6 +661,7 @@ __device__ void warp_topm_pair(const uint32_t* kk, int n, int m, const uint32_t*
   else
     select_exact(sk + kHalf, si + kHalf, cntB, m, nullptr, true, selB);
   __syncwarp();
+  return false;
 }
 
 // g~ of row ri (this lane's channels 2 lane, 2 lane + 1), its three bf16 terms (the A
@@ -717,20 +728,13 @@ __device__ __forceinline__ void kept_drift(const uint32_t* D, const SelPtrs& p,
 // The state after a round from the one before it: the restored blocks R join the kept set
 // and the dropped blocks X leave it, so g~ += sum_R P_k (z~_k - y~) - sum_X P_k (z~_k - y~)
 // and K += sum_R P_k - sum_X P_k over the 2m swapped blocks (exactly the kept-set sums of
-// Eq. 10-11 in exact arithmetic).  Same lane layout and staging as kept_drift.
-__device__ __forceinline__ void swap_drift(const uint32_t* R, const uint32_t* X, const SelPtrs& p,
-                                           const float* __restrict__ Prow,
-                                           const float* __restrict__ zt, float y0, float y1,
-                                           uint32_t* idx, float& g0, float& g1, float& K) {
+// Eq. 10-11 in exact arithmetic), taken in the order of their list (j | 0x8000 for a
+// dropped block).  Same lane layout and staging as kept_drift.
+__device__ __forceinline__ void swap_drift_list(const uint16_t* lst, int n,
+                                                const float* __restrict__ Prow,
+                                                const float* __restrict__ zt, float y0, float y1,
+                                                float& g0, float& g1, float& K) {
   const int lane = threadIdx.x & 31;
-  int n = 0;
-  for (int w = 0; w < p.words; ++w) {
-    const uint32_t sw = R[w] | X[w];
-    if ((sw >> lane) & 1u)
-      idx[n + __popc(sw & ((1u << lane) - 1u))] = (w * 32 + lane) | (((X[w] >> lane) & 1u) << 31);
-    n += __popc(sw);
-  }
-  __syncwarp();
   for (int k0 = 0; k0 < n; k0 += 8) {
     float pj[8];
     float2 z[8];
@@ -739,10 +743,10 @@ __device__ __forceinline__ void swap_drift(const uint32_t* R, const uint32_t* X,
       pj[u] = 0.f;
       z[u] = make_float2(y0, y1);
       if (k0 + u < n) {
-        const uint32_t e = idx[k0 + u];
-        const int j = (int)(e & 0x7fffffffu);
+        const uint32_t e = lst[k0 + u];
+        const int j = (int)(e & 0x7fffu);
         const float pv = Prow[j];
-        pj[u] = (e >> 31) ? -pv : pv;
+        pj[u] = (e >> 15) ? -pv : pv;
         z[u] = *reinterpret_cast<const float2*>(zt + (int64_t)j * 64 + 2 * lane);
       }
     }
@@ -759,9 +763,10 @@ __device__ __forceinline__ void swap_drift(const uint32_t* R, const uint32_t* X,
 // Per-warp scratch of the per-row kernels: keys [key_words(ld)] u32, survivor keys
 // [kSurvivors] u32, survivor indices [kSurvivors] u16, bitmask words (and, in the score
 // kernel, 256 radix counters after them).
-// The key area holds at least 256 words, so that it can serve as radix counters once the
-// keys are spent; the total is a multiple of 4 words (16-byte aligned per-warp areas).
-__host__ __device__ constexpr int key_words(int ld) { return ld > 256 ? ld : 256; }
+// The key area holds at least 320 words, so that once the keys are spent it can hold the
+// 256 radix counters and a list of up to 128 swapped blocks (u16); the total is a multiple
+// of 4 words (16-byte aligned per-warp areas).
+__host__ __device__ constexpr int key_words(int ld) { return ld > 320 ? ld : 320; }
 __host__ __device__ constexpr size_t warp_scratch_words(int ld, int words_per_warp) {
   return ((size_t)key_words(ld) + kSurvivors + kSurvivors / 2 + words_per_warp + 3) / 4 * 4;
 }
@@ -992,19 +997,40 @@ __global__ void __launch_bounds__(32 * kRowWarps, 10) k_round_rows(SelPtrs p, Bu
       if (j + u < p.ncand) top.add(k4[u], inD);
     }
   });
+  // the swapped blocks as a list: written by the selection itself on the common path
+  // (after the radix counters in the key area), else gathered from the bitmasks R and X
+  uint16_t* lst = reinterpret_cast<uint16_t*>(kk + 256);
+  int nl = 2 * m;
+  bool listed = false;
   if (m <= 64) {
-    warp_topm_pair(kk, p.ncand, m, Dw, top, Rw, Xw, p.words, sk, si);
+    listed = warp_topm_pair(kk, p.ncand, m, Dw, top, Rw, Xw, p.words, sk, si, lst);
   } else {
     warp_topm(kk, p.ncand, m, Rw, p.words, sk, si, Dw, true);
     warp_topm(kk, p.ncand, m, Xw, p.words, sk, si, Dw, false);
   }
-  for (int w = lane; w < p.words; w += 32) Dw[w] = (Dw[w] & ~Rw[w]) | Xw[w];
+  if (!listed) {
+    lst = reinterpret_cast<uint16_t*>(kk);  // 2 key_words >= 2m entries
+    nl = 0;
+    for (int w = 0; w < p.words; ++w) {
+      const uint32_t sw = Rw[w] | Xw[w];
+      if ((sw >> lane) & 1u)
+        lst[nl + __popc(sw & ((1u << lane) - 1u))] =
+            (uint16_t)((w * 32 + lane) | (((Xw[w] >> lane) & 1u) << 15));
+      nl += __popc(sw);
+    }
+    __syncwarp();
+  }
+  // every listed block changes sides: restores leave D, drops join it
+  for (int e = lane; e < nl; e += 32) {
+    const int j = lst[e] & 0x7fff;
+    atomicXor(&Dw[j >> 5], 1u << (j & 31));
+  }
   __syncwarp();
   // state of the new set (Eq. 10-12): the swapped blocks update g~ and K
   const float2 y = *reinterpret_cast<const float2*>(p.ytil + ri * 64 + 2 * lane);
   const float2 gold = *reinterpret_cast<const float2*>(p.gtil + ri * 64 + 2 * lane);
   float g0 = gold.x, g1 = gold.y, Kn = K;
-  swap_drift(Rw, Xw, p, Prow, zt_h, y.x, y.y, kk, g0, g1, Kn);
+  swap_drift_list(lst, nl, Prow, zt_h, y.x, y.y, g0, g1, Kn);
   const float Gn = warp_sum(g0 * g0 + g1 * g1);
   const float Kc = fmaxf(Kn, kEps);
   const float Jn = Gn / (Kc * Kc);
