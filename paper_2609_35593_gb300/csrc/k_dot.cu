@@ -194,10 +194,12 @@ __global__ void __launch_bounds__(kDotThreads)
         for (int k = 0; k < 32; ++k)
           if (jq + k < p.nb) ps += exp2f(o[k] - pm);
       } else {
+        // ||z~_j||^2 of this quarter's 32 blocks: one coalesced load, then by shuffle
         const int jq = j0 + 32 * q;
+        const float bl = (jq + lane < p.nb) ? p.b[(int64_t)h * p.nb + jq + lane] : 0.f;
 #pragma unroll
         for (int k = 0; k < 32; ++k) {
-          const float bz = (jq + k < p.nb) ? p.b[(int64_t)h * p.nb + jq + k] : 0.f;
+          const float bz = __shfl_sync(0xffffffffu, bl, k);
           o[k] = fmaxf(fmaf(-2.0f, __uint_as_float(v[k]), a + bz), 0.f);
         }
       }

@@ -770,8 +770,11 @@ __host__ __device__ constexpr int key_words(int ld) { return ld > 320 ? ld : 320
 __host__ __device__ constexpr size_t warp_scratch_words(int ld, int words_per_warp) {
   return ((size_t)key_words(ld) + kSurvivors + kSurvivors / 2 + words_per_warp + 3) / 4 * 4;
 }
-// the score kernel's words after the survivors: its drop-set mask, then 256 radix counters
-__host__ __device__ constexpr int score_mask_words(int words) { return (words + 3) / 4 * 4 + 256; }
+// the score kernel's words after the survivors: its drop-set mask, then (with the CDF rule,
+// which keeps the keys past the selection) 256 radix counters
+__host__ __device__ constexpr int score_mask_words(int words, bool cdf) {
+  return (words + 3) / 4 * 4 + (cdf ? 256 : 0);
+}
 
 
 
@@ -891,13 +894,14 @@ __global__ void __launch_bounds__(32 * kRowWarps, 8) k_score_rows(SelPtrs p, Bud
   const float* Prow = p.P + ri * p.ld;
   const float* qrow = p.q + ri * p.ld;
   const float* zt_h = p.ztil + (int64_t)h * p.nb * 64;
-  uint32_t* base =
-      reinterpret_cast<uint32_t*>(smem_raw) + (size_t)warp * warp_scratch_words(p.ld, score_mask_words(p.words));
+  uint32_t* base = reinterpret_cast<uint32_t*>(smem_raw) +
+                   (size_t)warp * warp_scratch_words(p.ld, score_mask_words(p.words, v.cdf > 0.f));
   uint32_t* kk = base;
   uint32_t* sk = base + key_words(p.ld);
   uint16_t* si = reinterpret_cast<uint16_t*>(sk + kSurvivors);
   uint32_t* sel = sk + kSurvivors + kSurvivors / 2;
-  uint32_t* hist = sel + (p.words + 3) / 4 * 4;  // radix counters (the keys stay for the CDF rule)
+  // radix counters: in the spent key area, or after the mask when the CDF rule needs the keys
+  uint32_t* hist = v.cdf > 0.f ? sel + (p.words + 3) / 4 * 4 : kk;
   row_keys(p.ncand, kk, [&](int j, uint32_t (&k4)[4]) {
     const float4 P4 = *reinterpret_cast<const float4*>(Prow + j);
     const float4 q4 = *reinterpret_cast<const float4*>(qrow + j);
@@ -1115,6 +1119,13 @@ __global__ void __launch_bounds__(1024) k_rowptr(const int32_t* __restrict__ kco
   if (t == 1023) row_ptr[R] = (int32_t)off;
 }
 
+// The kept blocks of one mask word w of a row, written from list position `at` on.
+__device__ __forceinline__ void csr_write_word(const CsrOut& o, uint32_t bits, int w, int at,
+                                               int expect, int64_t off) {
+  for (; bits; bits &= bits - 1u, ++at)
+    if (at < expect && off + at < o.cap) o.col_idx[off + at] = w * 32 + (__ffs(bits) - 1);
+}
+
 __global__ void k_csr(SelPtrs p, Budgets bud, CsrBases cb, int H, CsrOut o) {
   const int h = blockIdx.y, lane = threadIdx.x & 31;
   const int rpi = o.rows_per_item;
@@ -1140,41 +1151,47 @@ __global__ void k_csr(SelPtrs p, Budgets bud, CsrBases cb, int H, CsrOut o) {
                                                  : (int64_t)i * (c + ns));
     expect[r] = o.variable ? (int)(o.row_ptr[ri[r] + 1] - off[r]) : (dense[r] ? p.nb : c + ns);
   }
-  const uint32_t below = (1u << lane) - 1u;
+  // Lane l owns word w0 + l of each row: one warp scan of the lanes' kept counts gives
+  // every word's first list position, then each lane writes the blocks of its own word.
   int posU = 0;
   for (int w0 = 0; w0 < p.words; w0 += 32) {
-    // 32 words of each row per coalesced load, handed out by shuffle
-    uint32_t mine[2];
+    const int w = w0 + lane;
+    uint32_t keep[2] = {0u, 0u};
 #pragma unroll
     for (int r = 0; r < 2; ++r) {
-      mine[r] = (r < nr && !dense[r] && w0 + lane < p.words) ? p.bmask[ri[r] * p.words + w0 + lane] : 0u;
-      if (r < nr && o.drop_mask && w0 + lane < p.words) o.drop_mask[ri[r] * p.words + w0 + lane] = mine[r];
+      if (r < nr && w < p.words) {
+        const uint32_t dm = dense[r] ? 0u : p.bmask[ri[r] * p.words + w];
+        if (o.drop_mask) o.drop_mask[ri[r] * p.words + w] = dm;
+        keep[r] = ~dm & valid_bits(w, p.nb);
+      }
     }
-    const int nw = min(32, p.words - w0);
-    for (int k = 0; k < nw; ++k) {
-      const int w = w0 + k;
-      const uint32_t valid = valid_bits(w, p.nb);
-      uint32_t keep[2];
+    // a 128-token query block keeps its list for both 64-row halves of the tile
+    const uint32_t kb = rpi == 1 ? keep[0] : keep[1];
+    const uint32_t un = o.plist ? (keep[0] | kb) : 0u;
+    const int cAB = __popc(keep[0]) | (__popc(keep[1]) << 16), cU = __popc(un);
+    int iAB = cAB, iU = cU;
 #pragma unroll
-      for (int r = 0; r < 2; ++r) {
-        keep[r] = r < nr ? ~__shfl_sync(kFull, mine[r], k) & valid : 0u;
-        const int at = pos[r] + __popc(keep[r] & below);
-        if (((keep[r] >> lane) & 1u) && at < expect[r] && off[r] + at < o.cap)
-          o.col_idx[off[r] + at] = w * 32 + lane;
-        pos[r] += __popc(keep[r]);
-      }
-      if (o.plist) {
-        // a 128-token query block keeps its list for both 64-row halves of the tile
-        const uint32_t kb = rpi == 1 ? keep[0] : keep[1];
-        const uint32_t un = keep[0] | kb;
-        const int at = posU + __popc(un & below);
-        if (((un >> lane) & 1u) && off[0] + at < o.plist_cap) {
-          const int m = (int)((keep[0] >> lane) & 1u) | (int)(((kb >> lane) & 1u) << 1);
-          o.plist[off[0] + at] = (w * 32 + lane) | (m << 16);
-        }
-        posU += __popc(un);
+    for (int d = 1; d < 32; d <<= 1) {
+      const int yAB = __shfl_up_sync(kFull, iAB, d), yU = __shfl_up_sync(kFull, iU, d);
+      if (lane >= d) {
+        iAB += yAB;
+        iU += yU;
       }
     }
+    const int tAB = __shfl_sync(kFull, iAB, 31), tU = __shfl_sync(kFull, iU, 31);
+    csr_write_word(o, keep[0], w, pos[0] + ((iAB - cAB) & 0xffff), expect[0], off[0]);
+    csr_write_word(o, keep[1], w, pos[1] + ((iAB - cAB) >> 16), expect[1], off[1]);
+    if (o.plist) {
+      int au = posU + iU - cU;
+      for (uint32_t bits = un; bits; bits &= bits - 1u, ++au) {
+        const int b = __ffs(bits) - 1;
+        const int m = (int)((keep[0] >> b) & 1u) | (int)(((kb >> b) & 1u) << 1);
+        if (off[0] + au < o.plist_cap) o.plist[off[0] + au] = (w * 32 + b) | (m << 16);
+      }
+    }
+    pos[0] += tAB & 0xffff;
+    pos[1] += tAB >> 16;
+    posU += tU;
   }
   if (lane == 0) {
     for (int r = 0; r < nr; ++r) {
@@ -1225,7 +1242,8 @@ cudaError_t launch_score(const SelectArgs& a, cudaStream_t st) {
   if ((e = launch_logits(a, st)) != cudaSuccess) return e;
   if ((e = launch_yagg(a, st)) != cudaSuccess) return e;
   if ((e = launch_drift_norms(a, st)) != cudaSuccess) return e;
-  const size_t rsmem = (size_t)kRowWarps * warp_scratch_words(s.ld, score_mask_words(s.words)) * 4;
+  const size_t rsmem =
+      (size_t)kRowWarps * warp_scratch_words(s.ld, score_mask_words(s.words, a.v.cdf > 0.f)) * 4;
   e = cudaFuncSetAttribute(k_score_rows, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)rsmem);
   if (e != cudaSuccess) return e;
   k_score_rows<<<dim3((s.nqc + kRowWarps - 1) / kRowWarps, s.H), 32 * kRowWarps, rsmem, st>>>(

@@ -512,6 +512,46 @@ def test_selection_variants(name, variant, rounds):
     assert r["worst_row_rel"] <= G.DRIFT_REL and r["sum_rel_gpu_vs_oracle"] <= G.DRIFT_REL, r
 
 
+@pytest.mark.parametrize("name", ["tiny_v2", "vggt_v8"])
+@pytest.mark.parametrize("variant,rounds", [
+    (O.Variant(key="probability"), 3),
+    (O.Variant(key="random", seed=11), 2),
+    (O.Variant(maximize="swap"), 3),
+    (O.Variant(maximize="full"), 3),
+])
+def test_selection_variants_paper_grid(name, variant, rounds):
+    """The ablation variants on the paper's grid (128-token query blocks): identical drop
+    sets outside the decision margin, drift within 1e-3."""
+    wl = synth.WORKLOADS[name]
+    layer = G.Layer(synth.make_inputs(wl), wl.n_special, wl.budgets(), rounds, wl.rho,
+                    variant=variant, q_block=128).run(attention=False)
+    r = G.compare_selection(layer, layer.oracle_select())
+    assert r["mismatched"] == 0, r
+    assert r["exact"] >= 0.95 * (r["exact"] + r["near"]), r
+    assert r["worst_row_rel"] <= G.DRIFT_REL and r["sum_rel_gpu_vs_oracle"] <= G.DRIFT_REL, r
+
+
+def test_cdf_threshold_headline_shape_sampled():
+    """The CDF threshold at the 32-view headline shape: sampled rows of the drop sets against
+    the oracle, and every CSR row exactly the complement of its drop set."""
+    wl = synth.WORKLOADS["vggt_v32"]
+    variant = O.Variant(key="probability", cdf=0.9)
+    layer = G.Layer(synth.make_inputs(wl), wl.n_special, wl.budgets(), 0, wl.rho,
+                    variant=variant).run(attention=False)
+    rng = np.random.default_rng(7)
+    rows = [(int(h), int(i)) for h, i in zip(rng.integers(0, layer.H, 40),
+                                             rng.integers(0, layer.nqc, 40))]
+    r = G.compare_selection(layer, layer.oracle_select(rows))
+    assert r["mismatched"] == 0, r
+    assert r["worst_row_rel"] <= G.DRIFT_REL, r
+    rp, ci = layer.csr()
+    D = layer.drop_sets()
+    assert rp[-1] == int((~D[:, :layer.nqc]).sum()) + layer.H * (layer.nq - layer.nqc) * layer.nb
+    for h, i in rows:
+        k = ci[rp[h * layer.nq + i]:rp[h * layer.nq + i + 1]]
+        assert np.array_equal(k, np.nonzero(~D[h, i])[0])
+
+
 @pytest.mark.parametrize("name,q_block", [("tiny_v2", 64), ("vggt_v8", 64), ("vggt_v8", 128)])
 @pytest.mark.parametrize("variant", [
     O.Variant(key="probability", cdf=0.9),  # SparseVGGT's rule: top-k plus the CDF threshold
