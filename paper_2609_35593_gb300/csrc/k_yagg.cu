@@ -6,8 +6,11 @@
 // k_dot left in lstat.  P overwrites L in place; y~ is written in fp32, as three bf16
 // terms (the row operand of the drift-norm products) and as ||y~_i||^2.
 //
-// One CTA per 128 candidate rows of a head, 544 threads, 64 key blocks per chunk, two
-// pipeline stages:
+// One CTA per 128 candidate rows of a head and part of the key blocks (the blocks are split
+// into `parts` consecutive ranges of chunks when that fills more of the GPU; each part's
+// partial y~ goes to scratch and the CTA that finishes last sums the parts in their order and
+// writes the outputs, so the result does not depend on which finishes first), 544 threads,
+// 64 key blocks per chunk, two pipeline stages:
 //   warp 16    lane 0 loads chunk c + 1 by TMA (L: two 32-column fp32 boxes; z~: its three
 //              bf16 term tiles, 64 blocks x 64 channels) while the chunk c is converted;
 //              then the converged warp, one elected lane, issues the chunk's MMAs
@@ -53,6 +56,7 @@ struct __align__(1024) YSmem {
   uint64_t done;
   uint32_t tmem_base;
   int abort;
+  int last;  // this CTA sums the parts
 };
 
 struct YParams {
@@ -64,6 +68,9 @@ struct YParams {
   float* ny;        // [H, nb]
   int64_t term_words;  // H nb 32
   uint32_t* status;
+  int parts;           // key-block parts per stripe of 128 rows
+  float* part_buf;     // [parts][H][nq][64] partial y~ (parts > 1)
+  uint32_t* arrivals;  // [H][stripes] parts done, zero before the launch (parts > 1)
 };
 
 // (A term, B term) of product q of the six, smallest first (as in k_dot).
@@ -79,6 +86,11 @@ __device__ __forceinline__ bool y_wait(uint64_t* bar, uint32_t parity, volatile 
   return ok != 0;
 }
 
+// Barrier among the converter warps only (named barrier 1; the MMA warp takes no part).
+__device__ __forceinline__ void conv_sync() {
+  asm volatile("bar.sync 1, %0;" ::"n"(32 * kConvWarps) : "memory");
+}
+
 __device__ __forceinline__ void y_give_up(YSmem& S, uint32_t* status) {
   flag_status(status, kStatusTimeout);
   *reinterpret_cast<volatile int*>(&S.abort) = 1;
@@ -90,9 +102,12 @@ __global__ void __launch_bounds__(kYThreads, 1)
   extern __shared__ uint8_t smem_raw[];
   YSmem& S = *reinterpret_cast<YSmem*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) &
                                        ~static_cast<uintptr_t>(1023));
-  const int h = blockIdx.y, i0 = blockIdx.x * kYRows;
+  const int h = blockIdx.y, i0 = blockIdx.x * kYRows, part = blockIdx.z;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   volatile int* abort = &S.abort;
+  // this part's chunks [c0, c1); the pipeline counts them from 0
+  const int c0 = (int)((int64_t)p.nchunks * part / p.parts);
+  const int nch = (int)((int64_t)p.nchunks * (part + 1) / p.parts) - c0;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < kYStages; ++s) {
@@ -126,7 +141,7 @@ __global__ void __launch_bounds__(kYThreads, 1)
       const int s = c % kYStages, u = c / kYStages;
       if (u > 0 && !y_wait(&S.empty[s], (u - 1) & 1, abort)) return false;
       if (lane == 0) {
-        const int j0 = c * kYChunk;
+        const int j0 = (c0 + c) * kYChunk;
         mbar_arrive_expect_tx(&S.full[s], 2 * 16384 + 3 * 8192);
         tma_load_3d(S.L[s][0], &tmL, &S.full[s], j0, i0, h);
         tma_load_3d(S.L[s][1], &tmL, &S.full[s], j0 + 32, i0, h);
@@ -139,8 +154,8 @@ __global__ void __launch_bounds__(kYThreads, 1)
     };
     const uint32_t idesc = idesc_bf16_f32(kYRows, 64, true);
     if (!failed && !produce(0)) failed = true;
-    for (int c = 0; c < p.nchunks && !failed; ++c) {
-      if (c + 1 < p.nchunks && !produce(c + 1)) {
+    for (int c = 0; c < nch && !failed; ++c) {
+      if (c + 1 < nch && !produce(c + 1)) {
         failed = true;
         break;
       }
@@ -161,7 +176,7 @@ __global__ void __launch_bounds__(kYThreads, 1)
                         (c > 0 || q > 0 || k > 0) ? 1u : 0u);
         }
         mma_commit(&S.empty[s]);
-        if (c + 1 == p.nchunks) mma_commit(&S.done);
+        if (c + 1 == nch) mma_commit(&S.done);
       }
       __syncwarp();
       ++consumed;
@@ -199,13 +214,13 @@ __global__ void __launch_bounds__(kYThreads, 1)
     }
     float* Prow = p.P + (row_ok ? ri : 0) * p.ld;
     bool failed = false;
-    for (int c = 0; c < p.nchunks; ++c) {
+    for (int c = 0; c < nch; ++c) {
       const int s = c % kYStages, par = (c / kYStages) & 1;
       if (!y_wait(&S.full[s], par, abort)) {
         failed = true;
         break;
       }
-      const int jb = c * kYChunk + 16 * qq;  // first block of this thread's 16
+      const int jb = (c0 + c) * kYChunk + 16 * qq;  // first block of this thread's 16
       // L: box qq / 2, 16-byte chunks 4 (qq mod 2) .. + 3 of row r
       const uint8_t* lrow = S.L[s][qq >> 1] + r * 128;
       float pv[16];
@@ -242,10 +257,55 @@ __global__ void __launch_bounds__(kYThreads, 1)
     if (failed && lane == 0) y_give_up(S, p.status);
     // ---- epilogue: y~ row r, channels 16 qq .. 16 qq + 15 ------------------------------
     float nyp = 0.f;
+    bool have = false;
+    uint32_t v[16];
     if (!failed && y_wait(&S.done, 0, abort)) {
       tc_fence_after();
-      uint32_t v[16];
       RESS_TMEM_LD16(tmem + ((uint32_t)(32 * (warp & 3)) << 16) + 16 * qq, v);
+      have = true;
+    } else if (lane == 0) {
+      y_give_up(S, p.status);
+    }
+    if (p.parts > 1) {
+      // this part's sums to scratch; the last part to arrive adds all parts in order
+      float* mine = p.part_buf + (((int64_t)part * gridDim.y + h) * p.nq + (row_ok ? i : 0)) * 64 + 16 * qq;
+      if (have && row_ok) {
+#pragma unroll
+        for (int k = 0; k < 4; ++k)
+          *reinterpret_cast<float4*>(mine + 4 * k) =
+              make_float4(__uint_as_float(v[4 * k]), __uint_as_float(v[4 * k + 1]),
+                          __uint_as_float(v[4 * k + 2]), __uint_as_float(v[4 * k + 3]));
+      }
+      __threadfence();
+      conv_sync();
+      if (threadIdx.x == 0) {
+        const uint32_t before = atomicAdd(&p.arrivals[h * gridDim.x + blockIdx.x], 1u);
+        S.last = before == (uint32_t)(p.parts - 1);
+        if (S.last) p.arrivals[h * gridDim.x + blockIdx.x] = 0u;  // ready for the next call
+      }
+      conv_sync();
+      have = have && S.last;
+      if (have && row_ok) {
+        __threadfence();
+        float acc[16];
+#pragma unroll
+        for (int k = 0; k < 16; ++k) acc[k] = 0.f;
+        for (int t = 0; t < p.parts; ++t) {
+          const float* src = p.part_buf + (((int64_t)t * gridDim.y + h) * p.nq + i) * 64 + 16 * qq;
+#pragma unroll
+          for (int k = 0; k < 4; ++k) {
+            const float4 q4 = __ldcg(reinterpret_cast<const float4*>(src + 4 * k));
+            acc[4 * k] += q4.x;
+            acc[4 * k + 1] += q4.y;
+            acc[4 * k + 2] += q4.z;
+            acc[4 * k + 3] += q4.w;
+          }
+        }
+#pragma unroll
+        for (int k = 0; k < 16; ++k) v[k] = __float_as_uint(acc[k]);
+      }
+    }
+    if (have) {
       if (row_ok) {
         float* yrow = p.ytil + ri * 64 + 16 * qq;
 #pragma unroll
@@ -270,14 +330,12 @@ __global__ void __launch_bounds__(kYThreads, 1)
 #pragma unroll
         for (int k = 0; k < 16; ++k) nyp = fmaf(__uint_as_float(v[k]), __uint_as_float(v[k]), nyp);
       }
-    } else if (lane == 0) {
-      y_give_up(S, p.status);
     }
     S.ny_part[qq][r] = nyp;
   }
   tc_fence_before();
   __syncthreads();
-  if (threadIdx.x < kYRows) {
+  if (threadIdx.x < kYRows && (p.parts == 1 || S.last)) {
     const int i = i0 + threadIdx.x;
     if (i < p.nqc && !*abort)
       p.ny[(int64_t)h * p.nq + i] = (S.ny_part[0][threadIdx.x] + S.ny_part[1][threadIdx.x]) +
@@ -312,10 +370,29 @@ cudaError_t launch_yagg(const SelectArgs& a, cudaStream_t st) {
   p.ny = (float*)(a.ws + a.L.ny);
   p.term_words = (int64_t)s.H * s.nq * 32;
   p.status = (uint32_t*)(a.ws + a.L.status);
+  // One CTA per SM: when the stripes of rows leave SMs idle, split the key blocks into as
+  // many parts (up to 3) as still run in one wave.  (A second wave costs more than the
+  // split saves: measured at 32 views on 64-token query blocks, 96 stripes.)
+  const int stripes = (s.nqc + kYRows - 1) / kYRows;
+  int dev = 0, sms = 1;
+  cudaGetDevice(&dev);
+  cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  p.parts = 1;
+  // (the partial sums of k parts take 64 k of the ld floats per row of the gains array)
+  for (int k = 2; k <= 3 && k <= p.nchunks && 64 * k <= s.ld; ++k)
+    if ((int64_t)stripes * s.H * k <= sms) p.parts = k;
+  // scratch while the selection scores: the gains array (partial y~) and the attention
+  // items' length array (arrival counts), both unused until the restoration rounds
+  p.part_buf = (float*)(a.ws + a.L.t);
+  p.arrivals = (uint32_t*)(a.ws + a.L.plen);
+  cudaError_t e;
+  if (p.parts > 1 &&
+      (e = cudaMemsetAsync(p.arrivals, 0, (size_t)stripes * s.H * sizeof(uint32_t), st)) != cudaSuccess)
+    return e;
   const size_t smem = sizeof(YSmem) + 1024;
-  cudaError_t e = cudaFuncSetAttribute(k_yagg, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  e = cudaFuncSetAttribute(k_yagg, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
-  k_yagg<<<dim3((s.nqc + kYRows - 1) / kYRows, s.H), kYThreads, smem, st>>>(tl, tz, p);
+  k_yagg<<<dim3(stripes, s.H, p.parts), kYThreads, smem, st>>>(tl, tz, p);
   note_launch();
   return cudaGetLastError();
 }
