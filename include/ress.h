@@ -296,6 +296,14 @@ int ress_sparse_attn_noalloc(const ress_dims* dims, const uint16_t* Q, const uin
                              const uint16_t* V, const int32_t* row_ptr, const int32_t* col_idx,
                              int64_t col_capacity, uint16_t* O, int32_t wait, void* stream);
 
+/* Failure detection without a fault, for tests of the error path: one thread waits on a
+ * shared-memory barrier that nothing arrives at, with the bounded wait the kernels use
+ * (limit_us microseconds, 1..100000), gives up and records RESS_ETIMEOUT in the workspace
+ * status word exactly as a kernel's timed-out wait does; ress_status then reports it and
+ * clears it, and the context stays usable.  ws: a workspace of any layer (only its status
+ * word is used).  RESS_EINVAL on a bad pointer or limit.  No paper counterpart. */
+int ress_wait_selftest(void* ws, size_t ws_bytes, uint32_t limit_us, void* stream);
+
 /* Synchronises `stream`, returns the workspace status word as a ress_status_code
  * (RESS_OK, RESS_ETIMEOUT or RESS_EDEVICE) and clears it. */
 int ress_status(void* ws, void* stream);

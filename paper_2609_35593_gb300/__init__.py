@@ -98,6 +98,7 @@ _SIGS = {
                                      _c.c_int32, _c.c_float, _P, _c.c_size_t, _P, _P, _c.c_int64,
                                      _P, _P]),
     "ress_status": (_c.c_int, [_P, _P]),
+    "ress_wait_selftest": (_c.c_int, [_P, _c.c_size_t, _c.c_uint32, _P]),
     "ress_score_variant": (_c.c_int, [_c.POINTER(Dims), _P, _P, _P, _P, _P, _c.POINTER(Variant), _P,
                                       _c.c_size_t, _P]),
     "ress_restore_variant": (_c.c_int, [_c.POINTER(Dims), _P, _c.c_int32, _c.c_float,
@@ -335,6 +336,13 @@ def sparse_attn_noalloc(d: Dims, Q, K, V, row_ptr, col_idx, O, wait: bool = True
                                          _dev(V, _bf16(), "V"), _dev(row_ptr, (torch.int32,), "row_ptr"),
                                          _dev(col_idx, (torch.int32,), "col_idx"), col_idx.numel(),
                                          _dev(O, _bf16(), "O"), 1 if wait else 0, _stream(stream)))
+
+
+def wait_selftest(ws, limit_us: int = 20000, stream=None):
+    """ress_wait_selftest: a bounded wait that nothing completes, recorded as RESS_ETIMEOUT in
+    the workspace status word (read it with status())."""
+    _check(_lib.ress_wait_selftest(_dev(ws, None, "ws"), ws.numel() * ws.element_size(),
+                                   int(limit_us), _stream(stream)))
 
 
 def status(ws, stream=None):

@@ -19,6 +19,7 @@
 #include <stddef.h>
 
 #include "ress_internal.cuh"
+#include "sm100_ptx.cuh"
 
 namespace ress {
 
@@ -1202,6 +1203,38 @@ __global__ void k_csr(SelPtrs p, Budgets bud, CsrBases cb, int H, CsrOut o) {
     if (!o.variable && h == H - 1 && u == items - 1) o.row_ptr[(int64_t)H * p.nq] = (int32_t)cb.base[H];
     if (o.plist) o.plen[(int64_t)h * items + u] = posU;
   }
+}
+
+// ------------------------------------------------------------------------------------
+// Failure detection without a fault: one thread waits on a shared-memory barrier that
+// nothing arrives at, with the bounded wait of the kernels (a time limit, here also an
+// iteration limit), and records the timeout in the status word as a kernel's wait does.
+// ------------------------------------------------------------------------------------
+__global__ void k_wait_selftest(uint32_t* status, uint64_t limit_ns) {
+  __shared__ uint64_t bar;
+  if (threadIdx.x == 0) {
+    ptx::mbar_init(&bar, 1);
+    ptx::fence_barrier_init();
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    bool done = false;
+    const uint64_t t0 = ptx::globaltimer();
+    for (uint32_t it = 0; it < (1u << 24); ++it) {
+      if (ptx::mbar_try_wait(&bar, 0)) {
+        done = true;
+        break;
+      }
+      if (ptx::globaltimer() - t0 > limit_ns) break;
+    }
+    if (!done) flag_status(status, kStatusTimeout);
+  }
+}
+
+cudaError_t launch_wait_selftest(uint32_t* status, uint64_t limit_ns, cudaStream_t st) {
+  k_wait_selftest<<<1, 32, 0, st>>>(status, limit_ns);
+  note_launch();
+  return cudaGetLastError();
 }
 
 // ------------------------------------------------------------------------------------

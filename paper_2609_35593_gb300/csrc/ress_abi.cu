@@ -164,6 +164,7 @@ int check_variant(const ress_variant* v, ress::Variant* out) {
 
 namespace ress {
 void note_launch() { g_kernel_launches.fetch_add(1, std::memory_order_relaxed); }
+cudaError_t launch_wait_selftest(uint32_t* status, uint64_t limit_ns, cudaStream_t st);  // k_select.cu
 }  // namespace ress
 
 extern "C" {
@@ -483,6 +484,18 @@ int ress_forward_host(const ress_dims* d, const uint16_t* Q_host, const uint16_t
   if (je == cudaSuccess) je = cudaStreamWaitEvent(st, o->copied, 0);
   if (ce != cudaSuccess) return cuda_fail(ce, "ress_forward_host attention chunk");
   if (je != cudaSuccess) return cuda_fail(je, "ress_forward_host join");
+  return ok();
+}
+
+int ress_wait_selftest(void* ws, size_t ws_bytes, uint32_t limit_us, void* stream) {
+  int e = check_ptr(ws, 256, "ws");
+  if (e) return e;
+  if (ws_bytes < 64) return fail(RESS_EWORKSPACE, "workspace has %zu bytes, needs 64", ws_bytes);
+  if (limit_us < 1 || limit_us > 100000)
+    return fail(RESS_EINVAL, "limit_us %u outside 1..100000", limit_us);
+  cudaError_t ce = ress::launch_wait_selftest(static_cast<uint32_t*>(ws), 1000ull * limit_us,
+                                              static_cast<cudaStream_t>(stream));
+  if (ce != cudaSuccess) return cuda_fail(ce, "ress_wait_selftest");
   return ok();
 }
 

@@ -134,6 +134,15 @@ def test_variant_names_map_to_the_header_values():
     assert (ress.variant().key, ress.variant().direction) == (0, 0)
 
 
+def test_wait_selftest_validates_before_launch():
+    """The bounded-wait self-test rejects a bad limit or workspace on the host."""
+    ptr = ctypes.c_void_p(1 << 20)
+    assert ress._lib.ress_wait_selftest(ptr, 4096, 0, None) == EINVAL
+    assert ress._lib.ress_wait_selftest(ptr, 4096, 100001, None) == EINVAL
+    assert ress._lib.ress_wait_selftest(ptr, 16, 1000, None) == EWORKSPACE
+    assert ress._lib.ress_wait_selftest(None, 4096, 1000, None) == EINVAL
+
+
 def test_cdf_variant_capacity_and_validation():
     """A CDF threshold may keep every block: the capacity is H * nq * nb.  Out-of-range
     thresholds, a maximising direction, a nonzero reserved field and restoration rounds

@@ -601,6 +601,25 @@ def test_cdf_threshold_variant(name, q_block, variant):
     assert a["max_abs"] <= G.ATT_MAX_ABS and a["mean_rel"] <= G.ATT_MEAN_REL, a
 
 
+def test_timed_out_wait_is_reported_and_context_stays_usable(tiny):
+    """Failure detection without a fault: a kernel's bounded wait on a barrier that nothing
+    completes gives up after its limit, the status word reports RESS_ETIMEOUT once (then is
+    clear), and the next forward on the same context gives the same bits as before."""
+    import paper_2609_35593_gb300 as ress
+    layer, _ = layer_for("tiny_v2")
+    r, b = layer.ress, layer.buf
+    r.prepare_wo(layer.d, layer.W, b.F)
+    r.wait_selftest(b.ws, 20000)
+    with pytest.raises(ress.RessError) as e:
+        r.status(b.ws)
+    assert e.value.code == -5
+    r.status(b.ws)  # cleared
+    r.forward(layer.d, layer.Q, layer.K, layer.V, b.F, layer.c_h, layer.rounds, layer.rho, b.ws,
+              b.row_ptr, b.col_idx, b.O, b.J_best)
+    r.status(b.ws)
+    assert torch.equal(b.O.view(torch.int16), tiny.buf.O.view(torch.int16))
+
+
 def test_invalid_variant_is_rejected(tiny):
     import paper_2609_35593_gb300 as ress
     bad = ress.Variant(7, 0, 0)
