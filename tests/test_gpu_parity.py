@@ -315,6 +315,56 @@ def test_large_shapes_sampled(name, kw):
     assert a["max_abs"] <= G.ATT_MAX_ABS and a["mean_rel"] <= G.ATT_MEAN_REL, a
 
 
+def test_maximum_shape_sampled():
+    """The largest sequence the library takes (RESS_MAX_BLOCKS = 4096 key blocks, 262,144
+    tokens; 2 heads): a budget above 128 per row (the all-keys selection of the score
+    kernel) and a first round with m > 64 (the bitmask path of the rounds).  Sampled rows of
+    the selection and of the attention against the oracle, and the invariants on every row."""
+    N, H, ns = 64 * 4096, 2, 5
+    inp = synth.make_random_layer(N, H, 64 * H, seed=4096)
+    nc = O.n_candidates(N, ns)
+    c = int(round(0.1 * nc))
+    layer = G.Layer(inp, ns, [c] * H, 2).run()
+    assert layer.nb == 4096 and layer.ncand == nc
+    rng = np.random.default_rng(3)
+    rows = [(int(h), int(i)) for h, i in zip(rng.integers(0, H, 6), rng.integers(0, nc, 6))]
+    r = G.compare_selection(layer, layer.oracle_select(rows + [(H - 1, nc - 1)]))
+    assert r["mismatched"] == 0, r
+    assert r["worst_row_rel"] <= G.DRIFT_REL, r
+    J0 = layer.ws("J0", shape=(H, layer.nb))
+    Jb = layer.buf.J_best.cpu().numpy().reshape(H, layer.nb)
+    assert np.all(Jb[:, :nc] <= J0[:, :nc])
+    rp, ci = layer.csr()
+    assert rp[-1] == ci.size == H * (nc * (c + layer.nb - nc) + (layer.nb - nc) * layer.nb)
+    a = G.compare_attention(layer, rows[:4] + [(0, layer.nb - 1)])
+    assert a["max_abs"] <= G.ATT_MAX_ABS and a["mean_rel"] <= G.ATT_MEAN_REL, a
+
+
+@pytest.mark.parametrize("q_block", [64, 128])
+def test_equal_keys_keep_the_lowest_indices(q_block):
+    """Ties: with every key token equal, every pooled probability of a row is the same, so
+    the probability rule keeps the c_h candidates of lowest index (the tie order of Eq. 7's
+    top-c in this build and in the oracle) on every row; the rounds then follow the oracle."""
+    N, H, ns = 64 * 40, 2, 5
+    inp = synth.make_random_layer(N, H, 64 * H, seed=40)
+    inp["K"][:] = inp["K"][0:1]
+    nc = O.n_candidates(N, ns)
+    c = 11
+    layer = G.Layer(inp, ns, [c] * H, 0, variant=O.Variant(key="probability"),
+                    q_block=q_block).run(attention=False)
+    D = layer.drop_sets()
+    want = np.ones(layer.nb, dtype=bool)
+    want[:c] = False
+    want[nc:] = False
+    for h in range(H):
+        for i in range(layer.nqc):
+            assert np.array_equal(D[h, i], want), (h, i)
+    layer3 = G.Layer(inp, ns, [c] * H, 3, variant=O.Variant(key="probability"),
+                     q_block=q_block).run(attention=False)
+    r = G.compare_selection(layer3, layer3.oracle_select())
+    assert r["mismatched"] == 0, r
+
+
 @pytest.mark.parametrize("name,q_block", [("tiny_v2", 64), ("tiny_v2", 128), ("vggt_v8", 64)])
 def test_forward_host_equals_forward(name, q_block):
     """ress_forward_host (copies in, selection, then the attention in chunks of query rows
