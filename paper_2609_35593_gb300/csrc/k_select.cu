@@ -885,7 +885,7 @@ __device__ void cdf_extend(const uint32_t* kk, const float* __restrict__ Prow, u
 // The variant picks the key: the Eq. 7 drift key (ReSS), the pooled probability, or the top
 // 24 bits of SplitMix64 at seed + (h 4096 + i) 4096 + j; the full sign flip keeps the
 // smallest keys (complemented keys, ties still to the lower index).
-__global__ void __launch_bounds__(32 * kRowWarps, 8) k_score_rows(SelPtrs p, Budgets bud,
+__global__ void __launch_bounds__(32 * kRowWarps, 9) k_score_rows(SelPtrs p, Budgets bud,
                                                                   Variant v) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
