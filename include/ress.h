@@ -7,7 +7,11 @@
  *   ress_restore     R budget-neutral restoration rounds with track-best and the kept-block
  *                    lists (Sec. 4.3, Eq. 10-17)
  *   ress_sparse_attn exact attention over the kept 64x64 blocks (Sec. 3 step (3))
- *   ress_forward     the three in order on one stream
+ *   ress_forward     the three in order on one stream (ress_forward_host: from and to
+ *                    host buffers, the output copied back while the attention runs)
+ * Also: the ablation variants of the selection (ress_score_variant, ress_restore_variant),
+ * the residual update and token-level drift (ress_out_proj, ress_token_drift), an
+ * allocation-free attention entry point, and a bounded-wait self-test of the error path.
  *
  * Conventions shared by every call
  *   - Pointers named "device" point to GPU memory owned by the caller; the library never
@@ -222,7 +226,10 @@ int ress_sparse_attn_f32(const ress_dims* dims, const uint16_t* Q, const uint16_
                          const uint16_t* V, const int32_t* row_ptr, const int32_t* col_idx,
                          int64_t col_capacity, float* O, void* ws, size_t ws_bytes, void* stream);
 
-/* ress_score, ress_restore and ress_sparse_attn in order on one stream. */
+/* ress_score, ress_restore and ress_sparse_attn in order on one stream.  Inside the forward
+ * the CSR kernel also writes the attention items' union lists into the workspace, so the
+ * attention starts without the union pass of ress_sparse_attn; O, the CSR and J_best are
+ * bit for bit those of the three separate calls. */
 int ress_forward(const ress_dims* dims, const uint16_t* Q, const uint16_t* K, const uint16_t* V,
                  const float* F, const int32_t* c_h_host, int32_t rounds, float rho, void* ws,
                  size_t ws_bytes, int32_t* row_ptr, int32_t* col_idx, int64_t col_capacity,
@@ -241,7 +248,8 @@ int ress_forward(const ress_dims* dims, const uint16_t* Q, const uint16_t* K, co
  * example cudaHostAlloc) for the copies to overlap other work; every buffer belongs to the
  * caller and must stay untouched until the stream has passed the call.  Two calls on two
  * streams with separate device buffers, workspaces and CSR arrays overlap one layer's copies
- * with another's compute.  Q_host, K_host, V_host, O_host: bf16 [N, H, 64]; the other
+ * with another's compute (their attention chunks and output copies share the library's two
+ * streams of the device, so those parts of the two calls run one after the other).  Q_host, K_host, V_host, O_host: bf16 [N, H, 64]; the other
  * arguments as ress_forward.  Returns as ress_forward, or RESS_ECUDA if a copy could not be
  * enqueued; arguments are checked before anything is enqueued. */
 int ress_forward_host(const ress_dims* dims, const uint16_t* Q_host, const uint16_t* K_host,
