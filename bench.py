@@ -427,6 +427,23 @@ def run_ours(a, wl):
     st = np.array([[e[i].elapsed_time(e[i + 1]) for i in range(3)] for e in evs])
     score_ms, restore_ms, attn_ms = (float(x) for x in np.median(st, axis=0))
 
+    # ---- the rounds against the fp32 roofline: a round's time is restore(R) - restore(0)
+    #      over R; its arithmetic is the gain products, 2 H |P|_rows |P| 64 fp32 flop -----
+    csr_t = []
+    for k in range(nst):
+        ress.score(d, Q, K, V, buf.F, c_h, buf.ws)
+        e = evs[k]
+        e[0].record(stream)
+        ress.restore(d, c_h, 0, wl.rho, buf.ws, buf.row_ptr, buf.col_idx, buf.J_best)
+        e[1].record(stream)
+    torch.cuda.synchronize()
+    csr_ms = float(np.median([e[0].elapsed_time(e[1]) for e in evs]))
+    ress.score(d, Q, K, V, buf.F, c_h, buf.ws)  # back to the R-round state read below
+    ress.restore(d, c_h, wl.rounds, wl.rho, buf.ws, buf.row_ptr, buf.col_idx, buf.J_best)
+    torch.cuda.synchronize()
+    props = torch.cuda.get_device_properties(torch.cuda.current_device())
+    round_flop = 2.0 * H * ress.num_query_candidates(d) * ress.num_candidates(d) * 64
+
     rp = buf.row_ptr.cpu().numpy()
     ci = buf.col_idx.cpu().numpy()
     flops = kept_flops(rp, ci, N, H, nb, a.q_block)
@@ -622,6 +639,19 @@ def run_ours(a, wl):
                 "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h},
         "clocks": clk.summary(),
     }
+    if wl.rounds > 0:
+        # fp32 SIMT peak: 128 FMA lanes per SM at the SM clock seen under load (2070 MHz max)
+        mhz = line["clocks"].get("sm_max_mhz") or 2070.0
+        fp32_peak = props.multi_processor_count * 128 * 2 * mhz * 1e6 / 1e12
+        round_ms = max(restore_ms - csr_ms, 1e-9) / wl.rounds
+        line["rounds"] = {
+            "ms_per_round": round_ms, "csr_ms": csr_ms,
+            "fp32_gain_flop_per_round": round_flop,
+            "gain_tflops_over_round": round_flop / round_ms / 1e9,
+            "fp32_simt_peak_tflops": fp32_peak,
+            "frac_of_fp32_simt": round_flop / round_ms / 1e9 / fp32_peak,
+            "note": "a round = the gain products (tensor cores, three-term bf16) plus the per-row "
+                    "selection and update; its time bounds the gain arithmetic rate from below"}
 
     if pool is not None:
         kept = {(h, i): ci[rp[h * nb + i]:rp[h * nb + i + 1]] for h in range(H) for i in range(nb)}
