@@ -288,10 +288,13 @@ __device__ __forceinline__ uint32_t order_key(float x) {
 //    <= the m-th largest key overall (those 32 ceil(m/32) values include m entries);
 // 2. survivors: the participating keys >= that bound (usually about 1.5 m of them) are
 //    compacted, in block order, into a short list;
-// 3. the m-th largest survivor T is found bit by bit (count of survivors >= T), and the
+// 3. the m-th largest survivor T is found by a radix select over the survivors (8-bit
+//    digits; select_radix), or bit by bit without radix counters (select_exact), and the
 //    survivors > T plus the lowest-index ones == T are chosen.
 // When m needs more than kTopK candidates per lane, or too many keys tie at the bound,
-// step 3 runs on all participating keys instead (same result, slower).
+// step 3 runs bit by bit on all participating keys instead (same result, slower).  The
+// restoration rounds use warp_topm_pair below, which selects on both sides of the drop set
+// at once.
 // ------------------------------------------------------------------------------------
 constexpr int kTopK = 4;          // lane-local candidates: fast path for m <= 128
 constexpr int kSurvivors = 256;   // capacity of the survivor list
