@@ -622,7 +622,8 @@ def run_ours(a, wl):
         "select_overhead_pct": 100.0 * sel_ms / (sel_ms + attn_ms),
         "attn_tflops": flops / attn_ms / 1e9,
         "selection": {"algorithmic_bytes": sel_bytes, "gbs": sel_bytes / sel_ms / 1e6,
-                      "frac_of_hbm": sel_bytes / sel_ms / 1e6 / hbm, "hbm_peak_gbs": hbm},
+                      "frac_of_hbm": sel_bytes / sel_ms / 1e6 / hbm, "hbm_peak_gbs": hbm,
+                      "frac_of_nominal_8tbs": sel_bytes / sel_ms / 1e6 / 8000.0},
         "kept_tflop": flops / 1e12, "realized_pair_sparsity": 1.0 - kept_pairs / (H * nq * nb),
         "drift": {"sum_J_best": float(Jb[cand_rows].sum()), "sum_J0": float(J0[cand_rows].sum())},
         "dense": dense,
