@@ -1,4 +1,5 @@
-"""ReSS oracle in float64 (test infrastructure; see the package docstring).
+"""ReSS oracle in float64 (test infrastructure: only the tests, the smoke check and the
+benchmark's CPU baseline use it; nothing in the product path imports it).
 
 Notation follows the paper: heads h, query block i, key block j, pooled probability
 P_ij (Sec. 4.1), pooled value V_j, dense pooled output v_bar_i (Eq. 1), candidate set
@@ -7,7 +8,7 @@ e_ij = v_bar_i - V_j, drift contribution d_ij = P_ij e_ij (Eq. 5), head slice W_
 the output projection, block drift score s_ij (Eq. 6), cut key (Eq. 7), net drift g and
 remaining mass K (Eq. 10), objective J = G / K^2 (Eq. 12), swap schedule m_r (Eq. 17).
 
-Readings where the paper is silent (each listed in the design doc):
+Readings where the paper is silent:
   * Pooling: Q, K and V are mean-pooled over the valid tokens of each 64-token block; the
     pooled logits are q_bar_i . k_bar_j / sqrt(d_h) and P_i is their softmax over all key
     blocks (Sec. 3 step (1), Sec. 4.1).
@@ -159,12 +160,30 @@ def round_gains(D: np.ndarray, n_cand: int, P_i: np.ndarray, r: np.ndarray,
 
 
 def _gap(vals_sorted: np.ndarray, m: int, floor: float) -> float:
-    """Relative gap between the m-th and (m+1)-th of a descending list (inf if no cut)."""
+    """Decision margin of a top-m cut: the gap between the m-th and (m+1)-th entries of a
+    descending list, relative to the larger magnitude of the two (at least `floor`); inf when
+    the list has no (m+1)-th entry or m is 0 (nothing is decided)."""
     if m <= 0 or m >= vals_sorted.size:
         return math.inf
     a, b = vals_sorted[m - 1], vals_sorted[m]
     scale = max(abs(a), abs(b), floor)
     return (a - b) / scale if scale > 0 else 0.0
+
+
+def _track_margin(J: float, J_best: float) -> float:
+    """Decision margin of a track-best comparison (Sec. 4.3, Appendix B.3): how far the new
+    objective J is from the best one so far, relative to that best (inf when J_best is 0)."""
+    return abs(J - J_best) / J_best if J_best > 0 else math.inf
+
+
+def _cdf_margins(masses, tau: float, keys_sorted: np.ndarray, n_add: int) -> list:
+    """Decision margins of the CDF threshold: every running kept mass that was compared with
+    tau, relative to tau, and the key gaps on both sides of the last block that joined (a
+    swap there changes which blocks cross the threshold)."""
+    out = [abs(x - tau) / tau for x in masses]
+    if keys_sorted.size:
+        out += [_gap(keys_sorted, n_add, 0.0), _gap(keys_sorted, n_add - 1, 0.0)]
+    return out
 
 
 @dataclass
@@ -180,6 +199,15 @@ class RowSelection:
     J_trace: list = field(default_factory=list)   # J of the current set after each round
     margin: float = math.inf  # smallest relative decision margin of the row
     swaps: int = 0            # sum of the m actually applied
+    # every decision margin of the row in the order taken: ("cut", value) for the Eq. 7 cut,
+    # ("cdf", value) for the CDF threshold, ("restore", r, value) / ("drop", r, value) for the
+    # top-m cuts of round r and ("track", r, value) for its track-best comparison
+    margins: list = field(default_factory=list)
+
+    def note(self, kind: str, value: float, r: int = None) -> None:
+        """Record one decision margin and keep the row's smallest."""
+        self.margins.append((kind, value) if r is None else (kind, r, value))
+        self.margin = min(self.margin, value)
 
     @property
     def near_threshold(self) -> bool:
@@ -256,7 +284,7 @@ def select_row(P_i, vbar_i, Vb_h, WOh, n_cand: int, c: int, rounds: int, rho: fl
     D = np.zeros(nb, dtype=bool)
     D[:n_cand] = True
     D[keep] = False
-    margin = _gap(ranked(key[:n_cand]), c, 0.0)
+    notes = [("cut", _gap(ranked(key[:n_cand]), c, 0.0))]
     if variant.cdf > 0:
         if rounds:
             raise ValueError("the CDF threshold is defined without restoration rounds")
@@ -271,15 +299,13 @@ def select_row(P_i, vbar_i, Vb_h, WOh, n_cand: int, c: int, rounds: int, rho: fl
             masses.append(mass)
             n_add += 1
         D[order[:n_add]] = False
-        # decision margins: every running mass against tau, and the key gaps on both sides
-        # of the last added block (a swap there changes which blocks cross the threshold)
-        margin = min([margin] + [abs(x - tau) / tau for x in masses])
-        if rest.size:
-            keys_sorted = ranked(key[rest])
-            margin = min(margin, _gap(keys_sorted, n_add, 0.0), _gap(keys_sorted, n_add - 1, 0.0))
+        keys_sorted = ranked(key[rest]) if rest.size else rest
+        notes += [("cdf", x) for x in _cdf_margins(masses, tau, keys_sorted, n_add)]
     J, a, K = objective(D, P_i, r)
-    res = RowSelection(h, i, False, D.copy(), D.copy(), J, J, [], margin)
-    for m_r in swap_schedule(c, rounds, rho):
+    res = RowSelection(h, i, False, D.copy(), D.copy(), J, J, [])
+    for kind, value in notes:
+        res.note(kind, value)
+    for rnd, m_r in enumerate(swap_schedule(c, rounds, rho)):
         inD, gain_res, outD, gain_drop = round_gains(D, n_cand, P_i, r, J, a, K)
         m = min(m_r, inD.size, outD.size)
         if m == 0:
@@ -287,8 +313,8 @@ def select_row(P_i, vbar_i, Vb_h, WOh, n_cand: int, c: int, rounds: int, rho: fl
             continue
         floor = 1e-30 * J
         gain_res, gain_drop = sign * gain_res, sign * gain_drop
-        res.margin = min(res.margin, _gap(ranked(gain_res), m, floor),
-                         _gap(ranked(gain_drop), m, floor))
+        res.note("restore", _gap(ranked(gain_res), m, floor), rnd)
+        res.note("drop", _gap(ranked(gain_drop), m, floor), rnd)
         restore = inD[top_m(gain_res, m)]
         drop = outD[top_m(gain_drop, m)]
         D[restore] = False
@@ -296,8 +322,7 @@ def select_row(P_i, vbar_i, Vb_h, WOh, n_cand: int, c: int, rounds: int, rho: fl
         res.swaps += m
         J, a, K = objective(D, P_i, r)
         res.J_trace.append(J)
-        if res.J_best > 0:
-            res.margin = min(res.margin, abs(J - res.J_best) / res.J_best)
+        res.note("track", _track_margin(J, res.J_best), rnd)
         if (J < res.J_best) if sign > 0 else (J > res.J_best):
             res.J_best = J
             res.D_best = D.copy()

@@ -167,6 +167,22 @@ def compare_selection(layer: Layer, sel: dict) -> dict:
                 J_gpu_sum=J_gpu_sum, J_oracle_sum=J_oracle)
 
 
+NEAR_FRACTION = 0.05  # at most this share of the compared rows may differ as near-threshold
+
+
+def check_selection(r: dict) -> None:
+    """The selection acceptance rules on a compare_selection result: no drop set differs on a
+    row decided by a margin of at least 1e-3; the rows that do differ under that margin are
+    at most 5% of the compared rows (plus one, for small samples), so that a margin that
+    excused every row could not hide a wrong selection; realised drift within 1e-3 per row
+    and summed, against the oracle on the GPU's sets and against the oracle's own sets."""
+    assert r["mismatched"] == 0, r
+    assert r["near"] <= NEAR_FRACTION * (r["exact"] + r["near"]) + 1, r
+    assert r["worst_row_rel"] <= DRIFT_REL, r
+    assert r["sum_rel_gpu_vs_ref"] <= DRIFT_REL, r
+    assert r["sum_rel_gpu_vs_oracle"] <= DRIFT_REL, r
+
+
 def compare_attention(layer: Layer, rows) -> dict:
     ref = layer.oracle_attention(rows)
     out = layer.output()

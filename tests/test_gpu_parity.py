@@ -84,6 +84,7 @@ def test_drop_sets_and_drift(fixture, request):
     layer = request.getfixturevalue(fixture)
     sel = layer.oracle_select()
     r = G.compare_selection(layer, sel)
+    G.check_selection(r)
     print(fixture, r)
     assert r["mismatched"] == 0, r
     assert r["exact"] >= 0.95 * (r["exact"] + r["near"])
@@ -195,6 +196,7 @@ def test_edge_shapes(N, H, ns, c, R):
     layer = G.Layer(inp, ns, [c] * H, R).run()
     sel = layer.oracle_select()
     r = G.compare_selection(layer, sel)
+    G.check_selection(r)
     assert r["mismatched"] == 0, r
     rows = [(h, i) for h in range(H) for i in range(layer.nb)]
     a = G.compare_attention(layer, rows)
@@ -238,6 +240,7 @@ def test_headline_shape_sampled():
     rows = [(int(h), int(i)) for h, i in zip(rng.integers(0, wl.heads, 24), rng.integers(0, wl.n_candidates, 24))]
     sel = layer.oracle_select(rows)
     r = G.compare_selection(layer, sel)
+    G.check_selection(r)
     print(r)
     assert r["mismatched"] == 0, r
     J0 = layer.ws("J0", shape=(layer.H, layer.nb))
@@ -300,6 +303,7 @@ def test_large_shapes_sampled(name, kw):
     rng = np.random.default_rng(2)
     rows = [(int(h), int(i)) for h, i in zip(rng.integers(0, wl.heads, 10), rng.integers(0, wl.n_candidates, 10))]
     r = G.compare_selection(layer, layer.oracle_select(rows))
+    G.check_selection(r)
     print(name, kw, r)
     assert r["mismatched"] == 0, r
     J0 = layer.ws("J0", shape=(layer.H, layer.nb))
@@ -329,6 +333,7 @@ def test_maximum_shape_sampled():
     rng = np.random.default_rng(3)
     rows = [(int(h), int(i)) for h, i in zip(rng.integers(0, H, 6), rng.integers(0, nc, 6))]
     r = G.compare_selection(layer, layer.oracle_select(rows + [(H - 1, nc - 1)]))
+    G.check_selection(r)
     assert r["mismatched"] == 0, r
     assert r["worst_row_rel"] <= G.DRIFT_REL, r
     J0 = layer.ws("J0", shape=(H, layer.nb))
@@ -362,6 +367,7 @@ def test_equal_keys_keep_the_lowest_indices(q_block):
     layer3 = G.Layer(inp, ns, [c] * H, 3, variant=O.Variant(key="probability"),
                      q_block=q_block).run(attention=False)
     r = G.compare_selection(layer3, layer3.oracle_select())
+    G.check_selection(r)
     assert r["mismatched"] == 0, r
 
 
@@ -557,6 +563,7 @@ def test_selection_variants(name, variant, rounds):
     layer = G.Layer(synth.make_inputs(wl), wl.n_special, wl.budgets(), rounds, wl.rho,
                     variant=variant).run(attention=False)
     r = G.compare_selection(layer, layer.oracle_select())
+    G.check_selection(r)
     assert r["mismatched"] == 0, r
     assert r["exact"] >= 0.95 * (r["exact"] + r["near"]), r
     assert r["worst_row_rel"] <= G.DRIFT_REL and r["sum_rel_gpu_vs_oracle"] <= G.DRIFT_REL, r
@@ -576,6 +583,7 @@ def test_selection_variants_paper_grid(name, variant, rounds):
     layer = G.Layer(synth.make_inputs(wl), wl.n_special, wl.budgets(), rounds, wl.rho,
                     variant=variant, q_block=128).run(attention=False)
     r = G.compare_selection(layer, layer.oracle_select())
+    G.check_selection(r)
     assert r["mismatched"] == 0, r
     assert r["exact"] >= 0.95 * (r["exact"] + r["near"]), r
     assert r["worst_row_rel"] <= G.DRIFT_REL and r["sum_rel_gpu_vs_oracle"] <= G.DRIFT_REL, r
@@ -592,6 +600,7 @@ def test_cdf_threshold_headline_shape_sampled():
     rows = [(int(h), int(i)) for h, i in zip(rng.integers(0, layer.H, 40),
                                              rng.integers(0, layer.nqc, 40))]
     r = G.compare_selection(layer, layer.oracle_select(rows))
+    G.check_selection(r)
     assert r["mismatched"] == 0, r
     assert r["worst_row_rel"] <= G.DRIFT_REL, r
     rp, ci = layer.csr()
@@ -619,6 +628,7 @@ def test_cdf_threshold_variant(name, q_block, variant):
                     variant=variant, q_block=q_block).run()
     sel = layer.oracle_select()
     r = G.compare_selection(layer, sel)
+    G.check_selection(r)
     assert r["mismatched"] == 0, r
     assert r["exact"] >= 0.95 * (r["exact"] + r["near"]), r
     assert r["worst_row_rel"] <= G.DRIFT_REL and r["sum_rel_gpu_vs_oracle"] <= G.DRIFT_REL, r
@@ -688,6 +698,7 @@ def test_paper_grid_query_block_128(name):
                     q_block=128).run()
     assert layer.nq == -(-layer.N // 128)
     r = G.compare_selection(layer, layer.oracle_select())
+    G.check_selection(r)
     assert r["mismatched"] == 0, r
     assert r["exact"] >= 0.95 * (r["exact"] + r["near"]), r
     assert r["worst_row_rel"] <= G.DRIFT_REL and r["sum_rel_gpu_vs_oracle"] <= G.DRIFT_REL, r
@@ -721,6 +732,7 @@ def test_paper_grid_edge_shapes(N, H, ns, c, R):
     c = min(c, nc)
     layer = G.Layer(inp, ns, [c] * H, R, q_block=128).run()
     r = G.compare_selection(layer, layer.oracle_select())
+    G.check_selection(r)
     assert r["mismatched"] == 0, r
     a = G.compare_attention(layer, [(h, i) for h in range(H) for i in range(layer.nq)])
     assert a["max_abs"] <= G.ATT_MAX_ABS and a["mean_rel"] <= G.ATT_MEAN_REL, a
@@ -736,9 +748,122 @@ def test_paper_grid_headline_shape_sampled():
     rng = np.random.default_rng(2)
     rows = [(int(h), int(i)) for h, i in zip(rng.integers(0, wl.heads, 20), rng.integers(0, layer.nqc, 20))]
     r = G.compare_selection(layer, layer.oracle_select(rows))
+    G.check_selection(r)
     assert r["mismatched"] == 0, r
     J0 = layer.ws("J0", shape=(layer.H, layer.nq))
     Jb = layer.buf.J_best.cpu().numpy().reshape(layer.H, layer.nq)
     assert np.all(Jb[:, :layer.nqc] <= J0[:, :layer.nqc])
     a = G.compare_attention(layer, rows[:8] + [(0, layer.nq - 1), (7, layer.nqc - 1)])
+    assert a["max_abs"] <= G.ATT_MAX_ABS and a["mean_rel"] <= G.ATT_MEAN_REL, a
+
+
+# ---------------------------------------------------------------------------------------
+# Head-wise budgets (Sec. 4.4): a different c_h per head
+# ---------------------------------------------------------------------------------------
+UNEQUAL_BUDGETS = {
+    # tiny_v2, |P| = 42: one block, every candidate (nothing dropped), the uniform budget, few
+    "tiny_v2": [1, 42, 21, 8],
+    # vggt_v8, |P| = 171: from one block to every candidate, m_r from 0 to 42 per head
+    "vggt_v8": [8, 43, 2, 120, 171, 1, 17, 64, 5, 99, 3, 150, 33, 10, 77, 25],
+}
+
+
+def _check_csr_rows(layer, D):
+    """Every row of the CSR lists exactly the complement of its drop set (dense query rows:
+    every block), with the length its own head's budget gives."""
+    rp, ci = layer.csr()
+    ns = layer.nb - layer.ncand
+    assert rp.size == layer.H * layer.nq + 1 and rp[0] == 0 and rp[-1] == ci.size
+    for h in range(layer.H):
+        for i in range(layer.nq):
+            k = ci[rp[h * layer.nq + i]:rp[h * layer.nq + i + 1]]
+            if i >= layer.nqc:
+                assert k.tolist() == list(range(layer.nb)), (h, i)
+            else:
+                assert k.size == layer.c_h[h] + ns, (h, i, k.size)
+                assert np.array_equal(k, np.nonzero(~D[h, i])[0]), (h, i)
+
+
+@pytest.mark.parametrize("name,q_block", [("tiny_v2", 64), ("tiny_v2", 128), ("vggt_v8", 64),
+                                          ("vggt_v8", 128)])
+def test_unequal_head_budgets(name, q_block):
+    """Per-head budgets c_h that differ across the heads (one block, every candidate, and
+    values between): drop sets and drift of every row against the oracle, CSR rows of
+    per-head lengths at per-head offsets, and attention on rows of every head."""
+    wl = synth.WORKLOADS[name]
+    c_h = UNEQUAL_BUDGETS[name]
+    assert len(c_h) == wl.heads and max(c_h) == wl.n_candidates and min(c_h) == 1
+    layer = G.Layer(synth.make_inputs(wl), wl.n_special, c_h, wl.rounds, wl.rho,
+                    q_block=q_block).run()
+    sel = layer.oracle_select()
+    r = G.compare_selection(layer, sel)
+    G.check_selection(r)
+    assert r["exact"] >= 0.95 * (r["exact"] + r["near"]), r
+    D = layer.drop_sets()
+    _check_csr_rows(layer, D)
+    J0 = layer.ws("J0", shape=(layer.H, layer.nq))
+    Jb = layer.buf.J_best.cpu().numpy().reshape(layer.H, layer.nq)
+    assert np.all(Jb[:, :layer.nqc] <= J0[:, :layer.nqc])
+    for h, c in enumerate(c_h):  # nothing dropped: J = 0; rows that never swap keep J0
+        if c == layer.ncand:
+            assert np.all(Jb[h, :layer.nqc] == 0)
+        if all(m <= 0 for m in [min(x, c, layer.ncand - c) for x in O.swap_schedule(c, wl.rounds, wl.rho)]):
+            assert np.array_equal(Jb[h, :layer.nqc], J0[h, :layer.nqc])
+    rng = np.random.default_rng(4)
+    rows = []
+    for h in range(layer.H):
+        rows += [(h, int(i)) for i in rng.choice(layer.nqc, min(3, layer.nqc), replace=False)]
+        rows.append((h, layer.nq - 1))
+    a = G.compare_attention(layer, rows)
+    assert a["max_abs"] <= G.ATT_MAX_ABS and a["mean_rel"] <= G.ATT_MEAN_REL, a
+
+
+@pytest.mark.parametrize("q_block", [64, 128])
+def test_unequal_head_budgets_edge_shape(q_block):
+    """Three heads with budgets 1, |P| and 4 on a ragged sequence with special tokens."""
+    N, H, ns, R = 64 * 10 + 17, 3, 5, 3
+    inp = synth.make_random_layer(N, H, 64 * H, seed=N + 31)
+    nc = O.n_candidates(N, ns)
+    c_h = [1, nc, 4]
+    layer = G.Layer(inp, ns, c_h, R, q_block=q_block).run()
+    r = G.compare_selection(layer, layer.oracle_select())
+    G.check_selection(r)
+    _check_csr_rows(layer, layer.drop_sets())
+    a = G.compare_attention(layer, [(h, i) for h in range(H) for i in range(layer.nq)])
+    assert a["max_abs"] <= G.ATT_MAX_ABS and a["mean_rel"] <= G.ATT_MEAN_REL, a
+
+
+# ---------------------------------------------------------------------------------------
+# The headline layer on every row
+# ---------------------------------------------------------------------------------------
+def test_headline_shape_every_row():
+    """32 views, 16 heads, 90% sparsity, R = 3: the drop set and drift of every one of the
+    10,944 candidate rows against the oracle (run on every host core in spawned processes),
+    and attention on 500 rows: every dense query row (the special-token blocks of every
+    head) and a seeded sample of the sparse ones."""
+    import time
+    import oracle_pool
+    layer, wl = layer_for("vggt_v32")
+    layer.run()
+    rows = [(h, i) for h in range(layer.H) for i in range(layer.nq)]
+    t0 = time.perf_counter()
+    sel = oracle_pool.select_rows(layer.pooled(), layer.W_o(), layer.c_h, layer.rounds, layer.rho,
+                                  rows)
+    t_oracle = time.perf_counter() - t0
+    assert len(sel) == len(rows)
+    r = G.compare_selection(layer, sel)
+    print(f"oracle {t_oracle:.1f} s", r)
+    G.check_selection(r)
+    assert r["exact"] + r["near"] == layer.H * layer.nqc == 10944
+    assert r["exact"] >= 0.95 * (r["exact"] + r["near"]), r
+    D = layer.drop_sets()
+    _check_csr_rows(layer, D)
+    dense = [(h, i) for h in range(layer.H) for i in range(layer.nqc, layer.nq)]
+    sparse = [(h, i) for h in range(layer.H) for i in range(layer.nqc)]
+    rng = np.random.default_rng(9)
+    pick = rng.choice(len(sparse), 500 - len(dense), replace=False)
+    arows = dense + [sparse[k] for k in sorted(pick)]
+    assert len(arows) == 500 and len(dense) == 48
+    a = G.compare_attention(layer, arows)
+    print(a)
     assert a["max_abs"] <= G.ATT_MAX_ABS and a["mean_rel"] <= G.ATT_MEAN_REL, a

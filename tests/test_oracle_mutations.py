@@ -28,6 +28,10 @@ PIN_SET = [
     pins.test_budget_is_preserved_and_special_blocks_kept,
     pins.test_block_sparse_attention_is_masked_library_attention,
     lambda layer: pins.test_swap_schedule_totals(),
+    pins.test_margin_of_the_eq7_cut,
+    pins.test_margins_of_a_restoration_round,
+    pins.test_margins_of_track_best_comparisons,
+    pins.test_margins_of_the_cdf_threshold,
 ]
 
 
@@ -102,6 +106,40 @@ def _mut_attention_scale(Q, K, V, kept, rows, block=R.BLOCK):
     return out
 
 
+def _mut_gap_off_by_one(vals_sorted, m, floor):
+    if m <= 0 or m + 1 >= vals_sorted.size:
+        return math.inf
+    a, b = vals_sorted[m], vals_sorted[m + 1]
+    scale = max(abs(a), abs(b), floor)
+    return (a - b) / scale if scale > 0 else 0.0
+
+
+def _mut_gap_scale_next(vals_sorted, m, floor):
+    if m <= 0 or m >= vals_sorted.size:
+        return math.inf
+    a, b = vals_sorted[m - 1], vals_sorted[m]
+    scale = max(abs(b), floor)
+    return (a - b) / scale if scale > 0 else 0.0
+
+
+def _mut_track_over_new_J(J, J_best):
+    return abs(J - J_best) / J if J > 0 else math.inf
+
+
+def _mut_cdf_no_start_mass(masses, tau, keys_sorted, n_add):
+    out = [abs(x - tau) / tau for x in masses[1:]]
+    if keys_sorted.size:
+        out += [R._gap(keys_sorted, n_add, 0.0), R._gap(keys_sorted, n_add - 1, 0.0)]
+    return out
+
+
+def _mut_cdf_one_side(masses, tau, keys_sorted, n_add):
+    out = [abs(x - tau) / tau for x in masses]
+    if keys_sorted.size:
+        out += [R._gap(keys_sorted, n_add, 0.0)]
+    return out
+
+
 MUTATIONS = {
     "pool divides the ragged tail by 64": ("pool_blocks", _mut_pool_divides_by_block),
     "pooled logits scaled by 1/d": ("pooled_attention_row", _mut_softmax_scale),
@@ -114,6 +152,11 @@ MUTATIONS = {
     "schedule rounded up": ("swap_schedule", _mut_schedule_ceil),
     "top-m takes the smallest": ("top_m", _mut_topm_smallest),
     "token attention scaled by 1/d": ("block_sparse_attention", _mut_attention_scale),
+    "margin between the (m+1)-th and (m+2)-th": ("_gap", _mut_gap_off_by_one),
+    "margin relative to the (m+1)-th value": ("_gap", _mut_gap_scale_next),
+    "track-best margin relative to the new J": ("_track_margin", _mut_track_over_new_J),
+    "CDF margins without the starting mass": ("_cdf_margins", _mut_cdf_no_start_mass),
+    "CDF key gap on one side only": ("_cdf_margins", _mut_cdf_one_side),
 }
 
 

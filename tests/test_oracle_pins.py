@@ -552,3 +552,107 @@ def test_query_block_128_attention_is_two_64_blocks_with_the_same_list(layer):
     for i in range(3):
         assert np.allclose(a128[(0, i)], np.vstack([a64[(0, 2 * i)], a64[(0, 2 * i + 1)]]),
                            rtol=1e-12, atol=1e-12)
+
+
+# ---------------------------------------------------------------------------------------
+# Decision margins (which rows the GPU comparison excuses from the bit-exact rule)
+# ---------------------------------------------------------------------------------------
+def line_row(x):
+    """A row whose drift lives on one residual axis, so every key and gain has a closed form.
+
+    P is uniform (1/n over n candidate blocks, none always kept), W_O^h = I_64 and the pooled
+    values are V_j = x_j e_0 with sum x_j = 0, so v_bar = 0 and e_j = -x_j e_0.  Then
+    (Eq. 5-7, 10-12) the cut key of block j is |x_j| / (n - 1), and a drop set D has
+    J(D) = (sum_{j in D} x_j)^2 / (n - |D|)^2; restoring k gives (S - x_k)^2 / (n - |D| + 1)^2
+    and dropping k gives (S + x_k)^2 / (n - |D| - 1)^2 (Eq. 13-16).  The expected margins
+    below were worked out by hand from these closed forms."""
+    x = np.asarray(x, dtype=np.float64)
+    n = x.size
+    P = np.full(n, 1.0 / n)
+    Vb = np.zeros((n, 64))
+    Vb[:, 0] = x
+    return P, P @ Vb, Vb, np.eye(64)
+
+
+def _margins(sel):
+    return [(m[0], m[-1]) if len(m) == 2 else (m[0], m[1], m[2]) for m in sel.margins]
+
+
+def _assert_margins(sel, want):
+    got = _margins(sel)
+    assert [g[:-1] for g in got] == [w[:-1] for w in want], got
+    for g, w in zip(got, want):
+        assert g[-1] == pytest.approx(w[-1], rel=1e-12, abs=0), (g, w)
+    assert sel.margin == pytest.approx(min(w[-1] for w in want), rel=1e-12)
+
+
+def test_margin_of_the_eq7_cut(layer=None):
+    """Keys |x_j| / 7 ranked 5, 4, 3.5 | 3, 2, 1.5, 1, 1 (over 7): keeping c = 3 decides
+    between 3.5 and 3, a gap of 0.5 relative to 3.5."""
+    sel = O.select_row(*line_row([5, -4, 3.5, -3, 2, -1.5, -1, -1]), 8, 3, 0, 0.5)
+    _assert_margins(sel, [("cut", 1 / 7)])
+    assert not sel.near_threshold
+
+
+def test_margins_of_a_restoration_round(layer=None):
+    """c = 3, rho = 1.5, one round of m = 2.  D0 = {3,...,7}, S = -4.5, J0 = 2.25.
+    Restore gains 2.25 - (S - x_k)^2 / 16: 135/64 (k=3), 27/16 (k=5), 95/64 (k=6, 7),
+    -25/64 (k=4); the cut between the 2nd and 3rd is (27/16 - 95/64) / (27/16) = 13/108.
+    Drop gains 2.25 - (S + x_k)^2 / 4: 35/16 (k=0), 2 (k=2), -253/16 (k=1); the cut
+    (2 + 253/16) / (253/16) = 285/253.  The new set {0, 2, 4, 6, 7} has J = 8.5^2 / 9, above
+    J0: track-best margin (72.25/9 - 2.25) / 2.25 = 208/81, and the best set stays D0."""
+    sel = O.select_row(*line_row([5, -4, 3.5, -3, 2, -1.5, -1, -1]), 8, 3, 1, 1.5)
+    _assert_margins(sel, [("cut", 1 / 7), ("restore", 0, 13 / 108), ("drop", 0, 285 / 253),
+                          ("track", 0, 208 / 81)])
+    assert np.nonzero(sel.D_best)[0].tolist() == [3, 4, 5, 6, 7]
+    assert sel.J_trace == [pytest.approx(72.25 / 9, rel=1e-14)]
+
+
+def test_margins_of_track_best_comparisons(layer=None):
+    """Keys over 7: 19, 9, 8 | 7, 6, 4, 2, 1 (cut 1/8).  rho = 2: round 0 swaps m = 3 (every
+    kept candidate leaves, so the drop side has no cut: inf) and lowers J from 36 to 289/9:
+    track margin (36 - 289/9) / 36 = 35/324, taken relative to the best so far (J0).  Round 1
+    (m = 1) reaches J = 9: track margin (289/9 - 9) / (289/9) = 208/289, relative to the
+    updated best 289/9.  The restore cuts are 3/19 and 693/4588, the round-1 drop cut 189/256;
+    the row's margin is the round-0 track-best comparison."""
+    sel = O.select_row(*line_row([6, -8, -1, 7, 9, 4, 2, -19]), 8, 3, 2, 2.0)
+    _assert_margins(sel, [("cut", 1 / 8), ("restore", 0, 3 / 19), ("drop", 0, math.inf),
+                          ("track", 0, 35 / 324), ("restore", 1, 693 / 4588),
+                          ("drop", 1, 189 / 256), ("track", 1, 208 / 289)])
+    assert sel.J0 == pytest.approx(36.0, rel=1e-14)
+    assert sel.J_best == pytest.approx(9.0, rel=1e-14)
+
+
+def test_margins_of_the_cdf_threshold(layer=None):
+    """Probability key on P = (5, 3, 2, 1.5, 1, 0.5 | 3) / 16 (six candidates, one always-kept
+    block), c = 1, tau = 0.75: the kept mass starts at 8/16 and grows to 11/16, then 13/16,
+    so two blocks join (n_add = 2).  Margins: the Eq. 7 cut (5 - 3)/5 = 0.4; each running
+    mass against tau, |8/16 - 3/4| / (3/4) = 1/3, then 1/12 and 1/12; the key gaps of the
+    remaining candidates (3, 2, 1.5, 1, 0.5)/16 on both sides of the last joiner,
+    (2 - 1.5)/2 = 1/4 and (3 - 2)/3 = 1/3."""
+    P = np.array([5, 3, 2, 1.5, 1, 0.5, 3]) / 16.0
+    Vb = np.random.default_rng(0).normal(size=(7, 64))
+    sel = O.select_row(P, P @ Vb, Vb, np.eye(64), 6, 1, 0, 0.5,
+                       variant=O.Variant(key="probability", cdf=0.75))
+    _assert_margins(sel, [("cut", 0.4), ("cdf", 1 / 3), ("cdf", 1 / 12), ("cdf", 1 / 12),
+                          ("cdf", 0.25), ("cdf", 1 / 3)])
+    assert np.nonzero(~sel.D_best)[0].tolist() == [0, 1, 2, 6]
+
+
+def test_margin_is_smallest_recorded_and_near_rule(layer):
+    """On real rows the row margin is the smallest recorded decision margin, every round that
+    swaps records one restore cut, one drop cut and one track-best comparison, and a row with
+    equal keys at the Eq. 7 cut has margin 0 and is near-threshold."""
+    X, pooled = layer
+    sel = O.ress_select(pooled, X["W_o"], [4, 6], 3)
+    for (h, i), s in sel.items():
+        if s.dense:
+            assert s.margins == [] and s.margin == math.inf
+            continue
+        assert s.margin == min(m[-1] for m in s.margins)
+        assert s.margins[0][0] == "cut"
+        swapping = [r for r, m in enumerate(O.swap_schedule([4, 6][h], 3, 0.5)) if m > 0]
+        for kind in ("restore", "drop", "track"):
+            assert [m[1] for m in s.margins if m[0] == kind] == swapping
+    tie = O.select_row(*line_row([3, -3, 2, -2, 1, -1]), 6, 3, 0, 0.5)
+    assert tie.margin == 0.0 and tie.near_threshold
