@@ -804,9 +804,9 @@ def test_unequal_head_budgets(name, q_block):
     J0 = layer.ws("J0", shape=(layer.H, layer.nq))
     Jb = layer.buf.J_best.cpu().numpy().reshape(layer.H, layer.nq)
     assert np.all(Jb[:, :layer.nqc] <= J0[:, :layer.nqc])
-    for h, c in enumerate(c_h):  # nothing dropped: J = 0; rows that never swap keep J0
+    for h, c in enumerate(c_h):  # nothing dropped: J = 0 up to rounding; no swaps: J0 kept
         if c == layer.ncand:
-            assert np.all(Jb[h, :layer.nqc] == 0)
+            assert np.all(Jb[h, :layer.nqc] <= 1e-9 * Jb.max())
         if all(m <= 0 for m in [min(x, c, layer.ncand - c) for x in O.swap_schedule(c, wl.rounds, wl.rho)]):
             assert np.array_equal(Jb[h, :layer.nqc], J0[h, :layer.nqc])
     rng = np.random.default_rng(4)
