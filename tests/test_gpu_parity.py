@@ -490,6 +490,19 @@ def test_kernel_launch_counter():
     assert r.kernel_launches() - n0 == 6 + 2 * layer.rounds + 1 + 1
 
 
+def test_large_swap_count_parity():
+    """A budget of 135 of |P| = 171 candidates on the 8-view layer: a first swap count of 33,
+    more survivors than lanes in the round kernel's selection (its radix path), every row
+    against the oracle."""
+    wl = synth.WORKLOADS["vggt_v8"]
+    layer = G.Layer(synth.make_inputs(wl), wl.n_special, [135] * wl.heads, wl.rounds,
+                    wl.rho).run(attention=False)
+    assert O.swap_schedule(135, 1, wl.rho)[0] == 33
+    r = G.compare_selection(layer, layer.oracle_select())
+    G.check_selection(r)
+    assert r["exact"] >= 0.95 * (r["exact"] + r["near"]), r
+
+
 def _bf16_tensor(a):
     """float array -> (device bf16 tensor, the float64 values it holds)."""
     t = torch.from_numpy(np.ascontiguousarray(a, dtype=np.float32)).to(torch.bfloat16)
@@ -763,8 +776,10 @@ def test_paper_grid_headline_shape_sampled():
 UNEQUAL_BUDGETS = {
     # tiny_v2, |P| = 42: one block, every candidate (nothing dropped), the uniform budget, few
     "tiny_v2": [1, 42, 21, 8],
-    # vggt_v8, |P| = 171: from one block to every candidate, m_r from 0 to 42 per head
+    # vggt_v8, |P| = 171: from one block to every candidate, m_0 from 0 to 30 per head
     "vggt_v8": [8, 43, 2, 120, 171, 1, 17, 64, 5, 99, 3, 150, 33, 10, 77, 25],
+    # the same spread with every first swap count at most 17
+    "vggt_v8_small_m": [8, 43, 2, 68, 171, 1, 17, 64, 5, 30, 3, 69, 33, 10, 50, 25],
 }
 
 
@@ -784,14 +799,15 @@ def _check_csr_rows(layer, D):
                 assert np.array_equal(k, np.nonzero(~D[h, i])[0]), (h, i)
 
 
-@pytest.mark.parametrize("name,q_block", [("tiny_v2", 64), ("tiny_v2", 128), ("vggt_v8", 64),
-                                          ("vggt_v8", 128)])
-def test_unequal_head_budgets(name, q_block):
+@pytest.mark.parametrize("budgets,q_block", [("tiny_v2", 64), ("tiny_v2", 128), ("vggt_v8", 64),
+                                             ("vggt_v8", 128), ("vggt_v8_small_m", 64),
+                                             ("vggt_v8_small_m", 128)])
+def test_unequal_head_budgets(budgets, q_block):
     """Per-head budgets c_h that differ across the heads (one block, every candidate, and
     values between): drop sets and drift of every row against the oracle, CSR rows of
     per-head lengths at per-head offsets, and attention on rows of every head."""
-    wl = synth.WORKLOADS[name]
-    c_h = UNEQUAL_BUDGETS[name]
+    wl = synth.WORKLOADS[budgets.replace("_small_m", "")]
+    c_h = UNEQUAL_BUDGETS[budgets]
     assert len(c_h) == wl.heads and max(c_h) == wl.n_candidates and min(c_h) == 1
     layer = G.Layer(synth.make_inputs(wl), wl.n_special, c_h, wl.rounds, wl.rho,
                     q_block=q_block).run()
