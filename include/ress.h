@@ -40,7 +40,7 @@
 extern "C" {
 #endif
 
-#define RESS_ABI_VERSION 5
+#define RESS_ABI_VERSION 6
 #define RESS_HEAD_DIM 64
 #define RESS_BLOCK 64
 #define RESS_MAX_HEADS 32
@@ -95,6 +95,8 @@ typedef struct {
   int64_t lstat;       /* float2 [H, nq, ceil(nb/128)]: per 128-block slice of a row of
                           pooled logits, its max and sum of exp(logit - max)               */
   int64_t kcount;      /* int32 [H, nq]: key blocks kept by each candidate query row       */
+  int64_t prow;        /* int32 [H, ceil(nb/2)]: query blocks a | b << 16 of each attention
+                          item that ress_forward pairs by the overlap of their kept lists   */
   int64_t ld;          /* row stride of P, q, t                                          */
   int64_t words;       /* uint32 words per drop-set bitmask = ceil(nb / 32)              */
   int64_t total;       /* bytes                                                          */

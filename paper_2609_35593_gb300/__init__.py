@@ -67,7 +67,7 @@ class WsLayout(ctypes.Structure):
     _fields_ = [(n, ctypes.c_int64) for n in
                 ("status", "counter", "qbar", "kbar", "vbar", "ztil", "ytil", "gtil", "P", "q", "t",
                  "K", "G", "J", "Jbest", "J0", "dmask", "bmask", "plen", "asplit", "ksplit", "zsplit",
-                 "cdot", "ny", "nz", "lstat", "kcount", "ld", "words", "total")]
+                 "cdot", "ny", "nz", "lstat", "kcount", "prow", "ld", "words", "total")]
 
 
 _c = ctypes

@@ -1,14 +1,18 @@
 // Block-sparse attention forward over the kept 64x64 blocks (Sec. 3 step (3)) on sm_103a.
 //
-// Work item = (head h, pair of adjacent query blocks 2p, 2p+1): their 128 query rows form
-// the M = 128 operand of tcgen05.mma, and the CTA walks the union of the two kept lists
-// (built by k_pairs, ascending).  Each union entry carries a 2-bit mask saying which of the
-// two query blocks keeps it; rows of a block that does not keep the tile get P = 0, so
-// every row sees exactly its own kept blocks (softmax renormalised among them).
+// Work item = (head h, pair of query blocks): their 128 query rows form the M = 128 operand
+// of tcgen05.mma, and the CTA walks the union of the two kept lists (ascending; built by
+// k_pairs, or by a forward's CSR kernel).  The pair is the adjacent blocks 2p, 2p+1, or,
+// in a forward on the 64-token grid, the two candidate blocks that the pairing table names
+// (paired by the overlap of their kept lists, so fewer union entries are kept by one block
+// only).  Each union entry carries a 2-bit mask saying which of the two query blocks keeps
+// it; rows of a block that does not keep the tile get P = 0, so every row sees exactly its
+// own kept blocks (softmax renormalised among them).
 //
 // Warp roles (192 threads, 2 CTAs per SM):
-//   warp 0     TMA producer: Q tile (128 x 64) per item, K/V tiles (64 x 64) per entry into
-//              a 5-stage ring, 128-byte swizzled (UMMA canonical layouts).
+//   warp 0     TMA producer: Q tile (two 64 x 64 halves, one per query block) per item,
+//              K/V tiles (64 x 64) per entry into a 5-stage ring, 128-byte swizzled (UMMA
+//              canonical layouts).
 //   warp 1     TMEM owner and single-thread MMA issuer:
 //                S[g % 2] = Q K_g^T              (M128 N64 K64, Q from TMEM, K from shared memory)
 //                O       += P_{g-1} [V_{g-1} | 1]  (M128 N80 K64, P from TMEM, V MN-major)
@@ -82,6 +86,8 @@ struct AttnParams {
   const int32_t* row_ptr;
   const int32_t* plist;  // union lists: entry = j | mask << 16, at row_ptr[h*nb + 2p]
   const int32_t* plen;   // [H * npairs]
+  const int32_t* prow;   // items p < npaired: query blocks a | b << 16 (64-token grid), or NULL
+  int npaired;
   void* O;               // bf16 or float32 [N, H, 64]
   uint32_t* status;
   uint32_t* counter;
@@ -110,6 +116,20 @@ __device__ __forceinline__ void item_pair(const AttnParams& a, int item, int& h,
 // traffic low) and the verdict is broadcast, so that no lane leaves a loop its neighbours
 // stay in (the warp runs .sync.aligned code); __syncwarp orders the other lanes' later reads
 // after lane 0's acquire.
+// First tokens of the two 64-row halves of item (h, p): the query blocks of its table entry
+// when the forward paired them, else rows 128 p .. 128 p + 127 (adjacent 64-token blocks,
+// or one 128-token block).  A half past the sequence starts at or past N.
+__device__ __forceinline__ void item_tokens(const AttnParams& a, int h, int p, int& t0, int& t1) {
+  if (p < a.npaired) {
+    const int32_t pr = a.prow[(int64_t)h * a.npairs + p];
+    t0 = 64 * (pr & 0xffff);
+    t1 = 64 * (pr >> 16);
+  } else {
+    t0 = kRows * p;
+    t1 = kRows * p + 64;
+  }
+}
+
 __device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, volatile int* abort) {
   if (__all_sync(0xffffffffu, mbar_try_wait(bar, parity))) return true;
   int ok = 1;
@@ -245,8 +265,11 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
         break;
       }
       if (lane == 0) {
+        int t0, t1;
+        item_tokens(a, h, p, t0, t1);
         mbar_arrive_expect_tx(&S.q_full, kRows * 128);
-        tma_load_3d(S.Q, &tmQ, &S.q_full, 0, h, kRows * p);
+        tma_load_3d(S.Q, &tmQ, &S.q_full, 0, h, t0);               // rows 0..63
+        tma_load_3d(S.Q + 64 * 128, &tmQ, &S.q_full, 0, h, t1);    // rows 64..127
       }
       q_loaded = true;
       for (int e0 = 0; e0 < n && !failed; e0 += 32) {
@@ -515,10 +538,11 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
           break;
         }
         tc_fence_after();
-        int h, p;
+        int h, p, t0, t1;
         item_pair(a, info.item, h, p);
-        const int token = kRows * p + r;
-        const bool row_exists = (2 * p + half) < a.nb && token < a.N;
+        item_tokens(a, h, p, t0, t1);
+        const int token = (half ? t1 : t0) + (r & 63);
+        const bool row_exists = token < a.N;
         uint32_t o[2][32], ls[16];
         RESS_TMEM_LD32(tmem + lane_base + kColO, o[0]);
         RESS_TMEM_LD32(tmem + lane_base + kColO + 32, o[1]);
@@ -623,7 +647,7 @@ cudaError_t launch_attn_range(const AttnArgs& x, int p0, int p1, int slot, cudaS
   if (p0 < 0 || p1 > npairs || p0 >= p1 || slot < 0 || slot >= kAttnCounterSlots)
     return cudaErrorInvalidValue;
   CUtensorMap tq, tk, tv;
-  if (!make_map(&tq, x.Q, s.N, s.H, kRows) || !make_map(&tk, x.K, s.N, s.H, 64) ||
+  if (!make_map(&tq, x.Q, s.N, s.H, 64) || !make_map(&tk, x.K, s.N, s.H, 64) ||
       !make_map(&tv, x.V, s.N, s.H, 64))
     return cudaErrorInvalidValue;
   const int items = s.H * (p1 - p0);
@@ -643,6 +667,8 @@ cudaError_t launch_attn_range(const AttnArgs& x, int p0, int p1, int slot, cudaS
   p.row_ptr = x.row_ptr;
   p.plist = x.plist;
   p.plen = x.plen;
+  p.prow = x.prow;
+  p.npaired = x.prow ? x.npaired : 0;
   p.O = x.O;
   p.status = x.status;
   p.counter = x.counter + slot;

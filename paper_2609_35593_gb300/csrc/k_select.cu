@@ -1057,6 +1057,78 @@ __global__ void __launch_bounds__(32 * kRowWarps, 10) k_round_rows(SelPtrs p, Bu
 }
 
 // ------------------------------------------------------------------------------------
+// Pairing of query blocks for the attention items (64-token grid, fixed budgets).  The
+// attention runs two 64-row query blocks as one M = 128 tile over the union of their kept
+// lists, so every key block kept by only one of them is half a tile of wasted tensor work.
+// Within each window of kPairWindow candidate query blocks of a head, blocks are paired by
+// the overlap of their best kept candidate sets: in ascending order, each block not yet
+// paired takes the unpaired block of the window that shares most kept blocks with it (ties
+// to the nearer one).  Output: prow[h, 32 w + k] = a | b << 16 for the k-th pair of window
+// w.  Which blocks share a tile changes no row's result: a row attends its own kept blocks
+// in ascending order either way.  grid (windows, H) x 512 threads: all warps form the
+// window's overlaps, then the first warp pairs (one warp-wide maximum per pair).
+// ------------------------------------------------------------------------------------
+__global__ void __launch_bounds__(512) k_pairing(const uint32_t* __restrict__ bmask, int nq,
+                                                 int words, int ncand, int npaired, int items,
+                                                 int32_t* __restrict__ prow) {
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  constexpr int W = kPairWindow;
+  const int ks = words | 1;  // odd row stride: the rows one load touches fall in distinct banks
+  uint32_t* kept = reinterpret_cast<uint32_t*>(smem_raw);     // [W][ks]
+  uint16_t* ov = reinterpret_cast<uint16_t*>(kept + W * ks);  // [W][W]
+  const int h = blockIdx.y, w = blockIdx.x, t = threadIdx.x;
+  const int r0 = W * w;
+  const int n = min(W, 2 * npaired - r0);  // even
+  if (n <= 0) return;
+  for (int idx = t; idx < W * words; idx += blockDim.x) {  // rows past n: empty
+    const int r = idx / words, wd = idx - r * words;
+    kept[r * ks + wd] =
+        r < n ? ~bmask[((int64_t)h * nq + r0 + r) * words + wd] & valid_bits(wd, ncand) : 0u;
+  }
+  __syncthreads();
+  {  // thread t: row a = t / 8 against the blocks g, g + 8, .., g + 56 (g = t mod 8)
+    const int a = t >> 3, g = t & 7;
+    int c[8];
+#pragma unroll
+    for (int j = 0; j < 8; ++j) c[j] = 0;
+    if (a < n) {
+#pragma unroll 2
+      for (int wd = 0; wd < words; ++wd) {
+        const uint32_t ka = kept[a * ks + wd];
+#pragma unroll
+        for (int j = 0; j < 8; ++j) c[j] += __popc(ka & kept[(g + 8 * j) * ks + wd]);
+      }
+#pragma unroll
+      for (int j = 0; j < 8; ++j) ov[a * W + g + 8 * j] = (uint16_t)min(c[j], 2047);
+    }
+  }
+  __syncthreads();
+  if (t >= 32) return;
+  const int lane = t;
+  uint64_t freeb = n == 64 ? ~0ull : ((1ull << n) - 1ull);  // unpaired blocks of the window
+  int k = 0;
+  for (int a = 0; a < n - 1; ++a) {
+    if (!((freeb >> a) & 1ull)) continue;  // uniform across the warp
+    // the overlap, then the nearer block: candidates b > a (every earlier block is paired)
+    uint32_t key = 0u;
+#pragma unroll
+    for (int s = 0; s < W / 32; ++s) {
+      const int b = lane + 32 * s;
+      if (b > a && b < n && ((freeb >> b) & 1ull)) {
+        const uint32_t kb = ((uint32_t)ov[a * W + b] << 12) | (uint32_t)(4095 - (b - a));
+        key = max(key, kb);
+      }
+    }
+    const uint32_t best = __reduce_max_sync(0xffffffffu, key);
+    if (best == 0u) break;  // not reached: n is even, so a later block is always free
+    const int b = a + 4095 - (int)(best & 4095u);
+    freeb &= ~((1ull << a) | (1ull << b));
+    if (lane == 0) prow[(int64_t)h * items + W / 2 * w + k] = (r0 + a) | ((r0 + b) << 16);
+    ++k;
+  }
+}
+
+// ------------------------------------------------------------------------------------
 // Kept-block lists (CSR) from the best drop sets; special query rows keep everything.
 // One warp per attention item: query rows 2u and 2u + 1 on the 64-token grid, row u on the
 // 128-token grid.  With plist set the warp also writes the item's list for the attention
@@ -1078,6 +1150,8 @@ struct CsrOut {
   int32_t* plist;        // optional: attention item lists
   int32_t* plen;         // [H * items] with plist
   int64_t plist_cap;
+  const int32_t* prow;   // optional: rows of items u < npaired (k_pairing), else adjacent
+  int npaired;
   uint32_t* status;
   int rows_per_item;     // 2 on the 64-token grid, 1 on the 128-token grid
   bool variable;         // row offsets from row_ptr (k_rowptr) instead of the fixed budgets
@@ -1137,7 +1211,10 @@ __global__ void k_csr(SelPtrs p, Budgets bud, CsrBases cb, int H, CsrOut o) {
   const int u = blockIdx.x * 8 + (threadIdx.x >> 5);
   if (u >= items) return;
   const int i0 = u * rpi;
-  const int nr = min(rpi, p.nq - i0);  // rows of this item: 1 or 2
+  const bool paired = o.prow && u < o.npaired;
+  const int32_t pr = paired ? o.prow[(int64_t)h * items + u] : 0;
+  const int rowi[2] = {paired ? (pr & 0xffff) : i0, paired ? (pr >> 16) : i0 + 1};
+  const int nr = paired ? 2 : min(rpi, p.nq - i0);  // rows of this item: 1 or 2
   const int ns = p.nb - p.ncand;        // always-kept key blocks
   const int c = bud.c[h];
   int64_t ri[2], off[2];
@@ -1145,7 +1222,7 @@ __global__ void k_csr(SelPtrs p, Budgets bud, CsrBases cb, int H, CsrOut o) {
   bool dense[2];
 #pragma unroll
   for (int r = 0; r < 2; ++r) {
-    const int i = min(i0 + r, p.nq - 1);
+    const int i = min(rowi[r], p.nq - 1);
     ri[r] = (int64_t)h * p.nq + i;
     dense[r] = i >= p.nqc;
     // fixed budgets: offsets by formula; variable lengths: the offsets k_rowptr wrote
@@ -1155,6 +1232,9 @@ __global__ void k_csr(SelPtrs p, Budgets bud, CsrBases cb, int H, CsrOut o) {
                                                  : (int64_t)i * (c + ns));
     expect[r] = o.variable ? (int)(o.row_ptr[ri[r] + 1] - off[r]) : (dense[r] ? p.nb : c + ns);
   }
+  // an item's union list goes to its slot, the CSR span of rows rpi u .. rpi u + rpi - 1;
+  // a paired item's two candidate rows have the slot's two lengths (fixed budgets)
+  const int64_t uoff = paired ? cb.base[h] + (int64_t)i0 * (c + ns) : off[0];
   // Lane l owns word w0 + l of each row: one warp scan of the lanes' kept counts gives
   // every word's first list position, then each lane writes the blocks of its own word.
   int posU = 0;
@@ -1190,7 +1270,7 @@ __global__ void k_csr(SelPtrs p, Budgets bud, CsrBases cb, int H, CsrOut o) {
       for (uint32_t bits = un; bits; bits &= bits - 1u, ++au) {
         const int b = __ffs(bits) - 1;
         const int m = (int)((keep[0] >> b) & 1u) | (int)(((kb >> b) & 1u) << 1);
-        if (off[0] + au < o.plist_cap) o.plist[off[0] + au] = (w * 32 + b) | (m << 16);
+        if (uoff + au < o.plist_cap) o.plist[uoff + au] = (w * 32 + b) | (m << 16);
       }
     }
     pos[0] += tAB & 0xffff;
@@ -1306,7 +1386,7 @@ cudaError_t launch_round(const SelectArgs& a, int round, float rho, cudaStream_t
 cudaError_t launch_csr(const SelectArgs& a, const int64_t* head_base, int32_t* row_ptr,
                        int32_t* col_idx, int64_t col_capacity, float* J_best,
                        uint32_t* drop_mask, int32_t* plist, int32_t* plen, int64_t plist_cap,
-                       cudaStream_t st) {
+                       const int32_t* prow, cudaStream_t st) {
   const Shape& s = a.s;
   SelPtrs p = sel_ptrs(s, a.ws, a.L);
   CsrBases cb;
@@ -1323,12 +1403,33 @@ cudaError_t launch_csr(const SelectArgs& a, const int64_t* head_base, int32_t* r
   o.status = (uint32_t*)(a.ws + a.L.status);
   o.rows_per_item = s.qb == 128 ? 1 : 2;
   o.variable = a.v.cdf > 0.f;
+  o.prow = prow;
+  o.npaired = prow ? paired_items(s) : 0;
   if (o.variable) {
     k_rowptr<<<1, 1024, 0, st>>>(p.kcount, s.H, s.nq, s.nqc, s.nb, row_ptr);
     note_launch();
   }
   const int items = (s.nq + o.rows_per_item - 1) / o.rows_per_item;
   k_csr<<<dim3((items + 7) / 8, s.H), 256, 0, st>>>(p, budgets_of(a), cb, s.H, o);
+  note_launch();
+  return cudaGetLastError();
+}
+
+bool pairing_active(const Shape& s, const Variant& v) {
+  return s.qb == kBlock && v.cdf <= 0.f && paired_items(s) > 0;
+}
+
+int paired_items(const Shape& s) { return s.nqc / 2; }
+
+cudaError_t launch_pairing(const SelectArgs& a, int32_t* prow, cudaStream_t st) {
+  const Shape& s = a.s;
+  const int npaired = paired_items(s);
+  const int windows = (2 * npaired + kPairWindow - 1) / kPairWindow;
+  const size_t smem = (size_t)kPairWindow * (s.words | 1) * 4 + (size_t)kPairWindow * kPairWindow * 2;
+  cudaError_t e = cudaFuncSetAttribute(k_pairing, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+  if (e != cudaSuccess) return e;
+  k_pairing<<<dim3(windows, s.H), 512, smem, st>>>((const uint32_t*)(a.ws + a.L.bmask), s.nq, s.words,
+                                                   s.ncand, npaired, (s.nb + 1) / 2, prow);
   note_launch();
   return cudaGetLastError();
 }

@@ -300,8 +300,15 @@ static int restore_impl(const ress_dims* d, const int32_t* c_h, int32_t rounds, 
   char* w = static_cast<char*>(ws);
   int32_t* plist = items ? reinterpret_cast<int32_t*>(w + L.t) : nullptr;  // t is free by now
   int32_t* plen = items ? reinterpret_cast<int32_t*>(w + L.plen) : nullptr;
+  // a forward pairs the query blocks of its attention items by the overlap of their kept lists
+  int32_t* prow = nullptr;
+  if (items && ress::pairing_active(s, a.v)) {
+    prow = reinterpret_cast<int32_t*>(w + L.prow);
+    cudaError_t ce = ress::launch_pairing(a, prow, st);
+    if (ce != cudaSuccess) return cuda_fail(ce, "ress_restore pairing");
+  }
   cudaError_t ce = ress::launch_csr(a, base, row_ptr, col_idx, col_capacity, J_best, drop_mask,
-                                    plist, plen, (int64_t)s.H * s.nq * s.ld, st);
+                                    plist, plen, (int64_t)s.H * s.nq * s.ld, prow, st);
   if (ce != cudaSuccess) return cuda_fail(ce, "ress_restore csr");
   return ok();
 }
@@ -343,7 +350,18 @@ static ress::AttnArgs attn_args(const ress::Shape& s, const ress_ws_layout& L,
   a.plist = reinterpret_cast<int32_t*>(w + L.t);  // the gains buffer is free during attention
   a.plen = reinterpret_cast<int32_t*>(w + L.plen);
   a.scratch_cap = (int64_t)s.H * s.nq * s.ld;  // entries of the t array
+  a.prow = nullptr;  // adjacent query blocks; a forward sets its pairing table
+  a.npaired = 0;
   return a;
+}
+
+// The attention of a forward uses the item table its CSR step wrote (ReSS, no variant).
+static void use_forward_pairing(ress::AttnArgs* a, const ress::Shape& s, const ress_ws_layout& L,
+                                void* ws) {
+  if (ress::pairing_active(s, ress::Variant{0, 0, 0ull, 0.0f})) {
+    a->prow = reinterpret_cast<const int32_t*>(static_cast<char*>(ws) + L.prow);
+    a->npaired = ress::paired_items(s);
+  }
 }
 
 static int sparse_attn_impl(const ress_dims* d, const uint16_t* Q, const uint16_t* K,
@@ -403,7 +421,8 @@ int ress_forward(const ress_dims* d, const uint16_t* Q, const uint16_t* K, const
   if ((e = restore_impl(d, c_h, rounds, rho, nullptr, ws, ws_bytes, row_ptr, col_idx, col_capacity,
                         J_best, nullptr, true, stream)))
     return e;
-  const ress::AttnArgs a = attn_args(s, L, Q, K, V, row_ptr, col_idx, col_capacity, O, false, ws);
+  ress::AttnArgs a = attn_args(s, L, Q, K, V, row_ptr, col_idx, col_capacity, O, false, ws);
+  use_forward_pairing(&a, s, L, ws);
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   cudaError_t ce = cudaMemsetAsync(a.counter, 0, sizeof(uint32_t), st);
   if (ce == cudaSuccess) ce = ress::launch_attn_range(a, 0, ress::attn_num_pairs(s), 0, st);
@@ -454,8 +473,9 @@ int ress_forward_host(const ress_dims* d, const uint16_t* Q_host, const uint16_t
   const ress::Shape s = ress::make_shape(*d);
   ress_ws_layout L;
   if ((e = check_ws(s, ws, ws_bytes, &L))) return e;
-  const ress::AttnArgs a =
+  ress::AttnArgs a =
       attn_args(s, L, Q_dev, K_dev, V_dev, row_ptr, col_idx, col_capacity, O_dev, false, ws);
+  use_forward_pairing(&a, s, L, ws);
   std::lock_guard<std::mutex> lock(g_overlap_mu);
   OverlapStreams* o = nullptr;
   cudaError_t ce = overlap_streams(&o);
@@ -467,8 +487,16 @@ int ress_forward_host(const ress_dims* d, const uint16_t* Q_host, const uint16_t
   const int np = ress::attn_num_pairs(s);
   const int chunks = np < kOutChunks ? np : kOutChunks;
   const size_t row_bytes = bytes / (size_t)d->n_tokens;  // one token: H * 64 bf16
+  // chunk boundaries among the paired items fall on whole pairing windows, so that every
+  // chunk's items hold exactly the query rows [128 p0, 128 p1)
+  auto bound = [&](int c) {
+    int b = (int)((int64_t)np * c / chunks);
+    if (b < a.npaired) b = b / (ress::kPairWindow / 2) * (ress::kPairWindow / 2);
+    return b;
+  };
   for (int c = 0; c < chunks && ce == cudaSuccess; ++c) {
-    const int p0 = (int)((int64_t)np * c / chunks), p1 = (int)((int64_t)np * (c + 1) / chunks);
+    const int p0 = bound(c), p1 = c + 1 == chunks ? np : bound(c + 1);
+    if (p1 <= p0) continue;
     cudaStream_t cs = (c & 1) ? o->aux : st;
     const int64_t t0 = 128 * (int64_t)p0;
     const int64_t t1 = 128 * (int64_t)p1 < d->n_tokens ? 128 * (int64_t)p1 : d->n_tokens;
@@ -664,6 +692,8 @@ extern "C" int ress_sparse_attn_noalloc(const ress_dims* d, const uint16_t* Q, c
   a.plen = reinterpret_cast<int32_t*>(w + kNoallocPlen);
   a.plist = reinterpret_cast<int32_t*>(w + kNoallocPlen + plen_bytes);
   a.scratch_cap = list_entries;
+  a.prow = nullptr;  // items of adjacent query blocks
+  a.npaired = 0;
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   cudaError_t ce = ress::launch_sparse_attn(a, st);
   if (ce != cudaSuccess) return cuda_fail(ce, "ress_sparse_attn_noalloc");

@@ -84,6 +84,7 @@ inline ress_ws_layout make_layout(const Shape& s) {
   L.nz = take((int64_t)s.H * s.nb * 4);
   L.lstat = take((int64_t)s.H * s.nq * ((s.nb + 127) / 128) * 8);
   L.kcount = take(row);
+  L.prow = take((int64_t)s.H * ((s.nb + 1) / 2) * 4);
   L.ld = s.ld;
   L.words = s.words;
   L.total = off;
@@ -182,7 +183,16 @@ cudaError_t launch_yagg(const SelectArgs& a, cudaStream_t st);
 cudaError_t launch_csr(const SelectArgs& a, const int64_t* head_base, int32_t* row_ptr,
                        int32_t* col_idx, int64_t col_capacity, float* J_best,
                        uint32_t* drop_mask, int32_t* plist, int32_t* plen, int64_t plist_cap,
-                       cudaStream_t st);
+                       const int32_t* prow, cudaStream_t st);
+// Attention items of a forward on the 64-token grid with fixed budgets: the candidate query
+// blocks are paired by the overlap of their best kept lists, within windows of
+// kPairWindow blocks (prow, see ress_ws_layout); items of the window hold pair indices
+// [kPairWindow/2 * w, ...).  pairing_active says whether a forward on this shape and
+// variant uses the table; paired_items is the number of table entries per head.
+constexpr int kPairWindow = 64;
+bool pairing_active(const Shape& s, const Variant& v);
+int paired_items(const Shape& s);
+cudaError_t launch_pairing(const SelectArgs& a, int32_t* prow, cudaStream_t st);
 
 struct AttnArgs {
   Shape s;
@@ -196,6 +206,8 @@ struct AttnArgs {
   int32_t* plist;       // scratch: union lists of query-block pairs (>= scratch_cap entries)
   int32_t* plen;        // scratch: [H * ceil(nb / 2)] union lengths
   int64_t scratch_cap;
+  const int32_t* prow;  // item table of a paired forward (items p < npaired), or NULL
+  int npaired;
 };
 cudaError_t launch_sparse_attn(const AttnArgs& a, cudaStream_t st);
 // The two halves of launch_sparse_attn, for callers that split the attention: the union

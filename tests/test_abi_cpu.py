@@ -23,7 +23,7 @@ def test_every_declared_function_is_exported():
         assert hasattr(ress._lib, n), n
     for n in ("ress_score", "ress_restore", "ress_sparse_attn", "ress_forward"):
         assert n in names
-    assert ress._lib.ress_abi_version() == 5
+    assert ress._lib.ress_abi_version() == 6
 
 
 @pytest.mark.parametrize("name", list(synth.WORKLOADS))
