@@ -292,9 +292,14 @@ int ress_token_drift(const ress_dims* dims, const uint16_t* O_a, const uint16_t*
  * called.
  *   - Limit: col_capacity must not exceed (4 MiB - 256 - 4*H*ceil(nb/2) rounded up to 256) / 4
  *     entries (about one million: enough for 16 heads x 32 views at 90% sparsity);
- *     larger requests return RESS_EWORKSPACE with the limit in the message.
+ *     larger requests return RESS_EWORKSPACE with the limit in the message.  The check is on
+ *     col_capacity as passed, not on the entries the CSR uses (row_ptr's last value): pass
+ *     the used length when the buffer is larger.
  *   - Set-up: the first call on each device looks up the array's device address (with that
- *     device current) and caches it; make that first call before any stream capture.
+ *     device current) and caches it for the life of the process; make that first call
+ *     before any stream capture.  A cudaDeviceReset (or anything else that reloads this
+ *     library's module in a new primary context) leaves that cached address stale: do not
+ *     call this entry point after resetting a device it was already called on.
  *   - Every call shares the one array, and it keeps the last call's contents: calls that
  *     may overlap on the GPU (other streams, other host threads) race and must be ordered
  *     by the caller.  The tile counter is cleared by each call.

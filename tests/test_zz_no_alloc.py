@@ -60,3 +60,32 @@ def test_noalloc_rejects_requests_beyond_its_scratch():
     assert rc == -2  # RESS_EWORKSPACE, nothing launched
     msg = layer.ress._lib.ress_last_error().decode()
     assert "scratch" in msg and "ress_sparse_attn" in msg
+
+
+def test_noalloc_asynchronous_call_then_waiting_call():
+    """wait == 0 returns without synchronising; a following call with wait != 0 on the same
+    stream gives the same bits (the shared scratch is rewritten by every call)."""
+    wl = synth.WORKLOADS["tiny_v2"]
+    layer = G.Layer(synth.make_inputs(wl), wl.n_special, wl.budgets(), wl.rounds, wl.rho).run()
+    O1 = torch.full_like(layer.buf.O, float("nan"))
+    O2 = torch.full_like(layer.buf.O, float("nan"))
+    assert _call(layer, O1, wait=0) == 0, layer.ress._lib.ress_last_error()
+    assert _call(layer, O2, wait=1) == 0, layer.ress._lib.ress_last_error()
+    torch.cuda.synchronize()
+    assert torch.equal(O1.view(torch.int16), layer.buf.O.view(torch.int16))
+    assert torch.equal(O2.view(torch.int16), layer.buf.O.view(torch.int16))
+
+
+def test_noalloc_device_error_is_reported_once():
+    """A CSR entry out of range (caught by the union kernel's own bounds check, no memory
+    access past the arrays) is reported as RESS_EDEVICE by the waiting call, and the next
+    call on a good CSR returns RESS_OK: the recorded failure was cleared."""
+    wl = synth.WORKLOADS["tiny_v2"]
+    layer = G.Layer(synth.make_inputs(wl), wl.n_special, wl.budgets(), wl.rounds, wl.rho).run()
+    good = layer.buf.col_idx.clone()
+    layer.buf.col_idx[5] = layer.nb + 100
+    O = torch.empty_like(layer.buf.O)
+    assert _call(layer, O, wait=1) == -6  # RESS_EDEVICE
+    layer.buf.col_idx.copy_(good)
+    assert _call(layer, O, wait=1) == 0, layer.ress._lib.ress_last_error()
+    assert torch.equal(O.view(torch.int16), layer.buf.O.view(torch.int16))
