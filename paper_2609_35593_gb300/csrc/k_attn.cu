@@ -30,7 +30,12 @@
 //   warps 2-5  one query row per thread: tcgen05.ld of S, online softmax in the exp2 domain
 //              with lazy rescaling of the TMEM accumulator (only when the running max grows
 //              by more than 2^20, done after P is written so that the exponentials overlap
-//              the previous P V), tcgen05.st of P, epilogue O / l.
+//              the previous P V), tcgen05.st of P, epilogue O / l.  The exponentials are
+//              taken against the row's current reference maximum while the tile's maximum
+//              is formed (they use different pipes), and redone in the rare case that the
+//              maximum grew past the threshold.  The producer announces each item through a
+//              small ring of item slots and the softmax warps read its union list from
+//              global memory themselves, so that their per-tile work waits only for S.
 // Every mbarrier wait is bounded; a wait that gives up records RESS_ETIMEOUT in the status
 // word, makes the whole CTA leave its loops, drains in-flight copies and MMAs, frees TMEM
 // and returns.
@@ -54,6 +59,7 @@ constexpr int kNO = 80;  // O columns: 64 output channels, the row sum, 15 unuse
 constexpr uint64_t kWaitNs = 2000000000ull;  // 2 s per wait
 constexpr uint64_t kDrainNs = 200000000ull;  // 0.2 s to drain after an abort
 constexpr int kFirst = 1, kLast = 2, kTerm = 4;
+constexpr int kItemSlots = 4;  // items announced to the softmax warps ahead of their tiles
 constexpr uint32_t kTileBytes = 64 * 128;    // one 64 x 64 bf16 tile
 // log2 units: rescale only when the running max grows by more than 2^20.  P is bf16 and O
 // and its row sum accumulate in fp32, so p <= 2^20 over at most 2^18 keys stays far from
@@ -73,6 +79,8 @@ struct __align__(1024) AttnSmem {
   uint64_t q_full, q_empty;
   uint64_t s_full[2], p_full[2];
   uint64_t drain;
+  uint64_t it_full[kItemSlots], it_empty[kItemSlots];
+  int item_q[kItemSlots];  // item index, or -1: no more items
   TileInfo info[kStages];
   uint32_t tmem_base;
   int abort;
@@ -226,6 +234,10 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
       mbar_init(&S.p_full[b], 4);
     }
     mbar_init(&S.drain, 1);
+    for (int q = 0; q < kItemSlots; ++q) {
+      mbar_init(&S.it_full[q], 1);
+      mbar_init(&S.it_empty[q], 4);
+    }
     S.abort = 0;
     fence_barrier_init();
     prefetch_tensormap(&tmQ);
@@ -248,8 +260,20 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
     // =============================== producer ====================================
     // All lanes walk the list together (32 entries per coalesced load, broadcast by
     // shuffle); lane 0 issues the barrier operations and the TMA copies.
-    int g = 0, it = 0;
+    int g = 0, it = 0, pub = 0;
     bool failed = false, q_loaded = false;
+    // announce an item (or -1: none left) to the softmax warps, which walk its list themselves
+    auto publish = [&](int item) -> bool {
+      const int slot = pub % kItemSlots, u = pub / kItemSlots;
+      if (u > 0 && !warp_wait(&S.it_empty[slot], (u - 1) & 1, abort)) return false;
+      if (lane == 0) {
+        S.item_q[slot] = item;
+        mbar_arrive(&S.it_full[slot]);
+      }
+      __syncwarp();
+      ++pub;
+      return true;
+    };
     for (;;) {
       int item = 0;
       if (lane == 0) item = (int)atomicAdd(a.counter, 1u);
@@ -260,6 +284,10 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
       const int n = a.plen[h * a.npairs + p];
       if (n <= 0) continue;
       const int32_t* lst = a.plist + a.row_ptr[(int64_t)h * a.rows_per_head + a.row_step * p];
+      if (!publish(item)) {
+        failed = true;
+        break;
+      }
       if (it > 0 && !warp_wait(&S.q_empty, (it - 1) & 1, abort)) {
         failed = true;
         break;
@@ -307,6 +335,7 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
         S.info[s] = TileInfo{0, 0, kTerm, -1};
         mbar_arrive(&S.kv_full[s]);
       }
+      if (!failed && !publish(-1)) failed = true;
     }
     if (failed && lane == 0) {
       give_up(S, a.status);
@@ -422,164 +451,194 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
     __syncwarp();
   } else {
     // ================================ softmax =====================================
+    // Each warp walks the announced items' union lists itself (32 entries per coalesced
+    // load, the next 32 loaded while the current ones are used), so a tile costs it only
+    // the wait for S.
     const int quarter = warp & 3;
     const int r = quarter * 32 + lane;  // query row within the 128-row tile
     const int half = r >> 6;
     const uint32_t lane_base = (uint32_t)(quarter * 32) << 16;
     const float kScale = 1.4426950408889634f * 0.125f;  // log2(e) / sqrt(64)
+    // p = 2^(s * log2(e)/8 - m) of this row's 64 columns, two columns per packed FMA
+    auto exps = [&](const float (&x)[64], float m, uint32_t (&w)[32]) {
+      const float nm = -m;
+#pragma unroll
+      for (int e = 0; e < 32; ++e) {
+        float t0, t1;
+        fma2(t0, t1, x[2 * e], x[2 * e + 1], kScale, kScale, nm, nm);
+        w[e] = pack_bf16x2(ex2(t0), ex2(t1));
+      }
+    };
+    // the row maximum of the raw scores (the scale is positive) as a tree of 3-input maxima
+    auto row_max = [&](const float (&x)[64]) -> float {
+      float m1[22];
+#pragma unroll
+      for (int k = 0; k < 21; ++k) m1[k] = fmax3(x[3 * k], x[3 * k + 1], x[3 * k + 2]);
+      m1[21] = x[63];
+      float m2[8];
+#pragma unroll
+      for (int k = 0; k < 7; ++k) m2[k] = fmax3(m1[3 * k], m1[3 * k + 1], m1[3 * k + 2]);
+      m2[7] = m1[21];
+      return fmax3(fmax3(m2[0], m2[1], m2[2]), fmax3(m2[3], m2[4], m2[5]), fmaxf(m2[6], m2[7]));
+    };
     int g = 0;
-    float m_use = -INFINITY;
-    int tile_in_item = 0;
-    for (;;) {
-      const int s = g % kStages;
-      if (!warp_wait(&S.kv_full[s], (g / kStages) & 1, abort)) {
+    bool stop = false;
+    for (int pub = 0; !stop; ++pub) {
+      const int slot = pub % kItemSlots;
+      if (!warp_wait(&S.it_full[slot], (pub / kItemSlots) & 1, abort)) {
         give_up(S, a.status);
         break;
       }
-      const TileInfo info = S.info[s];
-      if (info.flags & kTerm) break;
-      if (info.flags & kFirst) {
-        m_use = -INFINITY;
-        tile_in_item = 0;
-      }
-      const int b = g & 1;
-      // S_g complete implies every earlier MMA complete, P_{g-2} V_{g-2} included
-      if (!warp_wait(&S.s_full[b], (g >> 1) & 1, abort)) {
-        give_up(S, a.status);
-        break;
-      }
-      tc_fence_after();
-      const bool active = (info.mask >> half) & 1;  // warp-uniform
-      const uint32_t tS = tmem + lane_base + kColS0 + 64 * b;
-      if (active) {
-        float x[64];
-        {
-          uint32_t v[64];
-          RESS_TMEM_LD64(tS, v);
-#pragma unroll
-          for (int c = 0; c < 64; ++c) x[c] = __uint_as_float(v[c]);
-        }
-        if (info.j == a.nb - 1) {  // ragged last key block: keys past N do not exist
-          const int valid = a.N - 64 * info.j;
-#pragma unroll
-          for (int c = 0; c < 64; ++c)
-            if (c >= valid) x[c] = -INFINITY;
-        }
-        // row max of the raw scores (the scale is positive) as a tree of 3-input maxima
-        float m1[22];
-#pragma unroll
-        for (int k = 0; k < 21; ++k) m1[k] = fmax3(x[3 * k], x[3 * k + 1], x[3 * k + 2]);
-        m1[21] = x[63];
-        float m2[8];
-#pragma unroll
-        for (int k = 0; k < 7; ++k) m2[k] = fmax3(m1[3 * k], m1[3 * k + 1], m1[3 * k + 2]);
-        m2[7] = m1[21];
-        const float mr =
-            fmax3(fmax3(m2[0], m2[1], m2[2]), fmax3(m2[3], m2[4], m2[5]), fmaxf(m2[6], m2[7]));
-        const float mt = mr * kScale;
-        float alpha = 1.f;
-        bool rescale = false;
-        if (m_use == -INFINITY) {
-          m_use = mt;  // first kept tile of this row: O row is still zero
-        } else if (mt > m_use + kLazyThreshold) {
-          alpha = ex2(m_use - mt);
-          m_use = mt;
-          rescale = true;
-        }
-        // p = 2^(s * log2(e)/8 - m), two columns per packed FMA
-        const float nm = -m_use;
-        uint32_t w[32];
-#pragma unroll
-        for (int e = 0; e < 32; ++e) {
-          float t0, t1;
-          fma2(t0, t1, x[2 * e], x[2 * e + 1], kScale, kScale, nm, nm);
-          w[e] = pack_bf16x2(ex2(t0), ex2(t1));
-        }
-        RESS_TMEM_ST32(tS, w);  // P_g over the first 32 columns of S_g
-        if (__any_sync(0xffffffffu, rescale)) {
-          // the previous P V must have landed before the accumulator row is rescaled; the
-          // exponentials above ran while it was in flight
-          if (!warp_wait(&S.kv_empty[(g - 1) % kStages], ((g - 1) / kStages) & 1, abort)) {
+      const int item = S.item_q[slot];
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&S.it_empty[slot]);
+      if (item < 0) break;
+      int h, p, t0, t1;
+      item_pair(a, item, h, p);
+      item_tokens(a, h, p, t0, t1);
+      const int n = a.plen[h * a.npairs + p];
+      const int32_t* lst = a.plist + a.row_ptr[(int64_t)h * a.rows_per_head + a.row_step * p];
+      float m_use = -INFINITY;  // this row's reference maximum (log2 units); warp-uniform -inf
+      int mine = lane < n ? lst[lane] : 0;
+      for (int e0 = 0; e0 < n && !stop; e0 += 32) {
+        const int nxt = (e0 + 32 + lane < n) ? lst[e0 + 32 + lane] : 0;
+        const int cnt = min(32, n - e0);
+        for (int k = 0; k < cnt; ++k) {
+          const int ent = __shfl_sync(0xffffffffu, mine, k);
+          const int j = ent & 0xffff;
+          const bool active = (ent >> (16 + half)) & 1;  // warp-uniform
+          const int b = g & 1;
+          // S_g complete implies every earlier MMA complete, P_{g-2} V_{g-2} included
+          if (!warp_wait(&S.s_full[b], (g >> 1) & 1, abort)) {
             give_up(S, a.status);
+            stop = true;
             break;
           }
           tc_fence_after();
+          const uint32_t tS = tmem + lane_base + kColS0 + 64 * b;
+          if (active) {
+            float x[64];
+            {
+              uint32_t v[64];
+              RESS_TMEM_LD64(tS, v);
 #pragma unroll
-          for (int hc = 0; hc < 2; ++hc) {
-            uint32_t v[32];
-            RESS_TMEM_LD32(tmem + lane_base + kColO + 32 * hc, v);
+              for (int c = 0; c < 64; ++c) x[c] = __uint_as_float(v[c]);
+            }
+            if (j == a.nb - 1) {  // ragged last key block: keys past N do not exist
+              const int valid = a.N - 64 * j;
 #pragma unroll
-            for (int c = 0; c < 32; ++c) v[c] = __float_as_uint(__uint_as_float(v[c]) * alpha);
-            RESS_TMEM_ST32(tmem + lane_base + kColO + 32 * hc, v);
-          }
-          {  // the row sum (column 64) and the unused columns after it
-            uint32_t v[16];
-            RESS_TMEM_LD16(tmem + lane_base + kColO + 64, v);
+              for (int c = 0; c < 64; ++c)
+                if (c >= valid) x[c] = -INFINITY;
+            }
+            uint32_t w[32];
+            float alpha = 1.f;
+            bool rescale = false;
+            if (m_use == -INFINITY) {
+              // first kept tile of this row: O row is still zero
+              m_use = row_max(x) * kScale;
+              exps(x, m_use, w);
+            } else {
+              // the exponentials against the current reference run alongside the maximum;
+              // a row whose maximum grew by more than 2^20 (rare) takes the new maximum
+              // and the warp recomputes, so P is the same as with the maximum taken first
+              exps(x, m_use, w);
+              const float mt = row_max(x) * kScale;
+              const bool grow = mt > m_use + kLazyThreshold;
+              if (__any_sync(0xffffffffu, grow)) {
+                if (grow) {
+                  alpha = ex2(m_use - mt);
+                  m_use = mt;
+                  rescale = true;
+                }
+                exps(x, m_use, w);
+              }
+            }
+            RESS_TMEM_ST32(tS, w);  // P_g over the first 32 columns of S_g
+            if (__any_sync(0xffffffffu, rescale)) {
+              // the previous P V must have landed before the accumulator row is rescaled;
+              // the exponentials above ran while it was in flight
+              if (!warp_wait(&S.kv_empty[(g - 1) % kStages], ((g - 1) / kStages) & 1, abort)) {
+                give_up(S, a.status);
+                stop = true;
+                break;
+              }
+              tc_fence_after();
 #pragma unroll
-            for (int c = 0; c < 16; ++c) v[c] = __float_as_uint(__uint_as_float(v[c]) * alpha);
-            RESS_TMEM_ST16(tmem + lane_base + kColO + 64, v);
-          }
-        }
-      } else {
-        uint32_t w[32];
+              for (int hc = 0; hc < 2; ++hc) {
+                uint32_t v[32];
+                RESS_TMEM_LD32(tmem + lane_base + kColO + 32 * hc, v);
 #pragma unroll
-        for (int e = 0; e < 32; ++e) w[e] = 0u;
-        RESS_TMEM_ST32(tS, w);
-      }
-      tc_fence_before();
-      __syncwarp();
-      if (lane == 0) mbar_arrive(&S.p_full[b]);
-      ++tile_in_item;
-
-      if (info.flags & kLast) {
-        // epilogue: O / l for this row once the last P V has landed
-        if (!warp_wait(&S.kv_empty[g % kStages], (g / kStages) & 1, abort)) {
-          give_up(S, a.status);
-          break;
-        }
-        tc_fence_after();
-        int h, p, t0, t1;
-        item_pair(a, info.item, h, p);
-        item_tokens(a, h, p, t0, t1);
-        const int token = (half ? t1 : t0) + (r & 63);
-        const bool row_exists = token < a.N;
-        uint32_t o[2][32], ls[16];
-        RESS_TMEM_LD32(tmem + lane_base + kColO, o[0]);
-        RESS_TMEM_LD32(tmem + lane_base + kColO + 32, o[1]);
-        RESS_TMEM_LD16(tmem + lane_base + kColO + 64, ls);
-        const float l = __uint_as_float(ls[0]);  // row sum of the bf16 probabilities
-        if (row_exists) {
-          if (!(l > 0.f)) flag_status(a.status, kStatusBadRow);
-          const float inv = l > 0.f ? 1.0f / l : 0.f;
-          const int64_t off = ((int64_t)token * a.H + h) * 64;
-          if (kOutF32) {
-            float4* dst = reinterpret_cast<float4*>(static_cast<float*>(a.O) + off);
+                for (int c = 0; c < 32; ++c) v[c] = __float_as_uint(__uint_as_float(v[c]) * alpha);
+                RESS_TMEM_ST32(tmem + lane_base + kColO + 32 * hc, v);
+              }
+              {  // the row sum (column 64) and the unused columns after it
+                uint32_t v[16];
+                RESS_TMEM_LD16(tmem + lane_base + kColO + 64, v);
 #pragma unroll
-            for (int ch = 0; ch < 16; ++ch) {
-              const int c = ch * 4;
-              dst[ch] = make_float4(__uint_as_float(o[c >> 5][c & 31]) * inv,
-                                    __uint_as_float(o[(c + 1) >> 5][(c + 1) & 31]) * inv,
-                                    __uint_as_float(o[(c + 2) >> 5][(c + 2) & 31]) * inv,
-                                    __uint_as_float(o[(c + 3) >> 5][(c + 3) & 31]) * inv);
+                for (int c = 0; c < 16; ++c) v[c] = __float_as_uint(__uint_as_float(v[c]) * alpha);
+                RESS_TMEM_ST16(tmem + lane_base + kColO + 64, v);
+              }
             }
           } else {
-            uint4* dst = reinterpret_cast<uint4*>(static_cast<uint16_t*>(a.O) + off);
+            uint32_t w[32];
 #pragma unroll
-            for (int ch = 0; ch < 8; ++ch) {
-              uint32_t w[4];
-#pragma unroll
-              for (int e = 0; e < 4; ++e) {
-                const int c = ch * 8 + 2 * e;
-                w[e] = pack_bf16x2(__uint_as_float(o[c >> 5][c & 31]) * inv,
-                                   __uint_as_float(o[(c + 1) >> 5][(c + 1) & 31]) * inv);
-              }
-              dst[ch] = make_uint4(w[0], w[1], w[2], w[3]);
-            }
+            for (int e = 0; e < 32; ++e) w[e] = 0u;
+            RESS_TMEM_ST32(tS, w);
           }
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&S.p_full[b]);
+
+          if (e0 + k == n - 1) {
+            // epilogue: O / l for this row once the last P V has landed
+            if (!warp_wait(&S.kv_empty[g % kStages], (g / kStages) & 1, abort)) {
+              give_up(S, a.status);
+              stop = true;
+              break;
+            }
+            tc_fence_after();
+            const int token = (half ? t1 : t0) + (r & 63);
+            const bool row_exists = token < a.N;
+            uint32_t o[2][32], ls[16];
+            RESS_TMEM_LD32(tmem + lane_base + kColO, o[0]);
+            RESS_TMEM_LD32(tmem + lane_base + kColO + 32, o[1]);
+            RESS_TMEM_LD16(tmem + lane_base + kColO + 64, ls);
+            const float l = __uint_as_float(ls[0]);  // row sum of the bf16 probabilities
+            if (row_exists) {
+              if (!(l > 0.f)) flag_status(a.status, kStatusBadRow);
+              const float inv = l > 0.f ? 1.0f / l : 0.f;
+              const int64_t off = ((int64_t)token * a.H + h) * 64;
+              if (kOutF32) {
+                float4* dst = reinterpret_cast<float4*>(static_cast<float*>(a.O) + off);
+#pragma unroll
+                for (int ch = 0; ch < 16; ++ch) {
+                  const int c = ch * 4;
+                  dst[ch] = make_float4(__uint_as_float(o[c >> 5][c & 31]) * inv,
+                                        __uint_as_float(o[(c + 1) >> 5][(c + 1) & 31]) * inv,
+                                        __uint_as_float(o[(c + 2) >> 5][(c + 2) & 31]) * inv,
+                                        __uint_as_float(o[(c + 3) >> 5][(c + 3) & 31]) * inv);
+                }
+              } else {
+                uint4* dst = reinterpret_cast<uint4*>(static_cast<uint16_t*>(a.O) + off);
+#pragma unroll
+                for (int ch = 0; ch < 8; ++ch) {
+                  uint32_t wo[4];
+#pragma unroll
+                  for (int e = 0; e < 4; ++e) {
+                    const int c = ch * 8 + 2 * e;
+                    wo[e] = pack_bf16x2(__uint_as_float(o[c >> 5][c & 31]) * inv,
+                                        __uint_as_float(o[(c + 1) >> 5][(c + 1) & 31]) * inv);
+                  }
+                  dst[ch] = make_uint4(wo[0], wo[1], wo[2], wo[3]);
+                }
+              }
+            }
+            tc_fence_before();
+          }
+          ++g;
         }
-        tc_fence_before();
+        mine = nxt;
       }
-      ++g;
     }
   }
 
