@@ -53,6 +53,7 @@ struct __align__(1024) YSmem {
   uint8_t Z[kYStages][3][8192];   // z~ terms: 64 blocks x 64 channels bf16 (MN-major)
   float ny_part[4][kYRows];
   uint64_t full[kYStages], conv[kYStages], empty[kYStages];
+  uint64_t pdone[kYStages];  // every converter's P is in the stage's logits buffer
   uint64_t done;
   uint32_t tmem_base;
   int abort;
@@ -113,6 +114,7 @@ __global__ void __launch_bounds__(kYThreads, 1)
     for (int s = 0; s < kYStages; ++s) {
       mbar_init(&S.full[s], 1);
       mbar_init(&S.conv[s], kConvWarps);
+      mbar_init(&S.pdone[s], kConvWarps);
       mbar_init(&S.empty[s], 1);
     }
     mbar_init(&S.done, 1);
@@ -212,7 +214,6 @@ __global__ void __launch_bounds__(kYThreads, 1)
       }
       iz = 1.0f / z;
     }
-    float* Prow = p.P + (row_ok ? ri : 0) * p.ld;
     bool failed = false;
     for (int c = 0; c < nch; ++c) {
       const int s = c % kYStages, par = (c / kYStages) & 1;
@@ -222,7 +223,7 @@ __global__ void __launch_bounds__(kYThreads, 1)
       }
       const int jb = (c0 + c) * kYChunk + 16 * qq;  // first block of this thread's 16
       // L: box qq / 2, 16-byte chunks 4 (qq mod 2) .. + 3 of row r
-      const uint8_t* lrow = S.L[s][qq >> 1] + r * 128;
+      uint8_t* lrow = S.L[s][qq >> 1] + r * 128;
       float pv[16];
 #pragma unroll
       for (int k = 0; k < 4; ++k) {
@@ -232,12 +233,14 @@ __global__ void __launch_bounds__(kYThreads, 1)
         for (int e = 0; e < 4; ++e)
           pv[4 * k + e] = (row_ok && jb + 4 * k + e < p.nb) ? exp2f(lv[e] - m) * iz : 0.f;
       }
-      if (row_ok && jb < p.ld) {  // ld is a multiple of 16
+      // P back over this thread's logits in the stage buffer and its three bf16 terms into
+      // the A tiles; once every converter has done so, the chunk's 128 x 64 block of P goes
+      // to global memory as whole row segments (two 256-byte rows per warp and store
+      // instead of 32 rows of 16 bytes)
 #pragma unroll
-        for (int k = 0; k < 4; ++k)
-          *reinterpret_cast<float4*>(Prow + jb + 4 * k) =
-              make_float4(pv[4 * k], pv[4 * k + 1], pv[4 * k + 2], pv[4 * k + 3]);
-      }
+      for (int k = 0; k < 4; ++k)
+        *reinterpret_cast<float4*>(lrow + (((4 * (qq & 1) + k) ^ (r & 7)) << 4)) =
+            make_float4(pv[4 * k], pv[4 * k + 1], pv[4 * k + 2], pv[4 * k + 3]);
       // P terms: this thread's 16 blocks are 16-byte chunks 2 qq, 2 qq + 1 of row r
 #pragma unroll
       for (int k = 0; k < 2; ++k) {
@@ -249,6 +252,23 @@ __global__ void __launch_bounds__(kYThreads, 1)
         *reinterpret_cast<uint4*>(S.A[s][0] + off) = make_uint4(hi[0], hi[1], hi[2], hi[3]);
         *reinterpret_cast<uint4*>(S.A[s][1] + off) = make_uint4(mid[0], mid[1], mid[2], mid[3]);
         *reinterpret_cast<uint4*>(S.A[s][2] + off) = make_uint4(lo[0], lo[1], lo[2], lo[3]);
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&S.pdone[s]);
+      if (!y_wait(&S.pdone[s], par, abort)) {  // bounded: a converter that gave up ends it
+        failed = true;
+        break;
+      }
+#pragma unroll
+      for (int k = 0; k < 4; ++k) {
+        const int idx = (int)threadIdx.x + 32 * kConvWarps * k;  // float4 of the 128 x 16
+        const int rr = idx >> 4, c4 = idx & 15;
+        const int j = (c0 + c) * kYChunk + 4 * c4;
+        if (i0 + rr < p.nqc && j < p.ld) {  // ld is a multiple of 16
+          const float4 v4 = *reinterpret_cast<const float4*>(
+              S.L[s][c4 >> 3] + rr * 128 + (((c4 & 7) ^ (rr & 7)) << 4));
+          *reinterpret_cast<float4*>(p.P + ((int64_t)h * p.nq + i0 + rr) * p.ld + j) = v4;
+        }
       }
       fence_proxy_async_smem();
       __syncwarp();
