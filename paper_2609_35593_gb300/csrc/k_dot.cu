@@ -50,6 +50,7 @@ constexpr float kLogitScale = 0.125f * 1.4426950408889634f;  // 1/sqrt(64) * log
 struct __align__(1024) DotSmem {
   uint8_t A[3][kTermBytes];  // row-vector terms (hi, mid, lo) of rows i0 .. i0 + 127
   uint8_t B[3][kTermBytes];  // block-vector terms of blocks j0 .. j0 + 127
+  float bcol[kDotTile];      // drift norms: ||z~_j||^2 of the tile's blocks
   uint64_t full, done;
   uint32_t tmem_base;
   int abort;
@@ -103,6 +104,10 @@ __global__ void __launch_bounds__(kDotThreads)
     prefetch_tensormap(&tmA);
     prefetch_tensormap(&tmB);
     prefetch_tensormap(&tmOut);
+  }
+  if (MODE == kDotDist) {
+    const int j = j0 + (int)threadIdx.x;  // kDotThreads == kDotTile
+    S.bcol[threadIdx.x] = j < p.nb ? p.b[(int64_t)h * p.nb + j] : 0.f;
   }
   if (warp == 0) tmem_alloc(&S.tmem_base, kDotCols);
   tc_fence_before();
@@ -190,17 +195,25 @@ __global__ void __launch_bounds__(kDotThreads)
           ps = (pm == -INFINITY) ? 0.f : ps * exp2f(pm - cm);
           pm = cm;
         }
+        // the sum in four interleaved partial sums, with the SFU's exp2 (relative error
+        // about 2^-22: far below what the row's softmax needs, and half the instructions)
+        float sp[4] = {0.f, 0.f, 0.f, 0.f};
 #pragma unroll
         for (int k = 0; k < 32; ++k)
-          if (jq + k < p.nb) ps += exp2f(o[k] - pm);
+          if (jq + k < p.nb) sp[k & 3] += ex2(o[k] - pm);
+        ps += (sp[0] + sp[1]) + (sp[2] + sp[3]);
       } else {
-        // ||z~_j||^2 of this quarter's 32 blocks: one coalesced load, then by shuffle
-        const int jq = j0 + 32 * q;
-        const float bl = (jq + lane < p.nb) ? p.b[(int64_t)h * p.nb + jq + lane] : 0.f;
+        // ||z~_j||^2 of this quarter's 32 blocks, broadcast from shared memory
+        const float4* bq = reinterpret_cast<const float4*>(S.bcol + 32 * q);
 #pragma unroll
-        for (int k = 0; k < 32; ++k) {
-          const float bz = __shfl_sync(0xffffffffu, bl, k);
-          o[k] = fmaxf(fmaf(-2.0f, __uint_as_float(v[k]), a + bz), 0.f);
+        for (int k4 = 0; k4 < 8; ++k4) {
+          const float4 bz = bq[k4];
+          const float b4[4] = {bz.x, bz.y, bz.z, bz.w};
+#pragma unroll
+          for (int e = 0; e < 4; ++e) {
+            const int k = 4 * k4 + e;
+            o[k] = fmaxf(fmaf(-2.0f, __uint_as_float(v[k]), a + b4[e]), 0.f);
+          }
         }
       }
       uint8_t* row = stage + q * 16384 + r * 128;

@@ -231,7 +231,7 @@ __global__ void __launch_bounds__(kYThreads, 1)
         const float lv[4] = {v.x, v.y, v.z, v.w};
 #pragma unroll
         for (int e = 0; e < 4; ++e)
-          pv[4 * k + e] = (row_ok && jb + 4 * k + e < p.nb) ? exp2f(lv[e] - m) * iz : 0.f;
+          pv[4 * k + e] = (row_ok && jb + 4 * k + e < p.nb) ? ex2(lv[e] - m) * iz : 0.f;
       }
       // P back over this thread's logits in the stage buffer and its three bf16 terms into
       // the A tiles; once every converter has done so, the chunk's 128 x 64 block of P goes
