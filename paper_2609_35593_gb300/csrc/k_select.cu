@@ -1061,70 +1061,113 @@ __global__ void __launch_bounds__(32 * kRowWarps, 10) k_round_rows(SelPtrs p, Bu
 // attention runs two 64-row query blocks as one M = 128 tile over the union of their kept
 // lists, so every key block kept by only one of them is half a tile of wasted tensor work.
 // Within each window of kPairWindow candidate query blocks of a head, blocks are paired by
-// the overlap of their best kept candidate sets: in ascending order, each block not yet
-// paired takes the unpaired block of the window that shares most kept blocks with it (ties
-// to the nearer one).  Output: prow[h, 32 w + k] = a | b << 16 for the k-th pair of window
+// the overlap of their best kept candidate sets, greedily by weight: of all pairs of
+// unpaired blocks of the window, the one sharing most kept blocks is taken next (ties to
+// the nearer pair, then to the lower first block).  Output: prow[h, 32 w + k] = a | b << 16 for the k-th pair of window
 // w.  Which blocks share a tile changes no row's result: a row attends its own kept blocks
 // in ascending order either way.  grid (windows, H) x 512 threads: all warps form the
-// window's overlaps, then the first warp pairs (one warp-wide maximum per pair).
+// window's overlaps, then take the pairs by weight (one block-wide maximum per pair).
 // ------------------------------------------------------------------------------------
 __global__ void __launch_bounds__(512) k_pairing(const uint32_t* __restrict__ bmask, int nq,
                                                  int words, int ncand, int npaired, int items,
                                                  int32_t* __restrict__ prow) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
   constexpr int W = kPairWindow;
-  const int ks = words | 1;  // odd row stride: the rows one load touches fall in distinct banks
-  uint32_t* kept = reinterpret_cast<uint32_t*>(smem_raw);     // [W][ks]
-  uint16_t* ov = reinterpret_cast<uint16_t*>(kept + W * ks);  // [W][W]
+  // kept sets as rows of 64-bit words with an odd row stride, so that the eight rows one
+  // load touches fall in distinct bank pairs
+  const int words2 = (words + 1) >> 1, ks2 = words2 | 1;
+  uint2* kept = reinterpret_cast<uint2*>(smem_raw);  // [W][ks2]
   const int h = blockIdx.y, w = blockIdx.x, t = threadIdx.x;
   const int r0 = W * w;
   const int n = min(W, 2 * npaired - r0);  // even
   if (n <= 0) return;
-  for (int idx = t; idx < W * words; idx += blockDim.x) {  // rows past n: empty
-    const int r = idx / words, wd = idx - r * words;
-    kept[r * ks + wd] =
-        r < n ? ~bmask[((int64_t)h * nq + r0 + r) * words + wd] & valid_bits(wd, ncand) : 0u;
+  for (int idx = t; idx < W * words2; idx += blockDim.x) {  // rows past n: empty
+    const int r = idx / words2, wd = 2 * (idx - r * words2);
+    uint2 v = make_uint2(0u, 0u);
+    if (r < n) {
+      const uint32_t* row = bmask + ((int64_t)h * nq + r0 + r) * words;
+      v.x = ~row[wd] & valid_bits(wd, ncand);
+      if (wd + 1 < words) v.y = ~row[wd + 1] & valid_bits(wd + 1, ncand);
+    }
+    kept[r * ks2 + (wd >> 1)] = v;
   }
   __syncthreads();
-  {  // thread t: row a = t / 8 against the blocks g, g + 8, .., g + 56 (g = t mod 8)
-    const int a = t >> 3, g = t & 7;
-    int c[8];
+  // thread t: block a = t / 8 against the blocks g, g + 8, .., g + 56 (g = t mod 8); the
+  // counts stay with the thread, which forms the keys of exactly these pairs below
+  const int a = t >> 3, g = t & 7;
+  int c[8];
 #pragma unroll
-    for (int j = 0; j < 8; ++j) c[j] = 0;
-    if (a < n) {
+  for (int j = 0; j < 8; ++j) c[j] = 0;
+  if (a < n) {
 #pragma unroll 2
-      for (int wd = 0; wd < words; ++wd) {
-        const uint32_t ka = kept[a * ks + wd];
+    for (int wd = 0; wd < words2; ++wd) {
+      const uint2 ka = kept[a * ks2 + wd];
 #pragma unroll
-        for (int j = 0; j < 8; ++j) c[j] += __popc(ka & kept[(g + 8 * j) * ks + wd]);
+      for (int j = 0; j < 8; ++j) {
+        const uint2 kb = kept[(g + 8 * j) * ks2 + wd];
+        c[j] += __popc(ka.x & kb.x) + __popc(ka.y & kb.y);
       }
-#pragma unroll
-      for (int j = 0; j < 8; ++j) ov[a * W + g + 8 * j] = (uint16_t)min(c[j], 2047);
     }
   }
-  __syncthreads();
-  if (t >= 32) return;
-  const int lane = t;
-  uint64_t freeb = n == 64 ? ~0ull : ((1ull << n) - 1ull);  // unpaired blocks of the window
-  int k = 0;
-  for (int a = 0; a < n - 1; ++a) {
-    if (!((freeb >> a) & 1ull)) continue;  // uniform across the warp
-    // the overlap, then the nearer block: candidates b > a (every earlier block is paired)
-    uint32_t key = 0u;
+  // Greedy matching by weight (the pair of unpaired blocks that shares most kept blocks
+  // first; ties to the nearer pair, then to the lower first block), found in rounds: every
+  // unpaired block points at its best unpaired partner, and blocks pointing at each other
+  // are paired (the best remaining pair always is; 7 rounds on average at 32 views).  Eight
+  // threads per block (thread t: block a = t / 8, partners g + 8 j, g = t mod 8).
+  __shared__ int best_s[W], partner_s[W];
+  __shared__ unsigned long long matched_s[2], lower_s[2];
+  const int lane = t & 31;
+  const uint32_t gmask = 0xFFu << (8 * (lane >> 3));  // the eight lanes of block a
+  uint32_t key[8];
 #pragma unroll
-    for (int s = 0; s < W / 32; ++s) {
-      const int b = lane + 32 * s;
-      if (b > a && b < n && ((freeb >> b) & 1ull)) {
-        const uint32_t kb = ((uint32_t)ov[a * W + b] << 12) | (uint32_t)(4095 - (b - a));
-        key = max(key, kb);
+  for (int j = 0; j < 8; ++j) {
+    const int b = g + 8 * j;
+    const int d = b > a ? b - a : a - b, lo = min(a, b);
+    // overlap < 2048 (clamped), |b - a| and min(a, b) < 64: one key per pair, every valid
+    // key above 0; the pair's count is the same whichever of its blocks forms it
+    key[j] = (b != a && b < n && a < n)
+                 ? ((uint32_t)min(c[j], 2047) << 12) | ((uint32_t)(63 - d) << 6) | (uint32_t)(63 - lo)
+                 : 0u;
+  }
+  if (t < W) partner_s[t] = -1;
+  if (t < 2) matched_s[t] = 0ull;
+  uint64_t freeb = n == 64 ? ~0ull : ((1ull << n) - 1ull);  // unpaired blocks of the window
+  __syncthreads();
+  for (int round = 0; round < W && __popcll(freeb) >= 2; ++round) {
+    uint32_t k = 0u;
+    if ((freeb >> a) & 1ull) {
+#pragma unroll
+      for (int j = 0; j < 8; ++j)
+        if ((freeb >> (g + 8 * j)) & 1ull) k = max(k, key[j]);
+    }
+    k = __reduce_max_sync(gmask, k);
+    if (g == 0) {
+      const int d = 63 - (int)((k >> 6) & 63u), lo = 63 - (int)(k & 63u);
+      best_s[a] = k == 0u ? -1 : (lo == a ? a + d : lo);
+    }
+    __syncthreads();
+    if (g == 0 && ((freeb >> a) & 1ull)) {
+      const int b = best_s[a];
+      if (b >= 0 && best_s[b] == a) {
+        partner_s[a] = b;
+        atomicOr(&matched_s[round & 1], 1ull << a);
       }
     }
-    const uint32_t best = __reduce_max_sync(0xffffffffu, key);
-    if (best == 0u) break;  // not reached: n is even, so a later block is always free
-    const int b = a + 4095 - (int)(best & 4095u);
-    freeb &= ~((1ull << a) | (1ull << b));
-    if (lane == 0) prow[(int64_t)h * items + W / 2 * w + k] = (r0 + a) | ((r0 + b) << 16);
-    ++k;
+    __syncthreads();
+    freeb &= ~matched_s[round & 1];
+    if (t == 0) matched_s[(round + 1) & 1] = 0ull;  // read by every thread a round ago
+  }
+  // pair slots in the order of the pairs' first blocks
+  if (t < W) {
+    const bool low = partner_s[t] > t;
+    const uint32_t bl = __ballot_sync(0xffffffffu, low);
+    if (lane == 0) lower_s[t >> 5] = bl;
+  }
+  __syncthreads();
+  if (t < W && partner_s[t] > t) {
+    const uint64_t lowm = (uint64_t)(uint32_t)lower_s[0] | ((uint64_t)(uint32_t)lower_s[1] << 32);
+    const int k = __popcll(lowm & ((1ull << t) - 1ull));
+    prow[(int64_t)h * items + W / 2 * w + k] = (r0 + t) | ((r0 + partner_s[t]) << 16);
   }
 }
 
@@ -1425,7 +1468,7 @@ cudaError_t launch_pairing(const SelectArgs& a, int32_t* prow, cudaStream_t st) 
   const Shape& s = a.s;
   const int npaired = paired_items(s);
   const int windows = (2 * npaired + kPairWindow - 1) / kPairWindow;
-  const size_t smem = (size_t)kPairWindow * (s.words | 1) * 4 + (size_t)kPairWindow * kPairWindow * 2;
+  const size_t smem = (size_t)kPairWindow * ((((s.words + 1) >> 1) | 1) * 8);
   cudaError_t e = cudaFuncSetAttribute(k_pairing, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
   if (e != cudaSuccess) return e;
   k_pairing<<<dim3(windows, s.H), 512, smem, st>>>((const uint32_t*)(a.ws + a.L.bmask), s.nq, s.words,
