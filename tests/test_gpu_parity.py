@@ -139,6 +139,24 @@ def test_forward_equals_staged_calls(tiny):
     assert np.array_equal(layer.buf.J_best.cpu().numpy(), tiny.buf.J_best.cpu().numpy())
 
 
+def greedy_pairs(keep):
+    """Greedy matching by weight of the query blocks of one window (host restatement of
+    the pairing's definition): keep [n, nb] bool kept candidate sets; of all pairs of unpaired
+    blocks the one sharing most kept blocks (clamped at 2047) is taken next, ties to the
+    nearer pair, then to the lower first block.  Pairs (a, b), a < b, by ascending a."""
+    n = keep.shape[0]
+    ov = np.minimum(keep.astype(np.int64) @ keep.T.astype(np.int64), 2047)
+    order = sorted(((int(ov[a, b]), -(b - a), -a, a, b) for a in range(n) for b in range(a + 1, n)),
+                   reverse=True)
+    free = np.ones(n, bool)
+    pairs = []
+    for *_, a, b in order:
+        if free[a] and free[b]:
+            free[a] = free[b] = False
+            pairs.append((a, b))
+    return sorted(pairs)
+
+
 @pytest.mark.parametrize("name,q_block", [("tiny_v2", 64), ("tiny_v2", 128), ("vggt_v8", 64),
                                           ("vggt_v8", 128)])
 def test_forward_item_lists(name, q_block):
@@ -149,7 +167,7 @@ def test_forward_item_lists(name, q_block):
     union of its two rows' lists with the right masks, and the attention output is bit for
     bit the one over adjacent pairs (ress_sparse_attn on the same CSR: a row's result does
     not depend on the row it shares a tile with).  The pairing keeps fewer one-sided union
-    entries than adjacent pairs."""
+    entries than adjacent pairs, and is the greedy matching by overlap of the kept sets."""
     wl = synth.WORKLOADS[name]
     layer = G.Layer(synth.make_inputs(wl), wl.n_special, wl.budgets(), wl.rounds, wl.rho,
                     q_block=q_block)
@@ -198,6 +216,18 @@ def test_forward_item_lists(name, q_block):
     if npaired:
         print(name, "union efficiency", entries / 2 / union, "adjacent", entries / 2 / adjacent_union)
         assert union <= adjacent_union
+        # the table is exactly the greedy matching by overlap of the best kept sets, window
+        # by window, its pairs in the order of their first blocks
+        drop = layer.drop_sets("bmask")
+        cand = np.arange(layer.nb) < layer.ncand
+        for h in range(layer.H):
+            keep = ~drop[h] & cand
+            for w0 in range(0, 2 * npaired, 64):
+                n = min(64, 2 * npaired - w0)
+                want = [(w0 + a, w0 + b) for a, b in greedy_pairs(keep[w0:w0 + n])]
+                got = [(int(v) & 0xffff, int(v) >> 16)
+                       for v in prow[h * items + w0 // 2:h * items + w0 // 2 + n // 2]]
+                assert got == want, (h, w0)
     r.sparse_attn(layer.d, layer.Q, layer.K, layer.V, b.row_ptr, b.col_idx, b.O, b.ws)
     r.status(b.ws)
     assert torch.equal(O_f.view(torch.int16), b.O.view(torch.int16))
