@@ -17,10 +17,13 @@
 //                y~ += P_c^(a) z~_c^(b)   for the six term pairs (a, b) of k_dot,
 //              M128 N64 K16 x 4 each, P terms K-major, z~ terms MN-major, both from shared
 //              memory, and commits them to the stage's "empty" barrier;
-//   warps 0-15 one row and 16 of the chunk's blocks per thread: P from L, P back to global
-//              memory, P as three bf16 terms into the stage's A tiles (128-byte swizzle),
-//              then an arrive on the stage's "converted" barrier; after the last chunk the
-//              epilogue (warp w: TMEM lanes 32 (w mod 4).., columns 16 (w / 4)..).
+//   warps 0-15 one row and 16 of the chunk's blocks per thread: P from L, written back over
+//              its logits in the stage buffer and as three bf16 terms into the stage's A
+//              tiles (128-byte swizzle); once all converters have done so (a bounded
+//              mbarrier), the chunk's 128 x 64 block of P goes to global memory as whole
+//              256-byte row segments, then an arrive on the stage's "converted" barrier;
+//              after the last chunk the epilogue (warp w: TMEM lanes 32 (w mod 4)..,
+//              columns 16 (w / 4)..).
 // Every mbarrier wait is bounded; a wait that gives up records RESS_ETIMEOUT, lets copies
 // and MMAs already issued finish (again bounded), frees TMEM and returns.
 
