@@ -158,7 +158,7 @@ def greedy_pairs(keep):
 
 
 @pytest.mark.parametrize("name,q_block", [("tiny_v2", 64), ("tiny_v2", 128), ("vggt_v8", 64),
-                                          ("vggt_v8", 128)])
+                                          ("vggt_v8", 128), ("vggt_v32", 64)])
 def test_forward_item_lists(name, q_block):
     """ress_forward's CSR kernel also writes the attention items' lists (entry j | mask << 16
     at each item's slot, the CSR offset of rows 2u, 2u + 1; lengths in plen).  On the 64-token
