@@ -698,11 +698,21 @@ __device__ __forceinline__ void kept_drift(const uint32_t* D, const SelPtrs& p,
                                            const float* __restrict__ zt, float y0, float y1,
                                            uint32_t* idx, float& g0, float& g1, float& K) {
   const int lane = threadIdx.x & 31;
+  // lane l compacts mask word w0 + l: one warp scan of the words' kept counts gives each
+  // word's first list position, then each lane writes its own word's blocks (ascending)
   int n = 0;
-  for (int w = 0; w < p.words; ++w) {
-    const uint32_t keep = ~D[w] & valid_bits(w, p.nb);
-    if ((keep >> lane) & 1u) idx[n + __popc(keep & ((1u << lane) - 1u))] = w * 32 + lane;
-    n += __popc(keep);
+  for (int w0 = 0; w0 < p.words; w0 += 32) {
+    const int w = w0 + lane;
+    uint32_t keep = w < p.words ? ~D[w] & valid_bits(w, p.nb) : 0u;
+    const int c = __popc(keep);
+    int inc = c;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const int y = __shfl_up_sync(kFull, inc, o);
+      if (lane >= o) inc += y;
+    }
+    for (int pos = n + inc - c; keep; keep &= keep - 1u, ++pos) idx[pos] = w * 32 + __ffs(keep) - 1;
+    n += __shfl_sync(kFull, inc, 31);
   }
   __syncwarp();
   g0 = g1 = K = 0.f;
