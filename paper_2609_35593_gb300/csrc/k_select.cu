@@ -237,6 +237,7 @@ struct SelPtrs {
   float* cdot;           // [H, nb] y~_i . g~_i
   int64_t split_stride;  // H nb 32: uint32 words per term
   int32_t* kcount;       // [H, nq] key blocks kept by each candidate row
+  uint32_t* status;      // device status word (first error wins)
 };
 
 __host__ __device__ inline SelPtrs sel_ptrs(const Shape& s, char* ws, const ress_ws_layout& L) {
@@ -266,6 +267,7 @@ __host__ __device__ inline SelPtrs sel_ptrs(const Shape& s, char* ws, const ress
   p.cdot = (float*)(ws + L.cdot);
   p.split_stride = (int64_t)s.H * s.nq * 32;
   p.kcount = (int32_t*)(ws + L.kcount);
+  p.status = (uint32_t*)(ws + L.status);
   return p;
 }
 
@@ -1026,6 +1028,19 @@ __global__ void __launch_bounds__(32 * kRowWarps, 10) k_round_rows(SelPtrs p, Bu
     warp_topm(kk, p.ncand, m, Rw, p.words, sk, si, Dw, true);
     warp_topm(kk, p.ncand, m, Xw, p.words, sk, si, Dw, false);
   }
+  if (round == 0) {
+    // both selections took m blocks from their side only if the drop set holds that many on
+    // each; a workspace whose drop set cannot give them (one the scoring did not write, or
+    // one scored with other budgets) is reported instead of updated from.  Later rounds
+    // read the drop sets this round wrote, whose sizes the swaps keep.
+    int nd = 0;
+    for (int w = lane; w < p.words; w += 32) nd += __popc(Dw[w] & valid_bits(w, p.ncand));
+    nd = __reduce_add_sync(kFull, nd);
+    if (nd < m || p.ncand - nd < m) {
+      if (lane == 0) flag_status(p.status, kStatusBadRow);
+      return;
+    }
+  }
   if (!listed) {
     lst = reinterpret_cast<uint16_t*>(kk);  // 2 key_words >= 2m entries
     nl = 0;
@@ -1041,7 +1056,8 @@ __global__ void __launch_bounds__(32 * kRowWarps, 10) k_round_rows(SelPtrs p, Bu
   // every listed block changes sides: restores leave D, drops join it
   for (int e = lane; e < nl; e += 32) {
     const int j = lst[e] & 0x7fff;
-    atomicXor(&Dw[j >> 5], 1u << (j & 31));
+    if (j < p.ncand) atomicXor(&Dw[j >> 5], 1u << (j & 31));
+    else flag_status(p.status, kStatusBadIndex);
   }
   __syncwarp();
   // state of the new set (Eq. 10-12): the swapped blocks update g~ and K
