@@ -271,6 +271,14 @@ __host__ __device__ inline SelPtrs sel_ptrs(const Shape& s, char* ws, const ress
   return p;
 }
 
+// Square root by the SFU (sqrt.approx: a few ulp, against the IEEE-rounded sqrtf's longer
+// sequence); q >= 0 here, and sqrt of 0 is 0.
+__device__ __forceinline__ float sqrt_approx(float x) {
+  float y;
+  asm("sqrt.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
 // Order-preserving map of a float to uint32; every non-NaN value maps above 0, so 0 can
 // mark "not a candidate".  -0 is folded onto +0; NaN maps to the lowest candidate value.
 __device__ __forceinline__ uint32_t order_key(float x) {
@@ -900,6 +908,8 @@ __device__ void cdf_extend(const uint32_t* kk, const float* __restrict__ Prow, u
 // The variant picks the key: the Eq. 7 drift key (ReSS), the pooled probability, or the top
 // 24 bits of SplitMix64 at seed + (h 4096 + i) 4096 + j; the full sign flip keeps the
 // smallest keys (complemented keys, ties still to the lower index).
+// KEY: the key variant (v.key), a template parameter so that the per-block key has no branch.
+template <int KEY>
 __global__ void __launch_bounds__(32 * kRowWarps, 9) k_score_rows(SelPtrs p, Budgets bud,
                                                                   Variant v) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
@@ -925,9 +935,9 @@ __global__ void __launch_bounds__(32 * kRowWarps, 9) k_score_rows(SelPtrs p, Bud
 #pragma unroll
     for (int u = 0; u < 4; ++u) {
       uint32_t key;
-      if (v.key == 0)  // s_ij / max(1 - P_ij, eps), s_ij = P_ij sqrt(q_ij)
-        key = order_key(__fdividef(pv[u] * sqrtf(qv[u]), fmaxf(1.0f - pv[u], kEps)));
-      else if (v.key == 1)
+      if (KEY == 0)  // s_ij / max(1 - P_ij, eps), s_ij = P_ij sqrt(q_ij); the SFU's square root
+        key = order_key(__fdividef(pv[u] * sqrt_approx(qv[u]), fmaxf(1.0f - pv[u], kEps)));
+      else if (KEY == 1)
         key = order_key(pv[u]);
       else
         key = (uint32_t)(splitmix64(v.seed + ((unsigned long long)h * 4096ull + (unsigned long long)i) *
@@ -1429,9 +1439,10 @@ cudaError_t launch_score(const SelectArgs& a, cudaStream_t st) {
   if ((e = launch_drift_norms(a, st)) != cudaSuccess) return e;
   const size_t rsmem =
       (size_t)kRowWarps * warp_scratch_words(s.ld, score_mask_words(s.words, a.v.cdf > 0.f)) * 4;
-  e = cudaFuncSetAttribute(k_score_rows, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)rsmem);
+  auto kern = a.v.key == 0 ? k_score_rows<0> : a.v.key == 1 ? k_score_rows<1> : k_score_rows<2>;
+  e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)rsmem);
   if (e != cudaSuccess) return e;
-  k_score_rows<<<dim3((s.nqc + kRowWarps - 1) / kRowWarps, s.H), 32 * kRowWarps, rsmem, st>>>(
+  kern<<<dim3((s.nqc + kRowWarps - 1) / kRowWarps, s.H), 32 * kRowWarps, rsmem, st>>>(
       p, budgets_of(a), a.v);
   note_launch();
   return cudaGetLastError();
