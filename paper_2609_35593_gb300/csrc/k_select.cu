@@ -488,6 +488,28 @@ __device__ void select_radix(const uint32_t* keys, const uint16_t* idx, int n, i
   }
 }
 
+// The lower bound of step 1 with KT = ceil(m / 32) keys kept per lane: the m-th largest of
+// the lanes' KT largest participating keys.
+template <int KT>
+__device__ __forceinline__ uint32_t lane_topk_bound(const uint32_t* kk, int n, int m,
+                                                    const uint32_t* member, bool want) {
+  const int lane = threadIdx.x & 31;
+  uint32_t top[KT];
+#pragma unroll
+  for (int k = 0; k < KT; ++k) top[k] = 0u;
+#pragma unroll 2
+  for (int x = lane; x < n; x += 32) {
+    uint32_t v = takes_part(member, want, x) ? kk[x] : 0u;
+#pragma unroll
+    for (int k = 0; k < KT; ++k) {
+      const uint32_t hi = max(top[k], v);
+      v = min(top[k], v);
+      top[k] = hi;
+    }
+  }
+  return mth_largest(top, m);
+}
+
 // Requires m <= number of participating blocks.  sk/si: survivor scratch (kSurvivors);
 // hist: 256 words for select_radix on the survivors (NULL: bit-by-bit select_exact).
 __device__ void warp_topm(const uint32_t* kk, int n, int m, uint32_t* sel, int words,
@@ -503,24 +525,14 @@ __device__ void warp_topm(const uint32_t* kk, int n, int m, uint32_t* sel, int w
     __syncwarp();
     return;
   }
-  // 1. lane-local top-kTopK (descending) of the participating keys, then the lower bound
-  uint32_t top[kTopK];
-#pragma unroll
-  for (int k = 0; k < kTopK; ++k) top[k] = 0u;
-#pragma unroll 2
-  for (int x = lane; x < n; x += 32) {
-    uint32_t v = takes_part(member, want, x) ? kk[x] : 0u;
-#pragma unroll
-    for (int k = 0; k < kTopK; ++k) {
-      const uint32_t hi = max(top[k], v);
-      v = min(top[k], v);
-      top[k] = hi;
-    }
+  // 1. lane-local top-K (descending) of the participating keys, then the lower bound
+  uint32_t bound;
+  switch (K) {
+    case 1: bound = lane_topk_bound<1>(kk, n, m, member, want); break;
+    case 2: bound = lane_topk_bound<2>(kk, n, m, member, want); break;
+    case 3: bound = lane_topk_bound<3>(kk, n, m, member, want); break;
+    default: bound = lane_topk_bound<4>(kk, n, m, member, want); break;
   }
-#pragma unroll
-  for (int k = 0; k < kTopK; ++k)
-    if (k >= K) top[k] = 0u;
-  const uint32_t bound = mth_largest(top, m);
   // 2. survivors (participating, >= bound), compacted in block order
   int cnt = 0;
   for (int x0 = 0; x0 < n; x0 += 32) {
@@ -740,8 +752,11 @@ __device__ __forceinline__ void kept_drift(const uint32_t* D, const SelPtrs& p,
 #pragma unroll
     for (int u = 0; u < 8; ++u) {
       if (k0 + u < n) {
-        g0 = fmaf(pj[u], z[u].x - y0, g0);
-        g1 = fmaf(pj[u], z[u].y - y1, g1);
+        // g += P_j (z~_j - y~), both channels in packed instructions (z - y as an exact
+        // fma with 1, so the bits are those of the scalar form)
+        float d0, d1;
+        ptx::fma2(d0, d1, z[u].x, z[u].y, 1.0f, 1.0f, -y0, -y1);
+        ptx::fma2(g0, g1, pj[u], pj[u], d0, d1, g0, g1);
         K += pj[u];
       }
     }
