@@ -998,9 +998,12 @@ __global__ void __launch_bounds__(32 * kRowWarps, 9) k_score_rows(SelPtrs p, Bud
 // Restoration round r, per row: exact top-m restores and drops from the round-start state,
 // update, track-best.  grid (ceil(|P| / 4), H).  With a maximising variant the keys are the
 // increases of J and track-best keeps the largest J.
+// MAXIMIZE: a maximising variant (keys are the increases of J, track-best keeps the largest
+// J), a template parameter so that the per-block key has no select.
+template <int MAXIMIZE>
 __global__ void __launch_bounds__(32 * kRowWarps, 10) k_round_rows(SelPtrs p, Budgets bud,
-                                                                  int round, float rho,
-                                                                  int maximize) {
+                                                                  int round, float rho) {
+  constexpr bool maximize = MAXIMIZE != 0;
   extern __shared__ __align__(16) unsigned char smem_raw[];
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int h = blockIdx.y, i = blockIdx.x * kRowWarps + warp;
@@ -1470,10 +1473,11 @@ cudaError_t launch_round(const SelectArgs& a, int round, float rho, cudaStream_t
   cudaError_t e = launch_gain(a, round, rho, st);  // t_ij on the tensor cores
   if (e != cudaSuccess) return e;
   const size_t rsmem = (size_t)kRowWarps * warp_scratch_words(s.ld, 3 * s.words) * 4;
-  e = cudaFuncSetAttribute(k_round_rows, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)rsmem);
+  auto kern = a.v.direction != 0 ? k_round_rows<1> : k_round_rows<0>;
+  e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)rsmem);
   if (e != cudaSuccess) return e;
-  k_round_rows<<<dim3((s.nqc + kRowWarps - 1) / kRowWarps, s.H), 32 * kRowWarps, rsmem, st>>>(
-      p, budgets_of(a), round, rho, a.v.direction != 0 ? 1 : 0);
+  kern<<<dim3((s.nqc + kRowWarps - 1) / kRowWarps, s.H), 32 * kRowWarps, rsmem, st>>>(
+      p, budgets_of(a), round, rho);
   note_launch();
   return cudaGetLastError();
 }
