@@ -1,13 +1,16 @@
 // Block-sparse attention forward over the kept 64x64 blocks (Sec. 3 step (3)) on sm_103a.
 //
 // Work item = (head h, pair of query blocks): their 128 query rows form the M = 128 operand
-// of tcgen05.mma, and the CTA walks the union of the two kept lists (ascending; built by
-// k_pairs, or by a forward's CSR kernel).  The pair is the adjacent blocks 2p, 2p+1, or,
-// in a forward on the 64-token grid, the two candidate blocks that the pairing table names
+// of tcgen05.mma, and the CTA walks the union of the two kept lists (built by k_pairs, or
+// by a forward's CSR kernel: the blocks kept by one query block only, alternating between
+// the two, then the rest ascending).  The pair is the adjacent blocks 2p, 2p+1, or, in a
+// forward on the 64-token grid, the two candidate blocks that the pairing table names
 // (paired by the overlap of their kept lists, so fewer union entries are kept by one block
 // only).  Each union entry carries a 2-bit mask saying which of the two query blocks keeps
 // it; rows of a block that does not keep the tile get P = 0, so every row sees exactly its
-// own kept blocks (softmax renormalised among them).
+// own kept blocks (softmax renormalised among them).  A one-sided tile keeps only two of the
+// four softmax warps busy (rows 0-63 or 64-127); alternating the sides lets the next tile's
+// two warps start while the current tile's finish, since S is double-buffered.
 //
 // Warp roles (192 threads, 2 CTAs per SM):
 //   warp 0     TMA producer: Q tile (two 64 x 64 halves, one per query block) per item,
@@ -196,17 +199,39 @@ __global__ void __launch_bounds__(256) k_pairs(const int32_t* __restrict__ row_p
     atomicOr((x < ea ? bA : bB) + (j >> 5), 1u << (j & 31));
   }
   __syncwarp();
-  // union in ascending block order, 32 blocks per step: lane l looks at block 32 w + l
-  int pos = 0;
-  for (int w = 0; w < words; ++w) {
-    const uint32_t a = bA[w], b = qb128 ? a : bB[w], u = a | b;
-    if ((u >> lane) & 1u) {
-      const int m = (int)((a >> lane) & 1u) | (int)(((b >> lane) & 1u) << 1);
-      plist[sa + pos + __popc(u & ((1u << lane) - 1u))] = (w * 32 + lane) | (m << 16);
-    }
-    pos += __popc(u);
+  // Entry order: the k-th block kept by the first query block only and the k-th kept by the
+  // second only (k < P, the smaller of the two counts, both ascending) alternate at list
+  // positions 2k, 2k + 1, so that the two halves' softmax work of consecutive one-sided
+  // tiles overlaps; then the rest of the union in ascending order.  Lane l looks at block
+  // 32 w + l.
+  int nA = 0, nB = 0;
+  for (int w = lane; w < words; w += 32) {
+    const uint32_t a = bA[w], b = qb128 ? a : bB[w];
+    nA += __popc(a & ~b);
+    nB += __popc(b & ~a);
   }
-  if (lane == 0) plen[pair] = pos;
+  const int P = min(__reduce_add_sync(0xffffffffu, nA), __reduce_add_sync(0xffffffffu, nB));
+  const uint32_t below = (1u << lane) - 1u;
+  int cA = 0, cB = 0, cR = 0;  // first-only, second-only and other entries before word w
+  for (int w = 0; w < words; ++w) {
+    const uint32_t a = bA[w], b = qb128 ? a : bB[w];
+    const uint32_t oa = a & ~b, ob = b & ~a;
+    const int rA = cA + __popc(oa & below), rB = cB + __popc(ob & below);
+    const bool pa = ((oa >> lane) & 1u) && rA < P, pb = ((ob >> lane) & 1u) && rB < P;
+    const bool rest = (((a | b) >> lane) & 1u) && !pa && !pb;
+    const uint32_t restw = __ballot_sync(0xffffffffu, rest);
+    const int j = w * 32 + lane;
+    if (pa) plist[sa + 2 * rA] = j | (1 << 16);
+    if (pb) plist[sa + 2 * rB + 1] = j | (2 << 16);
+    if (rest) {
+      const int m = (int)((a >> lane) & 1u) | (int)(((b >> lane) & 1u) << 1);
+      plist[sa + 2 * P + cR + __popc(restw & below)] = j | (m << 16);
+    }
+    cA += __popc(oa);
+    cB += __popc(ob);
+    cR += __popc(restw);
+  }
+  if (lane == 0) plen[pair] = 2 * P + cR;
 }
 
 // ------------------------------------------------------------------------------------

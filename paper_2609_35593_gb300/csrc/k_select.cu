@@ -1118,8 +1118,9 @@ __global__ void __launch_bounds__(32 * kRowWarps, 10) k_round_rows(SelPtrs p, Bu
 // the overlap of their best kept candidate sets, greedily by weight: of all pairs of
 // unpaired blocks of the window, the one sharing most kept blocks is taken next (ties to
 // the nearer pair, then to the lower first block).  Output: prow[h, 32 w + k] = a | b << 16 for the k-th pair of window
-// w.  Which blocks share a tile changes no row's result: a row attends its own kept blocks
-// in ascending order either way.  grid (windows, H) x 512 threads: all warps form the
+// w.  A row attends exactly its own kept blocks whichever block shares its tile; the partner
+// decides only their order (the blocks kept by one of the two lead the list), so it moves a
+// result by rounding alone.  grid (windows, H) x 512 threads: all warps form the
 // window's overlaps, then take the pairs by weight (one block-wide maximum per pair).
 // ------------------------------------------------------------------------------------
 __global__ void __launch_bounds__(512) k_pairing(const uint32_t* __restrict__ bmask, int nq,
@@ -1229,9 +1230,10 @@ __global__ void __launch_bounds__(512) k_pairing(const uint32_t* __restrict__ bm
 // Kept-block lists (CSR) from the best drop sets; special query rows keep everything.
 // One warp per attention item: query rows 2u and 2u + 1 on the 64-token grid, row u on the
 // 128-token grid.  With plist set the warp also writes the item's list for the attention
-// kernel (what k_pairs builds from a caller's CSR): the union of its rows' lists in
-// ascending order, entry j | mask << 16 (bit 0: the item's first 64 query rows keep j, bit 1:
-// the second 64), at the offset of the item's first row, and the union's length in plen.
+// kernel (what k_pairs builds from a caller's CSR): the union of its rows' lists, entry
+// j | mask << 16 (bit 0: the item's first 64 query rows keep j, bit 1: the second 64), at the
+// offset of the item's first row, and the union's length in plen.  Order: the blocks kept by
+// one row only alternate between the rows first (see below), then the rest ascending.
 // grid (ceil(items / 8), H) x 256 threads.
 // ------------------------------------------------------------------------------------
 struct CsrBases {
@@ -1332,16 +1334,35 @@ __global__ void k_csr(SelPtrs p, Budgets bud, CsrBases cb, int H, CsrOut o) {
   // an item's union list goes to its slot, the CSR span of rows rpi u .. rpi u + rpi - 1;
   // a paired item's two candidate rows have the slot's two lengths (fixed budgets)
   const int64_t uoff = paired ? cb.base[h] + (int64_t)i0 * (c + ns) : off[0];
-  // Lane l owns word w0 + l of each row: one warp scan of the lanes' kept counts gives
-  // every word's first list position, then each lane writes the blocks of its own word.
-  int posU = 0;
+  // best drop set of row r in mask word w (none for a dense row), and its kept blocks
+  auto drop_word = [&](int r, int w) -> uint32_t {
+    return dense[r] ? 0u : p.bmask[ri[r] * p.words + w];
+  };
+  auto kept_word = [&](int r, int w) -> uint32_t { return ~drop_word(r, w) & valid_bits(w, p.nb); };
+  // Union list order: the k-th block kept by the first row only and the k-th kept by the
+  // second only (k < P, the smaller of the two counts, both ascending) alternate at
+  // positions 2k, 2k + 1, so that in the attention the two halves' softmax work of
+  // consecutive one-sided tiles overlaps; then the rest of the union in ascending order.
+  int P = 0;
+  if (o.plist && rpi == 2 && nr == 2) {
+    int nA = 0, nB = 0;
+    for (int w = lane; w < p.words; w += 32) {
+      const uint32_t ka = kept_word(0, w), kb = kept_word(1, w);
+      nA += __popc(ka & ~kb);
+      nB += __popc(kb & ~ka);
+    }
+    P = min(__reduce_add_sync(kFull, nA), __reduce_add_sync(kFull, nB));
+  }
+  // Lane l owns word w0 + l of each row: warp scans of the lanes' counts give every word's
+  // first list positions, then each lane writes the blocks of its own word.
+  int posU = 0, cA = 0, cB = 0, cR = 0;
   for (int w0 = 0; w0 < p.words; w0 += 32) {
     const int w = w0 + lane;
     uint32_t keep[2] = {0u, 0u};
 #pragma unroll
     for (int r = 0; r < 2; ++r) {
       if (r < nr && w < p.words) {
-        const uint32_t dm = dense[r] ? 0u : p.bmask[ri[r] * p.words + w];
+        const uint32_t dm = drop_word(r, w);
         if (o.drop_mask) o.drop_mask[ri[r] * p.words + w] = dm;
         keep[r] = ~dm & valid_bits(w, p.nb);
       }
@@ -1349,30 +1370,62 @@ __global__ void k_csr(SelPtrs p, Budgets bud, CsrBases cb, int H, CsrOut o) {
     // a 128-token query block keeps its list for both 64-row halves of the tile
     const uint32_t kb = rpi == 1 ? keep[0] : keep[1];
     const uint32_t un = o.plist ? (keep[0] | kb) : 0u;
+    const uint32_t oa = P ? keep[0] & ~kb : 0u, ob = P ? kb & ~keep[0] : 0u;  // one-sided
     const int cAB = __popc(keep[0]) | (__popc(keep[1]) << 16), cU = __popc(un);
-    int iAB = cAB, iU = cU;
+    const int cO = __popc(oa) | (__popc(ob) << 16);
+    int iAB = cAB, iU = cU, iO = cO;
 #pragma unroll
     for (int d = 1; d < 32; d <<= 1) {
       const int yAB = __shfl_up_sync(kFull, iAB, d), yU = __shfl_up_sync(kFull, iU, d);
+      const int yO = __shfl_up_sync(kFull, iO, d);
       if (lane >= d) {
         iAB += yAB;
         iU += yU;
+        iO += yO;
       }
     }
     const int tAB = __shfl_sync(kFull, iAB, 31), tU = __shfl_sync(kFull, iU, 31);
+    const int tO = __shfl_sync(kFull, iO, 31);
     csr_write_word(o, keep[0], w, pos[0] + ((iAB - cAB) & 0xffff), expect[0], off[0]);
     csr_write_word(o, keep[1], w, pos[1] + ((iAB - cAB) >> 16), expect[1], off[1]);
     if (o.plist) {
-      int au = posU + iU - cU;
-      for (uint32_t bits = un; bits; bits &= bits - 1u, ++au) {
-        const int b = __ffs(bits) - 1;
-        const int m = (int)((keep[0] >> b) & 1u) | (int)(((kb >> b) & 1u) << 1);
-        if (uoff + au < o.plist_cap) o.plist[uoff + au] = (w * 32 + b) | (m << 16);
+      // ranks of this word's first one-sided blocks; its lowest mA (mB) of them alternate
+      const int gA = cA + ((iO - cO) & 0xffff), gB = cB + ((iO - cO) >> 16);
+      const int mA = min(max(P - gA, 0), __popc(oa)), mB = min(max(P - gB, 0), __popc(ob));
+      const int cRest = cU - mA - mB;
+      int iR = cRest;
+#pragma unroll
+      for (int d = 1; d < 32; d <<= 1) {
+        const int y = __shfl_up_sync(kFull, iR, d);
+        if (lane >= d) iR += y;
       }
+      int kA = 0, kB = 0, at = 2 * P + cR + iR - cRest;
+      for (uint32_t bits = un; bits; bits &= bits - 1u) {
+        const int b = __ffs(bits) - 1;
+        const int j = w * 32 + b;
+        int64_t dst;
+        int e;
+        if ((oa >> b) & 1u) {
+          dst = kA < mA ? 2 * (gA + kA) : at++;
+          e = j | (1 << 16);
+          ++kA;
+        } else if ((ob >> b) & 1u) {
+          dst = kB < mB ? 2 * (gB + kB) + 1 : at++;
+          e = j | (2 << 16);
+          ++kB;
+        } else {
+          dst = at++;
+          e = j | (((int)((keep[0] >> b) & 1u) | (int)(((kb >> b) & 1u) << 1)) << 16);
+        }
+        if (uoff + dst < o.plist_cap) o.plist[uoff + dst] = e;
+      }
+      cR += __shfl_sync(kFull, iR, 31);
     }
     pos[0] += tAB & 0xffff;
     pos[1] += tAB >> 16;
     posU += tU;
+    cA += tO & 0xffff;
+    cB += tO >> 16;
   }
   if (lane == 0) {
     for (int r = 0; r < nr; ++r) {

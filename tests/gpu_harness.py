@@ -208,6 +208,23 @@ def check_selection(r: dict) -> None:
     assert r["sum_rel_gpu_vs_oracle"] <= DRIFT_REL, r
 
 
+def compare_attention_bf16(layer: Layer, rows) -> dict:
+    """The bf16 output (the forward's own attention) against the oracle.  Rounding the exact
+    value to bf16 alone moves it by up to 2^-8 of its size, so max_abs is the error beyond
+    that; mean_rel includes the rounding."""
+    ref = layer.oracle_attention(rows)
+    out = layer.output_bf16()
+    num = den = 0.0
+    mx = 0.0
+    for (h, i), o in ref.items():
+        g = out[i * layer.q_block:i * layer.q_block + o.shape[0], h, :]
+        diff = np.abs(g - o)
+        mx = max(mx, float((diff - 2.0 ** -8 * np.abs(o)).max()))
+        num += float(diff.sum())
+        den += float(np.abs(o).sum())
+    return dict(max_abs=mx, mean_rel=num / max(den, 1e-30))
+
+
 def compare_attention(layer: Layer, rows) -> dict:
     ref = layer.oracle_attention(rows)
     out = layer.output()

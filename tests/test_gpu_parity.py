@@ -131,12 +131,18 @@ def test_bf16_output_is_rounded_f32_output(fixture, request):
 
 
 def test_forward_equals_staged_calls(tiny):
+    """The forward gives the staged calls' kept lists, best objectives and float32 output (the
+    same ress_sparse_attn_f32 on the same CSR) bit for bit.  Its bf16 attention walks paired
+    query blocks, whose one-sided blocks lead the lists, so a row takes its kept blocks in
+    another order than over adjacent pairs: that output is checked against the oracle on
+    every row (error beyond its bf16 rounding within the attention tolerance)."""
     layer, _ = layer_for("tiny_v2")
     layer.run_forward()
     assert np.array_equal(layer.csr()[1], tiny.csr()[1])
-    assert np.array_equal(layer.output_bf16(), tiny.output_bf16())
     assert np.array_equal(layer.output(), tiny.output())
     assert np.array_equal(layer.buf.J_best.cpu().numpy(), tiny.buf.J_best.cpu().numpy())
+    r = G.compare_attention_bf16(layer, [(h, i) for h in range(layer.H) for i in range(layer.nq)])
+    assert r["max_abs"] <= G.ATT_MAX_ABS and r["mean_rel"] <= G.ATT_MEAN_REL, r
 
 
 def greedy_pairs(keep):
@@ -163,11 +169,15 @@ def test_forward_item_lists(name, q_block):
     """ress_forward's CSR kernel also writes the attention items' lists (entry j | mask << 16
     at each item's slot, the CSR offset of rows 2u, 2u + 1; lengths in plen).  On the 64-token
     grid the forward pairs the candidate query blocks within windows of 64 by the overlap of
-    their kept lists (table prow): the items partition the rows, each list is exactly the
-    union of its two rows' lists with the right masks, and the attention output is bit for
-    bit the one over adjacent pairs (ress_sparse_attn on the same CSR: a row's result does
-    not depend on the row it shares a tile with).  The pairing keeps fewer one-sided union
-    entries than adjacent pairs, and is the greedy matching by overlap of the kept sets."""
+    their kept lists (table prow): the items partition the rows, and each list is exactly the
+    union of its two rows' lists with the right masks, laid out as the k-th block kept by the
+    first row only and the k-th kept by the second only (k < P, the smaller count) at
+    positions 2k, 2k + 1, then the rest in ascending order.  Rows take their blocks in list
+    order, so the output over these pairs and the one over adjacent pairs (ress_sparse_attn
+    on the same CSR) differ by rounding: both are within the attention tolerance of the
+    exact result, and they are equal bit for bit on the 128-token grid, where both walk the
+    same lists.  The pairing keeps fewer one-sided union entries than adjacent pairs,
+    and is the greedy matching by overlap of the kept sets."""
     wl = synth.WORKLOADS[name]
     layer = G.Layer(synth.make_inputs(wl), wl.n_special, wl.budgets(), wl.rounds, wl.rho,
                     q_block=q_block)
@@ -199,12 +209,19 @@ def test_forward_item_lists(name, q_block):
             seen += rows
             la = kept(h, rows[0])
             lb = kept(h, rows[1]) if len(rows) > 1 else (la if rpi == 1 else np.zeros(0, int))
-            want = sorted(set(la) | set(lb))
-            masks = [int(j in set(la)) | (int(j in set(lb)) << 1) for j in want]
+            sa, sb = set(la), set(lb)
+            only_a, only_b = sorted(sa - sb), sorted(sb - sa)
+            P = min(len(only_a), len(only_b))
+            want = []
+            for k in range(P):
+                want += [only_a[k] | (1 << 16), only_b[k] | (2 << 16)]
+            paired_set = set(only_a[:P]) | set(only_b[:P])
+            want += [j | ((int(j in sa) | (int(j in sb) << 1)) << 16)
+                     for j in sorted((sa | sb) - paired_set)]
             s0, n = rp[h * layer.nq + u * rpi], plen[h * items + u]
             got = plist[s0:s0 + n]
             assert n == len(want), (h, u)
-            assert np.array_equal(got & 0xffff, want) and np.array_equal(got >> 16, masks), (h, u)
+            assert np.array_equal(got, want), (h, u)
             entries += len(la) + len(lb)
             union += n
             if u < npaired:  # the adjacent pair of the same slot, for comparison
@@ -230,7 +247,19 @@ def test_forward_item_lists(name, q_block):
                 assert got == want, (h, w0)
     r.sparse_attn(layer.d, layer.Q, layer.K, layer.V, b.row_ptr, b.col_idx, b.O, b.ws)
     r.status(b.ws)
-    assert torch.equal(O_f.view(torch.int16), b.O.view(torch.int16))
+    if q_block == 128:
+        assert torch.equal(O_f.view(torch.int16), b.O.view(torch.int16))
+    else:
+        # each within the tolerance of the exact result, beyond its rounding to bf16
+        a, s = O_f.float(), b.O.float()
+        assert bool(((a - s).abs() <= 2 * G.ATT_MAX_ABS + 2.0 ** -8 * (a.abs() + s.abs())).all())
+        assert float((a - s).abs().mean() / s.abs().mean()) <= 2 * G.ATT_MEAN_REL
+        b.O.copy_(O_f)
+        rng = np.random.default_rng(7)
+        rows = [(h, i) for h in range(layer.H) for i in range(layer.nq)]
+        rows = [rows[k] for k in sorted(rng.choice(len(rows), min(len(rows), 200), replace=False))]
+        r2 = G.compare_attention_bf16(layer, rows)
+        assert r2["max_abs"] <= G.ATT_MAX_ABS and r2["mean_rel"] <= G.ATT_MEAN_REL, r2
 
 
 def test_deterministic_bits():
@@ -277,6 +306,92 @@ def test_dense_csr_is_dense_attention(tiny):
     diff = (O_.float() - ref).abs()
     assert diff.max().item() <= G.ATT_MAX_ABS
     assert diff.sum().item() / ref.abs().sum().item() <= G.ATT_MEAN_REL
+
+
+def _caller_csr(layer, kept):
+    H, nq = layer.H, layer.nq
+    lens = [len(kept[(h, i)]) for h in range(H) for i in range(nq)]
+    rp = torch.tensor(np.concatenate([[0], np.cumsum(lens)]), dtype=torch.int32, device="cuda")
+    ci = torch.tensor(np.concatenate([kept[(h, i)] for h in range(H) for i in range(nq)]),
+                      dtype=torch.int32, device="cuda")
+    return rp, ci
+
+
+def _attn_f32(layer, kept):
+    rp, ci = _caller_csr(layer, kept)
+    out = torch.empty_like(layer.O32)
+    layer.ress.sparse_attn_f32(layer.d, layer.Q, layer.K, layer.V, rp, ci, out, layer.buf.ws)
+    layer.ress.status(layer.buf.ws)
+    return out
+
+
+def _bf16_p_bound(layer, kept, h, i):
+    """Exact attention of query block (h, i) over its kept blocks (float64) and a bound on
+    the kernel's error there: each probability is rounded to bf16 (8 significant bits,
+    relative error at most u = 2^-8) and the row sum is formed from the same rounded values,
+    so the output moves by at most u / (1 - u) sum_k w_k |v_k - o| <= 1.01 u (sum_k w_k |v_k|
+    + |o|); 2^-12 sum_k w_k |v_k| more covers the float32 scores, exponentials and
+    accumulations (about 2^-13 of it for 2,000 keys)."""
+    Q, K, V = (G.widen(layer.bits[n]) for n in ("Q", "K", "V"))
+    N = layer.N
+    q = Q[i * 64:min(N, (i + 1) * 64), h].astype(np.float64)
+    idx = np.concatenate([np.arange(j * 64, min(N, (j + 1) * 64)) for j in kept[(h, i)]])
+    k, v = K[idx, h].astype(np.float64), V[idx, h].astype(np.float64)
+    s = q @ k.T / 8.0
+    w = np.exp(s - s.max(1, keepdims=True))
+    w /= w.sum(1, keepdims=True)
+    o = w @ v
+    wv = w @ np.abs(v)
+    return o, 1.01 * 2.0 ** -8 * (wv + np.abs(o)) + 2.0 ** -12 * wv
+
+
+@pytest.mark.parametrize("case", ["disjoint", "leftover", "unequal"])
+def test_one_sided_lists(tiny, case):
+    """Caller lists in which the two query blocks of each adjacent pair keep (mostly) disjoint
+    key blocks, so that most union entries are one-sided (the other block's rows get P = 0)
+    and lead the list, alternating between the two blocks.  "disjoint": every entry is
+    one-sided.  "leftover": three alternating pairs, then one-sided entries of the second
+    block, shared blocks and the ragged last block.  In both every row still takes its blocks
+    in ascending order, and its float32 output is bit for bit that of the same row given a
+    partner with its own list (no one-sided entry at all): a row's result depends only on its
+    own blocks and their order.  "unequal": a third of the blocks against the rest, where the
+    alternation reorders rows' blocks.  In all three the output is within the bound of bf16
+    probability rounding of the exact attention, and the bf16 output is the rounding of the
+    float32 one."""
+    H, nb, nq = tiny.H, tiny.nb, tiny.nq
+    kept = {}
+    for h in range(H):
+        for i in range(nq):
+            if case == "disjoint":
+                ks = [j for j in range(nb - 1) if j % 2 == (i + h) % 2]
+            elif case == "leftover":
+                ks = ([1, 3, 5, nb - 3, nb - 2] if i % 2 == 0
+                      else list(range(0, nb - 4, 2)) + [nb - 3, nb - 2, nb - 1])
+            elif i % 2 == 0:
+                ks = [j for j in range(nb - 1) if j % 3 == 0]
+            else:
+                ks = [0] + [j for j in range(nb) if j % 3 != 0]
+            kept[(h, i)] = np.asarray(sorted(ks), dtype=np.int64)
+    got = _attn_f32(tiny, kept)
+    rp, ci = _caller_csr(tiny, kept)
+    O16 = torch.empty_like(tiny.buf.O)
+    tiny.ress.sparse_attn(tiny.d, tiny.Q, tiny.K, tiny.V, rp, ci, O16, tiny.buf.ws)
+    tiny.ress.status(tiny.buf.ws)
+    assert torch.equal(got.to(torch.bfloat16).view(torch.int16), O16.view(torch.int16))
+    got = got.cpu().numpy()
+    if case != "unequal":
+        alone = np.empty_like(got)
+        for par in (0, 1):  # rows of parity par, each sharing its tile with a copy of its list
+            same = {(h, i): kept[(h, min(nq - 1, i - i % 2 + par))] for h in range(H) for i in range(nq)}
+            o = _attn_f32(tiny, same).cpu().numpy()
+            for i in range(par, nq, 2):
+                alone[i * 64:(i + 1) * 64] = o[i * 64:(i + 1) * 64]
+        assert np.array_equal(got.view(np.uint32), alone.view(np.uint32))
+    for h in range(H):
+        for i in range(nq):
+            o, bound = _bf16_p_bound(tiny, kept, h, i)
+            g = got[i * 64:i * 64 + o.shape[0], h, :]
+            assert np.all(np.abs(g - o) <= bound), (h, i, float(np.abs(g - o).max()))
 
 
 def test_bad_csr_index_is_reported_not_faulted(tiny):
@@ -436,11 +551,11 @@ def test_equal_keys_keep_the_lowest_indices(q_block):
 def test_forward_host_equals_forward(name, q_block):
     """ress_forward_host (copies in, selection, then the attention in chunks of query rows
     whose output rows are copied out as each chunk completes, on library streams joined back
-    into the caller's) gives the bits of the staged device calls, and the caller's stream
-    alone orders the result: every output row is on the host once that stream is done."""
+    into the caller's) gives the bits of the device forward, and the caller's stream alone
+    orders the result: every output row is on the host once that stream is done."""
     wl = synth.WORKLOADS[name]
     ref = G.Layer(synth.make_inputs(wl), wl.n_special, wl.budgets(), wl.rounds, wl.rho,
-                  q_block=q_block).run()
+                  q_block=q_block).run_forward()
     layer = G.Layer(synth.make_inputs(wl), wl.n_special, wl.budgets(), wl.rounds, wl.rho,
                     q_block=q_block)
     r, b = layer.ress, layer.buf
@@ -743,7 +858,8 @@ def test_timed_out_wait_is_reported_and_context_stays_usable(tiny):
     import paper_2609_35593_gb300 as ress
     layer, _ = layer_for("tiny_v2")
     r, b = layer.ress, layer.buf
-    r.prepare_wo(layer.d, layer.W, b.F)
+    layer.run_forward()
+    before = b.O.clone()
     r.wait_selftest(b.ws, 20000)
     with pytest.raises(ress.RessError) as e:
         r.status(b.ws)
@@ -752,7 +868,7 @@ def test_timed_out_wait_is_reported_and_context_stays_usable(tiny):
     r.forward(layer.d, layer.Q, layer.K, layer.V, b.F, layer.c_h, layer.rounds, layer.rho, b.ws,
               b.row_ptr, b.col_idx, b.O, b.J_best)
     r.status(b.ws)
-    assert torch.equal(b.O.view(torch.int16), tiny.buf.O.view(torch.int16))
+    assert torch.equal(b.O.view(torch.int16), before.view(torch.int16))
 
 
 def test_invalid_variant_is_rejected(tiny):
