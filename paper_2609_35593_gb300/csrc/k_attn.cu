@@ -390,20 +390,28 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
     const uint32_t idesc_pv = idesc_bf16_f32(kRows, kNO, true);
     const uint32_t ones_addr = smem_u32(S.ONES);
     const uint32_t q_addr = smem_u32(S.Q);
+    // Descriptors of stage 0's K and V tiles (V with the ONES atom LBO bytes after it).  A
+    // descriptor's start address (bits 0-13, in 16-byte units) is below 2^14 for every
+    // shared-memory address here, so stage s and K16 slice k are plain adds: the stages
+    // lie kTileBytes apart, a K slice 32 bytes on and a V slice 2048 bytes on, and V's
+    // leading byte offset (bits 16-29, to ONES) shrinks by the same stage stride.
+    constexpr uint64_t kStageUnits = kTileBytes >> 4;
+    const uint64_t kdesc0 = sdesc_sw128(smem_u32(S.K[0]));
+    const uint32_t v0 = smem_u32(S.V[0]);
+    const uint64_t vdesc0 = (sdesc_sw128(v0) & ~(0x3FFFull << 16)) |
+                            ((uint64_t)(((ones_addr - v0) >> 4) & 0x3FFFu) << 16);
     bool prev_first = false;
     int it = 0;
     auto issue_pv = [&](int pg, bool first) -> bool {
       const int pb = pg & 1, ps = pg % kStages;
+      // the N = 80 B operand: atom 0 = V (channels), atom 1 = ONES, LBO bytes after it
+      const uint64_t vd = vdesc0 + (uint64_t)ps * kStageUnits - (((uint64_t)ps * kStageUnits) << 16);
       if (!warp_wait(&S.p_full[pb], (pg >> 1) & 1, abort)) return false;
       tc_fence_after();
-      const uint32_t v_addr = smem_u32(S.V[ps]);
-      // the N = 80 B operand: atom 0 = V (channels), atom 1 = ONES, LBO bytes after it
-      const uint64_t lbo = (uint64_t)(((ones_addr - v_addr) >> 4) & 0x3FFFu) << 16;
       if (leader) {
 #pragma unroll
         for (int k = 0; k < 4; ++k)
-          mma_bf16_ts(tmem + kColO, tmem + kColS0 + 64 * pb + 8 * k,
-                      (sdesc_sw128(v_addr + 2048 * k) & ~(0x3FFFull << 16)) | lbo, idesc_pv,
+          mma_bf16_ts(tmem + kColO, tmem + kColS0 + 64 * pb + 8 * k, vd + 128 * k, idesc_pv,
                       (k > 0 || !first) ? 1u : 0u);
         mma_commit(&S.kv_empty[ps]);  // also tells the softmax warps that P V has landed
       }
@@ -442,12 +450,12 @@ __global__ void __launch_bounds__(kAttnThreads, 2)
       // no thread-sync fence here: S_g overwrites what softmax read for tile g-2, and the
       // fence after waiting for P_{g-2} already orders every later tcgen05 operation
       const int s = g % kStages, b = g & 1;
-      const uint32_t k_addr = smem_u32(S.K[s]);
+      const uint64_t kd = kdesc0 + (uint64_t)s * kStageUnits;
       if (leader) {
 #pragma unroll
         for (int k = 0; k < 4; ++k)
-          mma_bf16_ts(tmem + kColS0 + 64 * b, tmem + kColQ + 8 * k, sdesc_sw128(k_addr + 32 * k),
-                      idesc_qk, k > 0 ? 1u : 0u);
+          mma_bf16_ts(tmem + kColS0 + 64 * b, tmem + kColQ + 8 * k, kd + 2 * k, idesc_qk,
+                      k > 0 ? 1u : 0u);
         mma_commit(&S.s_full[b]);
       }
       __syncwarp();
