@@ -163,6 +163,22 @@ def greedy_pairs(keep):
     return sorted(pairs)
 
 
+def item_list(la, lb):
+    """The attention item list of two query blocks' kept lists (host restatement of the
+    layout): the k-th block kept by the first only and the k-th kept by the second only
+    (k below the smaller count, both ascending) at positions 2k, 2k + 1, then the rest of the
+    union ascending; entry j | mask << 16 (bit 0: the first block keeps j, bit 1: the second)."""
+    sa, sb = set(int(j) for j in la), set(int(j) for j in lb)
+    only_a, only_b = sorted(sa - sb), sorted(sb - sa)
+    P = min(len(only_a), len(only_b))
+    out = []
+    for k in range(P):
+        out += [only_a[k] | (1 << 16), only_b[k] | (2 << 16)]
+    lead = set(only_a[:P]) | set(only_b[:P])
+    out += [j | ((int(j in sa) | (int(j in sb) << 1)) << 16) for j in sorted((sa | sb) - lead)]
+    return np.asarray(out, dtype=np.int64)
+
+
 @pytest.mark.parametrize("name,q_block", [("tiny_v2", 64), ("tiny_v2", 128), ("vggt_v8", 64),
                                           ("vggt_v8", 128), ("vggt_v32", 64)])
 def test_forward_item_lists(name, q_block):
@@ -209,15 +225,7 @@ def test_forward_item_lists(name, q_block):
             seen += rows
             la = kept(h, rows[0])
             lb = kept(h, rows[1]) if len(rows) > 1 else (la if rpi == 1 else np.zeros(0, int))
-            sa, sb = set(la), set(lb)
-            only_a, only_b = sorted(sa - sb), sorted(sb - sa)
-            P = min(len(only_a), len(only_b))
-            want = []
-            for k in range(P):
-                want += [only_a[k] | (1 << 16), only_b[k] | (2 << 16)]
-            paired_set = set(only_a[:P]) | set(only_b[:P])
-            want += [j | ((int(j in sa) | (int(j in sb) << 1)) << 16)
-                     for j in sorted((sa | sb) - paired_set)]
+            want = item_list(la, lb)
             s0, n = rp[h * layer.nq + u * rpi], plen[h * items + u]
             got = plist[s0:s0 + n]
             assert n == len(want), (h, u)
@@ -356,8 +364,8 @@ def test_one_sided_lists(tiny, case):
     partner with its own list (no one-sided entry at all): a row's result depends only on its
     own blocks and their order.  "unequal": a third of the blocks against the rest, where the
     alternation reorders rows' blocks.  In all three the output is within the bound of bf16
-    probability rounding of the exact attention, and the bf16 output is the rounding of the
-    float32 one."""
+    probability rounding of the exact attention, the bf16 output is the rounding of the
+    float32 one, and the lists k_pairs builds follow item_list's layout."""
     H, nb, nq = tiny.H, tiny.nb, tiny.nq
     kept = {}
     for h in range(H):
@@ -373,6 +381,18 @@ def test_one_sided_lists(tiny, case):
                 ks = [0] + [j for j in range(nb) if j % 3 != 0]
             kept[(h, i)] = np.asarray(sorted(ks), dtype=np.int64)
     got = _attn_f32(tiny, kept)
+    # the union lists k_pairs wrote for the adjacent pairs (2p, 2p + 1) of each head
+    plist = tiny.ws("t", torch.int32)
+    npairs = (nq + 1) // 2
+    plen = tiny.ws("plen", torch.int32)[:H * npairs]
+    offs = np.concatenate([[0], np.cumsum([len(kept[(h, i)]) for h in range(H) for i in range(nq)])])
+    for h in range(H):
+        for pp in range(npairs):
+            lb = kept[(h, 2 * pp + 1)] if 2 * pp + 1 < nq else np.zeros(0, np.int64)
+            want = item_list(kept[(h, 2 * pp)], lb)
+            s0 = offs[h * nq + 2 * pp]
+            assert plen[h * npairs + pp] == len(want), (h, pp)
+            assert np.array_equal(plist[s0:s0 + len(want)], want), (h, pp)
     rp, ci = _caller_csr(tiny, kept)
     O16 = torch.empty_like(tiny.buf.O)
     tiny.ress.sparse_attn(tiny.d, tiny.Q, tiny.K, tiny.V, rp, ci, O16, tiny.buf.ws)
