@@ -230,8 +230,12 @@ int ress_sparse_attn_f32(const ress_dims* dims, const uint16_t* Q, const uint16_
 
 /* ress_score, ress_restore and ress_sparse_attn in order on one stream.  Inside the forward
  * the CSR kernel also writes the attention items' union lists into the workspace, so the
- * attention starts without the union pass of ress_sparse_attn; O, the CSR and J_best are
- * bit for bit those of the three separate calls. */
+ * attention starts without the union pass of ress_sparse_attn.  The CSR and J_best are bit
+ * for bit those of the three separate calls.  O is too on the 128-token query grid; on the
+ * 64-token grid the forward pairs the candidate query blocks by the overlap of their kept
+ * lists (ress_sparse_attn pairs adjacent blocks), which changes only the order in which a
+ * row takes its own kept blocks, so O agrees with the separate calls' to rounding (and is
+ * deterministic). */
 int ress_forward(const ress_dims* dims, const uint16_t* Q, const uint16_t* K, const uint16_t* V,
                  const float* F, const int32_t* c_h_host, int32_t rounds, float rho, void* ws,
                  size_t ws_bytes, int32_t* row_ptr, int32_t* col_idx, int64_t col_capacity,
